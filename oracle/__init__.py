@@ -1,0 +1,210 @@
+"""Plain CPU oracle for the aTTT update step -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package.  The CUDA library never imports, links
+or calls it, and it shares no code with that library.
+
+The arithmetic lives in ``attt_oracle.c`` (fp64 sums over the bf16 inputs,
+Eqs. 8-10, Eq. 2 and Algorithm 1 of the aTTT paper); this module only builds
+it with gcc and marshals numpy arrays through ctypes.
+
+Every function here has a pin in ``tests/test_oracle_*.py`` (hand-worked
+example, brute force, two independent counters, finite differences, torch CPU
+library routines, closed forms); none is "parity unpinned".
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "attt_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile attt_oracle.c into liboracle.so next to it (gcc, OpenMP)."""
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off",
+           "-fno-fast-math", "-std=c11", _SRC, "-o", tmp, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        i64 = ctypes.c_int64
+        lib.oracle_count_naive.restype = i64
+        lib.oracle_count_naive.argtypes = [P, i64, P, ctypes.c_int]
+        lib.oracle_exposure_naive.restype = None
+        lib.oracle_exposure_naive.argtypes = [P, i64, P, i64, ctypes.c_int, P]
+        lib.oracle_exposure_sorted.restype = None
+        lib.oracle_exposure_sorted.argtypes = [P, i64, P, i64, ctypes.c_int, P]
+        lib.oracle_weights_from_exposure.restype = None
+        lib.oracle_weights_from_exposure.argtypes = [P, i64, ctypes.c_float, P]
+        lib.oracle_ce_rows.restype = None
+        lib.oracle_ce_rows.argtypes = [P, P, P, P, i64, i64, i64, P, i64, P, P, P]
+        lib.oracle_ce_loss.restype = ctypes.c_double
+        lib.oracle_ce_loss.argtypes = [P, P, P, P, i64, i64, i64, P, P, P]
+        lib.oracle_lora_grad.restype = None
+        lib.oracle_lora_grad.argtypes = [P, P, P, P, i64, i64, i64, ctypes.c_int,
+                                         ctypes.c_double, P, P]
+        lib.oracle_sgd_step.restype = None
+        lib.oracle_sgd_step.argtypes = [P, P, i64, ctypes.c_float]
+        lib.oracle_to_bf16.restype = None
+        lib.oracle_to_bf16.argtypes = [P, P, i64]
+        lib.oracle_num_threads.restype = ctypes.c_int
+        lib.oracle_num_threads.argtypes = []
+        lib.oracle_set_num_threads.restype = None
+        lib.oracle_set_num_threads.argtypes = [ctypes.c_int]
+        _lib = lib
+        return lib
+
+
+def _c(a, dtype):
+    a = np.ascontiguousarray(a, dtype=dtype)
+    return a, a.ctypes.data_as(ctypes.c_void_p)
+
+
+def num_threads() -> int:
+    return int(_load().oracle_num_threads())
+
+
+def set_num_threads(t: int) -> None:
+    _load().oracle_set_num_threads(int(t))
+
+
+# --------------------------------------------------------------------------
+# Eq. 8 / Eq. 9
+# --------------------------------------------------------------------------
+
+def count_naive(H, g) -> int:
+    """count(g, H) of Eq. 8: every start position, overlaps included."""
+    H, pH = _c(H, np.int32)
+    g, pg = _c(g, np.int32)
+    return int(_load().oracle_count_naive(pH, H.size, pg, g.size))
+
+
+def exposure(H, x, n: int, method: str = "sorted") -> np.ndarray:
+    """f_k(j) of Eq. 8 for every position j of x (int64)."""
+    H, pH = _c(H, np.int32)
+    x, px = _c(x, np.int32)
+    f = np.zeros(x.size, dtype=np.int64)
+    fn = {"naive": _load().oracle_exposure_naive,
+          "sorted": _load().oracle_exposure_sorted}[method]
+    fn(pH, H.size, px, x.size, int(n), f.ctypes.data_as(ctypes.c_void_p))
+    return f
+
+
+def weights_from_exposure(f, w_min: float) -> np.ndarray:
+    """w_{k,j} of Eq. 9 in fp32 (IEEE divide, then the floor)."""
+    f, pf = _c(f, np.int64)
+    w = np.zeros(f.size, dtype=np.float32)
+    _load().oracle_weights_from_exposure(pf, f.size, ctypes.c_float(w_min),
+                                         w.ctypes.data_as(ctypes.c_void_p))
+    return w
+
+
+def ngram_weights(H, x, n: int, w_min: float = 0.05, method: str = "sorted") -> np.ndarray:
+    """Algorithm 1's per-token weight loop: Eq. 8 then Eq. 9."""
+    return weights_from_exposure(exposure(H, x, n, method), w_min)
+
+
+# --------------------------------------------------------------------------
+# Eq. 10 and dh
+# --------------------------------------------------------------------------
+
+def ce_rows(h_bf16, W_bf16, tgt, w, rows, with_dh: bool = True):
+    """Per-row lse, nll and (optionally) dh of Eq. 10 for the given rows.
+
+    h_bf16 [L, d] and W_bf16 [V, d] are uint16 arrays holding bf16 bits."""
+    h, ph = _c(h_bf16, np.uint16)
+    W, pW = _c(W_bf16, np.uint16)
+    t, pt = _c(tgt, np.int32)
+    wv, pw = _c(w, np.float32)
+    rows, pr = _c(rows, np.int64)
+    L, d = h.shape
+    V = W.shape[0]
+    lse = np.zeros(rows.size, dtype=np.float64)
+    nll = np.zeros(rows.size, dtype=np.float64)
+    dh = np.zeros((rows.size, d), dtype=np.float64) if with_dh else None
+    _load().oracle_ce_rows(ph, pW, pt, pw, L, d, V, pr, rows.size,
+                           lse.ctypes.data_as(ctypes.c_void_p),
+                           nll.ctypes.data_as(ctypes.c_void_p),
+                           dh.ctypes.data_as(ctypes.c_void_p) if with_dh else None)
+    return lse, nll, dh
+
+
+def ce_loss(h_bf16, W_bf16, tgt, w, with_dh: bool = True):
+    """Eq. 10 over all rows: (loss, lse[L], nll[L], dh[L, d] or None)."""
+    h, ph = _c(h_bf16, np.uint16)
+    W, pW = _c(W_bf16, np.uint16)
+    t, pt = _c(tgt, np.int32)
+    wv, pw = _c(w, np.float32)
+    L, d = h.shape
+    V = W.shape[0]
+    lse = np.zeros(L, dtype=np.float64)
+    nll = np.zeros(L, dtype=np.float64)
+    dh = np.zeros((L, d), dtype=np.float64) if with_dh else None
+    loss = _load().oracle_ce_loss(ph, pW, pt, pw, L, d, V,
+                                  lse.ctypes.data_as(ctypes.c_void_p),
+                                  nll.ctypes.data_as(ctypes.c_void_p),
+                                  dh.ctypes.data_as(ctypes.c_void_p) if with_dh else None)
+    return float(loss), lse, nll, dh
+
+
+# --------------------------------------------------------------------------
+# LoRA gradients and the SGD step
+# --------------------------------------------------------------------------
+
+def lora_grad(x_bf16, dy_bf16, A_bf16, B_bf16, scale: float):
+    """(dA [din, r], dB [r, dout]) in fp64 for y = x W0 + s (x A) B."""
+    x, px = _c(x_bf16, np.uint16)
+    dy, pdy = _c(dy_bf16, np.uint16)
+    A, pA = _c(A_bf16, np.uint16)
+    B, pB = _c(B_bf16, np.uint16)
+    L, din = x.shape
+    dout = dy.shape[1]
+    r = A.shape[1]
+    assert dy.shape[0] == L and A.shape[0] == din and B.shape == (r, dout)
+    dA = np.zeros((din, r), dtype=np.float64)
+    dB = np.zeros((r, dout), dtype=np.float64)
+    _load().oracle_lora_grad(px, pdy, pA, pB, L, din, dout, r, float(scale),
+                             dA.ctypes.data_as(ctypes.c_void_p),
+                             dB.ctypes.data_as(ctypes.c_void_p))
+    return dA, dB
+
+
+def sgd_step(p32, g32, lr: float):
+    """Eq. 2: returns (p - lr*g in fp32, its bf16 refresh as uint16)."""
+    p = np.array(p32, dtype=np.float32, copy=True)
+    g, pg = _c(g32, np.float32)
+    _load().oracle_sgd_step(p.ctypes.data_as(ctypes.c_void_p), pg, p.size,
+                            ctypes.c_float(lr))
+    b = np.zeros(p.shape, dtype=np.uint16)
+    _load().oracle_to_bf16(p.ctypes.data_as(ctypes.c_void_p),
+                           b.ctypes.data_as(ctypes.c_void_p), p.size)
+    return p, b
+
+
+def to_bf16(p32) -> np.ndarray:
+    """fp32 -> bf16 bits, round to nearest even."""
+    p, pp = _c(p32, np.float32)
+    b = np.zeros(p.shape, dtype=np.uint16)
+    _load().oracle_to_bf16(pp, b.ctypes.data_as(ctypes.c_void_p), p.size)
+    return b

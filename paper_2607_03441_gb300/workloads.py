@@ -1,0 +1,230 @@
+"""Seeded synthetic inputs for the aTTT update step.
+
+This module only draws random inputs; it holds none of the method's
+arithmetic (no counting, no weighting, no loss, no gradients), so both the
+CUDA path and the CPU oracle may take their inputs from it.
+
+Recipe (stands in for the paper's ALFWorld / SWE-bench update texts and the
+Qwen / Gemma weights, none of which are available here):
+
+* Token ids: truncated Zipf(1.1) over the vocabulary, P(k) proportional to
+  k^-1.1 for k = 1..V, drawn by inverse CDF over an fp64 cumulative table,
+  id = k - 1 (no permutation, so low ids are the hot ones).
+* History: iid Zipf ids of the stated length.
+* Repeated spans: a fraction ``frac`` of the update's positions is overwritten
+  by spans copied from the history.  Span lengths are uniform in [8, 32]
+  (the last one truncated so exactly round(frac * L) positions are covered),
+  source starts are uniform in the history, and the spans are laid out in a
+  random order with uniformly random gaps between them (no overlaps).
+* Dense tensors: fp32 normal samples rounded once to bf16 (round to nearest
+  even); hidden ~ N(0, 1), LM head ~ N(0, 0.02), LoRA A ~ N(0, 0.02),
+  B = 0.01 * N(0, 1), activations x and upstream grads dy ~ N(0, 1).
+
+Every array comes from its own numpy PCG64 stream keyed by (seed, name).
+"""
+from __future__ import annotations
+
+import dataclasses
+import functools
+import zlib
+from typing import Dict, List, Optional, Tuple
+
+import numpy as np
+
+W_MIN = 0.05          # the paper's weight floor (Appendix C)
+LORA_LR = 5e-4        # the paper's learning rate (Appendix C)
+
+
+def rng_for(seed: int, name: str) -> np.random.Generator:
+    """Independent, reproducible stream for one named array of one config."""
+    return np.random.default_rng([int(seed), zlib.crc32(name.encode())])
+
+
+@functools.lru_cache(maxsize=8)
+def _zipf_cdf(V: int, a: float) -> np.ndarray:
+    k = np.arange(1, V + 1, dtype=np.float64)
+    c = np.cumsum(k ** (-a))
+    return c / c[-1]
+
+
+def zipf_ids(rng: np.random.Generator, n: int, V: int, a: float = 1.1) -> np.ndarray:
+    """n iid token ids in [0, V) from a truncated Zipf(a) (inverse CDF)."""
+    u = rng.random(n)
+    ids = np.searchsorted(_zipf_cdf(int(V), float(a)), u, side="right")
+    return np.minimum(ids, V - 1).astype(np.int32)
+
+
+def copy_spans(rng: np.random.Generator, x: np.ndarray, H: np.ndarray, frac: float) -> np.ndarray:
+    """Overwrite round(frac*len(x)) positions of x with spans copied from H."""
+    x = np.array(x, dtype=np.int32, copy=True)
+    L = x.size
+    target = int(round(frac * L))
+    if target <= 0 or H.size == 0:
+        return x
+    target = min(target, L)
+    max_len = int(min(32, H.size))
+    min_len = int(min(8, max_len))
+    lens: List[int] = []
+    while sum(lens) < target:
+        lens.append(int(rng.integers(min_len, max_len + 1)))
+    lens[-1] -= sum(lens) - target
+    if lens[-1] <= 0:
+        lens.pop()
+    k = len(lens)
+    gap_total = L - target
+    # random composition of gap_total into k+1 non-negative gaps
+    cuts = np.sort(rng.integers(0, gap_total + 1, size=k))
+    gaps = np.diff(np.concatenate([[0], cuts, [gap_total]]))
+    pos = 0
+    for i, ln in enumerate(lens):
+        pos += int(gaps[i])
+        src = int(rng.integers(0, H.size - ln + 1))
+        x[pos:pos + ln] = H[src:src + ln]
+        pos += ln
+    return x
+
+
+def bf16_bits(a: np.ndarray) -> np.ndarray:
+    """fp32 array -> bf16 bit patterns (uint16), round to nearest even."""
+    a = np.ascontiguousarray(a, dtype=np.float32)
+    out = np.empty(a.shape, dtype=np.uint16)
+    flat_in = a.reshape(-1).view(np.uint32)
+    flat_out = out.reshape(-1)
+    step = 1 << 24
+    for s in range(0, flat_in.size, step):
+        u = flat_in[s:s + step].astype(np.uint64)
+        lsb = (u >> 16) & 1
+        flat_out[s:s + step] = ((u + 0x7FFF + lsb) >> 16).astype(np.uint16)
+    return out
+
+
+def bf16_to_f32(b: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns (uint16) -> fp32 values (exact)."""
+    return (np.asarray(b, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def normal_bf16(seed: int, name: str, shape: Tuple[int, ...], std: float = 1.0) -> np.ndarray:
+    """bf16 bits of fp32 N(0, std^2) samples, generated in chunks."""
+    rng = rng_for(seed, name)
+    n = int(np.prod(shape))
+    out = np.empty(n, dtype=np.uint16)
+    step = 1 << 24
+    for s in range(0, n, step):
+        m = min(step, n - s)
+        v = rng.standard_normal(m, dtype=np.float32)
+        if std != 1.0:
+            v *= np.float32(std)
+        out[s:s + m] = bf16_bits(v)
+    return out.reshape(shape)
+
+
+# --------------------------------------------------------------------------
+# The five workloads
+# --------------------------------------------------------------------------
+
+@dataclasses.dataclass
+class LoraProj:
+    name: str
+    din: int
+    dout: int
+    x_group: str          # projections with the same x_group share one x
+
+
+@dataclasses.dataclass
+class Workload:
+    name: str
+    seed: int
+    L: int                # update tokens
+    V: int                # vocabulary
+    n: int                # n-gram size
+    hist_len: int         # prior-update history length
+    frac: float           # repeated-span fraction
+    d: int = 0            # hidden size (0: integer path only)
+    r: int = 0            # LoRA rank
+    projs: Tuple[LoraProj, ...] = ()
+    updates: int = 1      # sequential updates (long episode)
+    w_min: float = W_MIN
+
+    @property
+    def scale(self) -> float:
+        """LoRA scale s = alpha / r with alpha = 2r (the paper's 16 / 8)."""
+        return 2.0
+
+
+def _qkvo(d: int, kv: int) -> Tuple[LoraProj, ...]:
+    return (LoraProj("q", d, d, "attn"), LoraProj("k", d, kv, "attn"),
+            LoraProj("v", d, kv, "attn"), LoraProj("o", d, d, "o"))
+
+
+WORKLOADS: Dict[str, Workload] = {
+    "tiny": Workload("tiny", 0, L=256, V=8192, n=4, hist_len=2048, frac=0.30, d=512, r=8,
+                     projs=(LoraProj("proj", 512, 512, "x"),)),
+    "7b": Workload("7b", 1, L=2048, V=152064, n=4, hist_len=65536, frac=0.40, d=3584, r=16,
+                   projs=(LoraProj("q", 3584, 3584, "attn"), LoraProj("v", 3584, 512, "attn"))),
+    "stress": Workload("stress", 2, L=8192, V=128256, n=4, hist_len=1 << 20, frac=0.30),
+    "long": Workload("long", 3, L=4096, V=128256, n=4, hist_len=0, frac=0.05, d=4096, r=32,
+                     projs=_qkvo(4096, 1024) + (LoraProj("gate", 4096, 14336, "mlp"),
+                                                 LoraProj("up", 4096, 14336, "mlp"),
+                                                 LoraProj("down", 14336, 4096, "down")),
+                     updates=32),
+    "32b": Workload("32b", 4, L=8192, V=152064, n=4, hist_len=262144, frac=0.50, d=5120, r=64,
+                    projs=_qkvo(5120, 1024)),
+}
+
+
+def long_episode_frac(k: int, updates: int = 32) -> float:
+    """Repeat fraction of update k (1-based): 5% rising linearly to 80%."""
+    if updates <= 1:
+        return 0.05
+    return 0.05 + 0.75 * (k - 1) / (updates - 1)
+
+
+def history_tokens(wl: Workload, seed: Optional[int] = None) -> np.ndarray:
+    s = wl.seed if seed is None else seed
+    return zipf_ids(rng_for(s, "history"), wl.hist_len, wl.V)
+
+
+def update_tokens(wl: Workload, H: np.ndarray, frac: Optional[float] = None,
+                  tag: str = "update", seed: Optional[int] = None) -> np.ndarray:
+    s = wl.seed if seed is None else seed
+    x = zipf_ids(rng_for(s, tag + "/ids"), wl.L, wl.V)
+    return copy_spans(rng_for(s, tag + "/spans"), x, H, wl.frac if frac is None else frac)
+
+
+def stress_case(n: int, frac: float, seed: int = 2, L: int = 8192, hist_len: int = 1 << 20,
+                V: int = 128256) -> Tuple[np.ndarray, np.ndarray]:
+    """(history, update) for one point of the n-gram stress sweep."""
+    H = zipf_ids(rng_for(seed, "stress/history"), hist_len, V)
+    x = zipf_ids(rng_for(seed, f"stress/ids/n{n}/f{frac:.2f}"), L, V)
+    x = copy_spans(rng_for(seed, f"stress/spans/n{n}/f{frac:.2f}"), x, H, frac)
+    return H, x
+
+
+def long_episode_updates(wl: Workload) -> List[np.ndarray]:
+    """The 32 update texts of the long episode; each copies spans from the
+    concatenation of the updates before it."""
+    out: List[np.ndarray] = []
+    H = np.zeros(0, dtype=np.int32)
+    for k in range(1, wl.updates + 1):
+        x = update_tokens(wl, H, frac=long_episode_frac(k, wl.updates), tag=f"update{k}")
+        out.append(x)
+        H = np.concatenate([H, x])
+    return out
+
+
+def dense_inputs(wl: Workload, with_lm_head: bool = True) -> Dict[str, np.ndarray]:
+    """bf16 bit arrays for the CE and LoRA parts of one update."""
+    s = wl.seed
+    out: Dict[str, np.ndarray] = {}
+    out["h"] = normal_bf16(s, "hidden", (wl.L, wl.d), 1.0)
+    if with_lm_head:
+        out["W"] = normal_bf16(s, "lm_head", (wl.V, wl.d), 0.02)
+    groups = {}
+    for p in wl.projs:
+        if p.x_group not in groups:
+            groups[p.x_group] = normal_bf16(s, f"x/{p.x_group}", (wl.L, p.din), 1.0)
+        out[f"x/{p.name}"] = groups[p.x_group]
+        out[f"A/{p.name}"] = normal_bf16(s, f"A/{p.name}", (p.din, wl.r), 0.02)
+        out[f"B/{p.name}"] = normal_bf16(s, f"B/{p.name}", (wl.r, p.dout), 0.01)
+        out[f"dy/{p.name}"] = normal_bf16(s, f"dy/{p.name}", (wl.L, p.dout), 1.0)
+    return out
