@@ -1,0 +1,224 @@
+/*
+ * attt.h -- C ABI of libattt, the GB300 (sm_103a) hot path of the aTTT
+ * in-episode update step ("Agentic Test-Time Training", Sec. 3.3,
+ * Algorithm 1).
+ *
+ * One update k of Algorithm 1, in call order:
+ *
+ *   attt_ngram_weights      Algorithm 1's loop over j: Eq. 8 exposure f_k(j)
+ *                           against the history table, then Eq. 9 weights.
+ *   attt_weighted_ce_fwd_bwd  Eq. 10 loss and its gradient w.r.t. the final
+ *                           hidden states (the input of the frozen LM head).
+ *   attt_lora_grad          the adapter gradients of the Eq. 2 / Algorithm 1
+ *                           gradient step, given the upstream gradient dy of
+ *                           each adapted projection.
+ *   attt_lora_step          the Eq. 2 SGD step on the adapter parameters.
+ *   attt_history_insert     Algorithm 1's last line: append x_k to the token
+ *                           history H (a concatenation, Sec. 3.3).
+ *
+ * Conventions shared by every call:
+ *   - Pointers named d_* are device pointers on the current CUDA device; the
+ *     caller owns them.  The library owns only attt_history objects.
+ *   - bf16 tensors are passed as attt_bf16 (the IEEE binary32 upper half).
+ *   - Matrices are row-major with the last dimension contiguous.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL = the
+ *     legacy default stream).  Argument errors are returned synchronously and
+ *     launch nothing.  Errors found on the device set a per-device status
+ *     word read by attt_device_status() (or attt_history_status()).
+ *   - No call aborts, traps or throws.  Every device-side wait is bounded;
+ *     a wait that runs out sets ATTT_ERR_TIMEOUT and the kernel returns.
+ *   - Inputs must not alias outputs unless a call says so.
+ */
+#ifndef ATTT_H
+#define ATTT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define ATTT_API __attribute__((visibility("default")))
+#else
+#define ATTT_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t attt_bf16;              /* bf16 bit pattern */
+typedef struct CUstream_st *attt_stream; /* same handle as cudaStream_t */
+
+typedef enum attt_status {
+    ATTT_OK = 0,
+    ATTT_ERR_INVALID_ARG = 1,  /* null/misaligned pointer, bad size or mode    */
+    ATTT_ERR_TABLE_FULL = 2,   /* history table probe sequence exhausted       */
+    ATTT_ERR_TOKEN_RANGE = 3,  /* a CE target outside [0, V)                   */
+    ATTT_ERR_TIMEOUT = 4,      /* a bounded device-side wait ran out           */
+    ATTT_ERR_WORKSPACE = 5,    /* workspace missing or smaller than required   */
+    ATTT_ERR_CUDA = 6,         /* a CUDA runtime call failed                   */
+    ATTT_ERR_UNSUPPORTED = 7,  /* not a GB300-class (sm_103) device, or shape  */
+    ATTT_ERR_CAPACITY = 8      /* history would exceed its max_tokens          */
+} attt_status;
+
+/* Human-readable name of a status code.  Never NULL. */
+ATTT_API const char *attt_status_string(int status);
+
+/* ABI version of this header (major * 100 + minor). */
+ATTT_API int attt_abi_version(void);
+
+/*
+ * Reads and clears the device-side status word of the current device after
+ * synchronising `stream`.  Returns the first error any kernel of this library
+ * recorded since the last read (ATTT_ERR_TIMEOUT, ATTT_ERR_TOKEN_RANGE), or
+ * ATTT_ERR_CUDA if the synchronisation itself failed.
+ */
+ATTT_API attt_status attt_device_status(attt_stream stream);
+
+/* ------------------------------------------------------------------------ */
+/* Token history H (Sec. 3.3: every earlier update's tokens of the episode, */
+/* joined end to end) and its exact n-gram count table.                     */
+/* ------------------------------------------------------------------------ */
+
+typedef struct attt_history attt_history;
+
+/*
+ * Creates an empty history for n-grams of size n (1 <= n <= 16) that can
+ * hold up to max_tokens tokens (>= 0) on the current device.  The library
+ * allocates the token stream (4 B/token) and an exact n-gram count table of
+ * 16 B slots, at least twice as many slots as max_tokens.  *out is set on
+ * success.  Allocation failure returns ATTT_ERR_CUDA.
+ */
+ATTT_API attt_status attt_history_create(int n, int64_t max_tokens, attt_history **out);
+
+/* Frees the history and its device memory (synchronises the device). */
+ATTT_API attt_status attt_history_destroy(attt_history *h);
+
+/*
+ * Empties the history (an episode boundary: the adapter and the history are
+ * reset between episodes, Sec. 4 / Appendix C).  Async on `stream`.
+ */
+ATTT_API attt_status attt_history_reset(attt_history *h, attt_stream stream);
+
+/*
+ * Algorithm 1, last line: H <- H || x_k.  Appends `len` tokens (any int32
+ * values) from d_tokens and counts every n-gram whose last token is new,
+ * including the n-1 n-grams that straddle the old tail and the new tokens,
+ * so insert(a); insert(b) equals insert(a||b).  Counts are exact (keys are
+ * compared token by token).  Returns ATTT_ERR_CAPACITY, launching nothing,
+ * if the history would exceed max_tokens.  A full probe sequence sets
+ * ATTT_ERR_TABLE_FULL in the history's status word.
+ */
+ATTT_API attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_t len,
+                                attt_stream stream);
+
+/* Current history length in tokens (host-side bookkeeping, no sync). */
+ATTT_API int64_t attt_history_length(const attt_history *h);
+
+/* n of the history. */
+ATTT_API int attt_history_ngram(const attt_history *h);
+
+/*
+ * Synchronises `stream`, then reads and clears the history's device status
+ * word (ATTT_ERR_TABLE_FULL, ATTT_ERR_TIMEOUT) and returns it.
+ */
+ATTT_API attt_status attt_history_status(attt_history *h, attt_stream stream);
+
+/*
+ * Eq. 8's count(g, H) for `m` n-grams: d_ngrams is [m, n] int32 (row i is one
+ * n-gram), d_counts is [m] uint32.  Exact.  Async on `stream`.
+ */
+ATTT_API attt_status attt_history_count(const attt_history *h, const int32_t *d_ngrams, int64_t m,
+                               uint32_t *d_counts, attt_stream stream);
+
+/*
+ * Algorithm 1's per-token loop (Eq. 8 then Eq. 9).  For the L tokens of the
+ * update x_k in d_tokens (int32 [L]) writes d_w (fp32 [L]):
+ *   c_s = count(x[s..s+n-1], H)                 for s = 0 .. L-n
+ *   f_j = max{ c_s : max(0, j-n+1) <= s <= min(j, L-n) }   (0 if empty)
+ *   w_j = max(w_min, 1.0f / (1.0f + (float)f_j))  -- IEEE fp32 RN divide
+ * Bit-exact.  0 < w_min <= 1.  L >= 0 (L = 0 launches nothing).
+ * H is not modified; positions of x_k do not count against themselves
+ * (count runs over the previous updates only, Eq. 8).
+ */
+ATTT_API attt_status attt_ngram_weights(const attt_history *h, const int32_t *d_tokens, int64_t L,
+                               float w_min, float *d_w, attt_stream stream);
+
+/* ------------------------------------------------------------------------ */
+/* Eq. 10: token-weighted next-token cross-entropy through the frozen LM    */
+/* head, forward and backward, without materialising the [L, V] logits.     */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Workspace bytes attt_weighted_ce_fwd_bwd needs for (L, d, V).
+ */
+ATTT_API size_t attt_ce_workspace_bytes(int64_t L, int64_t d, int64_t V);
+
+/*
+ * With h = d_h (bf16 [L, d], row j is the state that predicts target x_j),
+ * W = d_W (bf16 [V, d], the frozen LM head), z_j = h_j W^T:
+ *   lse_j  = log sum_v exp(z_jv)
+ *   *d_loss = (1/L) sum_j w_j (lse_j - z_{j, tgt_j})                 (Eq. 10)
+ *   d_dh[j, :] = (w_j / L) (sum_v softmax(z_j)_v W_v - W_{tgt_j})     (fp32)
+ * d_tgt int32 [L] in [0, V); d_w fp32 [L] (the Eq. 9 weights); d_lse fp32
+ * [L] receives lse_j when not NULL.  No gradient for W (it is frozen; only
+ * the adapter trains).  bf16 products, fp32 accumulation.
+ * Requirements: L >= 1, V >= 1, d >= 8 and d % 8 == 0, d_h / d_W / d_dh
+ * 16-byte aligned, d_ws at least attt_ce_workspace_bytes(L, d, V) bytes and
+ * 256-byte aligned.  A target outside [0, V) sets ATTT_ERR_TOKEN_RANGE in the
+ * device status word and makes the loss NaN.
+ */
+ATTT_API attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
+                                     const int32_t *d_tgt, const float *d_w,
+                                     int64_t L, int64_t d, int64_t V,
+                                     float *d_loss, float *d_dh, float *d_lse,
+                                     void *d_ws, size_t ws_bytes, attt_stream stream);
+
+/* ------------------------------------------------------------------------ */
+/* LoRA adapter gradients and the SGD step (Eq. 2; Appendix C adapter:       */
+/* y = x W0 + s (x A) B with A [din, r], B [r, dout], s = alpha / r).        */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Workspace bytes attt_lora_grad needs for `nproj` projections that share one
+ * input x of shape [L, din], with output widths dout[0..nproj-1] and rank r.
+ */
+ATTT_API size_t attt_lora_workspace_bytes(int64_t L, int64_t din, int nproj, const int64_t *dout, int r);
+
+/*
+ * For each projection p < nproj sharing the input x = d_x (bf16 [L, din]),
+ * with upstream gradient dy_p = d_dy[p] (bf16 [L, dout[p]]), adapter
+ * A_p = d_A[p] (bf16 [din, r]) and B_p = d_B[p] (bf16 [r, dout[p]]):
+ *   u_p = x A_p,  v_p = dy_p B_p^T                           ([L, r])
+ *   d_dB[p] = scale * u_p^T dy_p                              (fp32 [r, dout[p]])
+ *   d_dA[p] = scale * x^T v_p                                 (fp32 [din, r])
+ * u and v are rounded to bf16 before the second contraction; products are
+ * bf16, accumulation fp32.  The arrays d_dy, dout, d_A, d_B, d_dA, d_dB are
+ * HOST arrays of nproj entries holding device pointers / sizes.
+ * Requirements: 1 <= nproj <= 8, 1 <= r <= 64, L >= 1, din and every dout
+ * >= 8 and multiples of 8, all tensor pointers 16-byte aligned, d_ws at least
+ * attt_lora_workspace_bytes(...) bytes and 256-byte aligned.
+ */
+ATTT_API attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int nproj,
+                           const attt_bf16 *const *d_dy, const int64_t *dout,
+                           const attt_bf16 *const *d_A, const attt_bf16 *const *d_B,
+                           int r, float scale,
+                           float *const *d_dA, float *const *d_dB,
+                           void *d_ws, size_t ws_bytes, attt_stream stream);
+
+/*
+ * Eq. 2 / Algorithm 1 gradient step (plain SGD, no weight decay):
+ *   A32 <- A32 - lr * dA,  B32 <- B32 - lr * dB     (fp32: product, then
+ *                                                    difference, no FMA)
+ * then refreshes the bf16 copies A16, B16 (round to nearest even) when they
+ * are not NULL.  A32/dA/A16 are [din, r]; B32/dB/B16 are [r, dout].
+ * Bit-exact with the formula.  In-place on A32 and B32.
+ */
+ATTT_API attt_status attt_lora_step(float *d_A32, float *d_B32, const float *d_dA, const float *d_dB,
+                           int64_t din, int64_t dout, int r, float lr,
+                           attt_bf16 *d_A16, attt_bf16 *d_B16, attt_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ATTT_H */

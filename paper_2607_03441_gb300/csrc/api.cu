@@ -1,0 +1,130 @@
+// api.cu -- library-wide host plumbing of libattt: status codes, the device
+// check, the per-device status word, tensor-map encoding and the dynamic
+// shared-memory opt-in.
+#include <cudaTypedefs.h>
+
+#include <map>
+#include <mutex>
+#include <utility>
+
+#include "attt_host.h"
+
+namespace attt {
+
+namespace {
+
+std::mutex g_mu;
+std::map<int, int> g_sms;
+std::map<int, int *> g_status_words;
+std::map<std::pair<const void *, int>, size_t> g_smem_set;
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (!g_encode) {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    return g_encode;
+}
+
+}  // namespace
+
+attt_status current_device(int *dev) {
+    if (cudaGetDevice(dev) != cudaSuccess) return ATTT_ERR_CUDA;
+    int major = 0, minor = 0;
+    if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, *dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, *dev) != cudaSuccess)
+        return ATTT_ERR_CUDA;
+    // The kernels are compiled for sm_103a only.
+    if (major != 10 || minor != 3) return ATTT_ERR_UNSUPPORTED;
+    return ATTT_OK;
+}
+
+int num_sms(int dev) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto it = g_sms.find(dev);
+    if (it != g_sms.end()) return it->second;
+    int n = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+    g_sms[dev] = n;
+    return n;
+}
+
+int *device_status_word(int dev) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto it = g_status_words.find(dev);
+    if (it != g_status_words.end()) return it->second;
+    int *p = nullptr;
+    if (cudaMalloc(&p, 256) != cudaSuccess) return nullptr;
+    if (cudaMemset(p, 0, 256) != cudaSuccess) return nullptr;
+    g_status_words[dev] = p;
+    return p;
+}
+
+bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+                    uint32_t box_inner, uint32_t box_outer) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    if (!aligned16(base) || row_bytes % 16 != 0 || inner == 0 || outer == 0) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {row_bytes};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+bool set_smem_limit(const void *func, size_t bytes, int dev) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto key = std::make_pair(func, dev);
+    auto it = g_smem_set.find(key);
+    if (it != g_smem_set.end() && it->second >= bytes) return true;
+    if (cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes) != cudaSuccess)
+        return false;
+    g_smem_set[key] = bytes;
+    return true;
+}
+
+}  // namespace attt
+
+extern "C" {
+
+const char *attt_status_string(int status) {
+    switch (status) {
+        case ATTT_OK: return "ATTT_OK";
+        case ATTT_ERR_INVALID_ARG: return "ATTT_ERR_INVALID_ARG";
+        case ATTT_ERR_TABLE_FULL: return "ATTT_ERR_TABLE_FULL";
+        case ATTT_ERR_TOKEN_RANGE: return "ATTT_ERR_TOKEN_RANGE";
+        case ATTT_ERR_TIMEOUT: return "ATTT_ERR_TIMEOUT";
+        case ATTT_ERR_WORKSPACE: return "ATTT_ERR_WORKSPACE";
+        case ATTT_ERR_CUDA: return "ATTT_ERR_CUDA";
+        case ATTT_ERR_UNSUPPORTED: return "ATTT_ERR_UNSUPPORTED";
+        case ATTT_ERR_CAPACITY: return "ATTT_ERR_CAPACITY";
+        default: return "ATTT_ERR_UNKNOWN";
+    }
+}
+
+int attt_abi_version(void) { return 100; }
+
+attt_status attt_device_status(attt_stream stream) {
+    int dev;
+    attt_status st = attt::current_device(&dev);
+    if (st != ATTT_OK) return st;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return ATTT_ERR_CUDA;
+    int *w = attt::device_status_word(dev);
+    if (!w) return ATTT_ERR_CUDA;
+    int v = 0;
+    if (cudaMemcpy(&v, w, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return ATTT_ERR_CUDA;
+    if (v != 0 && cudaMemset(w, 0, sizeof v) != cudaSuccess) return ATTT_ERR_CUDA;
+    return (attt_status)v;
+}
+
+}  // extern "C"

@@ -1,0 +1,51 @@
+// attt_host.h -- host-side helpers shared by the translation units of libattt.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "attt.h"
+
+namespace attt {
+
+// Current device if it is a GB300-class part (compute capability 10.3), else
+// ATTT_ERR_UNSUPPORTED / ATTT_ERR_CUDA.
+attt_status current_device(int *dev);
+
+// Number of SMs of a device (cached).
+int num_sms(int dev);
+
+// Per-device status word used by the contraction kernels (lazily allocated).
+int *device_status_word(int dev);
+
+// Encodes a 2-D bf16 tensor map with 128-byte swizzle and zero fill for
+// out-of-range elements.  `inner` is the contiguous extent, `outer` the number
+// of rows, `row_bytes` the row pitch.  Returns false if the driver rejects it.
+bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
+                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
+
+// Raises the dynamic shared memory limit of `func` once per device.
+bool set_smem_limit(const void *func, size_t bytes, int dev);
+
+inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline bool aligned256(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 255u) == 0; }
+inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }
+inline int64_t round_up(int64_t a, int64_t b) { return cdiv(a, b) * b; }
+
+// Workspace carving: bump allocator over a caller-provided buffer, 256-byte
+// aligned pieces.
+struct Carve {
+    char *base;
+    size_t used;
+    template <class T>
+    T *take(size_t count) {
+        used = (size_t)round_up((int64_t)used, 256);
+        T *p = reinterpret_cast<T *>(base ? base + used : nullptr);
+        used += count * sizeof(T);
+        return p;
+    }
+};
+
+}  // namespace attt

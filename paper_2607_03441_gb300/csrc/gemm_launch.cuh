@@ -1,0 +1,94 @@
+// gemm_launch.cuh -- host-side set-up and launch of tc_gemm_kernel.
+#pragma once
+
+#include "attt_host.h"
+#include "tc_gemm.cuh"
+
+namespace attt {
+
+// Description of one contraction D = A * B^T (see tc_gemm.cuh).
+struct GemmProblem {
+    const void *a;        // A base pointer
+    int64_t a_rows_ld;    // A: K-major -> row pitch in elements of the [rows, K] matrix;
+                          //    MN-major -> row pitch of the [K, rows] matrix
+    int64_t a_rows, a_k;  // extents of A's storage (rows = M extent, k = K extent)
+    const void *b;
+    int64_t b_rows_ld;
+    int64_t b_rows, b_k;
+    int M, N, K;
+    int BN;
+    int a_m_off = 0, a_k_off = 0, b_n_off = 0, b_k_off = 0;
+    bool allow_split = false;  // epilogue reduces split-K partials with atomics
+};
+
+constexpr size_t kMaxSmem = 232448;  // 227 KB opt-in per CTA on sm_100-class parts
+
+inline int gemm_stages(int BN) {
+    int s = 8;
+    while (s > 2 && gemm_smem_bytes(BN, s) > kMaxSmem) --s;
+    return s;
+}
+
+inline uint32_t gemm_tmem_cols(int BN) {
+    uint32_t need = 2u * (uint32_t)BN, c = 32;
+    while (c < need) c <<= 1;
+    return c;
+}
+
+template <int EPI, bool A_MN, bool B_MN>
+attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cudaStream_t stream) {
+    if (p.BN < 16 || p.BN > 256 || p.BN % 16 != 0) return ATTT_ERR_INVALID_ARG;
+    if (B_MN && p.BN % 64 != 0) return ATTT_ERR_INVALID_ARG;
+    if (p.M <= 0 || p.N <= 0 || p.K <= 0) return ATTT_ERR_INVALID_ARG;
+    CUtensorMap ta, tb;
+    // K-major operand: storage [rows, K] (K contiguous), box 64 x rows_tile.
+    // MN-major operand: storage [K, rows] (rows contiguous), box 64 x 64.
+    bool ok;
+    if (!A_MN)
+        ok = make_tmap_bf16(&ta, p.a, (uint64_t)p.a_k, (uint64_t)p.a_rows, (uint64_t)p.a_rows_ld * 2, 64, 128);
+    else
+        ok = make_tmap_bf16(&ta, p.a, (uint64_t)p.a_rows, (uint64_t)p.a_k, (uint64_t)p.a_rows_ld * 2, 64, 64);
+    if (!ok) return ATTT_ERR_INVALID_ARG;
+    if (!B_MN)
+        ok = make_tmap_bf16(&tb, p.b, (uint64_t)p.b_k, (uint64_t)p.b_rows, (uint64_t)p.b_rows_ld * 2, 64,
+                            (uint32_t)p.BN);
+    else
+        ok = make_tmap_bf16(&tb, p.b, (uint64_t)p.b_rows, (uint64_t)p.b_k, (uint64_t)p.b_rows_ld * 2, 64, 64);
+    if (!ok) return ATTT_ERR_INVALID_ARG;
+
+    GemmArgs g{};
+    g.M = p.M;
+    g.N = p.N;
+    g.BN = p.BN;
+    g.stages = gemm_stages(p.BN);
+    g.tiles_m = (int)cdiv(p.M, 128);
+    g.tiles_n = (int)cdiv(p.N, p.BN);
+    g.kb_total = (int)cdiv(p.K, 64);
+    const int sms = num_sms(dev);
+    int splits = 1;
+    if (p.allow_split) {
+        const int tiles = g.tiles_m * g.tiles_n;
+        splits = (int)cdiv(sms, tiles);
+        if (splits > g.kb_total) splits = g.kb_total;
+        if (splits < 1) splits = 1;
+    }
+    g.kb_per_split = (int)cdiv(g.kb_total, splits);
+    g.splits = (int)cdiv(g.kb_total, g.kb_per_split);
+    g.a_m_off = p.a_m_off;
+    g.a_k_off = p.a_k_off;
+    g.b_n_off = p.b_n_off;
+    g.b_k_off = p.b_k_off;
+    g.tmem_cols = gemm_tmem_cols(p.BN);
+    g.status = device_status_word(dev);
+    g.ep = ep;
+
+    const size_t smem = gemm_smem_bytes(p.BN, g.stages);
+    auto kern = tc_gemm_kernel<EPI, A_MN, B_MN>;
+    if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
+    const int ntiles = g.tiles_m * g.tiles_n * g.splits;
+    const int grid = ntiles < sms ? ntiles : sms;
+    kern<<<grid, kGemmThreads, smem, stream>>>(ta, tb, g);
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+}  // namespace attt

@@ -1,0 +1,309 @@
+// ngram.cu -- Eq. 8 / Eq. 9 of aTTT on the GPU: the episode's token history
+// H (a concatenation of earlier update texts, Sec. 3.3), an exact n-gram
+// count table over it, and the per-token loss weights of an update.
+//
+// Table design (GB300-first):
+//   * open addressing, linear probing, power-of-two capacity >= 2 * max_tokens
+//     (load factor <= 1/2); one 16-byte slot = {key, count, unused}, so a
+//     probe touches exactly one 32-byte sector;
+//   * key = (32-bit hash tag << 32) | (history position + 1) of the n-gram's
+//     first occurrence, claimed with one 64-bit CAS; equality is decided by
+//     comparing the n tokens in the device-resident history stream (exact,
+//     any vocabulary, any n up to 16) after a tag match;
+//   * insertion aggregates equal n-grams inside a warp (match_any on the hash,
+//     ballot on token equality) so that hot keys cost one atomic per warp;
+//   * the weights kernel stages the update's tokens for a block in shared
+//     memory with coalesced loads, probes once per n-gram, takes the window
+//     max of the counts from shared memory and applies Eq. 9 with an IEEE
+//     round-to-nearest division (bit-exact with the definition).
+#include <cuda_runtime.h>
+
+#include <new>
+
+#include "attt_common.cuh"
+#include "attt_host.h"
+
+namespace attt {
+
+struct __align__(16) Slot {
+    unsigned long long key;  // 0 = empty
+    unsigned int count;
+    unsigned int unused;
+};
+
+constexpr int kMaxN = 16;
+constexpr int kMaxProbe = 1 << 16;
+
+__device__ __forceinline__ unsigned long long mix64(unsigned long long h) {
+    h ^= h >> 33;
+    h *= 0xff51afd7ed558ccdull;
+    h ^= h >> 33;
+    h *= 0xc4ceb9fe1a85ec53ull;
+    h ^= h >> 33;
+    return h;
+}
+
+// Hash of n consecutive tokens.
+__device__ __forceinline__ unsigned long long ngram_hash(const int32_t *t, int n) {
+    unsigned long long h = 0x9e3779b97f4a7c15ull * (unsigned long long)(n + 1);
+    for (int i = 0; i < n; ++i) h = mix64(h ^ (unsigned long long)(uint32_t)t[i]) + 0x632be59bd9b4e019ull;
+    return mix64(h);
+}
+
+__device__ __forceinline__ bool ngram_equal(const int32_t *a, const int32_t *b, int n) {
+    for (int i = 0; i < n; ++i)
+        if (a[i] != b[i]) return false;
+    return true;
+}
+
+// Finds the slot of n-gram `g` (n tokens, anywhere in memory) and returns its
+// count, or 0 if absent.  `hist` is the history token stream.
+__device__ __forceinline__ unsigned int table_lookup(const Slot *table, unsigned long long mask,
+                                                     const int32_t *hist, const int32_t *g, int n,
+                                                     unsigned long long hsh) {
+    const unsigned int tag = (unsigned int)(hsh >> 32);
+    unsigned long long idx = hsh & mask;
+    for (int probe = 0; probe < kMaxProbe; ++probe) {
+        const uint4 s = __ldcg(reinterpret_cast<const uint4 *>(table + idx));
+        const unsigned long long key = ((unsigned long long)s.y << 32) | s.x;
+        if (key == 0ull) return 0u;
+        if ((unsigned int)(key >> 32) == tag) {
+            const unsigned int pos = (unsigned int)key - 1u;
+            if (ngram_equal(hist + pos, g, n)) return s.z;
+        }
+        idx = (idx + 1) & mask;
+    }
+    return 0u;
+}
+
+// One thread per new n-gram start position p in [p_begin, p_begin + count).
+__global__ void __launch_bounds__(256) history_insert_kernel(const int32_t *__restrict__ hist, int64_t p_begin,
+                                                             int64_t count, int n, Slot *table,
+                                                             unsigned long long mask, int *status) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const bool active = i < count;
+    const unsigned amask = __ballot_sync(0xffffffffu, active);
+    if (!active) return;
+    const int lane = threadIdx.x & 31;
+    const int64_t p = p_begin + i;
+    const int32_t *g = hist + p;
+    const unsigned long long hsh = ngram_hash(g, n);
+
+    // Warp aggregation of equal n-grams (hot keys under Zipf text).
+    const unsigned peers = __match_any_sync(amask, hsh);
+    const int leader = __ffs(peers) - 1;
+    const int64_t pl = __shfl_sync(peers, p, leader);
+    const bool same = (lane == leader) || ngram_equal(hist + pl, g, n);
+    const unsigned same_mask = __ballot_sync(peers, same);
+    unsigned int add;
+    if (lane == leader) add = __popc(same_mask);
+    else if (!same) add = 1u;  // 64-bit hash collision between different n-grams
+    else return;
+
+    const unsigned int tag = (unsigned int)(hsh >> 32);
+    const unsigned long long mykey = ((unsigned long long)tag << 32) | (unsigned long long)(uint32_t)(p + 1);
+    unsigned long long idx = hsh & mask;
+    for (int probe = 0; probe < kMaxProbe; ++probe) {
+        Slot *s = table + idx;
+        unsigned long long k = *reinterpret_cast<volatile unsigned long long *>(&s->key);
+        if (k == 0ull) {
+            const unsigned long long old = atomicCAS(&s->key, 0ull, mykey);
+            if (old == 0ull) {
+                atomicAdd(&s->count, add);
+                return;
+            }
+            k = old;
+        }
+        if ((unsigned int)(k >> 32) == tag && ngram_equal(hist + ((unsigned int)k - 1u), g, n)) {
+            atomicAdd(&s->count, add);
+            return;
+        }
+        idx = (idx + 1) & mask;
+    }
+    record_error(status, ATTT_ERR_TABLE_FULL);
+}
+
+// count(g, H) for m query n-grams stored row-major [m, n].
+__global__ void __launch_bounds__(256) history_count_kernel(const int32_t *__restrict__ hist, const Slot *table,
+                                                            unsigned long long mask, const int32_t *__restrict__ q,
+                                                            int64_t m, int n, unsigned int *out) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= m) return;
+    const int32_t *g = q + i * n;
+    out[i] = table_lookup(table, mask, hist, g, n, ngram_hash(g, n));
+}
+
+constexpr int kWTile = 256;  // positions j per block
+
+// Eq. 8 then Eq. 9 for positions [j0, j0 + kWTile) of the update.
+__global__ void __launch_bounds__(kWTile) ngram_weights_kernel(const int32_t *__restrict__ x, int64_t L, int n,
+                                                               const int32_t *__restrict__ hist, int64_t hist_len,
+                                                               const Slot *table, unsigned long long mask,
+                                                               float w_min, float *__restrict__ w) {
+    __shared__ int32_t tok[kWTile + 2 * kMaxN];
+    __shared__ unsigned int cnt[kWTile + kMaxN];
+    const int64_t j0 = (int64_t)blockIdx.x * kWTile;
+    // Window starts s that cover some j in the tile: s in [j0-n+1, j0+kWTile-1]
+    // clipped to [0, L-n].  Tokens needed: x[s0 .. s1+n-1].
+    const int64_t s_lo = j0 - (n - 1);
+    const int64_t nwin = kWTile + n - 1;  // candidate windows, indexed by s - s_lo
+    // stage tokens x[s_lo .. s_lo + nwin + n - 2] (coalesced)
+    const int ntok = (int)(nwin + n - 1);
+    for (int i = threadIdx.x; i < ntok; i += blockDim.x) {
+        const int64_t pos = s_lo + i;
+        tok[i] = (pos >= 0 && pos < L) ? __ldg(x + pos) : 0;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < nwin; i += blockDim.x) {
+        const int64_t s = s_lo + i;
+        unsigned int c = 0u;
+        if (s >= 0 && s + n <= L && hist_len >= n) c = table_lookup(table, mask, hist, tok + i, n, ngram_hash(tok + i, n));
+        cnt[i] = c;
+    }
+    __syncthreads();
+    const int64_t j = j0 + threadIdx.x;
+    if (j >= L) return;
+    // windows covering j: s in [j-n+1, j], i.e. indices [threadIdx.x, threadIdx.x + n - 1];
+    // invalid windows (s < 0 or s > L-n) hold count 0, which never changes the max.
+    unsigned int f = 0u;
+    for (int k = 0; k < n; ++k) f = max(f, cnt[threadIdx.x + k]);
+    const float q = __fdiv_rn(1.0f, __fadd_rn(1.0f, __uint2float_rn(f)));
+    w[j] = fmaxf(w_min, q);
+}
+
+}  // namespace attt
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+
+struct attt_history {
+    int n;
+    int device;
+    int64_t max_tokens;
+    int64_t len;
+    int32_t *d_tokens;
+    attt::Slot *d_table;
+    unsigned long long capacity;
+    int *d_status;
+};
+
+extern "C" {
+
+attt_status attt_history_create(int n, int64_t max_tokens, attt_history **out) {
+    if (!out || n < 1 || n > attt::kMaxN || max_tokens < 0 || max_tokens > ((int64_t)1 << 31) - 2)
+        return ATTT_ERR_INVALID_ARG;
+    *out = nullptr;
+    int dev;
+    attt_status st = attt::current_device(&dev);
+    if (st != ATTT_OK) return st;
+    unsigned long long cap = 1024;
+    while (cap < 2ull * (unsigned long long)max_tokens) cap <<= 1;
+    attt_history *h = new (std::nothrow) attt_history();
+    if (!h) return ATTT_ERR_CUDA;
+    h->n = n;
+    h->device = dev;
+    h->max_tokens = max_tokens;
+    h->len = 0;
+    h->capacity = cap;
+    if (cudaMalloc(&h->d_tokens, (size_t)(max_tokens > 0 ? max_tokens : 1) * sizeof(int32_t)) != cudaSuccess ||
+        cudaMalloc(&h->d_table, cap * sizeof(attt::Slot)) != cudaSuccess ||
+        cudaMalloc(&h->d_status, 256) != cudaSuccess) {
+        cudaFree(h->d_tokens);
+        cudaFree(h->d_table);
+        cudaFree(h->d_status);
+        delete h;
+        return ATTT_ERR_CUDA;
+    }
+    if (cudaMemset(h->d_table, 0, cap * sizeof(attt::Slot)) != cudaSuccess ||
+        cudaMemset(h->d_status, 0, 256) != cudaSuccess) {
+        cudaFree(h->d_tokens);
+        cudaFree(h->d_table);
+        cudaFree(h->d_status);
+        delete h;
+        return ATTT_ERR_CUDA;
+    }
+    *out = h;
+    return ATTT_OK;
+}
+
+attt_status attt_history_destroy(attt_history *h) {
+    if (!h) return ATTT_ERR_INVALID_ARG;
+    int prev = -1;
+    cudaGetDevice(&prev);
+    cudaSetDevice(h->device);
+    cudaDeviceSynchronize();
+    cudaFree(h->d_tokens);
+    cudaFree(h->d_table);
+    cudaFree(h->d_status);
+    if (prev >= 0) cudaSetDevice(prev);
+    delete h;
+    return ATTT_OK;
+}
+
+attt_status attt_history_reset(attt_history *h, attt_stream stream) {
+    if (!h) return ATTT_ERR_INVALID_ARG;
+    if (cudaMemsetAsync(h->d_table, 0, h->capacity * sizeof(attt::Slot), stream) != cudaSuccess)
+        return ATTT_ERR_CUDA;
+    h->len = 0;
+    return ATTT_OK;
+}
+
+int64_t attt_history_length(const attt_history *h) { return h ? h->len : -1; }
+
+int attt_history_ngram(const attt_history *h) { return h ? h->n : -1; }
+
+attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_t len, attt_stream stream) {
+    if (!h || len < 0 || (len > 0 && !d_tokens)) return ATTT_ERR_INVALID_ARG;
+    if (len == 0) return ATTT_OK;
+    if (h->len + len > h->max_tokens) return ATTT_ERR_CAPACITY;
+    if (cudaMemcpyAsync(h->d_tokens + h->len, d_tokens, (size_t)len * sizeof(int32_t), cudaMemcpyDeviceToDevice,
+                        stream) != cudaSuccess)
+        return ATTT_ERR_CUDA;
+    const int64_t new_len = h->len + len;
+    // New n-grams: every start p whose last token p+n-1 is new, i.e.
+    // p in [max(0, old_len - n + 1), new_len - n].
+    int64_t p_begin = h->len - (h->n - 1);
+    if (p_begin < 0) p_begin = 0;
+    const int64_t p_end = new_len - h->n;  // inclusive
+    h->len = new_len;
+    if (p_end < p_begin) return ATTT_OK;
+    const int64_t count = p_end - p_begin + 1;
+    const int threads = 256;
+    const int64_t blocks = (count + threads - 1) / threads;
+    attt::history_insert_kernel<<<(unsigned)blocks, threads, 0, stream>>>(h->d_tokens, p_begin, count, h->n,
+                                                                          h->d_table, h->capacity - 1, h->d_status);
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+attt_status attt_history_status(attt_history *h, attt_stream stream) {
+    if (!h) return ATTT_ERR_INVALID_ARG;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return ATTT_ERR_CUDA;
+    int v = 0;
+    if (cudaMemcpy(&v, h->d_status, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return ATTT_ERR_CUDA;
+    if (v != 0 && cudaMemset(h->d_status, 0, sizeof v) != cudaSuccess) return ATTT_ERR_CUDA;
+    return (attt_status)v;
+}
+
+attt_status attt_history_count(const attt_history *h, const int32_t *d_ngrams, int64_t m, uint32_t *d_counts,
+                               attt_stream stream) {
+    if (!h || m < 0 || (m > 0 && (!d_ngrams || !d_counts))) return ATTT_ERR_INVALID_ARG;
+    if (m == 0) return ATTT_OK;
+    const int threads = 256;
+    attt::history_count_kernel<<<(unsigned)((m + threads - 1) / threads), threads, 0, stream>>>(
+        h->d_tokens, h->d_table, h->capacity - 1, d_ngrams, m, h->n, d_counts);
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+attt_status attt_ngram_weights(const attt_history *h, const int32_t *d_tokens, int64_t L, float w_min, float *d_w,
+                               attt_stream stream) {
+    if (!h || L < 0 || (L > 0 && (!d_tokens || !d_w)) || !(w_min > 0.0f) || !(w_min <= 1.0f))
+        return ATTT_ERR_INVALID_ARG;
+    if (L == 0) return ATTT_OK;
+    const int64_t blocks = (L + attt::kWTile - 1) / attt::kWTile;
+    attt::ngram_weights_kernel<<<(unsigned)blocks, attt::kWTile, 0, stream>>>(
+        d_tokens, L, h->n, h->d_tokens, h->len, h->d_table, h->capacity - 1, w_min, d_w);
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+}  // extern "C"

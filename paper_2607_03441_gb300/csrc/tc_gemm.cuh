@@ -1,0 +1,393 @@
+// tc_gemm.cuh -- the tcgen05 contraction engine shared by the Eq. 10 CE
+// kernels and the LoRA adapter-gradient kernels.
+//
+// D[M x N] = A[M x K] * B[N x K]^T with bf16 operands and fp32 accumulation.
+//   * one CTA per SM, persistent over output tiles of 128 x BN (BN <= 256);
+//   * warp 0: TMA producer (one thread) filling a ring of `stages` shared-
+//     memory stages of 64-deep K blocks, 128-byte swizzled;
+//   * warp 1: allocates TMEM and issues tcgen05.mma (one thread), four
+//     M128 x N(BN) x K16 MMAs per stage, into one of two TMEM accumulators;
+//   * warps 2-5: epilogue, one accumulator row per thread (tcgen05.ld
+//     32x32b), overlapping the next tile's MMAs through the second
+//     accumulator.  The epilogue kinds fuse the work that follows the
+//     contraction so that nothing of size [M x N] goes back to HBM unless it
+//     is the result itself.
+// An operand is K-major (K contiguous in memory: a row-major [rows, K] matrix)
+// or MN-major (rows contiguous: a row-major [K, rows] matrix); both are
+// loaded by TMA with the 128-byte swizzle that tcgen05 reads natively.
+// Tiles past M, N or K are zero-filled by TMA and masked in the epilogue.
+// The K range of a tile may be split (split-K); split partial sums are
+// reduced with fp32 atomics by the epilogue kinds that support it.
+#pragma once
+
+#include "attt_common.cuh"
+
+namespace attt {
+
+enum EpiKind : int {
+    EPI_CE_STATS = 0,  // per (row, vocab tile): running max and sum of exp, target logit
+    EPI_CE_GRAD = 1,   // G = (w/L) (softmax - onehot) as bf16, for the dh contraction
+    EPI_F32_ACC = 2,   // out[m, n] (+)= acc   (fp32, row-major)
+    EPI_ATOMIC_T = 3,  // out[n, m] += alpha * acc   (fp32, transposed, split-K)
+    EPI_ATOMIC_N = 4,  // out_p[m, c] += alpha * acc for column n = p * rpad + c (split-K)
+};
+
+constexpr int kMaxProj = 8;
+
+struct EpiParams {
+    // CE
+    const int32_t *tgt;  // [M] target ids
+    float2 *part;        // [tiles_n, M] (max, sum) in log2 units
+    float *ztgt;         // [M] target logit
+    const float *lse;    // [M] natural-log logsumexp
+    const float *w;      // [M] Eq. 9 weights
+    float inv_L;         // 1 / L
+    int v0;              // vocab id of column 0 of this launch
+    __nv_bfloat16 *G;    // [M, G_ld]
+    int64_t G_ld;
+    // fp32 outputs
+    float *out;
+    int64_t out_ld;
+    int accumulate;
+    float alpha;
+    float *outp[kMaxProj];
+    int r;     // valid columns per projection block
+    int rpad;  // column block width per projection
+};
+
+struct GemmArgs {
+    int M, N;
+    int BN, stages;
+    int tiles_m, tiles_n, splits;
+    int kb_per_split, kb_total;
+    int a_m_off, a_k_off;  // coordinate offsets into A's tensor map
+    int b_n_off, b_k_off;  // coordinate offsets into B's tensor map
+    uint32_t tmem_cols;
+    int *status;
+    EpiParams ep;
+};
+
+constexpr uint32_t kABytes = 128 * 64 * 2;  // one A stage: 128 rows x 64 bf16
+constexpr int kGemmThreads = 192;
+
+__host__ __device__ inline uint32_t gemm_b_stage_bytes(int BN) { return (uint32_t)BN * 128u; }
+
+__host__ __device__ inline size_t gemm_smem_bytes(int BN, int stages) {
+    return 1024 + (size_t)stages * (kABytes + gemm_b_stage_bytes(BN)) + 8 * (2 * stages + 5) + 16;
+}
+
+__device__ __forceinline__ void decode_tile(const GemmArgs &g, int t, int &tm, int &tn, int &split) {
+    const int per = g.tiles_m * g.tiles_n;
+    split = t / per;
+    const int rem = t - split * per;
+    tn = rem / g.tiles_m;
+    tm = rem - tn * g.tiles_m;
+}
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ---------------------------------------------------------------------------
+// Epilogues.  Every thread owns accumulator row `row` of the tile; all 32
+// lanes of a warp execute the TMEM loads together even when their row is
+// past M (the loads are warp-collective); only stores are predicated.
+// ---------------------------------------------------------------------------
+
+template <int EPI>
+__device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn, int row, uint32_t taddr) {
+    const int gm = tm * 128 + row;
+    const bool rv = gm < g.M;
+    const int n_base = tn * g.BN;
+    const EpiParams &ep = g.ep;
+
+    if constexpr (EPI == EPI_CE_STATS) {
+        // Online logsumexp over this tile's columns, in log2 units.
+        const int t = rv ? __ldg(ep.tgt + gm) - ep.v0 : -1;
+        float mx = -INFINITY, sm = 0.f, zt = 0.f;
+        bool hit = false;
+        for (int c = 0; c < g.BN; c += 32) {
+            if (n_base + c >= g.N) break;
+            float v[32];
+            tmem_ld_x32(taddr + (uint32_t)c, v);
+            float cm = -INFINITY;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const int col = n_base + c + i;
+                if (col == t) { zt = v[i]; hit = true; }
+                v[i] = (col < g.N) ? v[i] * kLog2e : -INFINITY;
+                cm = fmaxf(cm, v[i]);
+            }
+            const float nm = fmaxf(mx, cm);
+            float s = sm * exp2f(mx - nm);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) s += exp2f(v[i] - nm);
+            sm = s;
+            mx = nm;
+        }
+        if (rv) {
+            ep.part[(int64_t)tn * g.M + gm] = make_float2(mx, sm);
+            if (hit) ep.ztgt[gm] = zt;
+        }
+    } else if constexpr (EPI == EPI_CE_GRAD) {
+        // G[j, v] = (w_j / L) (exp(z - lse_j) - [v == tgt_j]) in bf16; columns
+        // past N are written as zeros so the dh contraction may read them.
+        float l2 = 0.f, cw = 0.f;
+        int t = -1;
+        if (rv) {
+            l2 = __ldg(ep.lse + gm) * kLog2e;
+            cw = __ldg(ep.w + gm) * ep.inv_L;
+            t = __ldg(ep.tgt + gm) - ep.v0;
+        }
+        __nv_bfloat16 *grow = ep.G + (int64_t)gm * ep.G_ld;
+        for (int c = 0; c < g.BN; c += 32) {
+            float v[32];
+            tmem_ld_x32(taddr + (uint32_t)c, v);
+            uint32_t pk[16];
+#pragma unroll
+            for (int i = 0; i < 32; i += 2) {
+                const int col = n_base + c + i;
+                float g0 = 0.f, g1 = 0.f;
+                if (col < g.N) g0 = cw * (exp2f(fmaf(v[i], kLog2e, -l2)) - (col == t ? 1.f : 0.f));
+                if (col + 1 < g.N) g1 = cw * (exp2f(fmaf(v[i + 1], kLog2e, -l2)) - (col + 1 == t ? 1.f : 0.f));
+                __nv_bfloat162 b = __floats2bfloat162_rn(g0, g1);
+                pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
+            }
+            if (rv) {
+                uint4 *dst = reinterpret_cast<uint4 *>(grow + n_base + c);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+            }
+        }
+    } else if constexpr (EPI == EPI_F32_ACC) {
+        float *orow = ep.out + (int64_t)gm * ep.out_ld;
+        for (int c = 0; c < g.BN; c += 32) {
+            if (n_base + c >= g.N) break;
+            float v[32];
+            tmem_ld_x32(taddr + (uint32_t)c, v);
+            if (rv) {
+                const int col0 = n_base + c;
+                if (col0 + 32 <= g.N) {
+                    float4 *dst = reinterpret_cast<float4 *>(orow + col0);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) {
+                        float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                        if (ep.accumulate) {
+                            const float4 p = dst[q];
+                            o.x += p.x; o.y += p.y; o.z += p.z; o.w += p.w;
+                        }
+                        dst[q] = o;
+                    }
+                } else {
+                    for (int i = 0; i < 32 && col0 + i < g.N; ++i)
+                        orow[col0 + i] = ep.accumulate ? orow[col0 + i] + v[i] : v[i];
+                }
+            }
+        }
+    } else if constexpr (EPI == EPI_ATOMIC_T) {
+        for (int c = 0; c < g.BN; c += 16) {
+            if (n_base + c >= g.N) break;
+            float v[16];
+            tmem_ld_x16(taddr + (uint32_t)c, v);
+            if (rv) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int col = n_base + c + i;
+                    if (col < g.N && (col % ep.rpad) < ep.r)
+                        atomicAdd(ep.out + (int64_t)col * ep.out_ld + gm, ep.alpha * v[i]);
+                }
+            }
+        }
+    } else if constexpr (EPI == EPI_ATOMIC_N) {
+        for (int c = 0; c < g.BN; c += 16) {
+            if (n_base + c >= g.N) break;
+            float v[16];
+            tmem_ld_x16(taddr + (uint32_t)c, v);
+            if (rv) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const int col = n_base + c + i;
+                    if (col < g.N) {
+                        const int p = col / ep.rpad, cc = col - p * ep.rpad;
+                        if (cc < ep.r) atomicAdd(ep.outp[p] + (int64_t)gm * ep.r + cc, ep.alpha * v[i]);
+                    }
+                }
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// The kernel
+// ---------------------------------------------------------------------------
+
+template <int EPI, bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const GemmArgs g) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int S = g.stages;
+    const uint32_t b_bytes = gemm_b_stage_bytes(g.BN);
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + (size_t)S * kABytes;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + (size_t)S * b_bytes);
+    const uint32_t full0 = smem_u32(bars);
+    const uint32_t empty0 = smem_u32(bars + S);
+    const uint32_t tfull0 = smem_u32(bars + 2 * S);
+    const uint32_t tempty0 = smem_u32(bars + 2 * S + 2);
+    const uint32_t drain0 = smem_u32(bars + 2 * S + 4);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * S + 5);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full0 + 8 * s, 1);
+            mbar_init(empty0 + 8 * s, 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(tfull0 + 8 * a, 1);
+            mbar_init(tempty0 + 8 * a, 4);
+        }
+        mbar_init(drain0, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        tma_prefetch_desc(&tmA);
+        tma_prefetch_desc(&tmB);
+    }
+    if (warp == 1) {
+        tmem_alloc(smem_u32(tmem_slot), g.tmem_cols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    const int ntiles = g.tiles_m * g.tiles_n * g.splits;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------- TMA producer ----------------
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t issued_mask = 0, issued_parity = 0;  // per stage: last issue pending?
+            bool ok = true;
+            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+                int tm, tn, split;
+                decode_tile(g, t, tm, tn, split);
+                const int kb0 = split * g.kb_per_split;
+                const int kb1 = min(g.kb_total, kb0 + g.kb_per_split);
+                for (int kb = kb0; kb < kb1; ++kb) {
+                    if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
+                    const uint32_t fb = full0 + 8 * stage;
+                    mbar_arrive_expect_tx(fb, kABytes + b_bytes);
+                    const uint32_t a_dst = smem_u32(sA + (size_t)stage * kABytes);
+                    const uint32_t b_dst = smem_u32(sB + (size_t)stage * b_bytes);
+                    const int k = kb * 64;
+                    if (!A_MN) {
+                        tma_load_2d(a_dst, &tmA, fb, g.a_k_off + k, g.a_m_off + tm * 128);
+                    } else {
+                        tma_load_2d(a_dst, &tmA, fb, g.a_m_off + tm * 128, g.a_k_off + k);
+                        tma_load_2d(a_dst + 8192, &tmA, fb, g.a_m_off + tm * 128 + 64, g.a_k_off + k);
+                    }
+                    if (!B_MN) {
+                        tma_load_2d(b_dst, &tmB, fb, g.b_k_off + k, g.b_n_off + tn * g.BN);
+                    } else {
+                        for (int b = 0; b < g.BN / 64; ++b)
+                            tma_load_2d(b_dst + 8192 * b, &tmB, fb, g.b_n_off + tn * g.BN + 64 * b, g.b_k_off + k);
+                    }
+                    issued_mask |= 1u << stage;
+                    issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+                    if (++stage == S) { stage = 0; phase ^= 1u; }
+                }
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                record_error(g.status, ATTT_ERR_TIMEOUT);
+                // Let every load already issued land before the CTA retires.
+                for (int s = 0; s < S; ++s)
+                    if (issued_mask & (1u << s))
+                        (void)mbar_wait(full0 + 8 * s, (issued_parity >> s) & 1u, abort_flag);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ---------------- MMA issuer ----------------
+            const uint32_t idesc = idesc_bf16_f32((uint32_t)g.BN, A_MN, B_MN);
+            int stage = 0;
+            uint32_t phase = 0;
+            int it = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++it) {
+                int tm, tn, split;
+                decode_tile(g, t, tm, tn, split);
+                const int kb0 = split * g.kb_per_split;
+                const int kb1 = min(g.kb_total, kb0 + g.kb_per_split);
+                const int acc = it & 1;
+                if (!mbar_wait(tempty0 + 8 * acc, (((uint32_t)it >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * g.BN);
+                for (int kb = kb0; kb < kb1; ++kb) {
+                    if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t a_addr = smem_u32(sA + (size_t)stage * kABytes);
+                    const uint32_t b_addr = smem_u32(sB + (size_t)stage * b_bytes);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const uint64_t ad = A_MN ? smem_desc_sw128(a_addr + kk * 2048, 8192, 1024)
+                                                 : smem_desc_sw128(a_addr + kk * 32, 16, 1024);
+                        const uint64_t bd = B_MN ? smem_desc_sw128(b_addr + kk * 2048, 8192, 1024)
+                                                 : smem_desc_sw128(b_addr + kk * 32, 16, 1024);
+                        umma_bf16(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+                    }
+                    umma_commit(empty0 + 8 * stage);
+                    if (++stage == S) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+                umma_commit(tfull0 + 8 * acc);
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                record_error(g.status, ATTT_ERR_TIMEOUT);
+            }
+            // Drain: every MMA issued by this thread completes before TMEM is
+            // freed (bounded wait; on the normal path they are long done).
+            umma_commit(drain0);
+            volatile int no_abort = 0;
+            if (!mbar_wait(drain0, 0u, &no_abort)) record_error(g.status, ATTT_ERR_TIMEOUT);
+        }
+    } else {
+        // ---------------- epilogue (warps 2..5) ----------------
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        int it = 0;
+        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++it) {
+            int tm, tn, split;
+            decode_tile(g, t, tm, tn, split);
+            const int acc = it & 1;
+            const uint32_t par = ((uint32_t)it >> 1) & 1u;
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(tfull0 + 8 * acc, par, abort_flag) ? 1 : 0;
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) {
+                if (lane == 0) { *abort_flag = 1; record_error(g.status, ATTT_ERR_TIMEOUT); }
+                break;
+            }
+            (void)mbar_try_wait(tfull0 + 8 * acc, par);  // per-thread acquire of the completed phase
+            tc_fence_after();
+            const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * g.BN);
+            epilogue_tile<EPI>(g, tm, tn, row, taddr);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc(tmem_base, g.tmem_cols);
+}
+
+}  // namespace attt

@@ -1,0 +1,77 @@
+"""The C-ABI library builds, loads without a GPU and exports every entry point
+that include/attt.h declares; host-only calls answer without a device."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "attt.h")
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"ATTT_API[^;(]*?\b(attt_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib_path():
+    from paper_2607_03441_gb300 import build
+    return build.build()
+
+
+def test_header_declares_north_star_calls():
+    names = declared_symbols()
+    for must in ("attt_history_insert", "attt_ngram_weights", "attt_weighted_ce_fwd_bwd", "attt_lora_grad",
+                 "attt_lora_step"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(lib_path):
+    out = subprocess.run(["nm", "-D", "--defined-only", lib_path], capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (attt_\w+)", out))
+    missing = [s for s in declared_symbols() if s not in exported]
+    assert not missing, f"not exported: {missing}"
+    lib = ctypes.CDLL(lib_path)
+    for s in declared_symbols():
+        assert getattr(lib, s) is not None
+
+
+def test_host_only_calls(lib_path):
+    from paper_2607_03441_gb300 import attt
+    assert attt.attt_abi_version() == 100
+    assert attt.attt_status_string(0) == "ATTT_OK"
+    assert attt.attt_status_string(8) == "ATTT_ERR_CAPACITY"
+    assert attt.attt_status_string(99) == "ATTT_ERR_UNKNOWN"
+    assert attt.attt_ce_workspace_bytes(256, 512, 8192) > 0
+    assert attt.attt_ce_workspace_bytes(0, 512, 8192) == 0
+    assert attt.attt_lora_workspace_bytes(256, 512, [512], 8) > 0
+    assert attt.attt_lora_workspace_bytes(256, 512, [512], 65) == 0
+
+
+def test_product_has_no_oracle_or_cpu_path():
+    """Nothing on the product path imports the oracle or falls back to torch
+    compute: the binding only marshals arguments to libattt."""
+    pkg = os.path.join(ROOT, "paper_2607_03441_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                src = open(os.path.join(dirpath, f)).read()
+                assert "import oracle" not in src and "from oracle" not in src, f
+                assert "liboracle" not in src, f
+    binding = open(os.path.join(pkg, "attt.py")).read()
+    for forbidden in ("torch.matmul", "F.cross_entropy", "torch.nn.functional", "@ ", ".mm("):
+        assert forbidden not in binding
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    from paper_2607_03441_gb300 import attt
+    saved = attt._lib
+    try:
+        attt._lib = None
+        with pytest.raises(RuntimeError):
+            attt.load_library(str(tmp_path / "nope.so"))
+    finally:
+        attt._lib = saved

@@ -1,0 +1,121 @@
+"""GPU parity of the LoRA adapter gradients and the SGD step against the CPU
+oracle.  Gradients within 2e-2 relative L2 per tensor (bf16 inputs, fp32
+accumulation, u and v rounded to bf16 once); exact zeros where the
+mathematics gives zeros; the SGD step bit-exact."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_03441_gb300 import workloads as wk
+from tests.gpu_util import DEV, bf16_dev, f32_dev, rel_l2
+
+pytestmark = pytest.mark.gpu
+
+GRAD_RL2 = 2e-2
+
+
+@pytest.fixture(scope="module")
+def attt():
+    from paper_2607_03441_gb300 import attt as a
+    from paper_2607_03441_gb300 import build
+    build.build()
+    oracle.build()
+    return a
+
+
+def _group(attt, x, dys, As, Bs, scale):
+    dAs, dBs = attt.attt_lora_grad(bf16_dev(x), [bf16_dev(d) for d in dys], [bf16_dev(a) for a in As],
+                                   [bf16_dev(b) for b in Bs], scale)
+    assert attt.attt_device_status() == 0
+    return [t.cpu().numpy() for t in dAs], [t.cpu().numpy() for t in dBs]
+
+
+def _check_group(attt, x, dys, As, Bs, scale=2.0):
+    gA, gB = _group(attt, x, dys, As, Bs, scale)
+    for p in range(len(dys)):
+        rA, rB = oracle.lora_grad(x, dys[p], As[p], Bs[p], scale)
+        ea, eb = rel_l2(gA[p], rA), rel_l2(gB[p], rB)
+        assert ea < GRAD_RL2 and eb < GRAD_RL2, (p, ea, eb)
+    return gA, gB
+
+
+def _inputs(seed, L, din, douts, r):
+    x = wk.normal_bf16(seed, "x", (L, din), 1.0)
+    dys = [wk.normal_bf16(seed, f"dy{p}", (L, do), 1.0) for p, do in enumerate(douts)]
+    As = [wk.normal_bf16(seed, f"A{p}", (din, r), 0.02) for p in range(len(douts))]
+    Bs = [wk.normal_bf16(seed, f"B{p}", (r, do), 0.01) for p, do in enumerate(douts)]
+    return x, dys, As, Bs
+
+
+@pytest.mark.parametrize("L,din,douts,r", [(256, 512, [512], 8), (300, 200, [72, 136], 5), (100, 64, [64], 1),
+                                          (513, 384, [256, 128, 64], 64), (64, 8, [8], 16), (1000, 256, [1024], 32)])
+def test_shapes(attt, L, din, douts, r):
+    _check_group(attt, *_inputs(L + din, L, din, douts, r))
+
+
+def test_zero_B_and_zero_x(attt):
+    x, dys, As, Bs = _inputs(7, 200, 128, [96], 8)
+    gA, gB = _group(attt, x, dys, As, [np.zeros_like(Bs[0])], 2.0)
+    assert np.all(gA[0] == 0.0)
+    gA, gB = _group(attt, np.zeros_like(x), dys, As, Bs, 2.0)
+    assert np.all(gA[0] == 0.0) and np.all(gB[0] == 0.0)
+
+
+def test_tiny_chained_from_ce(attt):
+    """Tiny config: dy of the projection is the Eq. 10 gradient dh cast to bf16,
+    each side chaining its own dh (the oracle its fp64 dh)."""
+    wl = wk.WORKLOADS["tiny"]
+    H = wk.history_tokens(wl)
+    xt = wk.update_tokens(wl, H)
+    w = oracle.ngram_weights(H, xt, wl.n)
+    dense = wk.dense_inputs(wl)
+    _, dh, _ = attt.attt_weighted_ce_fwd_bwd(bf16_dev(dense["h"]), bf16_dev(dense["W"]),
+                                             torch.from_numpy(xt).to(DEV), f32_dev(w))
+    dy_gpu = dh.to(torch.bfloat16)
+    _, _, _, rdh = oracle.ce_loss(dense["h"], dense["W"], xt, w)
+    dy_ref = wk.bf16_bits(rdh.astype(np.float32))
+    x, A, B = dense["x/proj"], dense["A/proj"], dense["B/proj"]
+    dAs, dBs = attt.attt_lora_grad(bf16_dev(x), [dy_gpu], [bf16_dev(A)], [bf16_dev(B)], wl.scale)
+    rA, rB = oracle.lora_grad(x, dy_ref, A, B, wl.scale)
+    assert rel_l2(dAs[0].cpu().numpy(), rA) < GRAD_RL2
+    assert rel_l2(dBs[0].cpu().numpy(), rB) < GRAD_RL2
+    # and with the same dy on both sides
+    _check_group(attt, x, [dy_ref], [A], [B], wl.scale)
+
+
+def _workload_groups(name):
+    wl = wk.WORKLOADS[name]
+    dense = wk.dense_inputs(wl, with_lm_head=False)
+    groups = {}
+    for p in wl.projs:
+        groups.setdefault(p.x_group, []).append(p)
+    return wl, dense, groups
+
+
+@pytest.mark.parametrize("name", ["7b", "long", "32b"])
+def test_workload(attt, name):
+    wl, dense, groups = _workload_groups(name)
+    for g, projs in groups.items():
+        x = dense[f"x/{projs[0].name}"]
+        _check_group(attt, x, [dense[f"dy/{p.name}"] for p in projs], [dense[f"A/{p.name}"] for p in projs],
+                     [dense[f"B/{p.name}"] for p in projs], wl.scale)
+
+
+def test_sgd_step_bit_exact(attt):
+    din, dout, r = 384, 200, 16
+    rng = np.random.default_rng(0)
+    A = rng.standard_normal((din, r)).astype(np.float32) * 0.02
+    B = rng.standard_normal((r, dout)).astype(np.float32) * 0.01
+    dA = rng.standard_normal((din, r)).astype(np.float32)
+    dB = rng.standard_normal((r, dout)).astype(np.float32)
+    A32, B32 = f32_dev(A), f32_dev(B)
+    A16 = torch.empty(din, r, dtype=torch.bfloat16, device=DEV)
+    B16 = torch.empty(r, dout, dtype=torch.bfloat16, device=DEV)
+    attt.attt_lora_step(A32, B32, f32_dev(dA), f32_dev(dB), 5e-4, A16, B16)
+    pA, bA = oracle.sgd_step(A, dA, 5e-4)
+    pB, bB = oracle.sgd_step(B, dB, 5e-4)
+    np.testing.assert_array_equal(A32.cpu().numpy(), pA)
+    np.testing.assert_array_equal(B32.cpu().numpy(), pB)
+    np.testing.assert_array_equal(A16.view(torch.int16).cpu().numpy().view(np.uint16), bA)
+    np.testing.assert_array_equal(B16.view(torch.int16).cpu().numpy().view(np.uint16), bB)

@@ -1,0 +1,169 @@
+"""GPU parity of Eq. 8 / Eq. 9 (history insert + n-gram weights) against the
+CPU oracle: bit-exact weights on every workload, plus edge cases."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_03441_gb300 import workloads as wk
+from tests.gpu_util import DEV, bits, i32_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def attt():
+    from paper_2607_03441_gb300 import attt as a
+    from paper_2607_03441_gb300 import build
+    build.build()
+    oracle.build()
+    return a
+
+
+def _weights(attt, H, x, n, w_min=0.05, chunks=None, max_tokens=None):
+    h = attt.attt_history_create(n, max_tokens or max(len(H), 1))
+    if chunks is None:
+        chunks = [H]
+    for c in chunks:
+        if len(c):
+            attt.attt_history_insert(h, i32_dev(c))
+    w = attt.attt_ngram_weights(h, i32_dev(x), w_min).cpu().numpy()
+    assert attt.attt_history_status(h) == 0
+    h.close()
+    return w
+
+
+def _assert_bit_exact(w, ref):
+    diff = np.nonzero(bits(w) != bits(ref))[0]
+    assert diff.size == 0, f"{diff.size} weights differ, first at {diff[:5]}: {w[diff[:5]]} vs {ref[diff[:5]]}"
+
+
+def test_worked_examples(attt):
+    import json, os
+    cases = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "ngram_worked_examples.json")))["cases"]
+    for c in cases:
+        H = np.array(c["history"], np.int32)
+        x = np.array(c["update"], np.int32)
+        chunks = [np.array(ch, np.int32) for ch in c.get("history_chunks", [c["history"]])]
+        w = _weights(attt, H, x, c["n"], c["w_min"], chunks=chunks, max_tokens=max(len(H), 1))
+        assert [f"0x{b:08x}" for b in bits(w)] == c["w_bits"], c["name"]
+
+
+@pytest.mark.parametrize("name", ["tiny", "7b", "32b"])
+def test_workload_weights(attt, name):
+    wl = wk.WORKLOADS[name]
+    H = wk.history_tokens(wl)
+    x = wk.update_tokens(wl, H)
+    w = _weights(attt, H, x, wl.n)
+    _assert_bit_exact(w, oracle.ngram_weights(H, x, wl.n))
+
+
+@pytest.mark.parametrize("n", [3, 4, 5])
+@pytest.mark.parametrize("frac", [0.0, 0.3, 0.6, 0.9])
+def test_stress_sweep(attt, n, frac):
+    """8,192 update tokens against a 1,048,576-token history."""
+    H, x = wk.stress_case(n, frac)
+    w = _weights(attt, H, x, n)
+    _assert_bit_exact(w, oracle.ngram_weights(H, x, n))
+
+
+def test_long_episode(attt):
+    """32 sequential updates, each inserted before the next (Algorithm 1)."""
+    wl = wk.WORKLOADS["long"]
+    ups = wk.long_episode_updates(wl)
+    h = attt.attt_history_create(wl.n, wl.L * wl.updates)
+    H = np.zeros(0, np.int32)
+    for k, x in enumerate(ups):
+        w = attt.attt_ngram_weights(h, i32_dev(x), 0.05).cpu().numpy()
+        _assert_bit_exact(w, oracle.ngram_weights(H, x, wl.n))
+        if k == 0:
+            assert np.all(w == np.float32(1.0))
+        attt.attt_history_insert(h, i32_dev(x))
+        H = np.concatenate([H, x])
+    assert attt.attt_history_status(h) == 0
+    h.close()
+
+
+def test_chunked_insert_equals_single(attt):
+    rng = wk.rng_for(1, "chunks")
+    H = wk.zipf_ids(rng, 5000, 64)
+    x = wk.copy_spans(rng, wk.zipf_ids(rng, 700, 64), H, 0.5)
+    cuts = [0, 1, 2, 3, 50, 1234, 1235, 4999, 5000]
+    chunks = [H[a:b] for a, b in zip(cuts[:-1], cuts[1:])]
+    for n in (1, 2, 3, 5, 8):
+        w1 = _weights(attt, H, x, n)
+        w2 = _weights(attt, H, x, n, chunks=chunks, max_tokens=len(H))
+        _assert_bit_exact(w1, w2)
+        _assert_bit_exact(w1, oracle.ngram_weights(H, x, n))
+
+
+def test_counts_exact(attt):
+    """Table counts equal the brute-force count for present and absent n-grams."""
+    rng = wk.rng_for(2, "counts")
+    H = wk.zipf_ids(rng, 20000, 40)
+    n = 3
+    h = attt.attt_history_create(n, len(H))
+    attt.attt_history_insert(h, i32_dev(H))
+    q = np.concatenate([np.stack([H[p:p + n] for p in range(0, 2000, 7)]),
+                        rng.integers(0, 60, (300, n)).astype(np.int32)])
+    got = attt.attt_history_count(h, i32_dev(q)).cpu().numpy()
+    ref = [oracle.count_naive(H, g) for g in q]
+    np.testing.assert_array_equal(got, ref)
+    h.close()
+
+
+def test_edge_cases(attt):
+    rng = wk.rng_for(3, "edge")
+    H = wk.zipf_ids(rng, 3000, 16)
+    # L < n, L == n, L == 1, L == 0, and ragged tile tails
+    for L in (0, 1, 2, 3, 4, 5, 255, 256, 257, 511, 513):
+        x = wk.zipf_ids(rng, L, 16)
+        for n in (1, 4):
+            if L == 0:
+                h = attt.attt_history_create(n, len(H))
+                attt.attt_history_insert(h, i32_dev(H))
+                out = torch.empty(0, dtype=torch.float32, device=DEV)
+                attt.attt_ngram_weights(h, torch.empty(0, dtype=torch.int32, device=DEV), 0.05, out=out)
+                h.close()
+                continue
+            _assert_bit_exact(_weights(attt, H, x, n), oracle.ngram_weights(H, x, n))
+    # empty history
+    x = wk.zipf_ids(rng, 100, 16)
+    w = _weights(attt, np.zeros(0, np.int32), x, 3, max_tokens=10)
+    assert np.all(w == np.float32(1.0))
+    # history shorter than n
+    w = _weights(attt, np.array([1, 2], np.int32), x, 3, max_tokens=10)
+    assert np.all(w == np.float32(1.0))
+    # a different floor
+    _assert_bit_exact(_weights(attt, H, x, 2, w_min=0.2), oracle.ngram_weights(H, x, 2, 0.2))
+
+
+def test_reset_and_capacity(attt):
+    from paper_2607_03441_gb300.attt import AtttError
+    rng = wk.rng_for(4, "reset")
+    H = wk.zipf_ids(rng, 1000, 8)
+    x = wk.zipf_ids(rng, 64, 8)
+    h = attt.attt_history_create(2, 1000)
+    attt.attt_history_insert(h, i32_dev(H))
+    with pytest.raises(AtttError):
+        attt.attt_history_insert(h, i32_dev(H[:1]))  # would exceed max_tokens
+    attt.attt_history_reset(h)
+    assert attt.attt_history_length(h) == 0
+    w = attt.attt_ngram_weights(h, i32_dev(x), 0.05).cpu().numpy()
+    assert np.all(w == np.float32(1.0))
+    attt.attt_history_insert(h, i32_dev(H[:500]))
+    _assert_bit_exact(attt.attt_ngram_weights(h, i32_dev(x), 0.05).cpu().numpy(),
+                      oracle.ngram_weights(H[:500], x, 2))
+    h.close()
+
+
+def test_invalid_args(attt):
+    from paper_2607_03441_gb300.attt import AtttError
+    with pytest.raises(AtttError):
+        attt.attt_history_create(0, 10)
+    with pytest.raises(AtttError):
+        attt.attt_history_create(17, 10)
+    h = attt.attt_history_create(3, 10)
+    with pytest.raises(AtttError):
+        attt.attt_ngram_weights(h, i32_dev(np.zeros(4, np.int32)), 0.0)
+    h.close()
