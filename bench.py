@@ -1,0 +1,387 @@
+#!/usr/bin/env python3
+"""aTTT update-step benchmark: update tokens/sec on GB300.
+
+One step = one aTTT update (Algorithm 1) of the 7B-class workload:
+  Eq. 8/9 weights of the 2,048-token update against the n = 4 history
+  (65,536 prior tokens at start), Eq. 10 weighted CE forward + backward
+  through the frozen 152,064 x 3,584 bf16 LM head, LoRA rank-16 gradients of
+  the q (3584x3584) and v (3584x512) projections, the SGD step on both
+  adapters, and the history insert of the update.
+The whole step runs in libattt's CUDA kernels, called through the C ABI.
+
+Contract: `python bench.py --gpus N --steps K --warmup W` prints one JSON line.
+N > 1 runs N independent replicas (one per GPU, no data-path collective;
+value is the sum over ranks).  `--impl reference` times the CPU oracle on the
+host cores instead (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import shutil
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2607_03441_gb300 import workloads as wk  # noqa: E402
+
+METRIC = "aTTT update tokens/sec on 1 GB300 and % of roofline (tensor peak / HBM)"
+UNIT = "update tokens/s"
+WORKLOAD = "7b"
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16": float(p["bf16_tflops"]),
+                "bf16_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), "src": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "src": "fallback"}
+
+
+# ---------------------------------------------------------------------------
+# clocks sampled during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        if shutil.which("nvidia-smi") is None:
+            return
+        fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
+        os.close(fd)
+        self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                      "--format=csv,noheader,nounits", "-lms", "100"],
+                                     stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r) if v.lower() == "active"})
+        sm = [r[0] for r in rows]
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(r[1] for r in rows),
+                "samples": len(rows), "reasons": reasons}
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+
+class Update:
+    """Device-resident state of the 7B-class update and one step of it."""
+
+    def __init__(self, wl, dev, max_steps):
+        import torch
+        from paper_2607_03441_gb300 import attt
+        self.attt = attt
+        self.torch = torch
+        self.wl = wl
+        self.dev = dev
+        H = wk.history_tokens(wl)
+        self.x_host = wk.update_tokens(wl, H)
+        dense = wk.dense_inputs(wl)
+        self.dense = dense
+
+        def bf(a):
+            return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
+
+        self.hist = attt.attt_history_create(wl.n, wl.hist_len + wl.L * max_steps)
+        attt.attt_history_insert(self.hist, torch.from_numpy(H).to(dev))
+        self.x = torch.from_numpy(self.x_host).to(dev)
+        self.h = bf(dense["h"])
+        self.W = bf(dense["W"])
+        self.projs = list(wl.projs)
+        self.xin = bf(dense[f"x/{self.projs[0].name}"])
+        self.dy = [bf(dense[f"dy/{p.name}"]) for p in self.projs]
+        self.A32 = [torch.from_numpy(wk.bf16_to_f32(dense[f"A/{p.name}"])).to(dev) for p in self.projs]
+        self.B32 = [torch.from_numpy(wk.bf16_to_f32(dense[f"B/{p.name}"])).to(dev) for p in self.projs]
+        self.A16 = [bf(dense[f"A/{p.name}"]) for p in self.projs]
+        self.B16 = [bf(dense[f"B/{p.name}"]) for p in self.projs]
+        self.dA = [torch.empty_like(a) for a in self.A32]
+        self.dB = [torch.empty_like(b) for b in self.B32]
+        L, d, V, r = wl.L, wl.d, wl.V, wl.r
+        self.w = torch.empty(L, dtype=torch.float32, device=dev)
+        self.loss = torch.empty(1, dtype=torch.float32, device=dev)
+        self.dh = torch.empty(L, d, dtype=torch.float32, device=dev)
+        self.ws_ce = torch.empty(attt.attt_ce_workspace_bytes(L, d, V), dtype=torch.uint8, device=dev)
+        self.ws_lora = torch.empty(attt.attt_lora_workspace_bytes(L, self.projs[0].din,
+                                                                   [p.dout for p in self.projs], r),
+                                   dtype=torch.uint8, device=dev)
+        self.stream = torch.cuda.current_stream()
+
+    def step(self, ce_events=None):
+        a = self.attt
+        a.attt_ngram_weights(self.hist, self.x, self.wl.w_min, out=self.w)
+        if ce_events is not None:
+            ce_events[0].record()
+        a.attt_weighted_ce_fwd_bwd(self.h, self.W, self.x, self.w, loss=self.loss, dh=self.dh,
+                                   workspace=self.ws_ce)
+        if ce_events is not None:
+            ce_events[1].record()
+        a.attt_lora_grad(self.xin, self.dy, self.A16, self.B16, self.wl.scale, dAs=self.dA, dBs=self.dB,
+                         workspace=self.ws_lora)
+        for i in range(len(self.projs)):
+            a.attt_lora_step(self.A32[i], self.B32[i], self.dA[i], self.dB[i], wk.LORA_LR, self.A16[i], self.B16[i])
+        a.attt_history_insert(self.hist, self.x)
+
+
+def _ce_roofline(wl, t_ce_ms, peaks, traffic):
+    flops = 4.0 * wl.L * wl.V * wl.d
+    achieved = flops / (t_ce_ms * 1e-3) / 1e12
+    peak = peaks["bf16_sustained"]
+    return {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
+            "frac": round(achieved / peak, 4), "traffic": traffic,
+            "kernel": "attt_weighted_ce_fwd_bwd (Eq. 10 fwd+bwd; 4*L*V*d algorithmic FLOPs per call)",
+            "peak_kind": f"bf16 sustained, {peaks['src']}"}
+
+
+class OracleSample:
+    """The CPU oracle on a bounded sample of one update (test infrastructure
+    reused as the timed CPU baseline; never on the GPU path)."""
+
+    def __init__(self, wl, dense=None, x=None, H=None):
+        import oracle
+        oracle.build()
+        self.oracle = oracle
+        self.wl = wl
+        self.H = wk.history_tokens(wl) if H is None else H
+        self.x = wk.update_tokens(wl, self.H) if x is None else x
+        self.dense = wk.dense_inputs(wl) if dense is None else dense
+
+    def run(self, rows: int):
+        o, wl, dense = self.oracle, self.wl, self.dense
+        sel = np.sort(wk.rng_for(wl.seed, "cpu_sample").choice(wl.L, rows, replace=False)).astype(np.int64)
+        t0 = time.perf_counter()
+        w = o.ngram_weights(self.H, self.x, wl.n, wl.w_min)
+        o.ce_rows(dense["h"], dense["W"], self.x, w, sel)
+        xs = dense[f"x/{wl.projs[0].name}"][sel]
+        for p in wl.projs:
+            dA, dB = o.lora_grad(xs, dense[f"dy/{p.name}"][sel], dense[f"A/{p.name}"], dense[f"B/{p.name}"],
+                                 wl.scale)
+            o.sgd_step(wk.bf16_to_f32(dense[f"A/{p.name}"]), dA.astype(np.float32), wk.LORA_LR)
+            o.sgd_step(wk.bf16_to_f32(dense[f"B/{p.name}"]), dB.astype(np.float32), wk.LORA_LR)
+        dt = time.perf_counter() - t0
+        desc = (f"{rows} of {wl.L} update tokens of the {wl.name} workload per sample: full Eq. 8/9 weights, "
+                f"Eq. 10 lse+dh for {rows} rows over all {wl.V} vocab entries, LoRA grads and SGD for those "
+                f"rows; fp64 C oracle with OpenMP")
+        return dt, {"value": round(rows / dt, 3), "unit": UNIT, "cores": o.num_threads(), "kind": "oracle",
+                    "sample": desc + f", {dt:.1f} s"}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_gpu(args):
+    import torch
+    from paper_2607_03441_gb300 import attt
+    from paper_2607_03441_gb300 import build
+    ws, rank, local = _dist()
+    build.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+    wl = wk.WORKLOADS[args.workload]
+    peaks = _peaks()
+    max_steps = 2 * (args.warmup + args.steps) + 4
+    u = Update(wl, dev, max_steps)
+    torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        u.step()
+    torch.cuda.synchronize()
+    if attt.attt_device_status() != 0 or attt.attt_history_status(u.hist) != 0:
+        raise RuntimeError("device status error after warm-up")
+
+    def barrier():
+        if pg is not None:
+            pg.barrier()
+
+    # ---------------- device-timed region ----------------
+    ce_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+             for _ in range(args.steps)]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    n0 = attt.attt_kernel_launches()
+    e0.record()
+    for i in range(args.steps):
+        u.step(ce_ev[i])
+    e1.record()
+    torch.cuda.synchronize()
+    n1 = attt.attt_kernel_launches()
+    barrier()
+    clk = clocks.stop()
+    t_ms = e0.elapsed_time(e1)
+    t_ce = statistics.mean(a.elapsed_time(b) for a, b in ce_ev)
+    if attt.attt_device_status() != 0 or attt.attt_history_status(u.hist) != 0:
+        raise RuntimeError("device status error in the timed region")
+
+    # ---------------- end to end through host buffers ----------------
+    host_in = {
+        "tokens": torch.from_numpy(u.x_host).pin_memory(),
+        "h": torch.from_numpy(u.dense["h"].view(np.int16)).pin_memory(),
+        "x": torch.from_numpy(u.dense[f"x/{u.projs[0].name}"].view(np.int16)).pin_memory(),
+    }
+    for p in u.projs:
+        host_in[f"dy/{p.name}"] = torch.from_numpy(u.dense[f"dy/{p.name}"].view(np.int16)).pin_memory()
+    dev_in = {"tokens": u.x, "h": u.h.view(torch.int16), "x": u.xin.view(torch.int16)}
+    for i, p in enumerate(u.projs):
+        dev_in[f"dy/{p.name}"] = u.dy[i].view(torch.int16)
+    loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+    d2h = loss_host.numel() * loss_host.element_size()
+    barrier()
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record()
+    for _ in range(args.steps):
+        for k, t in host_in.items():
+            dev_in[k].copy_(t, non_blocking=True)
+        u.step()
+        loss_host.copy_(u.loss, non_blocking=True)
+    f1.record()
+    torch.cuda.synchronize()
+    barrier()
+    t_e2e = f0.elapsed_time(f1)
+
+    if pg is not None:
+        tt = torch.tensor([t_ms, t_e2e], device=dev)
+        pg.all_reduce(tt, op=pg.ReduceOp.MAX)
+        t_ms, t_e2e = tt.tolist()
+
+    tokens = wl.L * args.steps * ws
+    value = tokens / (t_ms * 1e-3)
+    e2e_value = tokens / (t_e2e * 1e-3)
+    out = None
+    if rank == 0:
+        traffic = None
+        prof = os.path.join(ROOT, "profiles", "ce_7b_traffic.json")
+        if os.path.exists(prof):
+            try:
+                traffic = json.load(open(prof)).get("traffic_bytes_per_call")
+            except Exception:
+                traffic = None
+        cpu = None
+        if ws == 1 and args.cpu_rows > 0:
+            _, cpu = OracleSample(wl, dense=u.dense, x=u.x_host).run(args.cpu_rows)
+        out = {
+            "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(t_ms / args.steps, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": (f"{wl.name}: one aTTT update, L={wl.L} tokens, V={wl.V}, d={wl.d}, n={wl.n}, "
+                                    f"history {wl.hist_len}+ tokens, LoRA r={wl.r} on q 3584x3584 and "
+                                    f"v 3584x512, one SGD step"),
+                       "global_batch": wl.L * ws, "seq_len": wl.L, "parallelism": f"replicas{ws}",
+                       "l2": "inputs larger than L2 (LM head 1.09 GB streamed every step)"},
+            "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": int(n1 - n0),
+            "roofline": _ce_roofline(wl, t_ce, peaks, traffic),
+            "ce_ms_per_call": round(t_ce, 4),
+            "clocks": clk,
+            "cpu_baseline": cpu,
+        }
+    if pg is not None:
+        pg.barrier()
+        pg.destroy_process_group()
+    u.hist.close()
+    return out
+
+
+# ---------------------------------------------------------------------------
+# the reference arm: the CPU oracle on the host cores
+# ---------------------------------------------------------------------------
+
+def run_reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return None
+    wl = wk.WORKLOADS[args.workload]
+    sample = OracleSample(wl)
+    for _ in range(args.warmup):
+        sample.run(1)
+    t = 0.0
+    last = None
+    for _ in range(args.steps):
+        dt, last = sample.run(args.ref_rows)
+        t += dt
+    value = args.ref_rows * args.steps / t
+    return {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * t / args.steps, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": f"{wl.name} (oracle sample of {args.ref_rows} update tokens per step)",
+                       "global_batch": wl.L, "seq_len": wl.L, "parallelism": "host cores"},
+            "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": last["cores"], "kind": "oracle",
+                             "sample": last["sample"]},
+            "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["attt", "reference"], default="attt")
+    ap.add_argument("--workload", default=WORKLOAD, choices=["tiny", "7b", "long", "32b"])
+    ap.add_argument("--cpu-rows", type=int, default=64, help="rows of the oracle CPU-baseline sample (0: skip)")
+    ap.add_argument("--ref-rows", type=int, default=4, help="rows per step of the reference arm")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    out = run_reference(args) if args.impl == "reference" else run_gpu(args)
+    if out is not None:
+        print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -66,6 +66,11 @@ ATTT_API const char *attt_status_string(int status);
 /* ABI version of this header (major * 100 + minor). */
 ATTT_API int attt_abi_version(void);
 
+/* Number of CUDA kernels this library has launched in this process (all
+ * devices, all threads).  Host-side counter; copies and memsets issued by the
+ * library are not kernels and are not counted. */
+ATTT_API uint64_t attt_kernel_launches(void);
+
 /*
  * Reads and clears the device-side status word of the current device after
  * synchronising `stream`.  Returns the first error any kernel of this library

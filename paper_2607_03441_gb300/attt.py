@@ -49,6 +49,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
         sig = {
             "attt_status_string": (ctypes.c_char_p, [i32]),
             "attt_abi_version": (i32, []),
+            "attt_kernel_launches": (ctypes.c_uint64, []),
             "attt_device_status": (i32, [P]),
             "attt_history_create": (i32, [i32, i64, ctypes.POINTER(P)]),
             "attt_history_destroy": (i32, [P]),
@@ -109,6 +110,11 @@ def attt_status_string(code: int) -> str:
 
 def attt_abi_version() -> int:
     return int(load_library().attt_abi_version())
+
+
+def attt_kernel_launches() -> int:
+    """Kernels launched by libattt in this process so far."""
+    return int(load_library().attt_kernel_launches())
 
 
 def attt_device_status(stream=None) -> int:

@@ -3,6 +3,7 @@
 // shared-memory opt-in.
 #include <cudaTypedefs.h>
 
+#include <atomic>
 #include <map>
 #include <mutex>
 #include <utility>
@@ -18,6 +19,7 @@ std::map<int, int> g_sms;
 std::map<int, int *> g_status_words;
 std::map<std::pair<const void *, int>, size_t> g_smem_set;
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::atomic<unsigned long long> g_launches{0};
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     std::lock_guard<std::mutex> lk(g_mu);
@@ -33,6 +35,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 }  // namespace
+
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 attt_status current_device(int *dev) {
     if (cudaGetDevice(dev) != cudaSuccess) return ATTT_ERR_CUDA;
@@ -113,6 +117,8 @@ const char *attt_status_string(int status) {
 }
 
 int attt_abi_version(void) { return 100; }
+
+uint64_t attt_kernel_launches(void) { return attt::g_launches.load(std::memory_order_relaxed); }
 
 attt_status attt_device_status(attt_stream stream) {
     int dev;

@@ -26,6 +26,9 @@ int *device_status_word(int dev);
 bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
                     uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
 
+// Counts one kernel launch (attt_kernel_launches).
+void count_launch();
+
 // Raises the dynamic shared memory limit of `func` once per device.
 bool set_smem_limit(const void *func, size_t bytes, int dev);
 

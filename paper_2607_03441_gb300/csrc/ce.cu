@@ -153,6 +153,7 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
     ce_finalize_kernel<<<(unsigned)c.nblk, kFinThreads, 0, stream>>>(c.part, (int)c.nvt, c.ztgt, d_tgt, d_w, (int)L,
                                                                      (int)V, lse, 1.0f / (float)L, c.block_sums,
                                                                      c.ticket, d_loss, status);
+    count_launch();
     if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
 
     // pass 2: per vocab chunk, G = (w/L)(softmax - onehot) then dh += G W_chunk

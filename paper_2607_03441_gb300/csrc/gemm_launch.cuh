@@ -88,6 +88,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     const int ntiles = g.tiles_m * g.tiles_n * g.splits;
     const int grid = ntiles < sms ? ntiles : sms;
     kern<<<grid, kGemmThreads, smem, stream>>>(ta, tb, g);
+    count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
 

@@ -150,6 +150,7 @@ attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int npr
         a.nproj = nproj; a.r = r; a.rpad = c.rpad; a.din = din; a.AT = c.AT;
         dim3 grid(grid_for(maxn, 256, dev), nproj);
         lora_prep_kernel<<<grid, 256, 0, stream>>>(a);
+        count_launch();
         if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
     }
     if (cudaMemsetAsync(c.uT32, 0, (size_t)2 * c.Nu * c.Lp * sizeof(float), stream) != cudaSuccess)
@@ -186,6 +187,7 @@ attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int npr
     {
         const int64_t n = (int64_t)2 * c.Nu * c.Lp;
         f32_to_bf16_kernel<<<grid_for(n, 256, dev), 256, 0, stream>>>(c.uT32, c.uT16, n);
+        count_launch();
         if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
     }
     // pass 2a: dA_p = s x^T v_p for every projection at once (x MN-major)
@@ -226,6 +228,7 @@ attt_status attt_lora_step(float *d_A32, float *d_B32, const float *d_dA, const 
     lora_step_kernel<<<grid_for(nA + nB, 256, dev), 256, 0, stream>>>(
         d_A32, d_dA, reinterpret_cast<__nv_bfloat16 *>(d_A16), nA, d_B32, d_dB,
         reinterpret_cast<__nv_bfloat16 *>(d_B16), nB, lr);
+    count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
 

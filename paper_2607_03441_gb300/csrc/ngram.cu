@@ -273,6 +273,7 @@ attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_
     const int64_t blocks = (count + threads - 1) / threads;
     attt::history_insert_kernel<<<(unsigned)blocks, threads, 0, stream>>>(h->d_tokens, p_begin, count, h->n,
                                                                           h->d_table, h->capacity - 1, h->d_status);
+    attt::count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
 
@@ -292,6 +293,7 @@ attt_status attt_history_count(const attt_history *h, const int32_t *d_ngrams, i
     const int threads = 256;
     attt::history_count_kernel<<<(unsigned)((m + threads - 1) / threads), threads, 0, stream>>>(
         h->d_tokens, h->d_table, h->capacity - 1, d_ngrams, m, h->n, d_counts);
+    attt::count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
 
@@ -303,6 +305,7 @@ attt_status attt_ngram_weights(const attt_history *h, const int32_t *d_tokens, i
     const int64_t blocks = (L + attt::kWTile - 1) / attt::kWTile;
     attt::ngram_weights_kernel<<<(unsigned)blocks, attt::kWTile, 0, stream>>>(
         d_tokens, L, h->n, h->d_tokens, h->len, h->d_table, h->capacity - 1, w_min, d_w);
+    attt::count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
 
