@@ -211,6 +211,39 @@ ATTT_API attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din
                            void *d_ws, size_t ws_bytes, attt_stream stream);
 
 /*
+ * attt_lora_grad_noalloc -- attt_lora_grad for callers that cannot allocate
+ * device memory.  (A deployment variant; the paper has no counterpart.)
+ *
+ * Who needs it: a process whose device memory is reserved up front by its
+ * own pool, where a cudaMalloc would fail or fragment the pool; a latency-
+ * critical loop that may not call the allocator because cudaMalloc/cudaFree
+ * can synchronise the device; a plugin whose host application owns all
+ * device allocations.  This call allocates nothing and calls no allocating
+ * routine: its scratch is a static array of ATTT_LORA_NOALLOC_SCRATCH_BYTES
+ * (16 MiB) inside the library's device memory, held by every GPU that loads
+ * the library until the process exits.
+ *
+ * Arguments, layouts and results are those of attt_lora_grad without the
+ * workspace; the caller still passes every input and output buffer.  A
+ * problem whose scratch (attt_lora_workspace_bytes) exceeds 16 MiB returns
+ * ATTT_ERR_WORKSPACE and launches nothing.
+ *
+ * The first call on a device (with that device current) looks up the static
+ * array's device address and caches it; make that first call before any
+ * stream capture begins.  Every call shares the one array per device and the
+ * array keeps the last call's contents (the call clears what must start at
+ * zero itself), so calls that overlap on the GPU -- on two streams, or from
+ * two host threads -- race and must be serialised by the caller.  A timed-out
+ * device wait of this call is reported by attt_device_status().
+ */
+#define ATTT_LORA_NOALLOC_SCRATCH_BYTES ((size_t)16 << 20)
+ATTT_API attt_status attt_lora_grad_noalloc(const attt_bf16 *d_x, int64_t L, int64_t din, int nproj,
+                                            const attt_bf16 *const *d_dy, const int64_t *dout,
+                                            const attt_bf16 *const *d_A, const attt_bf16 *const *d_B,
+                                            int r, float scale,
+                                            float *const *d_dA, float *const *d_dB, attt_stream stream);
+
+/*
  * Eq. 2 / Algorithm 1 gradient step (plain SGD, no weight decay):
  *   A32 <- A32 - lr * dA,  B32 <- B32 - lr * dB     (fp32: product, then
  *                                                    difference, no FMA)

@@ -65,6 +65,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_lora_workspace_bytes": (sz, [i64, i64, i32, P, i32]),
             "attt_lora_grad": (i32, [P, i64, i64, i32, P, P, P, P, i32, f32, P, P, P, sz, P]),
             "attt_lora_step": (i32, [P, P, P, P, i64, i64, i32, f32, P, P, P]),
+            "attt_lora_grad_noalloc": (i32, [P, i64, i64, i32, P, P, P, P, i32, f32, P, P, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -266,6 +267,27 @@ def attt_lora_grad(x: torch.Tensor, dys: Sequence[torch.Tensor], As: Sequence[to
     _check(load_library().attt_lora_grad(
         _bf16(x), L, din, k, arr(dys, _bf16), douts_arr, arr(As, _bf16), arr(Bs, _bf16), int(r), float(scale),
         arr(dAs, _ptr), arr(dBs, _ptr), _ptr(workspace), workspace.numel(), _stream(stream)), "attt_lora_grad")
+    return dAs, dBs
+
+
+LORA_NOALLOC_SCRATCH_BYTES = 16 << 20
+
+
+def attt_lora_grad_noalloc(x: torch.Tensor, dys: Sequence[torch.Tensor], As: Sequence[torch.Tensor],
+                           Bs: Sequence[torch.Tensor], scale: float, dAs: Sequence[torch.Tensor],
+                           dBs: Sequence[torch.Tensor], stream=None):
+    """attt_lora_grad without a workspace: the library uses its own static
+    16 MiB device scratch and allocates nothing.  The caller passes the output
+    tensors.  Returns (dAs, dBs)."""
+    L, din = x.shape
+    k = len(dys)
+    r = As[0].shape[1]
+    P = ctypes.c_void_p
+    arr = lambda ts, f: (P * k)(*[f(t) for t in ts])  # noqa: E731
+    douts_arr = (ctypes.c_int64 * k)(*[int(t.shape[1]) for t in dys])
+    _check(load_library().attt_lora_grad_noalloc(
+        _bf16(x), L, din, k, arr(dys, _bf16), douts_arr, arr(As, _bf16), arr(Bs, _bf16), int(r), float(scale),
+        arr(dAs, _ptr), arr(dBs, _ptr), _stream(stream)), "attt_lora_grad_noalloc")
     return dAs, dBs
 
 

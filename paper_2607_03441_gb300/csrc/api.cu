@@ -130,6 +130,13 @@ attt_status attt_device_status(attt_stream stream) {
     int v = 0;
     if (cudaMemcpy(&v, w, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return ATTT_ERR_CUDA;
     if (v != 0 && cudaMemset(w, 0, sizeof v) != cudaSuccess) return ATTT_ERR_CUDA;
+    if (v == 0) {
+        int *nw = attt::noalloc_status_word(dev);  // attt_lora_grad_noalloc's own word
+        if (nw) {
+            if (cudaMemcpy(&v, nw, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return ATTT_ERR_CUDA;
+            if (v != 0 && cudaMemset(nw, 0, sizeof v) != cudaSuccess) return ATTT_ERR_CUDA;
+        }
+    }
     return (attt_status)v;
 }
 

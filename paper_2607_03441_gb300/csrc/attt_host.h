@@ -32,6 +32,17 @@ void count_launch();
 // Raises the dynamic shared memory limit of `func` once per device.
 bool set_smem_limit(const void *func, size_t bytes, int dev);
 
+// Body of attt_lora_grad.  `status` is the device word for timed-out waits
+// (nullptr: the per-device status word).
+attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int nproj, const attt_bf16 *const *d_dy,
+                          const int64_t *dout, const attt_bf16 *const *d_A, const attt_bf16 *const *d_B, int r,
+                          float scale, float *const *d_dA, float *const *d_dB, void *d_ws, size_t ws_bytes,
+                          int *status, cudaStream_t stream);
+
+// Device address of attt_lora_grad_noalloc's static status word on `dev`, or
+// nullptr if that entry point has not been set up on the device.
+int *noalloc_status_word(int dev);
+
 inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline bool aligned256(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 255u) == 0; }
 inline int64_t cdiv(int64_t a, int64_t b) { return (a + b - 1) / b; }

@@ -35,8 +35,11 @@ inline uint32_t gemm_tmem_cols(int BN) {
     return c;
 }
 
+// `status` is the device word that records a timed-out wait; nullptr selects
+// the library's per-device status word.
 template <int EPI, bool A_MN, bool B_MN>
-attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cudaStream_t stream) {
+attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cudaStream_t stream,
+                        int *status = nullptr) {
     if (p.BN < 16 || p.BN > 256 || p.BN % 16 != 0) return ATTT_ERR_INVALID_ARG;
     if (B_MN && p.BN % 64 != 0) return ATTT_ERR_INVALID_ARG;
     if (p.M <= 0 || p.N <= 0 || p.K <= 0) return ATTT_ERR_INVALID_ARG;
@@ -79,7 +82,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.b_n_off = p.b_n_off;
     g.b_k_off = p.b_k_off;
     g.tmem_cols = gemm_tmem_cols(p.BN);
-    g.status = device_status_word(dev);
+    g.status = status ? status : device_status_word(dev);
     g.ep = ep;
 
     const size_t smem = gemm_smem_bytes(p.BN, g.stages);

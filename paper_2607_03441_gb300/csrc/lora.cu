@@ -103,20 +103,10 @@ static unsigned grid_for(int64_t n, int threads, int dev) {
     return (unsigned)b;
 }
 
-}  // namespace attt
-
-extern "C" {
-
-size_t attt_lora_workspace_bytes(int64_t L, int64_t din, int nproj, const int64_t *dout, int r) {
-    if (L < 1 || din < 1 || nproj < 1 || nproj > attt::kMaxProj || !dout || r < 1 || r > 64) return 0;
-    return attt::lora_layout(nullptr, L, din, nproj, dout, r).bytes;
-}
-
-attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int nproj, const attt_bf16 *const *d_dy,
-                           const int64_t *dout, const attt_bf16 *const *d_A, const attt_bf16 *const *d_B, int r,
-                           float scale, float *const *d_dA, float *const *d_dB, void *d_ws, size_t ws_bytes,
-                           attt_stream stream) {
-    using namespace attt;
+attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int nproj, const attt_bf16 *const *d_dy,
+                          const int64_t *dout, const attt_bf16 *const *d_A, const attt_bf16 *const *d_B, int r,
+                          float scale, float *const *d_dA, float *const *d_dB, void *d_ws, size_t ws_bytes,
+                          int *status, cudaStream_t stream) {
     if (!d_x || !d_dy || !dout || !d_A || !d_B || !d_dA || !d_dB) return ATTT_ERR_INVALID_ARG;
     if (nproj < 1 || nproj > kMaxProj || r < 1 || r > 64 || L < 1 || din < 8 || din % 8 != 0)
         return ATTT_ERR_INVALID_ARG;
@@ -169,7 +159,7 @@ attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int npr
         p.M = (int)L; p.N = c.Nu; p.K = (int)din; p.BN = BNu; p.allow_split = true;
         EpiParams ep{};
         ep.out = c.uT32; ep.out_ld = c.Lp; ep.alpha = 1.0f; ep.r = c.rpad; ep.rpad = c.rpad;
-        st = launch_gemm<EPI_ATOMIC_T, false, false>(p, ep, dev, stream);
+        st = launch_gemm<EPI_ATOMIC_T, false, false>(p, ep, dev, stream, status);
         if (st != ATTT_OK) return st;
     }
     // pass 1b: v_p^T = (dy_p B_p^T)^T
@@ -181,7 +171,7 @@ attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int npr
         EpiParams ep{};
         ep.out = c.vT32 + (size_t)q * c.rpad * c.Lp; ep.out_ld = c.Lp; ep.alpha = 1.0f;
         ep.r = c.rpad; ep.rpad = c.rpad;
-        st = launch_gemm<EPI_ATOMIC_T, false, false>(p, ep, dev, stream);
+        st = launch_gemm<EPI_ATOMIC_T, false, false>(p, ep, dev, stream, status);
         if (st != ATTT_OK) return st;
     }
     {
@@ -199,7 +189,7 @@ attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int npr
         EpiParams ep{};
         for (int q = 0; q < nproj; ++q) ep.outp[q] = d_dA[q];
         ep.alpha = scale; ep.r = r; ep.rpad = c.rpad;
-        st = launch_gemm<EPI_ATOMIC_N, true, false>(p, ep, dev, stream);
+        st = launch_gemm<EPI_ATOMIC_N, true, false>(p, ep, dev, stream, status);
         if (st != ATTT_OK) return st;
     }
     // pass 2b: dB_p^T = s dy_p^T u_p (dy MN-major), stored transposed into dB_p
@@ -211,10 +201,27 @@ attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int npr
         p.M = (int)dout[q]; p.N = c.rpad; p.K = (int)L; p.BN = c.rpad; p.allow_split = true;
         EpiParams ep{};
         ep.out = d_dB[q]; ep.out_ld = dout[q]; ep.alpha = scale; ep.r = r; ep.rpad = c.rpad;
-        st = launch_gemm<EPI_ATOMIC_T, true, false>(p, ep, dev, stream);
+        st = launch_gemm<EPI_ATOMIC_T, true, false>(p, ep, dev, stream, status);
         if (st != ATTT_OK) return st;
     }
     return ATTT_OK;
+}
+
+}  // namespace attt
+
+extern "C" {
+
+size_t attt_lora_workspace_bytes(int64_t L, int64_t din, int nproj, const int64_t *dout, int r) {
+    if (L < 1 || din < 1 || nproj < 1 || nproj > attt::kMaxProj || !dout || r < 1 || r > 64) return 0;
+    return attt::lora_layout(nullptr, L, din, nproj, dout, r).bytes;
+}
+
+attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int nproj, const attt_bf16 *const *d_dy,
+                           const int64_t *dout, const attt_bf16 *const *d_A, const attt_bf16 *const *d_B, int r,
+                           float scale, float *const *d_dA, float *const *d_dB, void *d_ws, size_t ws_bytes,
+                           attt_stream stream) {
+    return attt::lora_grad_run(d_x, L, din, nproj, d_dy, dout, d_A, d_B, r, scale, d_dA, d_dB, d_ws, ws_bytes,
+                               nullptr, stream);
 }
 
 attt_status attt_lora_step(float *d_A32, float *d_B32, const float *d_dA, const float *d_dB, int64_t din,
