@@ -149,20 +149,25 @@ class Update:
                                    dtype=torch.uint8, device=dev)
         self.stream = torch.cuda.current_stream()
 
-    def step(self, ce_events=None):
+    def step(self, ce_events=None, part="all"):
         a = self.attt
-        a.attt_ngram_weights(self.hist, self.x, self.wl.w_min, out=self.w)
-        if ce_events is not None:
-            ce_events[0].record()
-        a.attt_weighted_ce_fwd_bwd(self.h, self.W, self.x, self.w, loss=self.loss, dh=self.dh,
-                                   workspace=self.ws_ce)
-        if ce_events is not None:
-            ce_events[1].record()
-        a.attt_lora_grad(self.xin, self.dy, self.A16, self.B16, self.wl.scale, dAs=self.dA, dBs=self.dB,
-                         workspace=self.ws_lora)
-        for i in range(len(self.projs)):
-            a.attt_lora_step(self.A32[i], self.B32[i], self.dA[i], self.dB[i], wk.LORA_LR, self.A16[i], self.B16[i])
-        a.attt_history_insert(self.hist, self.x)
+        if part in ("all", "ngram"):
+            a.attt_ngram_weights(self.hist, self.x, self.wl.w_min, out=self.w)
+        if part in ("all", "ce"):
+            if ce_events is not None:
+                ce_events[0].record()
+            a.attt_weighted_ce_fwd_bwd(self.h, self.W, self.x, self.w, loss=self.loss, dh=self.dh,
+                                       workspace=self.ws_ce)
+            if ce_events is not None:
+                ce_events[1].record()
+        if part in ("all", "lora"):
+            a.attt_lora_grad(self.xin, self.dy, self.A16, self.B16, self.wl.scale, dAs=self.dA, dBs=self.dB,
+                             workspace=self.ws_lora)
+            for i in range(len(self.projs)):
+                a.attt_lora_step(self.A32[i], self.B32[i], self.dA[i], self.dB[i], wk.LORA_LR, self.A16[i],
+                                 self.B16[i])
+        if part in ("all", "ngram"):
+            a.attt_history_insert(self.hist, self.x)
 
 
 def _ce_roofline(wl, t_ce_ms, peaks, traffic):
@@ -233,6 +238,24 @@ def run_gpu(args):
     max_steps = 2 * (args.warmup + args.steps) + 4
     u = Update(wl, dev, max_steps)
     torch.cuda.synchronize()
+
+    part = args.part
+    if part != "all":
+        # one stage alone, for profiling: a single timed loop, no e2e, no baseline
+        u.w.fill_(1.0)
+        for _ in range(args.warmup):
+            u.step(part=part)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(args.steps):
+            u.step(part=part)
+        e1.record()
+        torch.cuda.synchronize()
+        status = attt.attt_device_status()
+        u.hist.close()
+        return {"part": part, "workload": wl.name, "steps": args.steps,
+                "ms_per_step": round(e0.elapsed_time(e1) / args.steps, 4), "device_status": status}
 
     for _ in range(args.warmup):
         u.step()
@@ -372,7 +395,9 @@ def main():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["attt", "reference"], default="attt")
-    ap.add_argument("--workload", default=WORKLOAD, choices=["tiny", "7b", "long", "32b"])
+    ap.add_argument("--workload", default=WORKLOAD, choices=["tiny", "7b"])
+    ap.add_argument("--part", default="all", choices=["all", "ce", "lora", "ngram"],
+                    help="time one stage alone (profiling aid); 'all' is the benchmark")
     ap.add_argument("--cpu-rows", type=int, default=64, help="rows of the oracle CPU-baseline sample (0: skip)")
     ap.add_argument("--ref-rows", type=int, default=4, help="rows per step of the reference arm")
     args = ap.parse_args()

@@ -1,61 +1,123 @@
 // ce.cu -- Eq. 10 of aTTT on the GPU: the token-weighted next-token CE through
 // the frozen LM head, its value and its gradient with respect to the hidden
-// states, without ever holding the [L, V] logits in HBM.
+// states, in one sweep over the vocabulary (4*L*V*d tensor FLOPs: each logit
+// is computed once), never holding the [L, V] logits in HBM.
 //
-//   pass 1  tcgen05 contraction z = h W^T over 128 x 256 tiles; the epilogue
-//           keeps, per row and vocab tile, the running max and sum of exp
-//           (online logsumexp in log2 units) and the target logit.  HBM
-//           sees only [V/256, L] (max, sum) pairs.
-//   reduce  per row: merge the tile pairs into lse_j, nll_j = lse_j - z_{j,x_j};
-//           the weighted mean (1/L) sum_j w_j nll_j is summed in a fixed
-//           order (deterministic).
-//   pass 2  for each vocab chunk of Vc columns (Vc sized so the chunk's
-//           gradient block stays L2-resident): recompute z for the chunk and
-//           write G = (w_j/L)(softmax(z_j) - onehot(x_j)) as bf16 (fused
-//           epilogue), then dh (+)= G W_chunk with W read MN-major by TMA.
+// For each vocab chunk c of Vc columns (Vc sized so that the chunk's bf16
+// block stays L2-resident):
+//   GEMM1  z = h W_c^T on 128 x 256 tiles; the epilogue keeps per (row, tile)
+//          the max m_t and the sum of exp(z - m_t) (log2 units), writes
+//          E = exp(z - m_t) as bf16, and catches the target logit;
+//   rescale per row: the chunk max M_c over its tiles, E *= exp(m_t - M_c),
+//          and the online-softmax factors of the running max M:
+//          alpha = exp(M_old - M_new), beta = exp(M_c - M_new);
+//   GEMM2  D = E W_c (W read MN-major by TMA); the epilogue folds it into the
+//          fp32 accumulator: acc = alpha * acc + beta * D.
+// Then per row: lse from the (max, sum) pairs of every tile, the loss
+// (1/L) sum_j w_j (lse_j - z_{j,x_j}) summed in a fixed order, and
+//   dh_j = (w_j / L) (acc_j exp(M_j - lse_j) - W_{x_j}).
 // The LM head gets no gradient (frozen; only the adapter trains).
 #include "gemm_launch.cuh"
 
 namespace attt {
 
 constexpr int kCeBN = 256;
-constexpr int kFinThreads = 128;
+constexpr int kCeMaxTiles = 256;  // vocab tiles per chunk at most
+constexpr int kFinThreads = 256;
+constexpr int kFinRows = 32;
 
 struct CeLayout {
     int64_t nvt, Vc, nblk;
     float2 *part;
     float *ztgt, *lse_tmp, *block_sums;
+    float *mrun, *alpha, *beta;
     unsigned int *ticket;
     __nv_bfloat16 *G;
     size_t bytes;
 };
 
-static int64_t ce_chunk(int64_t L, int64_t V) {
-    // Gradient block of one chunk: L x Vc bf16, kept near 96 MB.
+// Upper bound of the vocab chunk: the chunk's bf16 gradient block L x Vc is
+// kept near 96 MB (L2 is 129 MB).  The workspace is sized for this bound.
+static int64_t ce_chunk_max(int64_t L, int64_t V) {
     int64_t vc = (96ll << 20) / (2 * L);
     vc = (vc / kCeBN) * kCeBN;
     if (vc < 4096) vc = 4096;
+    if (vc > kCeMaxTiles * kCeBN) vc = kCeMaxTiles * kCeBN;
     const int64_t vmax = round_up(V, kCeBN);
     if (vc > vmax) vc = vmax;
     return vc;
 }
 
+// Tile plan of pass 2 for `sms` SMs: the dh tile width BNd and the chunk
+// width Vc (<= the workspace bound) that minimise an estimate of the time,
+// counting whole waves of tiles (a partial wave costs a full one) plus a
+// per-launch cost.
+struct CePlan {
+    int64_t Vc;
+    int BNd;
+};
+
+static CePlan ce_plan(int64_t L, int64_t d, int64_t V, int sms) {
+    const double rate = 1.0e13;    // bf16 FLOP/s of one SM, order of magnitude
+    const double launch = 5.0e-6;  // seconds per launch, ramp-up and tail included
+    const int64_t tm = cdiv(L, 128);
+    CePlan best{ce_chunk_max(L, V), kCeBN};
+    double best_t = 1e30;
+    const int bnd_c[3] = {128, 192, 256};
+    int bnd = kCeBN;
+    double bnd_cost = 1e30;
+    for (int b : bnd_c) {
+        const int64_t tiles = tm * cdiv(d, b);
+        const double c = (double)cdiv(tiles, sms) * (b + 32);
+        if (c < bnd_cost) { bnd_cost = c; bnd = b; }
+    }
+    const int64_t vmax = ce_chunk_max(L, V);
+    for (int64_t vc = 4 * kCeBN; vc <= vmax; vc += kCeBN) {
+        double t = 0.0;
+        for (int64_t v0 = 0; v0 < V; v0 += vc) {
+            const int64_t nc = (V - v0 < vc) ? V - v0 : vc;
+            const double w1 = (double)cdiv(tm * cdiv(nc, kCeBN), sms);
+            const double w2 = (double)cdiv(tm * cdiv(d, bnd), sms);
+            t += w1 * 2.0 * 128 * kCeBN * d / rate + w2 * 2.0 * 128 * bnd * round_up(nc, 64) / rate + 2 * launch;
+        }
+        if (t < best_t) { best_t = t; best = CePlan{vc, bnd}; }
+        if (vc == vmax) break;
+    }
+    return best;
+}
+
 static CeLayout ce_layout(void *ws, int64_t L, int64_t V) {
     CeLayout c{};
     c.nvt = cdiv(V, kCeBN);
-    c.Vc = ce_chunk(L, V);
-    c.nblk = cdiv(L, kFinThreads);
+    c.Vc = ce_chunk_max(L, V);
+    c.nblk = cdiv(L, kFinRows);
     Carve cv{static_cast<char *>(ws), 0};
     c.part = cv.take<float2>((size_t)(c.nvt * L));
     c.ztgt = cv.take<float>((size_t)L);
     c.lse_tmp = cv.take<float>((size_t)L);
     c.block_sums = cv.take<float>((size_t)c.nblk);
+    c.mrun = cv.take<float>((size_t)L);
+    c.alpha = cv.take<float>((size_t)L);
+    c.beta = cv.take<float>((size_t)L);
     c.ticket = cv.take<unsigned int>(4);
     c.G = cv.take<__nv_bfloat16>((size_t)(L * c.Vc));
     c.bytes = (size_t)round_up((int64_t)cv.used, 256);
     return c;
 }
 
+// Merges two (max, sum) pairs of an online logsumexp in log2 units.
+__device__ __forceinline__ void lse_merge(float &m, float &s, float m2, float s2) {
+    const float mx = fmaxf(m, m2);
+    if (mx == -INFINITY) return;
+    s = s * exp2f(m - mx) + s2 * exp2f(m2 - mx);
+    m = mx;
+}
+
+// One block per kFinRows rows; warp w merges the vocab tiles i = w (mod 8) of
+// its 32 rows with coalesced loads of part[i, rows], then warp 0 merges the
+// 8 partial pairs per row and forms lse, the target NLL and the weighted sum.
+// The last block (atomic ticket) adds the block sums in block order, so the
+// loss is deterministic.
 __global__ void __launch_bounds__(kFinThreads) ce_finalize_kernel(const float2 *__restrict__ part, int nvt,
                                                                    const float *__restrict__ ztgt,
                                                                    const int32_t *__restrict__ tgt,
@@ -63,42 +125,43 @@ __global__ void __launch_bounds__(kFinThreads) ce_finalize_kernel(const float2 *
                                                                    float *__restrict__ lse_out, float inv_L,
                                                                    float *block_sums, unsigned int *ticket,
                                                                    float *loss, int *status) {
-    __shared__ float red[kFinThreads / 32];
+    constexpr int kWarps = kFinThreads / 32;
+    __shared__ float sm_m[kWarps][kFinRows], sm_s[kWarps][kFinRows];
     __shared__ bool last;
-    const int j = blockIdx.x * kFinThreads + threadIdx.x;
-    float contrib = 0.f;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j = blockIdx.x * kFinRows + lane;
+    float m = -INFINITY, s = 0.f;
     if (j < L) {
-        float m = -INFINITY, s = 0.f;
-        for (int i = 0; i < nvt; ++i) {
+        for (int i = warp; i < nvt; i += kWarps) {
             const float2 p = __ldcg(part + (int64_t)i * L + j);
-            if (p.x > m) {
-                s = s * exp2f(m - p.x) + p.y;
-                m = p.x;
-            } else {
-                s += p.y * exp2f(p.x - m);
-            }
+            lse_merge(m, s, p.x, p.y);
         }
-        const float lse = (m + log2f(s)) * 0.69314718055994531f;
-        lse_out[j] = lse;
-        const int t = tgt[j];
-        float nll;
-        if (t < 0 || t >= V) {
-            record_error(status, ATTT_ERR_TOKEN_RANGE);
-            nll = __int_as_float(0x7fc00000);
-        } else {
-            nll = lse - __ldcg(ztgt + j);
-        }
-        contrib = w[j] * nll;
     }
-    for (int o = 16; o > 0; o >>= 1) contrib += __shfl_xor_sync(0xffffffffu, contrib, o);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = contrib;
+    sm_m[warp][lane] = m;
+    sm_s[warp][lane] = s;
     __syncthreads();
-    if (threadIdx.x == 0) {
-        float b = 0.f;
-        for (int i = 0; i < kFinThreads / 32; ++i) b += red[i];
-        block_sums[blockIdx.x] = b;
-        __threadfence();
-        last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+    if (warp == 0) {
+        for (int k = 1; k < kWarps; ++k) lse_merge(m, s, sm_m[k][lane], sm_s[k][lane]);
+        float contrib = 0.f;
+        if (j < L) {
+            const float lse = (m + log2f(s)) * 0.69314718055994531f;
+            lse_out[j] = lse;
+            const int t = tgt[j];
+            float nll;
+            if (t < 0 || t >= V) {
+                record_error(status, ATTT_ERR_TOKEN_RANGE);
+                nll = __int_as_float(0x7fc00000);
+            } else {
+                nll = lse - __ldcg(ztgt + j);
+            }
+            contrib = w[j] * nll;
+        }
+        for (int o = 16; o > 0; o >>= 1) contrib += __shfl_xor_sync(0xffffffffu, contrib, o);
+        if (lane == 0) {
+            block_sums[blockIdx.x] = contrib;
+            __threadfence();
+            last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+        }
     }
     __syncthreads();
     if (last && threadIdx.x == 0) {
@@ -107,6 +170,84 @@ __global__ void __launch_bounds__(kFinThreads) ce_finalize_kernel(const float2 *
         for (unsigned i = 0; i < gridDim.x; ++i) total += __ldcg(block_sums + i);
         *loss = total * inv_L;
         *ticket = 0u;
+    }
+}
+
+// Per row j of chunk c (one block per row): the chunk max M_c over the
+// chunk's tiles, E[j, :] *= exp(m_t - M_c) tile by tile, and the running-max
+// factors for the dh accumulator.
+__global__ void __launch_bounds__(256) ce_rescale_kernel(const float2 *__restrict__ part, int tile0, int ntiles,
+                                                         int L, __nv_bfloat16 *G, int64_t G_ld, float *mrun,
+                                                         float *alpha, float *beta, int first) {
+    __shared__ float f[kCeMaxTiles];
+    __shared__ float red[8];
+    const int j = blockIdx.x;
+    float m = -INFINITY;
+    for (int t = threadIdx.x; t < ntiles; t += blockDim.x) {
+        const float mt = __ldcg(&part[(int64_t)(tile0 + t) * L + j].x);
+        f[t] = mt;
+        m = fmaxf(m, mt);
+    }
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
+    __syncthreads();
+    float mc = red[0];
+    for (int i = 1; i < (int)(blockDim.x >> 5); ++i) mc = fmaxf(mc, red[i]);
+    for (int t = threadIdx.x; t < ntiles; t += blockDim.x) f[t] = exp2f(f[t] - mc);
+    __syncthreads();
+    uint4 *row = reinterpret_cast<uint4 *>(G + (int64_t)j * G_ld);
+    const int nvec = ntiles * (kCeBN / 8);
+    for (int i = threadIdx.x; i < nvec; i += blockDim.x) {
+        const float sc = f[i / (kCeBN / 8)];
+        uint4 u = row[i];
+        uint32_t *w = reinterpret_cast<uint32_t *>(&u);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162 *>(&w[q]);
+            const float2 v = __bfloat1622float2(b);
+            b = __floats2bfloat162_rn(v.x * sc, v.y * sc);
+            w[q] = *reinterpret_cast<uint32_t *>(&b);
+        }
+        row[i] = u;
+    }
+    if (threadIdx.x == 0) {
+        const float mold = first ? -INFINITY : mrun[j];
+        const float mnew = fmaxf(mold, mc);
+        alpha[j] = (mold == -INFINITY) ? 0.f : exp2f(mold - mnew);
+        beta[j] = exp2f(mc - mnew);
+        mrun[j] = mnew;
+    }
+}
+
+// dh_j = (w_j / L) (acc_j exp(M_j - lse_j) - W_{x_j}); one block per row.
+__global__ void __launch_bounds__(256) ce_fixup_kernel(float *dh, int64_t d, const __nv_bfloat16 *__restrict__ W,
+                                                       const int32_t *__restrict__ tgt, const float *__restrict__ w,
+                                                       float inv_L, const float *__restrict__ mrun,
+                                                       const float *__restrict__ lse, int V) {
+    const int j = blockIdx.x;
+    const int t = tgt[j];
+    const float c = w[j] * inv_L;
+    const float sc = exp2f(mrun[j] - lse[j] * kLog2e);
+    float *row = dh + (int64_t)j * d;
+    if (t < 0 || t >= V) {
+        for (int64_t k = threadIdx.x; k < d; k += blockDim.x) row[k] = __int_as_float(0x7fc00000);
+        return;
+    }
+    const __nv_bfloat16 *wt = W + (int64_t)t * d;
+    // d % 8 == 0: 8 columns per step (one 16-byte load of W, two float4 of dh)
+    for (int64_t k = (int64_t)threadIdx.x * 8; k < d; k += (int64_t)blockDim.x * 8) {
+        const uint4 u = *reinterpret_cast<const uint4 *>(wt + k);
+        const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&u);
+        float4 *o = reinterpret_cast<float4 *>(row + k);
+        float4 a0 = o[0], a1 = o[1];
+        const float2 w0 = __bfloat1622float2(b[0]), w1 = __bfloat1622float2(b[1]);
+        const float2 w2 = __bfloat1622float2(b[2]), w3 = __bfloat1622float2(b[3]);
+        a0.x = c * (a0.x * sc - w0.x); a0.y = c * (a0.y * sc - w0.y);
+        a0.z = c * (a0.z * sc - w1.x); a0.w = c * (a0.w * sc - w1.y);
+        a1.x = c * (a1.x * sc - w2.x); a1.y = c * (a1.y * sc - w2.y);
+        a1.z = c * (a1.z * sc - w3.x); a1.w = c * (a1.w * sc - w3.y);
+        o[0] = a0;
+        o[1] = a1;
     }
 }
 
@@ -139,50 +280,48 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
     float *lse = d_lse ? d_lse : c.lse_tmp;
     if (cudaMemsetAsync(c.ticket, 0, sizeof(unsigned int), stream) != cudaSuccess) return ATTT_ERR_CUDA;
 
-    // pass 1: per-tile (max, sum exp) and the target logit
-    {
-        GemmProblem p{};
-        p.a = d_h; p.a_rows_ld = d; p.a_rows = L; p.a_k = d;
-        p.b = d_W; p.b_rows_ld = d; p.b_rows = V; p.b_k = d;
-        p.M = (int)L; p.N = (int)V; p.K = (int)d; p.BN = kCeBN;
-        EpiParams ep{};
-        ep.tgt = d_tgt; ep.part = c.part; ep.ztgt = c.ztgt; ep.v0 = 0;
-        st = launch_gemm<EPI_CE_STATS, false, false>(p, ep, dev, stream);
-        if (st != ATTT_OK) return st;
-    }
-    ce_finalize_kernel<<<(unsigned)c.nblk, kFinThreads, 0, stream>>>(c.part, (int)c.nvt, c.ztgt, d_tgt, d_w, (int)L,
-                                                                     (int)V, lse, 1.0f / (float)L, c.block_sums,
-                                                                     c.ticket, d_loss, status);
-    count_launch();
-    if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
-
-    // pass 2: per vocab chunk, G = (w/L)(softmax - onehot) then dh += G W_chunk
-    for (int64_t v0 = 0, ci = 0; v0 < V; v0 += c.Vc, ++ci) {
-        const int64_t Nc = (V - v0 < c.Vc) ? V - v0 : c.Vc;
-        {
+    const CePlan plan = ce_plan(L, d, V, num_sms(dev));
+    for (int64_t v0 = 0, ci = 0; v0 < V; v0 += plan.Vc, ++ci) {
+        const int64_t Nc = (V - v0 < plan.Vc) ? V - v0 : plan.Vc;
+        const int ntiles = (int)cdiv(Nc, kCeBN);
+        {   // GEMM1: logits of the chunk -> per-tile stats and E = exp(z - m_t)
             GemmProblem p{};
             p.a = d_h; p.a_rows_ld = d; p.a_rows = L; p.a_k = d;
             p.b = d_W; p.b_rows_ld = d; p.b_rows = V; p.b_k = d;
             p.M = (int)L; p.N = (int)Nc; p.K = (int)d; p.BN = kCeBN;
             p.b_n_off = (int)v0;
             EpiParams ep{};
-            ep.tgt = d_tgt; ep.lse = lse; ep.w = d_w; ep.inv_L = 1.0f / (float)L; ep.v0 = (int)v0;
+            ep.tgt = d_tgt; ep.part = c.part; ep.tile0 = (int)(v0 / kCeBN); ep.ztgt = c.ztgt; ep.v0 = (int)v0;
             ep.G = c.G; ep.G_ld = c.Vc;
-            st = launch_gemm<EPI_CE_GRAD, false, false>(p, ep, dev, stream);
+            st = launch_gemm<EPI_CE_EXP, false, false>(p, ep, dev, stream);
             if (st != ATTT_OK) return st;
         }
-        {
+        ce_rescale_kernel<<<(unsigned)L, 256, 0, stream>>>(c.part, (int)(v0 / kCeBN), ntiles, (int)L, c.G, c.Vc,
+                                                          c.mrun, c.alpha, c.beta, ci == 0 ? 1 : 0);
+        count_launch();
+        if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
+        {   // GEMM2: acc = alpha * acc + beta * (E W_c)
             GemmProblem p{};
             p.a = c.G; p.a_rows_ld = c.Vc; p.a_rows = L; p.a_k = c.Vc;
             p.b = d_W; p.b_rows_ld = d; p.b_rows = d; p.b_k = V;
-            p.M = (int)L; p.N = (int)d; p.K = (int)round_up(Nc, 64); p.BN = kCeBN;
+            p.M = (int)L; p.N = (int)d; p.K = (int)round_up(Nc, 64); p.BN = plan.BNd;
             p.b_k_off = (int)v0;
             EpiParams ep{};
             ep.out = d_dh; ep.out_ld = d; ep.accumulate = ci > 0 ? 1 : 0; ep.alpha = 1.0f;
+            ep.row_alpha = c.alpha; ep.row_beta = c.beta;
             st = launch_gemm<EPI_F32_ACC, false, true>(p, ep, dev, stream);
             if (st != ATTT_OK) return st;
         }
     }
+    ce_finalize_kernel<<<(unsigned)c.nblk, kFinThreads, 0, stream>>>(c.part, (int)c.nvt, c.ztgt, d_tgt, d_w, (int)L,
+                                                                     (int)V, lse, 1.0f / (float)L, c.block_sums,
+                                                                     c.ticket, d_loss, status);
+    count_launch();
+    if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
+    ce_fixup_kernel<<<(unsigned)L, 256, 0, stream>>>(d_dh, d, reinterpret_cast<const __nv_bfloat16 *>(d_W), d_tgt,
+                                                     d_w, 1.0f / (float)L, c.mrun, lse, (int)V);
+    count_launch();
+    if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
     return ATTT_OK;
 }
 

@@ -25,9 +25,8 @@
 namespace attt {
 
 enum EpiKind : int {
-    EPI_CE_STATS = 0,  // per (row, vocab tile): running max and sum of exp, target logit
-    EPI_CE_GRAD = 1,   // G = (w/L) (softmax - onehot) as bf16, for the dh contraction
-    EPI_F32_ACC = 2,   // out[m, n] (+)= acc   (fp32, row-major)
+    EPI_CE_EXP = 0,    // per (row, vocab tile): max m, E = exp(z - m) as bf16, sum of E, target logit
+    EPI_F32_ACC = 2,   // out[m, n] = (acc ? alpha_m out[m, n] : 0) + beta_m acc  (fp32, row-major)
     EPI_ATOMIC_T = 3,  // out[n, m] += alpha * acc   (fp32, transposed, split-K)
     EPI_ATOMIC_N = 4,  // out_p[m, c] += alpha * acc for column n = p * rpad + c (split-K)
 };
@@ -37,11 +36,9 @@ constexpr int kMaxProj = 8;
 struct EpiParams {
     // CE
     const int32_t *tgt;  // [M] target ids
-    float2 *part;        // [tiles_n, M] (max, sum) in log2 units
+    float2 *part;        // [vocab tiles, M] (max, sum of exp) in log2 units
+    int tile0;           // vocab tile index of column 0 of this launch
     float *ztgt;         // [M] target logit
-    const float *lse;    // [M] natural-log logsumexp
-    const float *w;      // [M] Eq. 9 weights
-    float inv_L;         // 1 / L
     int v0;              // vocab id of column 0 of this launch
     __nv_bfloat16 *G;    // [M, G_ld]
     int64_t G_ld;
@@ -50,6 +47,8 @@ struct EpiParams {
     int64_t out_ld;
     int accumulate;
     float alpha;
+    const float *row_alpha;  // [M] or nullptr (1)
+    const float *row_beta;   // [M] or nullptr (1)
     float *outp[kMaxProj];
     int r;     // valid columns per projection block
     int rpad;  // column block width per projection
@@ -99,44 +98,26 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
     const int n_base = tn * g.BN;
     const EpiParams &ep = g.ep;
 
-    if constexpr (EPI == EPI_CE_STATS) {
-        // Online logsumexp over this tile's columns, in log2 units.
+    if constexpr (EPI == EPI_CE_EXP) {
+        // Pass 1 over the tile's columns: the row max (log2 units) and the
+        // target logit.  Pass 2: E = exp(z - max) rounded to bf16 into the
+        // gradient block (columns past N as zeros), and the sum of the
+        // unrounded exponentials.
         const int t = rv ? __ldg(ep.tgt + gm) - ep.v0 : -1;
-        float mx = -INFINITY, sm = 0.f, zt = 0.f;
+        float mx = -INFINITY, zt = 0.f;
         bool hit = false;
         for (int c = 0; c < g.BN; c += 32) {
             if (n_base + c >= g.N) break;
             float v[32];
             tmem_ld_x32(taddr + (uint32_t)c, v);
-            float cm = -INFINITY;
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
                 const int col = n_base + c + i;
                 if (col == t) { zt = v[i]; hit = true; }
-                v[i] = (col < g.N) ? v[i] * kLog2e : -INFINITY;
-                cm = fmaxf(cm, v[i]);
+                if (col < g.N) mx = fmaxf(mx, v[i] * kLog2e);
             }
-            const float nm = fmaxf(mx, cm);
-            float s = sm * exp2f(mx - nm);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) s += exp2f(v[i] - nm);
-            sm = s;
-            mx = nm;
         }
-        if (rv) {
-            ep.part[(int64_t)tn * g.M + gm] = make_float2(mx, sm);
-            if (hit) ep.ztgt[gm] = zt;
-        }
-    } else if constexpr (EPI == EPI_CE_GRAD) {
-        // G[j, v] = (w_j / L) (exp(z - lse_j) - [v == tgt_j]) in bf16; columns
-        // past N are written as zeros so the dh contraction may read them.
-        float l2 = 0.f, cw = 0.f;
-        int t = -1;
-        if (rv) {
-            l2 = __ldg(ep.lse + gm) * kLog2e;
-            cw = __ldg(ep.w + gm) * ep.inv_L;
-            t = __ldg(ep.tgt + gm) - ep.v0;
-        }
+        float sm = 0.f;
         __nv_bfloat16 *grow = ep.G + (int64_t)gm * ep.G_ld;
         for (int c = 0; c < g.BN; c += 32) {
             float v[32];
@@ -145,10 +126,10 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
 #pragma unroll
             for (int i = 0; i < 32; i += 2) {
                 const int col = n_base + c + i;
-                float g0 = 0.f, g1 = 0.f;
-                if (col < g.N) g0 = cw * (exp2f(fmaf(v[i], kLog2e, -l2)) - (col == t ? 1.f : 0.f));
-                if (col + 1 < g.N) g1 = cw * (exp2f(fmaf(v[i + 1], kLog2e, -l2)) - (col + 1 == t ? 1.f : 0.f));
-                __nv_bfloat162 b = __floats2bfloat162_rn(g0, g1);
+                const float e0 = (col < g.N) ? exp2f(fmaf(v[i], kLog2e, -mx)) : 0.f;
+                const float e1 = (col + 1 < g.N) ? exp2f(fmaf(v[i + 1], kLog2e, -mx)) : 0.f;
+                sm += e0 + e1;
+                __nv_bfloat162 b = __floats2bfloat162_rn(e0, e1);
                 pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
             }
             if (rv) {
@@ -157,8 +138,15 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
                 for (int q = 0; q < 4; ++q) dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
             }
         }
+        if (rv) {
+            ep.part[(int64_t)(ep.tile0 + tn) * g.M + gm] = make_float2(mx, sm);
+            if (hit) ep.ztgt[gm] = zt;
+        }
     } else if constexpr (EPI == EPI_F32_ACC) {
         float *orow = ep.out + (int64_t)gm * ep.out_ld;
+        float ra = 1.f, rb = 1.f;
+        if (rv && ep.row_alpha) ra = __ldg(ep.row_alpha + gm);
+        if (rv && ep.row_beta) rb = __ldg(ep.row_beta + gm);
         for (int c = 0; c < g.BN; c += 32) {
             if (n_base + c >= g.N) break;
             float v[32];
@@ -169,16 +157,17 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
                     float4 *dst = reinterpret_cast<float4 *>(orow + col0);
 #pragma unroll
                     for (int q = 0; q < 8; ++q) {
-                        float4 o = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                        float4 o = make_float4(rb * v[4 * q], rb * v[4 * q + 1], rb * v[4 * q + 2], rb * v[4 * q + 3]);
                         if (ep.accumulate) {
                             const float4 p = dst[q];
-                            o.x += p.x; o.y += p.y; o.z += p.z; o.w += p.w;
+                            o.x = fmaf(ra, p.x, o.x); o.y = fmaf(ra, p.y, o.y);
+                            o.z = fmaf(ra, p.z, o.z); o.w = fmaf(ra, p.w, o.w);
                         }
                         dst[q] = o;
                     }
                 } else {
                     for (int i = 0; i < 32 && col0 + i < g.N; ++i)
-                        orow[col0 + i] = ep.accumulate ? orow[col0 + i] + v[i] : v[i];
+                        orow[col0 + i] = ep.accumulate ? fmaf(ra, orow[col0 + i], rb * v[i]) : rb * v[i];
                 }
             }
         }
