@@ -8,9 +8,12 @@
 //   GEMM1  z = h W_c^T on 128 x 256 tiles; the epilogue keeps per (row, tile)
 //          the max m_t and the sum of exp(z - m_t) (log2 units), writes
 //          E = exp(z - m_t) as bf16, and catches the target logit;
-//   rescale per row: the chunk max M_c over its tiles, E *= exp(m_t - M_c),
-//          and the online-softmax factors of the running max M:
-//          alpha = exp(M_old - M_new), beta = exp(M_c - M_new);
+//          From the second chunk on, E is written against the running max
+//          of the earlier chunks instead of the tile max;
+//   chunk  per row: the chunk max, a rewrite of E only where needed (the
+//          first chunk, or a row whose max jumped by more than 2^32), and the
+//          online-softmax factors of the accumulator's reference A:
+//          alpha = exp(A_old - A_new), beta = exp(R_E - A_new);
 //   GEMM2  D = E W_c (W read MN-major by TMA); the epilogue folds it into the
 //          fp32 accumulator: acc = alpha * acc + beta * D.
 // Then per row: lse from the (max, sum) pairs of every tile, the loss
@@ -30,7 +33,7 @@ struct CeLayout {
     int64_t nvt, Vc, nblk;
     float2 *part;
     float *ztgt, *lse_tmp, *block_sums;
-    float *mrun, *alpha, *beta;
+    float *aref, *mref, *alpha, *beta;
     unsigned int *ticket;
     __nv_bfloat16 *G;
     size_t bytes;
@@ -96,7 +99,8 @@ static CeLayout ce_layout(void *ws, int64_t L, int64_t V) {
     c.ztgt = cv.take<float>((size_t)L);
     c.lse_tmp = cv.take<float>((size_t)L);
     c.block_sums = cv.take<float>((size_t)c.nblk);
-    c.mrun = cv.take<float>((size_t)L);
+    c.aref = cv.take<float>((size_t)L);
+    c.mref = cv.take<float>((size_t)L);
     c.alpha = cv.take<float>((size_t)L);
     c.beta = cv.take<float>((size_t)L);
     c.ticket = cv.take<unsigned int>(4);
@@ -173,61 +177,66 @@ __global__ void __launch_bounds__(kFinThreads) ce_finalize_kernel(const float2 *
     }
 }
 
-// Per row j of chunk c (one block per row): the chunk max M_c over the
-// chunk's tiles, E[j, :] *= exp(m_t - M_c) tile by tile, and the running-max
-// factors for the dh accumulator.
-__global__ void __launch_bounds__(256) ce_rescale_kernel(const float2 *__restrict__ part, int tile0, int ntiles,
-                                                         int L, __nv_bfloat16 *G, int64_t G_ld, float *mrun,
-                                                         float *alpha, float *beta, int first) {
-    __shared__ float f[kCeMaxTiles];
-    __shared__ float red[8];
-    const int j = blockIdx.x;
-    float m = -INFINITY;
-    for (int t = threadIdx.x; t < ntiles; t += blockDim.x) {
-        const float mt = __ldcg(&part[(int64_t)(tile0 + t) * L + j].x);
-        f[t] = mt;
-        m = fmaxf(m, mt);
-    }
-    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = m;
-    __syncthreads();
-    float mc = red[0];
-    for (int i = 1; i < (int)(blockDim.x >> 5); ++i) mc = fmaxf(mc, red[i]);
-    for (int t = threadIdx.x; t < ntiles; t += blockDim.x) f[t] = exp2f(f[t] - mc);
-    __syncthreads();
+// Bookkeeping of chunk c, one warp per row j (log2 units throughout):
+//   M_c  = max over the chunk's tiles of the tile max m_t;
+//   R    = the running max of the earlier chunks (mref; -inf for the first).
+//   GEMM1 wrote tile t of E against R, or against m_t when m_t - R >
+//   kCeRefJump.  If any tile did (M_c - R > kCeRefJump), the row is rewritten
+//   against M_c tile by tile; otherwise it stays against R.  Rp = the
+//   reference E now has.
+//   acc = alpha * acc + beta * (E W_c) with A_new = max(A_old, Rp),
+//   alpha = exp2(A_old - A_new), beta = exp2(Rp - A_new);  mref <- max(R, M_c).
+__global__ void __launch_bounds__(256) ce_chunk_kernel(const float2 *__restrict__ part, int tile0, int ntiles, int L,
+                                                       __nv_bfloat16 *G, int64_t G_ld, float *aref, float *mref,
+                                                       float *alpha, float *beta, int first) {
+    const int j = blockIdx.x * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (j >= L) return;
+    float mc = -INFINITY;
+    for (int t = lane; t < ntiles; t += 32) mc = fmaxf(mc, __ldcg(&part[(int64_t)(tile0 + t) * L + j].x));
+    for (int o = 16; o > 0; o >>= 1) mc = fmaxf(mc, __shfl_xor_sync(0xffffffffu, mc, o));
+    const float r = first ? -INFINITY : mref[j];
     uint4 *row = reinterpret_cast<uint4 *>(G + (int64_t)j * G_ld);
-    const int nvec = ntiles * (kCeBN / 8);
-    for (int i = threadIdx.x; i < nvec; i += blockDim.x) {
-        const float sc = f[i / (kCeBN / 8)];
-        uint4 u = row[i];
-        uint32_t *w = reinterpret_cast<uint32_t *>(&u);
+    const int per_tile = kCeBN / 8;  // uint4 (8 x bf16) per tile row
+    float rp = r;
+    if (mc - r > kCeRefJump) {
+        rp = mc;
+        for (int t = 0; t < ntiles; ++t) {
+            const float mt = __ldcg(&part[(int64_t)(tile0 + t) * L + j].x);
+            const float sc = (mt - r > kCeRefJump) ? exp2f(mt - mc) : exp2f(r - mc);
+            for (int i = lane; i < per_tile; i += 32) {
+                uint4 u = row[t * per_tile + i];
+                uint32_t *w = reinterpret_cast<uint32_t *>(&u);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162 *>(&w[q]);
-            const float2 v = __bfloat1622float2(b);
-            b = __floats2bfloat162_rn(v.x * sc, v.y * sc);
-            w[q] = *reinterpret_cast<uint32_t *>(&b);
+                for (int q = 0; q < 4; ++q) {
+                    __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162 *>(&w[q]);
+                    const float2 v = __bfloat1622float2(b);
+                    b = __floats2bfloat162_rn(v.x * sc, v.y * sc);
+                    w[q] = *reinterpret_cast<uint32_t *>(&b);
+                }
+                row[t * per_tile + i] = u;
+            }
         }
-        row[i] = u;
     }
-    if (threadIdx.x == 0) {
-        const float mold = first ? -INFINITY : mrun[j];
-        const float mnew = fmaxf(mold, mc);
-        alpha[j] = (mold == -INFINITY) ? 0.f : exp2f(mold - mnew);
-        beta[j] = exp2f(mc - mnew);
-        mrun[j] = mnew;
+    if (lane == 0) {
+        const float aold = first ? -INFINITY : aref[j];
+        const float anew = fmaxf(aold, rp);
+        alpha[j] = (aold == -INFINITY) ? 0.f : exp2f(aold - anew);
+        beta[j] = exp2f(rp - anew);
+        aref[j] = anew;
+        mref[j] = fmaxf(r, mc);
     }
 }
 
-// dh_j = (w_j / L) (acc_j exp(M_j - lse_j) - W_{x_j}); one block per row.
+// dh_j = (w_j / L) (acc_j exp(A_j - lse_j) - W_{x_j}); one block per row.
 __global__ void __launch_bounds__(256) ce_fixup_kernel(float *dh, int64_t d, const __nv_bfloat16 *__restrict__ W,
                                                        const int32_t *__restrict__ tgt, const float *__restrict__ w,
-                                                       float inv_L, const float *__restrict__ mrun,
+                                                       float inv_L, const float *__restrict__ aref,
                                                        const float *__restrict__ lse, int V) {
     const int j = blockIdx.x;
     const int t = tgt[j];
     const float c = w[j] * inv_L;
-    const float sc = exp2f(mrun[j] - lse[j] * kLog2e);
+    const float sc = exp2f(aref[j] - lse[j] * kLog2e);
     float *row = dh + (int64_t)j * d;
     if (t < 0 || t >= V) {
         for (int64_t k = threadIdx.x; k < d; k += blockDim.x) row[k] = __int_as_float(0x7fc00000);
@@ -293,11 +302,13 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
             EpiParams ep{};
             ep.tgt = d_tgt; ep.part = c.part; ep.tile0 = (int)(v0 / kCeBN); ep.ztgt = c.ztgt; ep.v0 = (int)v0;
             ep.G = c.G; ep.G_ld = c.Vc;
+            ep.eref = ci == 0 ? nullptr : c.mref;
             st = launch_gemm<EPI_CE_EXP, false, false>(p, ep, dev, stream);
             if (st != ATTT_OK) return st;
         }
-        ce_rescale_kernel<<<(unsigned)L, 256, 0, stream>>>(c.part, (int)(v0 / kCeBN), ntiles, (int)L, c.G, c.Vc,
-                                                          c.mrun, c.alpha, c.beta, ci == 0 ? 1 : 0);
+        ce_chunk_kernel<<<(unsigned)cdiv(L, 8), 256, 0, stream>>>(c.part, (int)(v0 / kCeBN), ntiles, (int)L, c.G,
+                                                                  c.Vc, c.aref, c.mref, c.alpha, c.beta,
+                                                                  ci == 0 ? 1 : 0);
         count_launch();
         if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
         {   // GEMM2: acc = alpha * acc + beta * (E W_c)
@@ -319,7 +330,7 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
     count_launch();
     if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
     ce_fixup_kernel<<<(unsigned)L, 256, 0, stream>>>(d_dh, d, reinterpret_cast<const __nv_bfloat16 *>(d_W), d_tgt,
-                                                     d_w, 1.0f / (float)L, c.mrun, lse, (int)V);
+                                                     d_w, 1.0f / (float)L, c.aref, lse, (int)V);
     count_launch();
     if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
     return ATTT_OK;

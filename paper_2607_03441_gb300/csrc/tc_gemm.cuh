@@ -39,6 +39,7 @@ struct EpiParams {
     float2 *part;        // [vocab tiles, M] (max, sum of exp) in log2 units
     int tile0;           // vocab tile index of column 0 of this launch
     float *ztgt;         // [M] target logit
+    const float *eref;   // [M] reference (log2 units) E is written against; nullptr: the tile max
     int v0;              // vocab id of column 0 of this launch
     __nv_bfloat16 *G;    // [M, G_ld]
     int64_t G_ld;
@@ -85,6 +86,10 @@ __device__ __forceinline__ void decode_tile(const GemmArgs &g, int t, int &tm, i
 
 constexpr float kLog2e = 1.4426950408889634f;
 
+// A CE tile whose max exceeds the row reference by more than 2^kCeRefJump
+// (log2 units) writes E against its own max instead, so E <= 2^kCeRefJump.
+constexpr float kCeRefJump = 32.f;
+
 // ---------------------------------------------------------------------------
 // Epilogues.  Every thread owns accumulator row `row` of the tile; all 32
 // lanes of a warp execute the TMEM loads together even when their row is
@@ -118,6 +123,15 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
             }
         }
         float sm = 0.f;
+        // E = exp2(z2 - mx) * sc: against the row reference R given by the
+        // caller (sc = exp2(mx - R)), or against the tile max (sc = 1) when
+        // there is none or mx - R > kCeRefJump.  The sum is always taken
+        // against the tile max.
+        float sc = 1.f;
+        if (ep.eref && rv) {
+            const float jump = mx - __ldg(ep.eref + gm);
+            if (jump <= kCeRefJump) sc = exp2f(jump);
+        }
         __nv_bfloat16 *grow = ep.G + (int64_t)gm * ep.G_ld;
         for (int c = 0; c < g.BN; c += 32) {
             float v[32];
@@ -129,7 +143,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
                 const float e0 = (col < g.N) ? exp2f(fmaf(v[i], kLog2e, -mx)) : 0.f;
                 const float e1 = (col + 1 < g.N) ? exp2f(fmaf(v[i + 1], kLog2e, -mx)) : 0.f;
                 sm += e0 + e1;
-                __nv_bfloat162 b = __floats2bfloat162_rn(e0, e1);
+                __nv_bfloat162 b = __floats2bfloat162_rn(e0 * sc, e1 * sc);
                 pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
             }
             if (rv) {

@@ -152,3 +152,32 @@ def test_long_sampled(attt):
 @pytest.mark.slow
 def test_32b_sampled(attt):
     _sampled_check(attt, "32b", nrows=6)
+
+
+def test_multichunk_with_reference_jumps(attt):
+    """Several vocab chunks, with rows whose max logit jumps far above the
+    running max of the earlier chunks (2^92 in log2 units) and rows whose
+    later chunks sit far below it; sampled rows against the oracle."""
+    L, V, d = 2048, 80000, 64
+    rng = wk.rng_for(77, "jump")
+    h = wk.normal_bf16(77, "h", (L, d), 0.5)
+    W = wk.normal_bf16(77, "W", (V, d), 0.05)
+    hot_rows = [5, 77, 1500]
+    for j, v in zip(hot_rows, [60000, 79999, 30]):
+        h[j] = 0
+        h[j, 0] = wk.bf16_bits(np.array([8.0], np.float32))[0]
+        W[v, 0] = wk.bf16_bits(np.array([8.0], np.float32))[0]  # z[j, v] = 64
+    tgt = rng.integers(0, V, L).astype(np.int32)
+    tgt[5] = 60000
+    w = rng.choice(np.array([1.0, 0.5, 0.05], np.float32), L).astype(np.float32)
+    loss, dh, lse = _run(attt, h, W, tgt, w)
+    rows = np.array(hot_rows + [0, 1, 1000, L - 1], np.int64)
+    rlse, rnll, rdh = oracle.ce_rows(h, W, tgt, w, rows)
+    np.testing.assert_allclose(lse[rows], rlse, atol=LSE_ATOL, rtol=0)
+    for i in range(len(rows)):
+        e = rel_l2(dh[rows[i]], rdh[i])
+        assert e < DH_RL2, (rows[i], e)
+    hf = wk.bf16_to_f32(h).astype(np.float64)
+    zt = np.einsum("ld,ld->l", hf, wk.bf16_to_f32(W[tgt]).astype(np.float64))
+    ref_loss = float(np.sum(w.astype(np.float64) * (lse.astype(np.float64) - zt)) / L)
+    assert abs(loss - ref_loss) <= LOSS_RTOL * abs(ref_loss)
