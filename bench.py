@@ -17,6 +17,8 @@ host cores instead (rank 0 only).
 from __future__ import annotations
 
 import argparse
+import glob
+import hashlib
 import json
 import os
 import shutil
@@ -168,6 +170,33 @@ class Update:
                                  self.B16[i])
         if part in ("all", "ngram"):
             a.attt_history_insert(self.hist, self.x)
+
+
+def _sources_sha256() -> str:
+    """Hash of the CUDA sources and the C header, to tell whether a stored
+    ncu capture still describes the kernels that run."""
+    h = hashlib.sha256()
+    files = sorted(glob.glob(os.path.join(ROOT, "paper_2607_03441_gb300", "csrc", "*")))
+    files.append(os.path.join(ROOT, "include", "attt.h"))
+    for f in files:
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def _stored_traffic(wl):
+    """DRAM bytes per Eq. 10 call from the committed ncu capture, or None when
+    there is none for this workload or the kernels changed since."""
+    path = os.path.join(ROOT, "profiles", f"ce_{wl.name}_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    if rec.get("csrc_sha256") != _sources_sha256():
+        return None
+    return rec.get("traffic_bytes_per_call")
 
 
 def _ce_roofline(wl, t_ce_ms, peaks, traffic):
@@ -327,13 +356,7 @@ def run_gpu(args):
     e2e_value = tokens / (t_e2e * 1e-3)
     out = None
     if rank == 0:
-        traffic = None
-        prof = os.path.join(ROOT, "profiles", "ce_7b_traffic.json")
-        if os.path.exists(prof):
-            try:
-                traffic = json.load(open(prof)).get("traffic_bytes_per_call")
-            except Exception:
-                traffic = None
+        traffic = _stored_traffic(wl)
         cpu = None
         if ws == 1 and args.cpu_rows > 0:
             _, cpu = OracleSample(wl, dense=u.dense, x=u.x_host).run(args.cpu_rows)

@@ -51,39 +51,36 @@ static int64_t ce_chunk_max(int64_t L, int64_t V) {
     return vc;
 }
 
-// Tile plan of pass 2 for `sms` SMs: the dh tile width BNd and the chunk
-// width Vc (<= the workspace bound) that minimise an estimate of the time,
-// counting whole waves of tiles (a partial wave costs a full one) plus a
-// per-launch cost.
+// Tile plan for `sms` SMs.  Above 128 rows both contractions run on CTA pairs
+// (cta_group::2: 256 x 256 accumulator tiles), else on single CTAs (128 x 256).
+// The chunk width Vc (<= the workspace bound) minimises an estimate of the
+// time that counts whole waves of tiles (a partial wave costs a full one)
+// plus a per-launch cost.
 struct CePlan {
     int64_t Vc;
-    int BNd;
+    bool pair;
 };
 
 static CePlan ce_plan(int64_t L, int64_t d, int64_t V, int sms) {
     const double rate = 1.0e13;    // bf16 FLOP/s of one SM, order of magnitude
     const double launch = 5.0e-6;  // seconds per launch, ramp-up and tail included
-    const int64_t tm = cdiv(L, 128);
-    CePlan best{ce_chunk_max(L, V), kCeBN};
+    const bool pair = L > 128;
+    const int64_t rows = pair ? 256 : 128;       // accumulator rows per tile
+    const int64_t units = pair ? sms / 2 : sms;  // tiles in flight
+    const double tile_rate = rate * (pair ? 2.0 : 1.0);
+    const int64_t tm = cdiv(L, rows);
+    const double w2 = (double)cdiv(tm * cdiv(d, kCeBN), units);
+    CePlan best{ce_chunk_max(L, V), pair};
     double best_t = 1e30;
-    const int bnd_c[3] = {128, 192, 256};
-    int bnd = kCeBN;
-    double bnd_cost = 1e30;
-    for (int b : bnd_c) {
-        const int64_t tiles = tm * cdiv(d, b);
-        const double c = (double)cdiv(tiles, sms) * (b + 32);
-        if (c < bnd_cost) { bnd_cost = c; bnd = b; }
-    }
     const int64_t vmax = ce_chunk_max(L, V);
     for (int64_t vc = 4 * kCeBN; vc <= vmax; vc += kCeBN) {
         double t = 0.0;
         for (int64_t v0 = 0; v0 < V; v0 += vc) {
             const int64_t nc = (V - v0 < vc) ? V - v0 : vc;
-            const double w1 = (double)cdiv(tm * cdiv(nc, kCeBN), sms);
-            const double w2 = (double)cdiv(tm * cdiv(d, bnd), sms);
-            t += w1 * 2.0 * 128 * kCeBN * d / rate + w2 * 2.0 * 128 * bnd * round_up(nc, 64) / rate + 2 * launch;
+            const double w1 = (double)cdiv(tm * cdiv(nc, kCeBN), units);
+            t += (w1 * d + w2 * round_up(nc, 64)) * 2.0 * rows * kCeBN / tile_rate + 3 * launch;
         }
-        if (t < best_t) { best_t = t; best = CePlan{vc, bnd}; }
+        if (t < best_t) { best_t = t; best = CePlan{vc, pair}; }
         if (vc == vmax) break;
     }
     return best;
@@ -297,7 +294,7 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
             GemmProblem p{};
             p.a = d_h; p.a_rows_ld = d; p.a_rows = L; p.a_k = d;
             p.b = d_W; p.b_rows_ld = d; p.b_rows = V; p.b_k = d;
-            p.M = (int)L; p.N = (int)Nc; p.K = (int)d; p.BN = kCeBN;
+            p.M = (int)L; p.N = (int)Nc; p.K = (int)d; p.BN = kCeBN; p.pair = plan.pair;
             p.b_n_off = (int)v0;
             EpiParams ep{};
             ep.tgt = d_tgt; ep.part = c.part; ep.tile0 = (int)(v0 / kCeBN); ep.ztgt = c.ztgt; ep.v0 = (int)v0;
@@ -315,7 +312,7 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
             GemmProblem p{};
             p.a = c.G; p.a_rows_ld = c.Vc; p.a_rows = L; p.a_k = c.Vc;
             p.b = d_W; p.b_rows_ld = d; p.b_rows = d; p.b_k = V;
-            p.M = (int)L; p.N = (int)d; p.K = (int)round_up(Nc, 64); p.BN = plan.BNd;
+            p.M = (int)L; p.N = (int)d; p.K = (int)round_up(Nc, 64); p.BN = kCeBN; p.pair = plan.pair;
             p.b_k_off = (int)v0;
             EpiParams ep{};
             ep.out = d_dh; ep.out_ld = d; ep.accumulate = ci > 0 ? 1 : 0; ep.alpha = 1.0f;

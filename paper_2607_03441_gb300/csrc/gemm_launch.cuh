@@ -19,6 +19,7 @@ struct GemmProblem {
     int BN;
     int a_m_off = 0, a_k_off = 0, b_n_off = 0, b_k_off = 0;
     bool allow_split = false;  // epilogue reduces split-K partials with atomics
+    bool pair = false;         // run on CTA pairs (256-row tiles, cta_group::2)
 };
 
 constexpr size_t kMaxSmem = 232448;  // 227 KB opt-in per CTA on sm_100-class parts
@@ -41,7 +42,8 @@ template <int EPI, bool A_MN, bool B_MN>
 attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cudaStream_t stream,
                         int *status = nullptr) {
     if (p.BN < 16 || p.BN > 256 || p.BN % 16 != 0) return ATTT_ERR_INVALID_ARG;
-    if (B_MN && p.BN % 64 != 0) return ATTT_ERR_INVALID_ARG;
+    if (B_MN && (p.pair ? (p.BN / 2) % 64 : p.BN % 64) != 0) return ATTT_ERR_INVALID_ARG;
+    if (p.pair && p.BN < 32) return ATTT_ERR_INVALID_ARG;  // BN/2 B rows per CTA (a multiple of 8)
     if (p.M <= 0 || p.N <= 0 || p.K <= 0) return ATTT_ERR_INVALID_ARG;
     CUtensorMap ta, tb;
     // K-major operand: storage [rows, K] (K contiguous), box 64 x rows_tile.
@@ -54,7 +56,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     if (!ok) return ATTT_ERR_INVALID_ARG;
     if (!B_MN)
         ok = make_tmap_bf16(&tb, p.b, (uint64_t)p.b_k, (uint64_t)p.b_rows, (uint64_t)p.b_rows_ld * 2, 64,
-                            (uint32_t)p.BN);
+                            (uint32_t)(p.pair ? p.BN / 2 : p.BN));
     else
         ok = make_tmap_bf16(&tb, p.b, (uint64_t)p.b_rows, (uint64_t)p.b_k, (uint64_t)p.b_rows_ld * 2, 64, 64);
     if (!ok) return ATTT_ERR_INVALID_ARG;
@@ -63,15 +65,17 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.M = p.M;
     g.N = p.N;
     g.BN = p.BN;
-    g.stages = gemm_stages(p.BN);
+    const int bn_cta = p.pair ? p.BN / 2 : p.BN;  // B rows one CTA stages
+    g.stages = gemm_stages(bn_cta);
     g.tiles_m = (int)cdiv(p.M, 128);
     g.tiles_n = (int)cdiv(p.N, p.BN);
     g.kb_total = (int)cdiv(p.K, 64);
     const int sms = num_sms(dev);
+    const int units = p.pair ? sms / 2 : sms;  // concurrent tiles
+    const int tiles = (p.pair ? (g.tiles_m + 1) / 2 : g.tiles_m) * g.tiles_n;
     int splits = 1;
     if (p.allow_split) {
-        const int tiles = g.tiles_m * g.tiles_n;
-        splits = (int)cdiv(sms, tiles);
+        splits = (int)cdiv(units, tiles);
         if (splits > g.kb_total) splits = g.kb_total;
         if (splits < 1) splits = 1;
     }
@@ -85,12 +89,31 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.status = status ? status : device_status_word(dev);
     g.ep = ep;
 
-    const size_t smem = gemm_smem_bytes(p.BN, g.stages);
-    auto kern = tc_gemm_kernel<EPI, A_MN, B_MN>;
-    if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
-    const int ntiles = g.tiles_m * g.tiles_n * g.splits;
-    const int grid = ntiles < sms ? ntiles : sms;
-    kern<<<grid, kGemmThreads, smem, stream>>>(ta, tb, g);
+    const size_t smem = gemm_smem_bytes(bn_cta, g.stages);
+    const int ntiles = tiles * g.splits;
+    if (!p.pair) {
+        auto kern = tc_gemm_kernel<EPI, A_MN, B_MN>;
+        if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
+        const int grid = ntiles < sms ? ntiles : sms;
+        kern<<<grid, kGemmThreads, smem, stream>>>(ta, tb, g);
+    } else {
+        auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN>;
+        if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
+        const int pairs = ntiles < units ? ntiles : units;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)(2 * pairs));
+        cfg.blockDim = dim3(kGemmThreads);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = stream;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = 2;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        if (cudaLaunchKernelEx(&cfg, kern, ta, tb, g) != cudaSuccess) return ATTT_ERR_CUDA;
+    }
     count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }

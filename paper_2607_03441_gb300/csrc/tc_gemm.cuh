@@ -97,10 +97,16 @@ constexpr float kCeRefJump = 32.f;
 // ---------------------------------------------------------------------------
 
 template <int EPI>
-__device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn, int row, uint32_t taddr) {
-    const int gm = tm * 128 + row;
+__device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, int tn, int row, uint32_t taddr) {
+    const int gm = gm_base + row;
     const bool rv = gm < g.M;
     const int n_base = tn * g.BN;
+    // Columns this tile owns: [n_base, n_tile) within the tile, [n_base, n_end)
+    // within the problem.  TMEM is read in chunks of 32 (or 16) columns, so a
+    // chunk may run past the tile when BN is not a multiple of it; nothing
+    // past n_tile is ever stored (it belongs to the next tile).
+    const int n_tile = n_base + g.BN;
+    const int n_end = min(g.N, n_tile);
     const EpiParams &ep = g.ep;
 
     if constexpr (EPI == EPI_CE_EXP) {
@@ -112,14 +118,16 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
         float mx = -INFINITY, zt = 0.f;
         bool hit = false;
         for (int c = 0; c < g.BN; c += 32) {
-            if (n_base + c >= g.N) break;
+            if (n_base + c >= n_end) break;
             float v[32];
             tmem_ld_x32(taddr + (uint32_t)c, v);
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
                 const int col = n_base + c + i;
-                if (col == t) { zt = v[i]; hit = true; }
-                if (col < g.N) mx = fmaxf(mx, v[i] * kLog2e);
+                if (col < n_end) {
+                    if (col == t) { zt = v[i]; hit = true; }
+                    mx = fmaxf(mx, v[i] * kLog2e);
+                }
             }
         }
         float sm = 0.f;
@@ -140,16 +148,20 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
 #pragma unroll
             for (int i = 0; i < 32; i += 2) {
                 const int col = n_base + c + i;
-                const float e0 = (col < g.N) ? exp2f(fmaf(v[i], kLog2e, -mx)) : 0.f;
-                const float e1 = (col + 1 < g.N) ? exp2f(fmaf(v[i + 1], kLog2e, -mx)) : 0.f;
+                const float e0 = (col < n_end) ? exp2f(fmaf(v[i], kLog2e, -mx)) : 0.f;
+                const float e1 = (col + 1 < n_end) ? exp2f(fmaf(v[i + 1], kLog2e, -mx)) : 0.f;
                 sm += e0 + e1;
                 __nv_bfloat162 b = __floats2bfloat162_rn(e0 * sc, e1 * sc);
                 pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
             }
             if (rv) {
+                // zeros past N (inside the tile) are stored too: the dh
+                // contraction reads whole 64-column K blocks
                 uint4 *dst = reinterpret_cast<uint4 *>(grow + n_base + c);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+                for (int q = 0; q < 4; ++q)
+                    if (n_base + c + 8 * q < n_tile)
+                        dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
             }
         }
         if (rv) {
@@ -162,12 +174,12 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
         if (rv && ep.row_alpha) ra = __ldg(ep.row_alpha + gm);
         if (rv && ep.row_beta) rb = __ldg(ep.row_beta + gm);
         for (int c = 0; c < g.BN; c += 32) {
-            if (n_base + c >= g.N) break;
+            if (n_base + c >= n_end) break;
             float v[32];
             tmem_ld_x32(taddr + (uint32_t)c, v);
             if (rv) {
                 const int col0 = n_base + c;
-                if (col0 + 32 <= g.N) {
+                if (col0 + 32 <= n_end) {
                     float4 *dst = reinterpret_cast<float4 *>(orow + col0);
 #pragma unroll
                     for (int q = 0; q < 8; ++q) {
@@ -180,35 +192,35 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int tm, int tn,
                         dst[q] = o;
                     }
                 } else {
-                    for (int i = 0; i < 32 && col0 + i < g.N; ++i)
+                    for (int i = 0; i < 32 && col0 + i < n_end; ++i)
                         orow[col0 + i] = ep.accumulate ? fmaf(ra, orow[col0 + i], rb * v[i]) : rb * v[i];
                 }
             }
         }
     } else if constexpr (EPI == EPI_ATOMIC_T) {
         for (int c = 0; c < g.BN; c += 16) {
-            if (n_base + c >= g.N) break;
+            if (n_base + c >= n_end) break;
             float v[16];
             tmem_ld_x16(taddr + (uint32_t)c, v);
             if (rv) {
 #pragma unroll
                 for (int i = 0; i < 16; ++i) {
                     const int col = n_base + c + i;
-                    if (col < g.N && (col % ep.rpad) < ep.r)
+                    if (col < n_end && (col % ep.rpad) < ep.r)
                         atomicAdd(ep.out + (int64_t)col * ep.out_ld + gm, ep.alpha * v[i]);
                 }
             }
         }
     } else if constexpr (EPI == EPI_ATOMIC_N) {
         for (int c = 0; c < g.BN; c += 16) {
-            if (n_base + c >= g.N) break;
+            if (n_base + c >= n_end) break;
             float v[16];
             tmem_ld_x16(taddr + (uint32_t)c, v);
             if (rv) {
 #pragma unroll
                 for (int i = 0; i < 16; ++i) {
                     const int col = n_base + c + i;
-                    if (col < g.N) {
+                    if (col < n_end) {
                         const int p = col / ep.rpad, cc = col - p * ep.rpad;
                         if (cc < ep.r) atomicAdd(ep.outp[p] + (int64_t)gm * ep.r + cc, ep.alpha * v[i]);
                     }
@@ -380,7 +392,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             (void)mbar_try_wait(tfull0 + 8 * acc, par);  // per-thread acquire of the completed phase
             tc_fence_after();
             const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * g.BN);
-            epilogue_tile<EPI>(g, tm, tn, row, taddr);
+            epilogue_tile<EPI>(g, tm * 128, tn, row, taddr);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
@@ -391,6 +403,197 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __syncthreads();
     tc_fence_after();
     if (warp == 1) tmem_dealloc(tmem_base, g.tmem_cols);
+}
+
+// ---------------------------------------------------------------------------
+// The CTA-pair kernel: one 256 x BN accumulator tile per cluster of 2 CTAs
+// (tcgen05 cta_group::2).  Each CTA holds 128 rows of A and BN/2 rows of B
+// per stage and 128 rows of the accumulator; the even CTA issues the MMAs,
+// which read both CTAs' shared memory, and multicasts its commits to both
+// CTAs.  Both CTAs' TMA loads complete on the even CTA's stage barrier; both
+// CTAs' epilogues release the accumulator to the even CTA.  Per SM this moves
+// a third less shared-memory traffic per FLOP than the single-CTA kernel.
+// ---------------------------------------------------------------------------
+
+__device__ __forceinline__ void decode_tile_pair(const GemmArgs &g, int t, int &tm2, int &tn, int &split) {
+    const int tiles_m2 = (g.tiles_m + 1) / 2;
+    const int per = tiles_m2 * g.tiles_n;
+    split = t / per;
+    const int rem = t - split * per;
+    tn = rem / tiles_m2;
+    tm2 = rem - tn * tiles_m2;
+}
+
+template <int EPI, bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                        const GemmArgs g) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int S = g.stages;
+    const int BNh = g.BN / 2;  // B rows held by this CTA
+    const uint32_t b_bytes = gemm_b_stage_bytes(BNh);
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + (size_t)S * kABytes;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + (size_t)S * b_bytes);
+    const uint32_t full0 = smem_u32(bars);
+    const uint32_t empty0 = smem_u32(bars + S);
+    const uint32_t tfull0 = smem_u32(bars + 2 * S);
+    const uint32_t tempty0 = smem_u32(bars + 2 * S + 2);
+    const uint32_t drain0 = smem_u32(bars + 2 * S + 4);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * S + 5);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const bool leader = rank == 0;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            mbar_init(full0 + 8 * s, 1);
+            mbar_init(empty0 + 8 * s, 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(tfull0 + 8 * a, 1);
+            mbar_init(tempty0 + 8 * a, 8);
+        }
+        mbar_init(drain0, 1);
+        *abort_flag = 0;
+        fence_mbar_init();
+        tma_prefetch_desc(&tmA);
+        tma_prefetch_desc(&tmB);
+    }
+    cluster_sync();  // both CTAs' barriers exist before any cross-CTA signal
+    if (warp == 1) {
+        tmem_alloc_pair(smem_u32(tmem_slot), g.tmem_cols);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    const int tiles_m2 = (g.tiles_m + 1) / 2;
+    const int ntiles = tiles_m2 * g.tiles_n * g.splits;
+    const int cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
+    const uint32_t lead_full0 = mapa_shared(full0, 0);
+    const uint32_t lead_tempty0 = mapa_shared(tempty0, 0);
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------- TMA producer (both CTAs) ----------------
+            int stage = 0;
+            uint32_t phase = 0;
+            bool ok = true;
+            for (int t = cid; t < ntiles && ok; t += ncl) {
+                int tm2, tn, split;
+                decode_tile_pair(g, t, tm2, tn, split);
+                const int kb0 = split * g.kb_per_split;
+                const int kb1 = min(g.kb_total, kb0 + g.kb_per_split);
+                const int arow = g.a_m_off + tm2 * 256 + 128 * (int)rank;
+                const int brow = g.b_n_off + tn * g.BN + BNh * (int)rank;
+                for (int kb = kb0; kb < kb1; ++kb) {
+                    if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
+                    if (leader) mbar_arrive_expect_tx(full0 + 8 * stage, 2u * (kABytes + b_bytes));
+                    const uint32_t fb = lead_full0 + 8 * stage;
+                    const uint32_t a_dst = smem_u32(sA + (size_t)stage * kABytes);
+                    const uint32_t b_dst = smem_u32(sB + (size_t)stage * b_bytes);
+                    const int k = kb * 64;
+                    if (!A_MN) {
+                        tma_load_2d_pair(a_dst, &tmA, fb, g.a_k_off + k, arow);
+                    } else {
+                        tma_load_2d_pair(a_dst, &tmA, fb, arow, g.a_k_off + k);
+                        tma_load_2d_pair(a_dst + 8192, &tmA, fb, arow + 64, g.a_k_off + k);
+                    }
+                    if (!B_MN) {
+                        tma_load_2d_pair(b_dst, &tmB, fb, g.b_k_off + k, brow);
+                    } else {
+                        for (int b = 0; b < BNh / 64; ++b)
+                            tma_load_2d_pair(b_dst + 8192 * b, &tmB, fb, brow + 64 * b, g.b_k_off + k);
+                    }
+                    if (++stage == S) { stage = 0; phase ^= 1u; }
+                }
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                record_error(g.status, ATTT_ERR_TIMEOUT);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0 && leader) {
+            // ---------------- MMA issuer (even CTA) ----------------
+            const uint32_t idesc = idesc_bf16_f32((uint32_t)g.BN, A_MN, B_MN, 256);
+            int stage = 0;
+            uint32_t phase = 0;
+            int it = 0;
+            bool ok = true;
+            for (int t = cid; t < ntiles && ok; t += ncl, ++it) {
+                int tm2, tn, split;
+                decode_tile_pair(g, t, tm2, tn, split);
+                const int kb0 = split * g.kb_per_split;
+                const int kb1 = min(g.kb_total, kb0 + g.kb_per_split);
+                const int acc = it & 1;
+                if (!mbar_wait(tempty0 + 8 * acc, (((uint32_t)it >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * g.BN);
+                for (int kb = kb0; kb < kb1; ++kb) {
+                    if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t a_addr = smem_u32(sA + (size_t)stage * kABytes);
+                    const uint32_t b_addr = smem_u32(sB + (size_t)stage * b_bytes);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const uint64_t ad = A_MN ? smem_desc_sw128(a_addr + kk * 2048, 8192, 1024)
+                                                 : smem_desc_sw128(a_addr + kk * 32, 16, 1024);
+                        const uint64_t bd = B_MN ? smem_desc_sw128(b_addr + kk * 2048, 8192, 1024)
+                                                 : smem_desc_sw128(b_addr + kk * 32, 16, 1024);
+                        umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+                    }
+                    umma_commit_pair(empty0 + 8 * stage, 3);
+                    if (++stage == S) { stage = 0; phase ^= 1u; }
+                }
+                if (!ok) break;
+                umma_commit_pair(tfull0 + 8 * acc, 3);
+            }
+            if (!ok) {
+                *abort_flag = 1;
+                record_error(g.status, ATTT_ERR_TIMEOUT);
+            }
+            umma_commit_pair(drain0, 1);
+            volatile int no_abort = 0;
+            if (!mbar_wait(drain0, 0u, &no_abort)) record_error(g.status, ATTT_ERR_TIMEOUT);
+        }
+    } else {
+        // ---------------- epilogue (warps 2..5, both CTAs) ----------------
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        int it = 0;
+        for (int t = cid; t < ntiles; t += ncl, ++it) {
+            int tm2, tn, split;
+            decode_tile_pair(g, t, tm2, tn, split);
+            const int acc = it & 1;
+            const uint32_t par = ((uint32_t)it >> 1) & 1u;
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(tfull0 + 8 * acc, par, abort_flag) ? 1 : 0;
+            ok = __shfl_sync(0xffffffffu, ok, 0);
+            if (!ok) {
+                if (lane == 0) { *abort_flag = 1; record_error(g.status, ATTT_ERR_TIMEOUT); }
+                break;
+            }
+            (void)mbar_try_wait(tfull0 + 8 * acc, par);
+            tc_fence_after();
+            const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * g.BN);
+            epilogue_tile<EPI>(g, tm2 * 256 + 128 * (int)rank, tn, row, taddr);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(lead_tempty0 + 8 * acc);
+        }
+    }
+
+    tc_fence_before();
+    cluster_sync();  // no CTA leaves while the pair's MMAs or signals are in flight
+    tc_fence_after();
+    if (warp == 1) tmem_dealloc_pair(tmem_base, g.tmem_cols);
 }
 
 }  // namespace attt

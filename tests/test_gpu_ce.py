@@ -181,3 +181,17 @@ def test_multichunk_with_reference_jumps(attt):
     zt = np.einsum("ld,ld->l", hf, wk.bf16_to_f32(W[tgt]).astype(np.float64))
     ref_loss = float(np.sum(w.astype(np.float64) * (lse.astype(np.float64) - zt)) / L)
     assert abs(loss - ref_loss) <= LOSS_RTOL * abs(ref_loss)
+
+
+def test_launch_counter_counts_every_kernel(attt):
+    """One single-chunk call launches GEMM1, the chunk kernel, GEMM2, the
+    finalize and the fixup kernels: five kernels, all counted."""
+    L, V, d = 200, 1000, 64
+    h = wk.normal_bf16(8, "h", (L, d), 1.0)
+    W = wk.normal_bf16(8, "W", (V, d), 0.1)
+    tgt = wk.rng_for(8, "t").integers(0, V, L).astype(np.int32)
+    args = (bf16_dev(h), bf16_dev(W), i32_dev(tgt), f32_dev(np.ones(L, np.float32)))
+    attt.attt_weighted_ce_fwd_bwd(*args)
+    n0 = attt.attt_kernel_launches()
+    attt.attt_weighted_ce_fwd_bwd(*args)
+    assert attt.attt_kernel_launches() - n0 == 5

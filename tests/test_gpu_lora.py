@@ -119,3 +119,17 @@ def test_sgd_step_bit_exact(attt):
     np.testing.assert_array_equal(B32.cpu().numpy(), pB)
     np.testing.assert_array_equal(A16.view(torch.int16).cpu().numpy().view(np.uint16), bA)
     np.testing.assert_array_equal(B16.view(torch.int16).cpu().numpy().view(np.uint16), bB)
+
+
+def test_launch_counter_counts_every_kernel(attt):
+    """Two projections: prep, u, v (x2), bf16 cast, dA, dB (x2) = 8 kernels;
+    the SGD step is one more."""
+    x, dys, As, Bs = _inputs(9, 200, 128, [64, 128], 8)
+    n0 = attt.attt_kernel_launches()
+    _group(attt, x, dys, As, Bs, 2.0)
+    assert attt.attt_kernel_launches() - n0 == 8
+    A32 = f32_dev(np.zeros((128, 8), np.float32))
+    B32 = f32_dev(np.zeros((8, 64), np.float32))
+    n1 = attt.attt_kernel_launches()
+    attt.attt_lora_step(A32, B32, torch.zeros_like(A32), torch.zeros_like(B32), 5e-4)
+    assert attt.attt_kernel_launches() - n1 == 1
