@@ -384,7 +384,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             const uint32_t par = ((uint32_t)it >> 1) & 1u;
             int ok = 1;
             if (lane == 0) ok = mbar_wait(tfull0 + 8 * acc, par, abort_flag) ? 1 : 0;
-            ok = __shfl_sync(0xffffffffu, ok, 0);
+            // one decision for all four epilogue warps
+            ok = named_barrier_and(1, 128, __shfl_sync(0xffffffffu, ok, 0));
             if (!ok) {
                 if (lane == 0) { *abort_flag = 1; record_error(g.status, ATTT_ERR_TIMEOUT); }
                 break;
@@ -575,7 +576,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             const uint32_t par = ((uint32_t)it >> 1) & 1u;
             int ok = 1;
             if (lane == 0) ok = mbar_wait(tfull0 + 8 * acc, par, abort_flag) ? 1 : 0;
-            ok = __shfl_sync(0xffffffffu, ok, 0);
+            // one decision for all four epilogue warps
+            ok = named_barrier_and(1, 128, __shfl_sync(0xffffffffu, ok, 0));
             if (!ok) {
                 if (lane == 0) { *abort_flag = 1; record_error(g.status, ATTT_ERR_TIMEOUT); }
                 break;
