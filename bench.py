@@ -151,25 +151,80 @@ class Update:
                                    dtype=torch.uint8, device=dev)
         self.stream = torch.cuda.current_stream()
 
-    def step(self, ce_events=None, part="all"):
+    ROWS = ("ngram_weights", "weighted_ce_fwd_bwd", "lora_grad", "lora_step", "history_insert")
+
+    def step(self, events=None, part="all"):
+        """One update.  `events` (optional) maps each row name to a pair of
+        CUDA events recorded around that row's calls on the current stream."""
         a = self.attt
+
+        def mark(name, k):
+            if events is not None:
+                events[name][k].record()
+
         if part in ("all", "ngram"):
+            mark("ngram_weights", 0)
             a.attt_ngram_weights(self.hist, self.x, self.wl.w_min, out=self.w)
+            mark("ngram_weights", 1)
         if part in ("all", "ce"):
-            if ce_events is not None:
-                ce_events[0].record()
+            mark("weighted_ce_fwd_bwd", 0)
             a.attt_weighted_ce_fwd_bwd(self.h, self.W, self.x, self.w, loss=self.loss, dh=self.dh,
                                        workspace=self.ws_ce)
-            if ce_events is not None:
-                ce_events[1].record()
+            mark("weighted_ce_fwd_bwd", 1)
         if part in ("all", "lora"):
+            mark("lora_grad", 0)
             a.attt_lora_grad(self.xin, self.dy, self.A16, self.B16, self.wl.scale, dAs=self.dA, dBs=self.dB,
                              workspace=self.ws_lora)
+            mark("lora_grad", 1)
+            mark("lora_step", 0)
             for i in range(len(self.projs)):
                 a.attt_lora_step(self.A32[i], self.B32[i], self.dA[i], self.dB[i], wk.LORA_LR, self.A16[i],
                                  self.B16[i])
+            mark("lora_step", 1)
         if part in ("all", "ngram"):
+            mark("history_insert", 0)
             a.attt_history_insert(self.hist, self.x)
+            mark("history_insert", 1)
+
+
+def row_work(wl):
+    """Algorithmic work of each row of one update: (kind, amount, unit).
+    Bytes count each input read once and each output written once; FLOPs
+    count the contractions the method defines."""
+    L, V, d, n, r = wl.L, wl.V, wl.d, wl.n, wl.r
+    din = wl.projs[0].din
+    douts = [p.dout for p in wl.projs]
+    lora_bytes = 2 * L * din + sum(2 * L * do for do in douts)               # x once, each dy once
+    lora_bytes += sum(2 * din * r + 2 * r * do + 4 * din * r + 4 * r * do for do in douts)  # A, B in; dA, dB out
+    step_elems = sum(din * r + r * do for do in douts)
+    return {
+        # Eq. 8/9: tokens in, one 32 B table sector per probe, weights out
+        "ngram_weights": ("hbm", 4 * L + 32 * max(L - n + 1, 0) + 4 * L, "B"),
+        # Eq. 10: 4 L V d tensor FLOPs (logits once, dh once)
+        "weighted_ce_fwd_bwd": ("tensor", 4.0 * L * V * d, "FLOP"),
+        "lora_grad": ("hbm", lora_bytes, "B"),
+        # fp32 master + grad read, master written, bf16 copy written
+        "lora_step": ("hbm", 14 * step_elems, "B"),
+        # Algorithm 1 append: token in and one 32 B sector read + written per new n-gram
+        "history_insert": ("hbm", 4 * L + 64 * L, "B"),
+    }
+
+
+def row_report(wl, events, peaks):
+    out = {}
+    work = row_work(wl)
+    for name, evs in events.items():
+        ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+        kind, amount, _ = work[name]
+        if kind == "tensor":
+            ach = amount / (ms * 1e-3) / 1e12
+            out[name] = {"ms": round(ms, 4), "bound": "tensor", "achieved_tflops": round(ach, 1),
+                         "frac": round(ach / peaks["bf16_sustained"], 4), "flop": amount}
+        else:
+            ach = amount / (ms * 1e-3) / 1e9
+            out[name] = {"ms": round(ms, 4), "bound": "hbm", "achieved_gbs": round(ach, 1),
+                         "frac": round(ach / peaks["hbm_gbs"], 4), "bytes": int(amount)}
+    return out
 
 
 def _sources_sha256() -> str:
@@ -242,6 +297,22 @@ class OracleSample:
                     "sample": desc + f", {dt:.1f} s"}
 
 
+def max_over_ranks(vals, pg, device):
+    """Element-wise max of `vals` over the ranks of process group module `pg`
+    (the slowest rank decides each timing)."""
+    import torch
+    t = torch.tensor([float(v) for v in vals], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return t.tolist()
+
+
+def replica_throughput(tokens_per_step, steps, world_size, t_ms):
+    """Whole-job update tokens/s of `world_size` independent replicas that each
+    ran `steps` updates of `tokens_per_step` tokens within t_ms (the max over
+    ranks)."""
+    return tokens_per_step * steps * world_size / (t_ms * 1e-3)
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -297,8 +368,8 @@ def run_gpu(args):
             pg.barrier()
 
     # ---------------- device-timed region ----------------
-    ce_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-             for _ in range(args.steps)]
+    events = {name: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                     for _ in range(args.steps)] for name in Update.ROWS}
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
     clocks.start()
@@ -307,14 +378,15 @@ def run_gpu(args):
     n0 = attt.attt_kernel_launches()
     e0.record()
     for i in range(args.steps):
-        u.step(ce_ev[i])
+        u.step({k: v[i] for k, v in events.items()})
     e1.record()
     torch.cuda.synchronize()
     n1 = attt.attt_kernel_launches()
     barrier()
     clk = clocks.stop()
     t_ms = e0.elapsed_time(e1)
-    t_ce = statistics.mean(a.elapsed_time(b) for a, b in ce_ev)
+    rows = row_report(wl, events, peaks)
+    t_ce = rows["weighted_ce_fwd_bwd"]["ms"]
     if attt.attt_device_status() != 0 or attt.attt_history_status(u.hist) != 0:
         raise RuntimeError("device status error in the timed region")
 
@@ -347,13 +419,10 @@ def run_gpu(args):
     t_e2e = f0.elapsed_time(f1)
 
     if pg is not None:
-        tt = torch.tensor([t_ms, t_e2e], device=dev)
-        pg.all_reduce(tt, op=pg.ReduceOp.MAX)
-        t_ms, t_e2e = tt.tolist()
+        t_ms, t_e2e = max_over_ranks([t_ms, t_e2e], pg, dev)
 
-    tokens = wl.L * args.steps * ws
-    value = tokens / (t_ms * 1e-3)
-    e2e_value = tokens / (t_e2e * 1e-3)
+    value = replica_throughput(wl.L, args.steps, ws, t_ms)
+    e2e_value = replica_throughput(wl.L, args.steps, ws, t_e2e)
     out = None
     if rank == 0:
         traffic = _stored_traffic(wl)
@@ -374,6 +443,7 @@ def run_gpu(args):
             "gpu_launches": int(n1 - n0),
             "roofline": _ce_roofline(wl, t_ce, peaks, traffic),
             "ce_ms_per_call": round(t_ce, 4),
+            "rows": rows,
             "clocks": clk,
             "cpu_baseline": cpu,
         }
@@ -385,6 +455,69 @@ def run_gpu(args):
 
 
 # ---------------------------------------------------------------------------
+# the n-gram stress workload: 8,192 update tokens against a 1,048,576-token
+# history, n in {3, 4, 5}, repeated-span fraction in {0, 30, 60, 90}%
+# ---------------------------------------------------------------------------
+
+def run_stress(args):
+    import torch
+    from paper_2607_03441_gb300 import attt
+    from paper_2607_03441_gb300 import build
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peaks = _peaks()
+    reps = max(3, args.steps)
+    out = {"metric": "n-gram history insert and Eq. 8/9 weights, GB/s of algorithmic bytes vs HBM",
+           "workload": "stress: 8,192 update tokens vs a 1,048,576-token history, Zipf(1.1) over 128,256",
+           "hbm_peak_gbs": peaks["hbm_gbs"], "reps": reps, "cases": []}
+    for n in (3, 4, 5):
+        H, _ = wk.stress_case(n, 0.0)
+        Hd = torch.from_numpy(H).to(dev)
+        h = attt.attt_history_create(n, len(H))
+        ins_ms = []
+        for _ in range(args.warmup + reps):
+            attt.attt_history_reset(h)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            attt.attt_history_insert(h, Hd)
+            e1.record()
+            torch.cuda.synchronize()
+            ins_ms.append(e0.elapsed_time(e1))
+        if attt.attt_history_status(h) != 0:
+            raise RuntimeError("history status error")
+        ins_ms = statistics.median(ins_ms[args.warmup:])
+        ins_bytes = 4 * len(H) + 64 * (len(H) - n + 1)
+        case = {"n": n, "insert": {"tokens": len(H), "ms": round(ins_ms, 4), "bytes": ins_bytes,
+                                   "achieved_gbs": round(ins_bytes / ins_ms / 1e6, 1),
+                                   "frac": round(ins_bytes / ins_ms / 1e6 / peaks["hbm_gbs"], 4)},
+                "weights": []}
+        for frac in (0.0, 0.3, 0.6, 0.9):
+            _, x = wk.stress_case(n, frac)
+            xd = torch.from_numpy(x).to(dev)
+            w = torch.empty(len(x), dtype=torch.float32, device=dev)
+            for _ in range(args.warmup):
+                attt.attt_ngram_weights(h, xd, 0.05, out=w)
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(reps):
+                attt.attt_ngram_weights(h, xd, 0.05, out=w)
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1) / reps
+            wb = 4 * len(x) + 32 * (len(x) - n + 1) + 4 * len(x)
+            case["weights"].append({"frac": frac, "tokens": len(x), "ms": round(ms, 5), "bytes": wb,
+                                    "achieved_gbs": round(wb / ms / 1e6, 1),
+                                    "frac_of_hbm": round(wb / ms / 1e6 / peaks["hbm_gbs"], 4),
+                                    "tokens_per_s": round(len(x) / (ms * 1e-3), 1)})
+        h.close()
+        out["cases"].append(case)
+    return out
+
+
+# ---------------------------------------------------------------------------
 # the reference arm: the CPU oracle on the host cores
 # ---------------------------------------------------------------------------
 
@@ -392,7 +525,7 @@ def run_reference(args):
     ws, rank, _ = _dist()
     if rank != 0:
         return None
-    wl = wk.WORKLOADS[args.workload]
+    wl = wk.WORKLOADS[args.workload if args.workload != "stress" else WORKLOAD]
     sample = OracleSample(wl)
     for _ in range(args.warmup):
         sample.run(1)
@@ -418,7 +551,8 @@ def main():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["attt", "reference"], default="attt")
-    ap.add_argument("--workload", default=WORKLOAD, choices=["tiny", "7b"])
+    ap.add_argument("--workload", default=WORKLOAD, choices=["tiny", "7b", "stress"],
+                    help="'stress' times the n-gram insert and weights on the 1M-token history")
     ap.add_argument("--part", default="all", choices=["all", "ce", "lora", "ngram"],
                     help="time one stage alone (profiling aid); 'all' is the benchmark")
     ap.add_argument("--cpu-rows", type=int, default=64, help="rows of the oracle CPU-baseline sample (0: skip)")
@@ -426,7 +560,12 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
-    out = run_reference(args) if args.impl == "reference" else run_gpu(args)
+    if args.impl == "reference":
+        out = run_reference(args)
+    elif args.workload == "stress":
+        out = run_stress(args)
+    else:
+        out = run_gpu(args)
     if out is not None:
         print(json.dumps(out), flush=True)
 
