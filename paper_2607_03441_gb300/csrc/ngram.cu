@@ -4,14 +4,15 @@
 //
 // Table design (GB300-first):
 //   * open addressing, linear probing, power-of-two capacity >= 2 * max_tokens
-//     (load factor <= 1/2); one 16-byte slot = {key, count, unused}, so a
-//     probe touches exactly one 32-byte sector;
-//   * key = (32-bit hash tag << 32) | (history position + 1) of the n-gram's
-//     first occurrence, claimed with one 64-bit CAS; equality is decided by
-//     comparing the n tokens in the device-resident history stream (exact,
-//     any vocabulary, any n up to 16) after a tag match;
-//   * insertion aggregates equal n-grams inside a warp (match_any on the hash,
-//     ballot on token equality) so that hot keys cost one atomic per warp;
+//     (load factor <= 1/2) of 8-byte slots, one 64-bit word each:
+//       [63:48] 16-bit hash tag | [47:24] history position + 1 of the
+//       n-gram's first occurrence | [23:0] count
+//     (0 = empty).  A new n-gram costs one CAS that claims the slot with its
+//     count already set; a repeat costs one atomic add on the same word.  The
+//     history is therefore limited to 2^24 - 2 tokens (count and position fit
+//     24 bits).  Equality is decided by comparing the n tokens in the
+//     device-resident history stream (exact, any vocabulary, any n up to 16)
+//     after a tag match;
 //   * the weights kernel stages the update's tokens for a block in shared
 //     memory with coalesced loads, probes once per n-gram, takes the window
 //     max of the counts from shared memory and applies Eq. 9 with an IEEE
@@ -25,13 +26,14 @@
 
 namespace attt {
 
-struct __align__(16) Slot {
-    unsigned long long key;  // 0 = empty
-    unsigned int count;
-    unsigned int unused;
-};
+typedef unsigned long long Slot;  // tag16 | pos24 | count24, 0 = empty
 
 constexpr int kMaxN = 16;
+constexpr int64_t kMaxHistory = (1ll << 24) - 2;
+
+__device__ __forceinline__ unsigned int slot_tag(unsigned long long hsh) { return (unsigned int)(hsh >> 48); }
+__device__ __forceinline__ unsigned int slot_pos(Slot k) { return (unsigned int)((k >> 24) & 0xFFFFFFu) - 1u; }
+__device__ __forceinline__ unsigned int slot_count(Slot k) { return (unsigned int)(k & 0xFFFFFFu); }
 constexpr int kMaxProbe = 1 << 16;
 
 __device__ __forceinline__ unsigned long long mix64(unsigned long long h) {
@@ -61,61 +63,40 @@ __device__ __forceinline__ bool ngram_equal(const int32_t *a, const int32_t *b, 
 __device__ __forceinline__ unsigned int table_lookup(const Slot *table, unsigned long long mask,
                                                      const int32_t *hist, const int32_t *g, int n,
                                                      unsigned long long hsh) {
-    const unsigned int tag = (unsigned int)(hsh >> 32);
+    const unsigned int tag = slot_tag(hsh);
     unsigned long long idx = hsh & mask;
     for (int probe = 0; probe < kMaxProbe; ++probe) {
-        const uint4 s = __ldcg(reinterpret_cast<const uint4 *>(table + idx));
-        const unsigned long long key = ((unsigned long long)s.y << 32) | s.x;
-        if (key == 0ull) return 0u;
-        if ((unsigned int)(key >> 32) == tag) {
-            const unsigned int pos = (unsigned int)key - 1u;
-            if (ngram_equal(hist + pos, g, n)) return s.z;
-        }
+        const Slot k = __ldcg(table + idx);
+        if (k == 0ull) return 0u;
+        if ((unsigned int)(k >> 48) == tag && ngram_equal(hist + slot_pos(k), g, n)) return slot_count(k);
         idx = (idx + 1) & mask;
     }
     return 0u;
 }
 
 // One thread per new n-gram start position p in [p_begin, p_begin + count).
+// (Aggregating equal n-grams inside a warp with match_any was measured to
+// cost more than the atomics it saves on Zipf text, so every thread inserts
+// its own occurrence.)
 __global__ void __launch_bounds__(256) history_insert_kernel(const int32_t *__restrict__ hist, int64_t p_begin,
                                                              int64_t count, int n, Slot *table,
                                                              unsigned long long mask, int *status) {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const bool active = i < count;
-    const unsigned amask = __ballot_sync(0xffffffffu, active);
-    if (!active) return;
-    const int lane = threadIdx.x & 31;
+    if (i >= count) return;
     const int64_t p = p_begin + i;
     const int32_t *g = hist + p;
     const unsigned long long hsh = ngram_hash(g, n);
-
-    // Warp aggregation of equal n-grams (hot keys under Zipf text).
-    const unsigned peers = __match_any_sync(amask, hsh);
-    const int leader = __ffs(peers) - 1;
-    const int64_t pl = __shfl_sync(peers, p, leader);
-    const bool same = (lane == leader) || ngram_equal(hist + pl, g, n);
-    const unsigned same_mask = __ballot_sync(peers, same);
-    unsigned int add;
-    if (lane == leader) add = __popc(same_mask);
-    else if (!same) add = 1u;  // 64-bit hash collision between different n-grams
-    else return;
-
-    const unsigned int tag = (unsigned int)(hsh >> 32);
-    const unsigned long long mykey = ((unsigned long long)tag << 32) | (unsigned long long)(uint32_t)(p + 1);
+    const unsigned int tag = slot_tag(hsh);
+    const Slot claim = ((unsigned long long)tag << 48) | ((unsigned long long)(uint32_t)(p + 1) << 24) | 1ull;
     unsigned long long idx = hsh & mask;
     for (int probe = 0; probe < kMaxProbe; ++probe) {
         Slot *s = table + idx;
-        unsigned long long k = *reinterpret_cast<volatile unsigned long long *>(&s->key);
-        if (k == 0ull) {
-            const unsigned long long old = atomicCAS(&s->key, 0ull, mykey);
-            if (old == 0ull) {
-                atomicAdd(&s->count, add);
-                return;
-            }
-            k = old;
-        }
-        if ((unsigned int)(k >> 32) == tag && ngram_equal(hist + ((unsigned int)k - 1u), g, n)) {
-            atomicAdd(&s->count, add);
+        // Optimistic claim: one round trip for a new n-gram; an occupied slot
+        // returns its word, which is then compared.
+        const Slot k = atomicCAS(s, 0ull, claim);
+        if (k == 0ull) return;  // claimed with count 1
+        if ((unsigned int)(k >> 48) == tag && ngram_equal(hist + slot_pos(k), g, n)) {
+            atomicAdd(s, 1ull);  // count lives in the low 24 bits
             return;
         }
         idx = (idx + 1) & mask;
@@ -191,7 +172,7 @@ struct attt_history {
 extern "C" {
 
 attt_status attt_history_create(int n, int64_t max_tokens, attt_history **out) {
-    if (!out || n < 1 || n > attt::kMaxN || max_tokens < 0 || max_tokens > ((int64_t)1 << 31) - 2)
+    if (!out || n < 1 || n > attt::kMaxN || max_tokens < 0 || max_tokens > attt::kMaxHistory)
         return ATTT_ERR_INVALID_ARG;
     *out = nullptr;
     int dev;
