@@ -35,6 +35,11 @@ __device__ __forceinline__ void record_error(int *status, int code) {
     if (status) atomicCAS(status, 0, code);
 }
 
+// bar.sync on a named barrier shared by `count` threads (a multiple of 32).
+__device__ __forceinline__ void named_barrier_sync(uint32_t id, uint32_t count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // bar.red.and over a named barrier: 1 iff every participating thread passed
 // a non-zero predicate.
 __device__ __forceinline__ int named_barrier_and(uint32_t id, uint32_t count, int pred) {

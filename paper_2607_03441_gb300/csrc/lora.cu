@@ -10,8 +10,12 @@
 // Every contraction puts the long dimension (L, din or dout) on the 128-row
 // MMA side and the rank on N, so the tensor core streams x and dy once per
 // pass at HBM rate.  Reductions over L (or din/dout) are split across CTAs
-// and merged with fp32 atomics; u and v are rounded to bf16 in between.
+// and merged with fp32 atomics; u and v are rounded to bf16 in between (by
+// the split that finishes each tile last).  Three launches per call: prep
+// (adapters to K-major, every accumulator zeroed), pass 1 (u and every v_p,
+// grouped), pass 2 (dA and every dB_p, grouped).
 #include "gemm_launch.cuh"
+#include "tc_group.cuh"
 
 namespace attt {
 
@@ -22,6 +26,8 @@ struct LoraLayout {
     __nv_bfloat16 *BT[kMaxProj];  // [rpad, dout_p]
     float *uT32, *vT32;           // [Nu, Lp] each, contiguous
     __nv_bfloat16 *uT16, *vT16;   // [Nu, Lp] each, contiguous
+    unsigned int *tickets;        // pass-1 tile counters, (1 + nproj) x ntick
+    int64_t ntick;
     size_t bytes;
 };
 
@@ -37,6 +43,8 @@ static LoraLayout lora_layout(void *ws, int64_t L, int64_t din, int nproj, const
     c.vT32 = c.uT32 + (size_t)c.Nu * c.Lp;
     c.uT16 = cv.take<__nv_bfloat16>((size_t)(2 * c.Nu * c.Lp));
     c.vT16 = c.uT16 + (size_t)c.Nu * c.Lp;
+    c.ntick = cdiv(L, 128) * cdiv(c.Nu, 256);
+    c.tickets = cv.take<unsigned int>((size_t)((1 + nproj) * c.ntick));
     c.bytes = (size_t)round_up((int64_t)cv.used, 256);
     return c;
 }
@@ -45,19 +53,34 @@ struct PrepArgs {
     const __nv_bfloat16 *A[kMaxProj];
     const __nv_bfloat16 *B[kMaxProj];
     __nv_bfloat16 *BT[kMaxProj];
+    float *dA[kMaxProj];
+    float *dB[kMaxProj];
     int64_t dout[kMaxProj];
     int nproj, r, rpad;
     int64_t din;
     __nv_bfloat16 *AT;
+    float *acc;           // uT32 and vT32, contiguous
+    int64_t nacc;
+    unsigned int *tickets;
+    int64_t ntickets;
 };
 
 // AT[p*rpad + c, i] = A_p[i, c] (zero for c >= r); BT_p[c, o] = B_p[c, o]
-// (zero rows for c >= r).
+// (zero rows for c >= r); and every accumulator of the call set to zero
+// (u^T, v^T, dA_p, dB_p and the tile tickets), block row p of the grid doing
+// projection p's share.
 __global__ void lora_prep_kernel(PrepArgs a) {
     const int p = blockIdx.y;
     const int64_t nA = (int64_t)a.rpad * a.din;
     const int64_t nB = (int64_t)a.rpad * a.dout[p];
-    const int64_t n = nA > nB ? nA : nB;
+    const int64_t ndA = a.din * a.r, ndB = (int64_t)a.r * a.dout[p];
+    const int64_t zacc = (a.nacc + a.nproj - 1) / a.nproj;   // this row's slice of the u/v accumulators
+    const int64_t ztk = (a.ntickets + a.nproj - 1) / a.nproj;
+    int64_t n = nA > nB ? nA : nB;
+    if (ndA > n) n = ndA;
+    if (ndB > n) n = ndB;
+    if (zacc > n) n = zacc;
+    if (ztk > n) n = ztk;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         if (i < nA) {
             const int c = (int)(i / a.din);
@@ -69,12 +92,11 @@ __global__ void lora_prep_kernel(PrepArgs a) {
             const int c = (int)(i / a.dout[p]);
             a.BT[p][i] = c < a.r ? a.B[p][i] : __float2bfloat16_rn(0.f);
         }
+        if (i < ndA) a.dA[p][i] = 0.f;
+        if (i < ndB) a.dB[p][i] = 0.f;
+        if (i < zacc && p * zacc + i < a.nacc) a.acc[p * zacc + i] = 0.f;
+        if (i < ztk && p * ztk + i < a.ntickets) a.tickets[p * ztk + i] = 0u;
     }
-}
-
-__global__ void f32_to_bf16_kernel(const float *__restrict__ in, __nv_bfloat16 *__restrict__ out, int64_t n) {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
-        out[i] = __float2bfloat16_rn(in[i]);
 }
 
 // SGD: p <- p - lr * g (product then difference, both rounded), bf16 refresh.
@@ -103,6 +125,79 @@ static unsigned grid_for(int64_t n, int threads, int dev) {
     return (unsigned)b;
 }
 
+// One problem of a grouped launch (see tc_group.cuh).
+struct GroupSpec {
+    const void *a;
+    int64_t a_rows_ld, a_rows, a_k;  // as GemmProblem
+    const void *b;
+    int64_t b_rows_ld, b_rows, b_k;
+    int M, N, K;
+    int b_n_off;
+    int epi;
+    EpiParams ep;
+};
+
+// Launches every problem of `specs` in one grouped kernel.  K is split per
+// problem so that each CTA streams about the same number of K blocks.
+template <bool A_MN, bool B_MN>
+static attt_status launch_group(const GroupSpec *specs, int n, int BN, int dev, cudaStream_t stream, int *status) {
+    if (n < 1 || n > kMaxGroup || BN < 16 || BN > 256 || BN % 16 != 0) return ATTT_ERR_INVALID_ARG;
+    static_assert(!B_MN, "grouped B operands are K-major");
+    GroupMaps maps;
+    GroupArgs g{};
+    g.nprob = n;
+    g.BN = BN;
+    g.stages = gemm_stages(BN);
+    g.tmem_cols = gemm_tmem_cols(BN);
+    g.status = status ? status : device_status_word(dev);
+    const int sms = num_sms(dev);
+    int64_t work = 0;  // tile x K-block units of the whole group
+    for (int q = 0; q < n; ++q) {
+        const GroupSpec &sp = specs[q];
+        work += cdiv(sp.M, 128) * cdiv(sp.N, BN) * cdiv(sp.K, 64);
+    }
+    const int64_t per_cta = cdiv(work, sms) > 0 ? cdiv(work, sms) : 1;
+    int tiles = 0;
+    for (int q = 0; q < n; ++q) {
+        const GroupSpec &sp = specs[q];
+        if (sp.M <= 0 || sp.N <= 0 || sp.K <= 0) return ATTT_ERR_INVALID_ARG;
+        bool ok;
+        if (!A_MN)
+            ok = make_tmap_bf16(&maps.a[q], sp.a, (uint64_t)sp.a_k, (uint64_t)sp.a_rows, (uint64_t)sp.a_rows_ld * 2,
+                                64, 128);
+        else
+            ok = make_tmap_bf16(&maps.a[q], sp.a, (uint64_t)sp.a_rows, (uint64_t)sp.a_k, (uint64_t)sp.a_rows_ld * 2,
+                                64, 64);
+        if (!ok) return ATTT_ERR_INVALID_ARG;
+        if (!make_tmap_bf16(&maps.b[q], sp.b, (uint64_t)sp.b_k, (uint64_t)sp.b_rows, (uint64_t)sp.b_rows_ld * 2, 64,
+                            (uint32_t)BN))
+            return ATTT_ERR_INVALID_ARG;
+        GroupProblem &pr = g.prob[q];
+        pr.M = sp.M;
+        pr.N = sp.N;
+        pr.tiles_m = (int)cdiv(sp.M, 128);
+        pr.tiles_n = (int)cdiv(sp.N, BN);
+        pr.kb_total = (int)cdiv(sp.K, 64);
+        int splits = (int)cdiv(pr.kb_total, per_cta);
+        if (splits < 1) splits = 1;
+        pr.kb_per_split = (int)cdiv(pr.kb_total, splits);
+        pr.splits = (int)cdiv(pr.kb_total, pr.kb_per_split);
+        pr.b_n_off = sp.b_n_off;
+        pr.tile_begin = tiles;
+        pr.epi = sp.epi;
+        pr.ep = sp.ep;
+        tiles += pr.tiles_m * pr.tiles_n * pr.splits;
+    }
+    g.total_tiles = tiles;
+    const size_t smem = gemm_smem_bytes(BN, g.stages);
+    auto kern = tc_gemm_group_kernel<A_MN, B_MN>;
+    if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
+    const int grid = tiles < sms ? tiles : sms;
+    kern<<<grid, kGemmThreads, smem, stream>>>(maps, g);
+    count_launch();
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
 attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int nproj, const attt_bf16 *const *d_dy,
                           const int64_t *dout, const attt_bf16 *const *d_A, const attt_bf16 *const *d_B, int r,
                           float scale, float *const *d_dA, float *const *d_dB, void *d_ws, size_t ws_bytes,
@@ -124,9 +219,9 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
     if (st != ATTT_OK) return st;
 
     LoraLayout c = lora_layout(d_ws, L, din, nproj, dout, r);
-    const int BNu = c.Nu <= 256 ? c.Nu : 256;
+    const int BN = c.Nu <= 256 ? c.Nu : 256;
 
-    // adapters in K-major, rank padded to a multiple of 16 with zeros
+    // prep: adapters to K-major (rank padded with zeros), accumulators zeroed
     {
         PrepArgs a{};
         int64_t maxn = c.rpad * din;
@@ -134,74 +229,68 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
             a.A[p] = reinterpret_cast<const __nv_bfloat16 *>(d_A[p]);
             a.B[p] = reinterpret_cast<const __nv_bfloat16 *>(d_B[p]);
             a.BT[p] = c.BT[p];
+            a.dA[p] = d_dA[p];
+            a.dB[p] = d_dB[p];
             a.dout[p] = dout[p];
             if (c.rpad * dout[p] > maxn) maxn = c.rpad * dout[p];
         }
         a.nproj = nproj; a.r = r; a.rpad = c.rpad; a.din = din; a.AT = c.AT;
+        a.acc = c.uT32; a.nacc = (int64_t)2 * c.Nu * c.Lp;
+        a.tickets = c.tickets; a.ntickets = (1 + nproj) * c.ntick;
+        if (a.nacc / nproj > maxn) maxn = a.nacc / nproj + 1;
         dim3 grid(grid_for(maxn, 256, dev), nproj);
         lora_prep_kernel<<<grid, 256, 0, stream>>>(a);
         count_launch();
         if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
     }
-    if (cudaMemsetAsync(c.uT32, 0, (size_t)2 * c.Nu * c.Lp * sizeof(float), stream) != cudaSuccess)
-        return ATTT_ERR_CUDA;
-    for (int p = 0; p < nproj; ++p) {
-        if (cudaMemsetAsync(d_dA[p], 0, (size_t)din * r * sizeof(float), stream) != cudaSuccess ||
-            cudaMemsetAsync(d_dB[p], 0, (size_t)r * dout[p] * sizeof(float), stream) != cudaSuccess)
-            return ATTT_ERR_CUDA;
+
+    // pass 1: u^T = (x AT^T)^T and v_p^T = (dy_p BT_p^T)^T, fp32 sums then bf16
+    {
+        GroupSpec sp[kMaxGroup];
+        int n = 0;
+        GroupSpec &u = sp[n++];
+        u = GroupSpec{};
+        u.a = d_x; u.a_rows_ld = din; u.a_rows = L; u.a_k = din;
+        u.b = c.AT; u.b_rows_ld = din; u.b_rows = c.Nu; u.b_k = din;
+        u.M = (int)L; u.N = c.Nu; u.K = (int)din; u.epi = EPI_ATOMIC_T;
+        u.ep.out = c.uT32; u.ep.out_ld = c.Lp; u.ep.alpha = 1.0f; u.ep.r = c.rpad; u.ep.rpad = c.rpad;
+        u.ep.out16 = c.uT16; u.ep.tickets = c.tickets;
+        for (int q = 0; q < nproj; ++q) {
+            GroupSpec &v = sp[n++];
+            v = GroupSpec{};
+            v.a = d_dy[q]; v.a_rows_ld = dout[q]; v.a_rows = L; v.a_k = dout[q];
+            v.b = c.BT[q]; v.b_rows_ld = dout[q]; v.b_rows = c.rpad; v.b_k = dout[q];
+            v.M = (int)L; v.N = c.rpad; v.K = (int)dout[q]; v.epi = EPI_ATOMIC_T;
+            v.ep.out = c.vT32 + (size_t)q * c.rpad * c.Lp; v.ep.out_ld = c.Lp; v.ep.alpha = 1.0f;
+            v.ep.r = c.rpad; v.ep.rpad = c.rpad;
+            v.ep.out16 = c.vT16 + (size_t)q * c.rpad * c.Lp; v.ep.tickets = c.tickets + (1 + q) * c.ntick;
+        }
+        st = launch_group<false, false>(sp, n, BN, dev, stream, status);
+        if (st != ATTT_OK) return st;
     }
 
-    // pass 1a: u^T = (x AT^T)^T for every projection at once
+    // pass 2: dA_p = s x^T v_p (all p at once, x MN-major) and
+    //         dB_p^T = s dy_p^T u_p (dy MN-major), stored transposed into dB_p
     {
-        GemmProblem p{};
-        p.a = d_x; p.a_rows_ld = din; p.a_rows = L; p.a_k = din;
-        p.b = c.AT; p.b_rows_ld = din; p.b_rows = c.Nu; p.b_k = din;
-        p.M = (int)L; p.N = c.Nu; p.K = (int)din; p.BN = BNu; p.allow_split = true;
-        EpiParams ep{};
-        ep.out = c.uT32; ep.out_ld = c.Lp; ep.alpha = 1.0f; ep.r = c.rpad; ep.rpad = c.rpad;
-        st = launch_gemm<EPI_ATOMIC_T, false, false>(p, ep, dev, stream, status);
-        if (st != ATTT_OK) return st;
-    }
-    // pass 1b: v_p^T = (dy_p B_p^T)^T
-    for (int q = 0; q < nproj; ++q) {
-        GemmProblem p{};
-        p.a = d_dy[q]; p.a_rows_ld = dout[q]; p.a_rows = L; p.a_k = dout[q];
-        p.b = c.BT[q]; p.b_rows_ld = dout[q]; p.b_rows = c.rpad; p.b_k = dout[q];
-        p.M = (int)L; p.N = c.rpad; p.K = (int)dout[q]; p.BN = c.rpad; p.allow_split = true;
-        EpiParams ep{};
-        ep.out = c.vT32 + (size_t)q * c.rpad * c.Lp; ep.out_ld = c.Lp; ep.alpha = 1.0f;
-        ep.r = c.rpad; ep.rpad = c.rpad;
-        st = launch_gemm<EPI_ATOMIC_T, false, false>(p, ep, dev, stream, status);
-        if (st != ATTT_OK) return st;
-    }
-    {
-        const int64_t n = (int64_t)2 * c.Nu * c.Lp;
-        f32_to_bf16_kernel<<<grid_for(n, 256, dev), 256, 0, stream>>>(c.uT32, c.uT16, n);
-        count_launch();
-        if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
-    }
-    // pass 2a: dA_p = s x^T v_p for every projection at once (x MN-major)
-    {
-        GemmProblem p{};
-        p.a = d_x; p.a_rows_ld = din; p.a_rows = din; p.a_k = L;
-        p.b = c.vT16; p.b_rows_ld = c.Lp; p.b_rows = c.Nu; p.b_k = c.Lp;
-        p.M = (int)din; p.N = c.Nu; p.K = (int)L; p.BN = BNu; p.allow_split = true;
-        EpiParams ep{};
-        for (int q = 0; q < nproj; ++q) ep.outp[q] = d_dA[q];
-        ep.alpha = scale; ep.r = r; ep.rpad = c.rpad;
-        st = launch_gemm<EPI_ATOMIC_N, true, false>(p, ep, dev, stream, status);
-        if (st != ATTT_OK) return st;
-    }
-    // pass 2b: dB_p^T = s dy_p^T u_p (dy MN-major), stored transposed into dB_p
-    for (int q = 0; q < nproj; ++q) {
-        GemmProblem p{};
-        p.a = d_dy[q]; p.a_rows_ld = dout[q]; p.a_rows = dout[q]; p.a_k = L;
-        p.b = c.uT16; p.b_rows_ld = c.Lp; p.b_rows = c.Nu; p.b_k = c.Lp;
-        p.b_n_off = q * c.rpad;
-        p.M = (int)dout[q]; p.N = c.rpad; p.K = (int)L; p.BN = c.rpad; p.allow_split = true;
-        EpiParams ep{};
-        ep.out = d_dB[q]; ep.out_ld = dout[q]; ep.alpha = scale; ep.r = r; ep.rpad = c.rpad;
-        st = launch_gemm<EPI_ATOMIC_T, true, false>(p, ep, dev, stream, status);
+        GroupSpec sp[kMaxGroup];
+        int n = 0;
+        GroupSpec &a = sp[n++];
+        a = GroupSpec{};
+        a.a = d_x; a.a_rows_ld = din; a.a_rows = din; a.a_k = L;
+        a.b = c.vT16; a.b_rows_ld = c.Lp; a.b_rows = c.Nu; a.b_k = L;  // padding columns read as zeros
+        a.M = (int)din; a.N = c.Nu; a.K = (int)L; a.epi = EPI_ATOMIC_N;
+        for (int q = 0; q < nproj; ++q) a.ep.outp[q] = d_dA[q];
+        a.ep.alpha = scale; a.ep.r = r; a.ep.rpad = c.rpad;
+        for (int q = 0; q < nproj; ++q) {
+            GroupSpec &b = sp[n++];
+            b = GroupSpec{};
+            b.a = d_dy[q]; b.a_rows_ld = dout[q]; b.a_rows = dout[q]; b.a_k = L;
+            b.b = c.uT16; b.b_rows_ld = c.Lp; b.b_rows = c.Nu; b.b_k = L;
+            b.b_n_off = q * c.rpad;
+            b.M = (int)dout[q]; b.N = c.rpad; b.K = (int)L; b.epi = EPI_ATOMIC_T;
+            b.ep.out = d_dB[q]; b.ep.out_ld = dout[q]; b.ep.alpha = scale; b.ep.r = r; b.ep.rpad = c.rpad;
+        }
+        st = launch_group<true, false>(sp, n, BN, dev, stream, status);
         if (st != ATTT_OK) return st;
     }
     return ATTT_OK;

@@ -50,6 +50,8 @@ struct EpiParams {
     float alpha;
     const float *row_alpha;  // [M] or nullptr (1)
     const float *row_beta;   // [M] or nullptr (1)
+    __nv_bfloat16 *out16;    // grouped EPI_ATOMIC_T: bf16 copy of out, written by the last split
+    unsigned int *tickets;   // grouped EPI_ATOMIC_T: one counter per tile, starts at 0
     float *outp[kMaxProj];
     int r;     // valid columns per projection block
     int rpad;  // column block width per projection
