@@ -110,7 +110,9 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 
 class Update:
-    """Device-resident state of the 7B-class update and one step of it."""
+    """Device-resident state of one aTTT update of a workload and one step of
+    it.  Projections that share an input x (q/k/v; gate/up) form one group
+    and one attt_lora_grad call."""
 
     def __init__(self, wl, dev, max_steps):
         import torch
@@ -119,21 +121,30 @@ class Update:
         self.torch = torch
         self.wl = wl
         self.dev = dev
-        H = wk.history_tokens(wl)
-        self.x_host = wk.update_tokens(wl, H)
+        if wl.hist_len:
+            H = wk.history_tokens(wl)
+            self.x_host = wk.update_tokens(wl, H)
+        else:  # long episode: the last update against the 31 before it
+            ups = wk.long_episode_updates(wl)
+            H = np.concatenate(ups[:-1])
+            self.x_host = ups[-1]
         dense = wk.dense_inputs(wl)
         self.dense = dense
 
         def bf(a):
             return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
 
-        self.hist = attt.attt_history_create(wl.n, wl.hist_len + wl.L * max_steps)
+        self.H0 = H
+        self.hist = attt.attt_history_create(wl.n, len(H) + wl.L * max_steps)
         attt.attt_history_insert(self.hist, torch.from_numpy(H).to(dev))
         self.x = torch.from_numpy(self.x_host).to(dev)
         self.h = bf(dense["h"])
         self.W = bf(dense["W"])
         self.projs = list(wl.projs)
-        self.xin = bf(dense[f"x/{self.projs[0].name}"])
+        self.groups = {}
+        for i, p in enumerate(self.projs):
+            self.groups.setdefault(p.x_group, []).append(i)
+        self.xin = {gname: bf(dense[f"x/{self.projs[idx[0]].name}"]) for gname, idx in self.groups.items()}
         self.dy = [bf(dense[f"dy/{p.name}"]) for p in self.projs]
         self.A32 = [torch.from_numpy(wk.bf16_to_f32(dense[f"A/{p.name}"])).to(dev) for p in self.projs]
         self.B32 = [torch.from_numpy(wk.bf16_to_f32(dense[f"B/{p.name}"])).to(dev) for p in self.projs]
@@ -146,9 +157,9 @@ class Update:
         self.loss = torch.empty(1, dtype=torch.float32, device=dev)
         self.dh = torch.empty(L, d, dtype=torch.float32, device=dev)
         self.ws_ce = torch.empty(attt.attt_ce_workspace_bytes(L, d, V), dtype=torch.uint8, device=dev)
-        self.ws_lora = torch.empty(attt.attt_lora_workspace_bytes(L, self.projs[0].din,
-                                                                   [p.dout for p in self.projs], r),
-                                   dtype=torch.uint8, device=dev)
+        ws = max(attt.attt_lora_workspace_bytes(L, self.projs[idx[0]].din, [self.projs[i].dout for i in idx], r)
+                 for idx in self.groups.values())
+        self.ws_lora = torch.empty(ws, dtype=torch.uint8, device=dev)  # groups run one after another
         self.stream = torch.cuda.current_stream()
 
     ROWS = ("ngram_weights", "weighted_ce_fwd_bwd", "lora_grad", "lora_step", "history_insert")
@@ -173,8 +184,10 @@ class Update:
             mark("weighted_ce_fwd_bwd", 1)
         if part in ("all", "lora"):
             mark("lora_grad", 0)
-            a.attt_lora_grad(self.xin, self.dy, self.A16, self.B16, self.wl.scale, dAs=self.dA, dBs=self.dB,
-                             workspace=self.ws_lora)
+            for gname, idx in self.groups.items():
+                a.attt_lora_grad(self.xin[gname], [self.dy[i] for i in idx], [self.A16[i] for i in idx],
+                                 [self.B16[i] for i in idx], self.wl.scale, dAs=[self.dA[i] for i in idx],
+                                 dBs=[self.dB[i] for i in idx], workspace=self.ws_lora)
             mark("lora_grad", 1)
             mark("lora_step", 0)
             for i in range(len(self.projs)):
@@ -192,11 +205,14 @@ def row_work(wl):
     Bytes count each input read once and each output written once; FLOPs
     count the contractions the method defines."""
     L, V, d, n, r = wl.L, wl.V, wl.d, wl.n, wl.r
-    din = wl.projs[0].din
-    douts = [p.dout for p in wl.projs]
-    lora_bytes = 2 * L * din + sum(2 * L * do for do in douts)               # x once, each dy once
-    lora_bytes += sum(2 * din * r + 2 * r * do + 4 * din * r + 4 * r * do for do in douts)  # A, B in; dA, dB out
-    step_elems = sum(din * r + r * do for do in douts)
+    groups = {}
+    for p in wl.projs:
+        groups.setdefault(p.x_group, []).append(p)
+    lora_bytes = 0
+    for ps in groups.values():
+        lora_bytes += 2 * L * ps[0].din + sum(2 * L * p.dout for p in ps)     # each distinct x once, each dy once
+        lora_bytes += sum(6 * p.din * r + 6 * r * p.dout for p in ps)         # A, B in (bf16); dA, dB out (fp32)
+    step_elems = sum(p.din * r + r * p.dout for p in wl.projs)
     return {
         # Eq. 8/9: tokens in, one 32 B table sector per probe, weights out
         "ngram_weights": ("hbm", 4 * L + 32 * max(L - n + 1, 0) + 4 * L, "B"),
@@ -283,10 +299,9 @@ class OracleSample:
         t0 = time.perf_counter()
         w = o.ngram_weights(self.H, self.x, wl.n, wl.w_min)
         o.ce_rows(dense["h"], dense["W"], self.x, w, sel)
-        xs = dense[f"x/{wl.projs[0].name}"][sel]
         for p in wl.projs:
-            dA, dB = o.lora_grad(xs, dense[f"dy/{p.name}"][sel], dense[f"A/{p.name}"], dense[f"B/{p.name}"],
-                                 wl.scale)
+            dA, dB = o.lora_grad(dense[f"x/{p.name}"][sel], dense[f"dy/{p.name}"][sel], dense[f"A/{p.name}"],
+                                 dense[f"B/{p.name}"], wl.scale)
             o.sgd_step(wk.bf16_to_f32(dense[f"A/{p.name}"]), dA.astype(np.float32), wk.LORA_LR)
             o.sgd_step(wk.bf16_to_f32(dense[f"B/{p.name}"]), dB.astype(np.float32), wk.LORA_LR)
         dt = time.perf_counter() - t0
@@ -394,12 +409,13 @@ def run_gpu(args):
     host_in = {
         "tokens": torch.from_numpy(u.x_host).pin_memory(),
         "h": torch.from_numpy(u.dense["h"].view(np.int16)).pin_memory(),
-        "x": torch.from_numpy(u.dense[f"x/{u.projs[0].name}"].view(np.int16)).pin_memory(),
     }
-    for p in u.projs:
-        host_in[f"dy/{p.name}"] = torch.from_numpy(u.dense[f"dy/{p.name}"].view(np.int16)).pin_memory()
-    dev_in = {"tokens": u.x, "h": u.h.view(torch.int16), "x": u.xin.view(torch.int16)}
+    dev_in = {"tokens": u.x, "h": u.h.view(torch.int16)}
+    for gname, idx in u.groups.items():
+        host_in[f"x/{gname}"] = torch.from_numpy(u.dense[f"x/{u.projs[idx[0]].name}"].view(np.int16)).pin_memory()
+        dev_in[f"x/{gname}"] = u.xin[gname].view(torch.int16)
     for i, p in enumerate(u.projs):
+        host_in[f"dy/{p.name}"] = torch.from_numpy(u.dense[f"dy/{p.name}"].view(np.int16)).pin_memory()
         dev_in[f"dy/{p.name}"] = u.dy[i].view(torch.int16)
     loss_host = torch.empty(1, dtype=torch.float32).pin_memory()
     h2d = sum(t.numel() * t.element_size() for t in host_in.values())
@@ -428,16 +444,17 @@ def run_gpu(args):
         traffic = _stored_traffic(wl)
         cpu = None
         if ws == 1 and args.cpu_rows > 0:
-            _, cpu = OracleSample(wl, dense=u.dense, x=u.x_host).run(args.cpu_rows)
+            _, cpu = OracleSample(wl, dense=u.dense, x=u.x_host, H=u.H0).run(args.cpu_rows)
         out = {
             "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(t_ms / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": (f"{wl.name}: one aTTT update, L={wl.L} tokens, V={wl.V}, d={wl.d}, n={wl.n}, "
-                                    f"history {wl.hist_len}+ tokens, LoRA r={wl.r} on q 3584x3584 and "
-                                    f"v 3584x512, one SGD step"),
+                                    f"history {len(u.H0)} tokens at the start (+L per step), LoRA r={wl.r} on " +
+                                    ", ".join(f"{p.name} {p.din}x{p.dout}" for p in wl.projs) +
+                                    ", one SGD step"),
                        "global_batch": wl.L * ws, "seq_len": wl.L, "parallelism": f"replicas{ws}",
-                       "l2": "inputs larger than L2 (LM head 1.09 GB streamed every step)"},
+                       "l2": f"inputs larger than L2 (LM head {2 * wl.V * wl.d / 1e9:.2f} GB streamed every step)"},
             "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "gpu_launches": int(n1 - n0),
@@ -551,7 +568,7 @@ def main():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["attt", "reference"], default="attt")
-    ap.add_argument("--workload", default=WORKLOAD, choices=["tiny", "7b", "stress"],
+    ap.add_argument("--workload", default=WORKLOAD, choices=["tiny", "7b", "long", "32b", "stress"],
                     help="'stress' times the n-gram insert and weights on the 1M-token history")
     ap.add_argument("--part", default="all", choices=["all", "ce", "lora", "ngram"],
                     help="time one stage alone (profiling aid); 'all' is the benchmark")

@@ -147,7 +147,18 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, int dev, 
     GroupArgs g{};
     g.nprob = n;
     g.BN = BN;
-    g.stages = gemm_stages(BN);
+    // Up to four 64-deep K blocks per stage, so each operand row is fetched in
+    // runs of up to 512 bytes (better DRAM locality than one 128-byte piece per
+    // row per block), as long as at least two stages fit in shared memory.
+    g.kbs = 1;
+    g.stages = 0;
+    for (int kbs = 4; kbs >= 1 && g.stages == 0; kbs /= 2) {
+        const size_t per_stage = (size_t)kbs * (kABytes + gemm_b_stage_bytes(BN));
+        int st = 8;
+        while (st >= 2 && 1024 + st * per_stage + 8 * (2 * st + 5) + 16 > kMaxSmem) --st;
+        if (st >= 2) { g.kbs = kbs; g.stages = st; }
+    }
+    if (g.stages == 0) return ATTT_ERR_UNSUPPORTED;
     g.tmem_cols = gemm_tmem_cols(BN);
     g.status = status ? status : device_status_word(dev);
     const int sms = num_sms(dev);
@@ -180,7 +191,7 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, int dev, 
         pr.kb_total = (int)cdiv(sp.K, 64);
         int splits = (int)cdiv(pr.kb_total, per_cta);
         if (splits < 1) splits = 1;
-        pr.kb_per_split = (int)cdiv(pr.kb_total, splits);
+        pr.kb_per_split = (int)round_up(cdiv(pr.kb_total, splits), g.kbs);  // whole stages per split
         pr.splits = (int)cdiv(pr.kb_total, pr.kb_per_split);
         pr.b_n_off = sp.b_n_off;
         pr.tile_begin = tiles;
@@ -189,7 +200,8 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, int dev, 
         tiles += pr.tiles_m * pr.tiles_n * pr.splits;
     }
     g.total_tiles = tiles;
-    const size_t smem = gemm_smem_bytes(BN, g.stages);
+    const size_t smem =
+        1024 + (size_t)g.stages * g.kbs * (kABytes + gemm_b_stage_bytes(BN)) + 8 * (2 * g.stages + 5) + 16;
     auto kern = tc_gemm_group_kernel<A_MN, B_MN>;
     if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
     const int grid = tiles < sms ? tiles : sms;

@@ -34,6 +34,7 @@ struct GroupMaps {
 struct GroupArgs {
     int nprob, total_tiles;
     int BN, stages;
+    int kbs;  // 64-deep K blocks per pipeline stage (each row is fetched in kbs x 128 B runs)
     uint32_t tmem_cols;
     int *status;
     GroupProblem prob[kMaxGroup];
@@ -100,9 +101,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = g.stages;
-    const uint32_t b_bytes = gemm_b_stage_bytes(g.BN);
+    const int KBS = g.kbs;
+    const uint32_t a1 = kABytes, b1 = gemm_b_stage_bytes(g.BN);  // one K block
+    const uint32_t kABytesS = a1 * KBS;
+    const uint32_t b_bytes = b1 * KBS;
     uint8_t *sA = smem;
-    uint8_t *sB = smem + (size_t)S * kABytes;
+    uint8_t *sB = smem + (size_t)S * kABytesS;
     uint64_t *bars = reinterpret_cast<uint64_t *>(sB + (size_t)S * b_bytes);
     const uint32_t full0 = smem_u32(bars);
     const uint32_t empty0 = smem_u32(bars + S);
@@ -153,24 +157,26 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const CUtensorMap *tb = &maps.b[q];
                 const int kb0 = split * p.kb_per_split;
                 const int kb1 = min(p.kb_total, kb0 + p.kb_per_split);
-                for (int kb = kb0; kb < kb1; ++kb) {
+                for (int kb = kb0; kb < kb1; kb += KBS) {
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
                     const uint32_t fb = full0 + 8 * stage;
-                    mbar_arrive_expect_tx(fb, kABytes + b_bytes);
-                    const uint32_t a_dst = smem_u32(sA + (size_t)stage * kABytes);
-                    const uint32_t b_dst = smem_u32(sB + (size_t)stage * b_bytes);
-                    const int k = kb * 64;
-                    if (!A_MN) {
-                        tma_load_2d(a_dst, ta, fb, p.a_k_off + k, p.a_m_off + tm * 128);
-                    } else {
-                        tma_load_2d(a_dst, ta, fb, p.a_m_off + tm * 128, p.a_k_off + k);
-                        tma_load_2d(a_dst + 8192, ta, fb, p.a_m_off + tm * 128 + 64, p.a_k_off + k);
-                    }
-                    if (!B_MN) {
-                        tma_load_2d(b_dst, tb, fb, p.b_k_off + k, p.b_n_off + tn * g.BN);
-                    } else {
-                        for (int b = 0; b < g.BN / 64; ++b)
-                            tma_load_2d(b_dst + 8192 * b, tb, fb, p.b_n_off + tn * g.BN + 64 * b, p.b_k_off + k);
+                    mbar_arrive_expect_tx(fb, kABytesS + b_bytes);  // blocks past K arrive as zeros
+                    for (int j = 0; j < KBS; ++j) {
+                        const uint32_t a_dst = smem_u32(sA + (size_t)stage * kABytesS + (size_t)j * a1);
+                        const uint32_t b_dst = smem_u32(sB + (size_t)stage * b_bytes + (size_t)j * b1);
+                        const int k = (kb + j) * 64;
+                        if (!A_MN) {
+                            tma_load_2d(a_dst, ta, fb, p.a_k_off + k, p.a_m_off + tm * 128);
+                        } else {
+                            tma_load_2d(a_dst, ta, fb, p.a_m_off + tm * 128, p.a_k_off + k);
+                            tma_load_2d(a_dst + 8192, ta, fb, p.a_m_off + tm * 128 + 64, p.a_k_off + k);
+                        }
+                        if (!B_MN) {
+                            tma_load_2d(b_dst, tb, fb, p.b_k_off + k, p.b_n_off + tn * g.BN);
+                        } else {
+                            for (int b = 0; b < g.BN / 64; ++b)
+                                tma_load_2d(b_dst + 8192 * b, tb, fb, p.b_n_off + tn * g.BN + 64 * b, p.b_k_off + k);
+                        }
                     }
                     issued_mask |= 1u << stage;
                     issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
@@ -202,18 +208,20 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 if (!mbar_wait(tempty0 + 8 * acc, (((uint32_t)it >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * g.BN);
-                for (int kb = kb0; kb < kb1; ++kb) {
+                for (int kb = kb0; kb < kb1; kb += KBS) {
                     if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) { ok = false; break; }
                     tc_fence_after();
-                    const uint32_t a_addr = smem_u32(sA + (size_t)stage * kABytes);
-                    const uint32_t b_addr = smem_u32(sB + (size_t)stage * b_bytes);
+                    for (int j = 0; j < KBS; ++j) {
+                        const uint32_t a_addr = smem_u32(sA + (size_t)stage * kABytesS + (size_t)j * a1);
+                        const uint32_t b_addr = smem_u32(sB + (size_t)stage * b_bytes + (size_t)j * b1);
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk) {
-                        const uint64_t ad = A_MN ? smem_desc_sw128(a_addr + kk * 2048, 8192, 1024)
-                                                 : smem_desc_sw128(a_addr + kk * 32, 16, 1024);
-                        const uint64_t bd = B_MN ? smem_desc_sw128(b_addr + kk * 2048, 8192, 1024)
-                                                 : smem_desc_sw128(b_addr + kk * 32, 16, 1024);
-                        umma_bf16(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < 4; ++kk) {
+                            const uint64_t ad = A_MN ? smem_desc_sw128(a_addr + kk * 2048, 8192, 1024)
+                                                     : smem_desc_sw128(a_addr + kk * 32, 16, 1024);
+                            const uint64_t bd = B_MN ? smem_desc_sw128(b_addr + kk * 2048, 8192, 1024)
+                                                     : smem_desc_sw128(b_addr + kk * 32, 16, 1024);
+                            umma_bf16(d_tmem, ad, bd, idesc, (kb > kb0 || j > 0 || kk > 0) ? 1u : 0u);
+                        }
                     }
                     umma_commit(empty0 + 8 * stage);
                     if (++stage == S) { stage = 0; phase ^= 1u; }
