@@ -55,6 +55,21 @@ __device__ __forceinline__ int named_barrier_and(uint32_t id, uint32_t count, in
     return r;
 }
 
+// bar.red.or over a named barrier: 1 iff any participating thread passed a
+// non-zero predicate (a broadcast of one thread's decision).
+__device__ __forceinline__ int named_barrier_or(uint32_t id, uint32_t count, int pred) {
+    int r;
+    asm volatile(
+        "{\n\t.reg .pred pi, po;\n\t"
+        "setp.ne.s32 pi, %1, 0;\n\t"
+        "bar.red.or.pred po, %2, %3, pi;\n\t"
+        "selp.s32 %0, 1, 0, po;\n\t}"
+        : "=r"(r)
+        : "r"(pred), "r"(id), "r"(count)
+        : "memory");
+    return r;
+}
+
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -28,13 +28,19 @@ constexpr int kCeBN = 256;
 constexpr int kCeMaxTiles = 256;  // vocab tiles per chunk at most
 constexpr int kFinThreads = 256;
 constexpr int kFinRows = 32;
+// fp32 partials of 128 x kCeBN (128 KB each) for the tail split of the dh
+// contraction: enough for every CTA of a 160-SM part to hold one piece.
+constexpr int kCeSplitRegions = 160;
 
 struct CeLayout {
     int64_t nvt, Vc, nblk;
     float2 *part;
     float *ztgt, *lse_tmp, *block_sums;
     float *aref, *mref, *alpha, *beta;
-    unsigned int *ticket;
+    unsigned int *ticket;       // [4] loss ticket, then [split_regions] tail-split counters
+    unsigned int *split_tick;
+    int split_regions;
+    float *split_ws;
     __nv_bfloat16 *G;
     size_t bytes;
 };
@@ -86,8 +92,13 @@ static CePlan ce_plan(int64_t L, int64_t d, int64_t V, int sms) {
     return best;
 }
 
-static CeLayout ce_layout(void *ws, int64_t L, int64_t V) {
+static CeLayout ce_layout(void *ws, int64_t L, int64_t d, int64_t V) {
     CeLayout c{};
+    // tail split of the dh contraction: at most 4 pieces per tile and 2 CTAs
+    // per tile, so 8 regions per tile of the contraction bound the need
+    const int64_t rows = L > 128 ? 256 : 128;
+    const int64_t t2 = cdiv(L, rows) * cdiv(d, kCeBN);
+    c.split_regions = (int)(8 * t2 < kCeSplitRegions ? 8 * t2 : kCeSplitRegions);
     c.nvt = cdiv(V, kCeBN);
     c.Vc = ce_chunk_max(L, V);
     c.nblk = cdiv(L, kFinRows);
@@ -100,7 +111,9 @@ static CeLayout ce_layout(void *ws, int64_t L, int64_t V) {
     c.mref = cv.take<float>((size_t)L);
     c.alpha = cv.take<float>((size_t)L);
     c.beta = cv.take<float>((size_t)L);
-    c.ticket = cv.take<unsigned int>(4);
+    c.ticket = cv.take<unsigned int>(4 + (size_t)c.split_regions);
+    c.split_tick = c.ticket + 4;
+    c.split_ws = cv.take<float>((size_t)c.split_regions * 128 * kCeBN);
     c.G = cv.take<__nv_bfloat16>((size_t)(L * c.Vc));
     c.bytes = (size_t)round_up((int64_t)cv.used, 256);
     return c;
@@ -262,9 +275,8 @@ __global__ void __launch_bounds__(256) ce_fixup_kernel(float *dh, int64_t d, con
 extern "C" {
 
 size_t attt_ce_workspace_bytes(int64_t L, int64_t d, int64_t V) {
-    (void)d;
-    if (L <= 0 || V <= 0) return 0;
-    return attt::ce_layout(nullptr, L, V).bytes;
+    if (L <= 0 || V <= 0 || d <= 0) return 0;
+    return attt::ce_layout(nullptr, L, d, V).bytes;
 }
 
 attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W, const int32_t *d_tgt,
@@ -282,9 +294,10 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
     int *status = device_status_word(dev);
     if (!status) return ATTT_ERR_CUDA;
 
-    CeLayout c = ce_layout(d_ws, L, V);
+    CeLayout c = ce_layout(d_ws, L, d, V);
     float *lse = d_lse ? d_lse : c.lse_tmp;
-    if (cudaMemsetAsync(c.ticket, 0, sizeof(unsigned int), stream) != cudaSuccess) return ATTT_ERR_CUDA;
+    if (cudaMemsetAsync(c.ticket, 0, sizeof(unsigned int) * (4 + (size_t)c.split_regions), stream) != cudaSuccess)
+        return ATTT_ERR_CUDA;
 
     const CePlan plan = ce_plan(L, d, V, num_sms(dev));
     for (int64_t v0 = 0, ci = 0; v0 < V; v0 += plan.Vc, ++ci) {
@@ -317,6 +330,7 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
             EpiParams ep{};
             ep.out = d_dh; ep.out_ld = d; ep.accumulate = ci > 0 ? 1 : 0; ep.alpha = 1.0f;
             ep.row_alpha = c.alpha; ep.row_beta = c.beta;
+            p.split_ws = c.split_ws; p.split_tick = c.split_tick; p.split_regions = c.split_regions;
             st = launch_gemm<EPI_F32_ACC, false, true>(p, ep, dev, stream);
             if (st != ATTT_OK) return st;
         }

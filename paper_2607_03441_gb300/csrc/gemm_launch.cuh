@@ -18,9 +18,34 @@ struct GemmProblem {
     int M, N, K;
     int BN;
     int a_m_off = 0, a_k_off = 0, b_n_off = 0, b_k_off = 0;
-    bool allow_split = false;  // epilogue reduces split-K partials with atomics
-    bool pair = false;         // run on CTA pairs (256-row tiles, cta_group::2)
+    bool pair = false;  // run on CTA pairs (256-row tiles, cta_group::2)
+    // Tail split (EPI_F32_ACC): workspace for up to `split_regions` partials
+    // of 128 x BN fp32 and as many arrival counters (zero on entry).
+    float *split_ws = nullptr;
+    unsigned int *split_tick = nullptr;
+    int split_regions = 0;
 };
+
+// Pieces per tile for the tiles of a partial last wave: `tiles` tiles over
+// `units` concurrent tile slots leave r = tiles mod units tiles for the last
+// wave; cutting each into s K pieces (2 <= s <= 4, at least 8 K blocks each)
+// runs that wave in ceil(r s / units) / s of a tile's time.  Returns 1 when the
+// cut shortens the launch by less than a tenth (a long launch under the power
+// cap gains nothing from filling idle SMs) or the partials would not fit
+// `regions` (ranks per tile: `nranks`).
+inline int tail_pieces(int tiles, int units, int kb_total, int nranks, int regions) {
+    const int r = tiles % units;
+    if (r == 0) return 1;
+    int best_s = 1;
+    double best = 1.0;
+    for (int s = 2; s <= 4; ++s) {
+        if (kb_total < 8 * s || r * s * nranks > regions) break;
+        const double t = (double)cdiv(r * s, units) / s;
+        if (t < best - 1e-9) { best = t; best_s = s; }
+    }
+    const double waves = (double)(tiles / units) + 1.0;
+    return (1.0 - best) >= 0.1 * waves ? best_s : 1;
+}
 
 constexpr size_t kMaxSmem = 232448;  // 227 KB opt-in per CTA on sm_100-class parts
 
@@ -73,14 +98,19 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     const int sms = num_sms(dev);
     const int units = p.pair ? sms / 2 : sms;  // concurrent tiles
     const int tiles = (p.pair ? (g.tiles_m + 1) / 2 : g.tiles_m) * g.tiles_n;
-    int splits = 1;
-    if (p.allow_split) {
-        splits = (int)cdiv(units, tiles);
-        if (splits > g.kb_total) splits = g.kb_total;
-        if (splits < 1) splits = 1;
+    g.splits = 1;
+    g.kb_per_split = g.kb_total;
+    g.whole_tiles = tiles;
+    g.tail_s = 1;
+    if (EPI == EPI_F32_ACC && p.split_ws && p.split_tick && p.BN % 32 == 0) {
+        const int s = tail_pieces(tiles, units, g.kb_total, p.pair ? 2 : 1, p.split_regions);
+        if (s > 1) {
+            g.tail_s = s;
+            g.whole_tiles = tiles - tiles % units;
+            g.split_ws = p.split_ws;
+            g.split_tick = p.split_tick;
+        }
     }
-    g.kb_per_split = (int)cdiv(g.kb_total, splits);
-    g.splits = (int)cdiv(g.kb_total, g.kb_per_split);
     g.a_m_off = p.a_m_off;
     g.a_k_off = p.a_k_off;
     g.b_n_off = p.b_n_off;
@@ -90,7 +120,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.ep = ep;
 
     const size_t smem = gemm_smem_bytes(bn_cta, g.stages);
-    const int ntiles = tiles * g.splits;
+    const int ntiles = g.whole_tiles + (tiles - g.whole_tiles) * g.tail_s;  // work items
     if (!p.pair) {
         auto kern = tc_gemm_kernel<EPI, A_MN, B_MN>;
         if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;

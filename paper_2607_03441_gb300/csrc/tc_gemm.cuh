@@ -16,8 +16,10 @@
 // or MN-major (rows contiguous: a row-major [K, rows] matrix); both are
 // loaded by TMA with the 128-byte swizzle that tcgen05 reads natively.
 // Tiles past M, N or K are zero-filled by TMA and masked in the epilogue.
-// The K range of a tile may be split (split-K); split partial sums are
-// reduced with fp32 atomics by the epilogue kinds that support it.
+// When the tiles do not fill the last wave, the tiles of that wave may be
+// cut into K pieces spread over the idle SMs (EPI_F32_ACC): each piece
+// stores an fp32 partial and the last piece to arrive sums them in piece
+// order, so the result does not depend on which piece finishes last.
 #pragma once
 
 #include "attt_common.cuh"
@@ -67,6 +69,11 @@ struct GemmArgs {
     uint32_t tmem_cols;
     int *status;
     EpiParams ep;
+    // Tail split (tc_gemm_kernel / tc_gemm_pair_kernel): tiles [0, whole_tiles)
+    // run whole; every later tile runs as tail_s K pieces.
+    int whole_tiles, tail_s;
+    float *split_ws;           // [tail tile][piece][CTA rank] fp32 partials of 128 x BN, column-quad major
+    unsigned int *split_tick;  // [tail tile][CTA rank] arrival counters; 0 between launches
 };
 
 constexpr uint32_t kABytes = 128 * 64 * 2;  // one A stage: 128 rows x 64 bf16
@@ -78,12 +85,35 @@ __host__ __device__ inline size_t gemm_smem_bytes(int BN, int stages) {
     return 1024 + (size_t)stages * (kABytes + gemm_b_stage_bytes(BN)) + 8 * (2 * stages + 5) + 16;
 }
 
-__device__ __forceinline__ void decode_tile(const GemmArgs &g, int t, int &tm, int &tn, int &split) {
-    const int per = g.tiles_m * g.tiles_n;
-    split = t / per;
-    const int rem = t - split * per;
-    tn = rem / g.tiles_m;
-    tm = rem - tn * g.tiles_m;
+// One unit of work of tc_gemm_kernel / tc_gemm_pair_kernel: an output tile
+// (m fastest) and its K-block range; piece >= 0 marks a K piece of tail tile
+// `tail`.  `tiles_m` counts row tiles of the kernel's accumulator height.
+struct Work {
+    int tm, tn, kb0, kb1, piece, tail;
+};
+
+__device__ __forceinline__ Work work_item(const GemmArgs &g, int w, int tiles_m) {
+    Work k;
+    int t = w;
+    k.piece = -1;
+    k.tail = -1;
+    k.kb0 = 0;
+    k.kb1 = g.kb_total;
+    if (w >= g.whole_tiles) {
+        const int j = w - g.whole_tiles;
+        k.tail = j / g.tail_s;
+        k.piece = j - k.tail * g.tail_s;
+        t = g.whole_tiles + k.tail;
+        k.kb0 = (int)((int64_t)g.kb_total * k.piece / g.tail_s);
+        k.kb1 = (int)((int64_t)g.kb_total * (k.piece + 1) / g.tail_s);
+    }
+    k.tn = t / tiles_m;
+    k.tm = t - k.tn * tiles_m;
+    return k;
+}
+
+__device__ __forceinline__ int work_count(const GemmArgs &g, int tiles_m) {
+    return g.whole_tiles + (tiles_m * g.tiles_n - g.whole_tiles) * g.tail_s;
 }
 
 constexpr float kLog2e = 1.4426950408889634f;
@@ -91,6 +121,28 @@ constexpr float kLog2e = 1.4426950408889634f;
 // A CE tile whose max exceeds the row reference by more than 2^kCeRefJump
 // (log2 units) writes E against its own max instead, so E <= 2^kCeRefJump.
 constexpr float kCeRefJump = 32.f;
+
+// out[gm, col0 + i] = (accumulate ? ra * out : 0) + rb * v[i] for the 32
+// columns of one TMEM chunk (EPI_F32_ACC), nothing at or past n_end.
+__device__ __forceinline__ void f32_acc_store(const EpiParams &ep, float *orow, int col0, int n_end, float ra,
+                                              float rb, const float (&v)[32]) {
+    if (col0 + 32 <= n_end) {
+        float4 *dst = reinterpret_cast<float4 *>(orow + col0);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            float4 o = make_float4(rb * v[4 * q], rb * v[4 * q + 1], rb * v[4 * q + 2], rb * v[4 * q + 3]);
+            if (ep.accumulate) {
+                const float4 p = dst[q];
+                o.x = fmaf(ra, p.x, o.x); o.y = fmaf(ra, p.y, o.y);
+                o.z = fmaf(ra, p.z, o.z); o.w = fmaf(ra, p.w, o.w);
+            }
+            dst[q] = o;
+        }
+    } else {
+        for (int i = 0; i < 32 && col0 + i < n_end; ++i)
+            orow[col0 + i] = ep.accumulate ? fmaf(ra, orow[col0 + i], rb * v[i]) : rb * v[i];
+    }
+}
 
 // ---------------------------------------------------------------------------
 // Epilogues.  Every thread owns accumulator row `row` of the tile; all 32
@@ -179,25 +231,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
             if (n_base + c >= n_end) break;
             float v[32];
             tmem_ld_x32(taddr + (uint32_t)c, v);
-            if (rv) {
-                const int col0 = n_base + c;
-                if (col0 + 32 <= n_end) {
-                    float4 *dst = reinterpret_cast<float4 *>(orow + col0);
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) {
-                        float4 o = make_float4(rb * v[4 * q], rb * v[4 * q + 1], rb * v[4 * q + 2], rb * v[4 * q + 3]);
-                        if (ep.accumulate) {
-                            const float4 p = dst[q];
-                            o.x = fmaf(ra, p.x, o.x); o.y = fmaf(ra, p.y, o.y);
-                            o.z = fmaf(ra, p.z, o.z); o.w = fmaf(ra, p.w, o.w);
-                        }
-                        dst[q] = o;
-                    }
-                } else {
-                    for (int i = 0; i < 32 && col0 + i < n_end; ++i)
-                        orow[col0 + i] = ep.accumulate ? fmaf(ra, orow[col0 + i], rb * v[i]) : rb * v[i];
-                }
-            }
+            if (rv) f32_acc_store(ep, orow, n_base + c, n_end, ra, rb, v);
         }
     } else if constexpr (EPI == EPI_ATOMIC_T) {
         for (int c = 0; c < g.BN; c += 16) {
@@ -229,6 +263,68 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
                 }
             }
         }
+    }
+}
+
+// EPI_F32_ACC for K piece k.piece of tail tile k.tail, on the 128 accumulator
+// rows this CTA holds (CTA `rank` of `nranks`).  The four epilogue warps store
+// the piece's partial (column-quad major: a warp writes 512 contiguous bytes
+// per store), then one thread takes a ticket; the piece that arrives last
+// forms the sum P_0 + P_1 + ... in piece order, its own term read back from
+// TMEM, and applies the epilogue to it.  BN is a multiple of 32.
+__device__ __forceinline__ void epilogue_piece_f32_acc(const GemmArgs &g, const Work &k, int gm_base, int rank,
+                                                    int nranks, int row, uint32_t taddr) {
+    const int BN = g.BN;
+    const size_t region = (size_t)128 * (size_t)BN;
+    const size_t slot0 = (size_t)k.tail * (size_t)g.tail_s;
+    float4 *mine = reinterpret_cast<float4 *>(g.split_ws + ((slot0 + k.piece) * nranks + rank) * region) + row;
+    for (int c = 0; c < BN; c += 32) {
+        float v[32];
+        tmem_ld_x32(taddr + (uint32_t)c, v);
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            __stcg(mine + (size_t)(c / 4 + q) * 128, make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+    }
+    __threadfence();
+    named_barrier_sync(1, 128);
+    int last = 0;
+    if (row == 0) {
+        unsigned int *tk = g.split_tick + (size_t)k.tail * nranks + rank;
+        last = atomicAdd(tk, 1u) == (unsigned int)(g.tail_s - 1) ? 1 : 0;
+        if (last) atomicExch(tk, 0u);  // every piece has arrived: ready for the next launch
+        __threadfence();
+    }
+    if (!named_barrier_or(1, 128, last)) return;
+
+    const EpiParams &ep = g.ep;
+    const int gm = gm_base + row;
+    const bool rv = gm < g.M;
+    const int n_base = k.tn * BN;
+    const int n_end = min(g.N, n_base + BN);
+    float ra = 1.f, rb = 1.f;
+    if (rv && ep.row_alpha) ra = __ldg(ep.row_alpha + gm);
+    if (rv && ep.row_beta) rb = __ldg(ep.row_beta + gm);
+    float *orow = ep.out + (int64_t)gm * ep.out_ld;
+    for (int c = 0; c < BN; c += 32) {
+        if (n_base + c >= n_end) break;
+        float s[32];
+        for (int j = 0; j < g.tail_s; ++j) {
+            float v[32];
+            if (j == k.piece) {
+                tmem_ld_x32(taddr + (uint32_t)c, v);
+            } else {
+                const float4 *src =
+                    reinterpret_cast<const float4 *>(g.split_ws + ((slot0 + j) * nranks + rank) * region) + row;
+#pragma unroll
+                for (int q = 0; q < 8; ++q) {
+                    const float4 p = __ldcg(src + (size_t)(c / 4 + q) * 128);
+                    v[4 * q] = p.x; v[4 * q + 1] = p.y; v[4 * q + 2] = p.z; v[4 * q + 3] = p.w;
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 32; ++i) s[i] = (j == 0) ? v[i] : s[i] + v[i];
+        }
+        if (rv) f32_acc_store(ep, orow, n_base + c, n_end, ra, rb, s);
     }
 }
 
@@ -281,7 +377,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    const int ntiles = g.tiles_m * g.tiles_n * g.splits;
+    const int nwork = work_count(g, g.tiles_m);
 
     if (warp == 0) {
         if (lane == 0) {
@@ -290,12 +386,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_parity = 0;  // per stage: last issue pending?
             bool ok = true;
-            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
-                int tm, tn, split;
-                decode_tile(g, t, tm, tn, split);
-                const int kb0 = split * g.kb_per_split;
-                const int kb1 = min(g.kb_total, kb0 + g.kb_per_split);
-                for (int kb = kb0; kb < kb1; ++kb) {
+            for (int w = blockIdx.x; w < nwork && ok; w += gridDim.x) {
+                const Work wi = work_item(g, w, g.tiles_m);
+                const int tm = wi.tm, tn = wi.tn;
+                for (int kb = wi.kb0; kb < wi.kb1; ++kb) {
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
                     const uint32_t fb = full0 + 8 * stage;
                     mbar_arrive_expect_tx(fb, kABytes + b_bytes);
@@ -336,11 +430,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             uint32_t phase = 0;
             int it = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++it) {
-                int tm, tn, split;
-                decode_tile(g, t, tm, tn, split);
-                const int kb0 = split * g.kb_per_split;
-                const int kb1 = min(g.kb_total, kb0 + g.kb_per_split);
+            for (int w = blockIdx.x; w < nwork && ok; w += gridDim.x, ++it) {
+                const Work wi = work_item(g, w, g.tiles_m);
+                const int kb0 = wi.kb0, kb1 = wi.kb1;
                 const int acc = it & 1;
                 if (!mbar_wait(tempty0 + 8 * acc, (((uint32_t)it >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
                 tc_fence_after();
@@ -379,9 +471,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int q = warp & 3;
         const int row = q * 32 + lane;
         int it = 0;
-        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++it) {
-            int tm, tn, split;
-            decode_tile(g, t, tm, tn, split);
+        for (int w = blockIdx.x; w < nwork; w += gridDim.x, ++it) {
+            const Work wi = work_item(g, w, g.tiles_m);
             const int acc = it & 1;
             const uint32_t par = ((uint32_t)it >> 1) & 1u;
             int ok = 1;
@@ -395,7 +486,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             (void)mbar_try_wait(tfull0 + 8 * acc, par);  // per-thread acquire of the completed phase
             tc_fence_after();
             const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * g.BN);
-            epilogue_tile<EPI>(g, tm * 128, tn, row, taddr);
+            if constexpr (EPI == EPI_F32_ACC) {
+                if (wi.piece >= 0)
+                    epilogue_piece_f32_acc(g, wi, wi.tm * 128, 0, 1, row, taddr);
+                else
+                    epilogue_tile<EPI>(g, wi.tm * 128, wi.tn, row, taddr);
+            } else {
+                epilogue_tile<EPI>(g, wi.tm * 128, wi.tn, row, taddr);
+            }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
@@ -417,15 +515,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 // CTAs' epilogues release the accumulator to the even CTA.  Per SM this moves
 // a third less shared-memory traffic per FLOP than the single-CTA kernel.
 // ---------------------------------------------------------------------------
-
-__device__ __forceinline__ void decode_tile_pair(const GemmArgs &g, int t, int &tm2, int &tn, int &split) {
-    const int tiles_m2 = (g.tiles_m + 1) / 2;
-    const int per = tiles_m2 * g.tiles_n;
-    split = t / per;
-    const int rem = t - split * per;
-    tn = rem / tiles_m2;
-    tm2 = rem - tn * tiles_m2;
-}
 
 template <int EPI, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1)
@@ -477,7 +566,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t tmem_base = *tmem_slot;
 
     const int tiles_m2 = (g.tiles_m + 1) / 2;
-    const int ntiles = tiles_m2 * g.tiles_n * g.splits;
+    const int nwork = work_count(g, tiles_m2);
     const int cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
     const uint32_t lead_full0 = mapa_shared(full0, 0);
     const uint32_t lead_tempty0 = mapa_shared(tempty0, 0);
@@ -488,14 +577,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             int stage = 0;
             uint32_t phase = 0;
             bool ok = true;
-            for (int t = cid; t < ntiles && ok; t += ncl) {
-                int tm2, tn, split;
-                decode_tile_pair(g, t, tm2, tn, split);
-                const int kb0 = split * g.kb_per_split;
-                const int kb1 = min(g.kb_total, kb0 + g.kb_per_split);
-                const int arow = g.a_m_off + tm2 * 256 + 128 * (int)rank;
-                const int brow = g.b_n_off + tn * g.BN + BNh * (int)rank;
-                for (int kb = kb0; kb < kb1; ++kb) {
+            for (int w = cid; w < nwork && ok; w += ncl) {
+                const Work wi = work_item(g, w, tiles_m2);
+                const int arow = g.a_m_off + wi.tm * 256 + 128 * (int)rank;
+                const int brow = g.b_n_off + wi.tn * g.BN + BNh * (int)rank;
+                for (int kb = wi.kb0; kb < wi.kb1; ++kb) {
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
                     if (leader) mbar_arrive_expect_tx(full0 + 8 * stage, 2u * (kABytes + b_bytes));
                     const uint32_t fb = lead_full0 + 8 * stage;
@@ -530,11 +616,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             uint32_t phase = 0;
             int it = 0;
             bool ok = true;
-            for (int t = cid; t < ntiles && ok; t += ncl, ++it) {
-                int tm2, tn, split;
-                decode_tile_pair(g, t, tm2, tn, split);
-                const int kb0 = split * g.kb_per_split;
-                const int kb1 = min(g.kb_total, kb0 + g.kb_per_split);
+            for (int w = cid; w < nwork && ok; w += ncl, ++it) {
+                const Work wi = work_item(g, w, tiles_m2);
+                const int kb0 = wi.kb0, kb1 = wi.kb1;
                 const int acc = it & 1;
                 if (!mbar_wait(tempty0 + 8 * acc, (((uint32_t)it >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
                 tc_fence_after();
@@ -571,9 +655,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int q = warp & 3;
         const int row = q * 32 + lane;
         int it = 0;
-        for (int t = cid; t < ntiles; t += ncl, ++it) {
-            int tm2, tn, split;
-            decode_tile_pair(g, t, tm2, tn, split);
+        for (int w = cid; w < nwork; w += ncl, ++it) {
+            const Work wi = work_item(g, w, tiles_m2);
             const int acc = it & 1;
             const uint32_t par = ((uint32_t)it >> 1) & 1u;
             int ok = 1;
@@ -587,7 +670,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             (void)mbar_try_wait(tfull0 + 8 * acc, par);
             tc_fence_after();
             const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * g.BN);
-            epilogue_tile<EPI>(g, tm2 * 256 + 128 * (int)rank, tn, row, taddr);
+            const int gm_base = wi.tm * 256 + 128 * (int)rank;
+            if constexpr (EPI == EPI_F32_ACC) {
+                if (wi.piece >= 0)
+                    epilogue_piece_f32_acc(g, wi, gm_base, (int)rank, 2, row, taddr);
+                else
+                    epilogue_tile<EPI>(g, gm_base, wi.tn, row, taddr);
+            } else {
+                epilogue_tile<EPI>(g, gm_base, wi.tn, row, taddr);
+            }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(lead_tempty0 + 8 * acc);

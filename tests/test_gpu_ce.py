@@ -183,6 +183,29 @@ def test_multichunk_with_reference_jumps(attt):
     assert abs(loss - ref_loss) <= LOSS_RTOL * abs(ref_loss)
 
 
+@pytest.mark.parametrize("L,V,d", [(1280, 6000, 1280), (2048, 3000, 3584), (100, 20000, 3584)])
+def test_tail_pieces_deterministic(attt, L, V, d):
+    """Shapes whose dh contraction leaves a partial last wave on a 152-SM
+    part, so its tiles run as 2-4 K pieces (25 tiles: 3 pieces; 112 tiles:
+    2; 14 single-CTA tiles: 4): sampled rows against the oracle, and two calls
+    give the same bits whichever piece finishes last."""
+    h = wk.normal_bf16(L + 1, "h", (L, d), 1.0)
+    W = wk.normal_bf16(V + 1, "W", (V, d), 0.05)
+    rng = wk.rng_for(L + V, "t")
+    tgt = rng.integers(0, V, L).astype(np.int32)
+    w = rng.choice(np.array([1.0, 0.5, 0.05], np.float32), L).astype(np.float32)
+    loss, dh, lse = _run(attt, h, W, tgt, w)
+    loss2, dh2, lse2 = _run(attt, h, W, tgt, w)
+    assert loss == loss2
+    np.testing.assert_array_equal(dh.view(np.uint32), dh2.view(np.uint32))
+    np.testing.assert_array_equal(lse.view(np.uint32), lse2.view(np.uint32))
+    rows = np.unique(np.concatenate([[0, 1, L - 1], rng.choice(L, 9, replace=False)])).astype(np.int64)
+    rlse, _, rdh = oracle.ce_rows(h, W, tgt, w, rows)
+    np.testing.assert_allclose(lse[rows], rlse, atol=LSE_ATOL, rtol=0)
+    e = rel_l2(dh[rows], rdh)
+    assert e < DH_RL2, e
+
+
 def test_launch_counter_counts_every_kernel(attt):
     """One single-chunk call launches GEMM1, the chunk kernel, GEMM2, the
     finalize and the fixup kernels: five kernels, all counted."""
