@@ -3,31 +3,31 @@
 // states, in one sweep over the vocabulary (4*L*V*d tensor FLOPs: each logit
 // is computed once), never holding the [L, V] logits in HBM.
 //
-// For each vocab chunk c of Vc columns (Vc sized so that the chunk's bf16
-// block stays L2-resident):
-//   GEMM1  z = h W_c^T on 128 x 256 tiles; the epilogue keeps per (row, tile)
-//          the max m_t and the sum of exp(z - m_t) (log2 units), writes
-//          E = exp(z - m_t) as bf16, and catches the target logit;
-//          From the second chunk on, E is written against the running max
-//          of the earlier chunks instead of the tile max;
-//   chunk  per row: the chunk max, a rewrite of E only where needed (the
-//          first chunk, or a row whose max jumped by more than 2^32), and the
-//          online-softmax factors of the accumulator's reference A:
-//          alpha = exp(A_old - A_new), beta = exp(R_E - A_new);
+// First, per row j, a reference R_j: the target logit z_{j,x_j} (log2 units).
+// Then for each vocab chunk c of Vc columns:
+//   GEMM1  z = h W_c^T; the epilogue keeps per (row, tile) the max m_t and the
+//          sum of exp(z - m_t) (log2 units), writes E = exp(z - R) as bf16
+//          against the row's reference R (against m_t for a tile whose max
+//          exceeds R by more than 2^64), and catches the target logit;
+//   chunk  per row: the chunk max, the running (max, sum) of the logsumexp,
+//          a rewrite of E where a tile used its own max, the online-softmax
+//          factors of the accumulator's reference A, alpha = exp(A_old -
+//          A_new), beta = exp(R_E - A_new), and R <- max(R, chunk max);
 //   GEMM2  D = E W_c (W read MN-major by TMA); the epilogue folds it into the
 //          fp32 accumulator: acc = alpha * acc + beta * D.
-// Then per row: lse from the (max, sum) pairs of every tile, the loss
-// (1/L) sum_j w_j (lse_j - z_{j,x_j}) summed in a fixed order, and
-//   dh_j = (w_j / L) (acc_j exp(M_j - lse_j) - W_{x_j}).
-// The LM head gets no gradient (frozen; only the adapter trains).
+// The last chunk's bookkeeping also forms lse_j and the loss
+// (1/L) sum_j w_j (lse_j - z_{j,x_j}) (summed in a fixed order) and folds
+// the gradient's factors into alpha and beta, so that the last GEMM2 writes
+//   dh_j = (w_j / L) (acc_j exp(A_j - lse_j) - W_{x_j})
+// directly.  The LM head gets no gradient (frozen; only the adapter trains).
 #include "gemm_launch.cuh"
 
 namespace attt {
 
 constexpr int kCeBN = 256;
 constexpr int kCeMaxTiles = 256;  // vocab tiles per chunk at most
-constexpr int kFinThreads = 256;
-constexpr int kFinRows = 32;
+constexpr int kChunkWarps = 8;  // ce_chunk_kernel: 8 warps, 32 rows (one per lane) per block
+constexpr int kChunkRows = 32;
 // fp32 partials of 128 x kCeBN (128 KB each) for the tail split of the dh
 // contraction: enough for every CTA of a 160-SM part to hold one piece.
 constexpr int kCeSplitRegions = 160;
@@ -35,8 +35,8 @@ constexpr int kCeSplitRegions = 160;
 struct CeLayout {
     int64_t nvt, Vc, nblk;
     float2 *part;
-    float *ztgt, *lse_tmp, *block_sums;
-    float *aref, *mref, *alpha, *beta;
+    float *ztgt, *block_sums;
+    float *aref, *mref, *lm, *ls, *alpha, *beta, *gamma;
     unsigned int *ticket;       // [4] loss ticket, then [split_regions] tail-split counters
     unsigned int *split_tick;
     int split_regions;
@@ -101,16 +101,18 @@ static CeLayout ce_layout(void *ws, int64_t L, int64_t d, int64_t V) {
     c.split_regions = (int)(8 * t2 < kCeSplitRegions ? 8 * t2 : kCeSplitRegions);
     c.nvt = cdiv(V, kCeBN);
     c.Vc = ce_chunk_max(L, V);
-    c.nblk = cdiv(L, kFinRows);
+    c.nblk = cdiv(L, kChunkRows);
     Carve cv{static_cast<char *>(ws), 0};
     c.part = cv.take<float2>((size_t)(c.nvt * L));
     c.ztgt = cv.take<float>((size_t)L);
-    c.lse_tmp = cv.take<float>((size_t)L);
     c.block_sums = cv.take<float>((size_t)c.nblk);
     c.aref = cv.take<float>((size_t)L);
     c.mref = cv.take<float>((size_t)L);
+    c.lm = cv.take<float>((size_t)L);
+    c.ls = cv.take<float>((size_t)L);
     c.alpha = cv.take<float>((size_t)L);
     c.beta = cv.take<float>((size_t)L);
+    c.gamma = cv.take<float>((size_t)L);
     c.ticket = cv.take<unsigned int>(4 + (size_t)c.split_regions);
     c.split_tick = c.ticket + 4;
     c.split_ws = cv.take<float>((size_t)c.split_regions * 128 * kCeBN);
@@ -127,146 +129,186 @@ __device__ __forceinline__ void lse_merge(float &m, float &s, float m2, float s2
     m = mx;
 }
 
-// One block per kFinRows rows; warp w merges the vocab tiles i = w (mod 8) of
-// its 32 rows with coalesced loads of part[i, rows], then warp 0 merges the
-// 8 partial pairs per row and forms lse, the target NLL and the weighted sum.
-// The last block (atomic ticket) adds the block sums in block order, so the
-// loss is deterministic.
-__global__ void __launch_bounds__(kFinThreads) ce_finalize_kernel(const float2 *__restrict__ part, int nvt,
-                                                                   const float *__restrict__ ztgt,
-                                                                   const int32_t *__restrict__ tgt,
-                                                                   const float *__restrict__ w, int L, int V,
-                                                                   float *__restrict__ lse_out, float inv_L,
-                                                                   float *block_sums, unsigned int *ticket,
-                                                                   float *loss, int *status) {
-    constexpr int kWarps = kFinThreads / 32;
-    __shared__ float sm_m[kWarps][kFinRows], sm_s[kWarps][kFinRows];
-    __shared__ bool last;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int j = blockIdx.x * kFinRows + lane;
-    float m = -INFINITY, s = 0.f;
-    if (j < L) {
-        for (int i = warp; i < nvt; i += kWarps) {
-            const float2 p = __ldcg(part + (int64_t)i * L + j);
-            lse_merge(m, s, p.x, p.y);
-        }
-    }
-    sm_m[warp][lane] = m;
-    sm_s[warp][lane] = s;
-    __syncthreads();
-    if (warp == 0) {
-        for (int k = 1; k < kWarps; ++k) lse_merge(m, s, sm_m[k][lane], sm_s[k][lane]);
-        float contrib = 0.f;
-        if (j < L) {
-            const float lse = (m + log2f(s)) * 0.69314718055994531f;
-            lse_out[j] = lse;
-            const int t = tgt[j];
-            float nll;
-            if (t < 0 || t >= V) {
-                record_error(status, ATTT_ERR_TOKEN_RANGE);
-                nll = __int_as_float(0x7fc00000);
-            } else {
-                nll = lse - __ldcg(ztgt + j);
-            }
-            contrib = w[j] * nll;
-        }
-        for (int o = 16; o > 0; o >>= 1) contrib += __shfl_xor_sync(0xffffffffu, contrib, o);
-        if (lane == 0) {
-            block_sums[blockIdx.x] = contrib;
-            __threadfence();
-            last = atomicAdd(ticket, 1u) == gridDim.x - 1;
-        }
-    }
-    __syncthreads();
-    if (last && threadIdx.x == 0) {
-        __threadfence();
-        float total = 0.f;
-        for (unsigned i = 0; i < gridDim.x; ++i) total += __ldcg(block_sums + i);
-        *loss = total * inv_L;
-        *ticket = 0u;
-    }
-}
-
-// Bookkeeping of chunk c, one warp per row j (log2 units throughout):
-//   M_c  = max over the chunk's tiles of the tile max m_t;
-//   R    = the running max of the earlier chunks (mref; -inf for the first).
-//   GEMM1 wrote tile t of E against R, or against m_t when m_t - R >
-//   kCeRefJump.  If any tile did (M_c - R > kCeRefJump), the row is rewritten
-//   against M_c tile by tile; otherwise it stays against R.  Rp = the
-//   reference E now has.
-//   acc = alpha * acc + beta * (E W_c) with A_new = max(A_old, Rp),
-//   alpha = exp2(A_old - A_new), beta = exp2(Rp - A_new);  mref <- max(R, M_c).
-__global__ void __launch_bounds__(256) ce_chunk_kernel(const float2 *__restrict__ part, int tile0, int ntiles, int L,
-                                                       __nv_bfloat16 *G, int64_t G_ld, float *aref, float *mref,
-                                                       float *alpha, float *beta, int first) {
+// Reference of the first chunk, one warp per row: R_j = z_{j,x_j} log2 e (an
+// fp32 dot product), -inf for a target outside [0, V).  Any R_j at or below
+// the row max keeps E from overflowing; the target logit sits near the max
+// for the tokens a model is trained on, so E rarely needs a rewrite.
+__global__ void __launch_bounds__(256) ce_ref_kernel(const __nv_bfloat16 *__restrict__ h,
+                                                     const __nv_bfloat16 *__restrict__ W,
+                                                     const int32_t *__restrict__ tgt, int L, int64_t d, int V,
+                                                     float *__restrict__ mref) {
     const int j = blockIdx.x * 8 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (j >= L) return;
-    float mc = -INFINITY;
-    for (int t = lane; t < ntiles; t += 32) mc = fmaxf(mc, __ldcg(&part[(int64_t)(tile0 + t) * L + j].x));
-    for (int o = 16; o > 0; o >>= 1) mc = fmaxf(mc, __shfl_xor_sync(0xffffffffu, mc, o));
-    const float r = first ? -INFINITY : mref[j];
-    uint4 *row = reinterpret_cast<uint4 *>(G + (int64_t)j * G_ld);
-    const int per_tile = kCeBN / 8;  // uint4 (8 x bf16) per tile row
-    float rp = r;
-    if (mc - r > kCeRefJump) {
-        rp = mc;
-        for (int t = 0; t < ntiles; ++t) {
-            const float mt = __ldcg(&part[(int64_t)(tile0 + t) * L + j].x);
-            const float sc = (mt - r > kCeRefJump) ? exp2f(mt - mc) : exp2f(r - mc);
-            for (int i = lane; i < per_tile; i += 32) {
-                uint4 u = row[t * per_tile + i];
-                uint32_t *w = reinterpret_cast<uint32_t *>(&u);
+    const int t = tgt[j];
+    if (t < 0 || t >= V) {
+        if (lane == 0) mref[j] = -INFINITY;
+        return;
+    }
+    const __nv_bfloat16 *hr = h + (int64_t)j * d;
+    const __nv_bfloat16 *wr = W + (int64_t)t * d;
+    float acc = 0.f;
+    for (int64_t k = (int64_t)lane * 8; k < d; k += 256) {  // d % 8 == 0: 16-byte loads
+        const uint4 a = __ldg(reinterpret_cast<const uint4 *>(hr + k));
+        const uint4 b = __ldg(reinterpret_cast<const uint4 *>(wr + k));
+        const __nv_bfloat162 *a2 = reinterpret_cast<const __nv_bfloat162 *>(&a);
+        const __nv_bfloat162 *b2 = reinterpret_cast<const __nv_bfloat162 *>(&b);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162 *>(&w[q]);
-                    const float2 v = __bfloat1622float2(b);
-                    b = __floats2bfloat162_rn(v.x * sc, v.y * sc);
-                    w[q] = *reinterpret_cast<uint32_t *>(&b);
+        for (int e = 0; e < 4; ++e) {
+            const float2 x = __bfloat1622float2(a2[e]), y = __bfloat1622float2(b2[e]);
+            acc = fmaf(x.x, y.x, acc);
+            acc = fmaf(x.y, y.y, acc);
+        }
+    }
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) mref[j] = acc * kLog2e;
+}
+
+struct CeChunkArgs {
+    const float2 *part;  // [vocab tiles, L] (max, sum) of every tile (log2 units)
+    int tile0, ntiles, L, V;
+    __nv_bfloat16 *G;
+    int64_t G_ld;
+    float *aref, *mref, *lm, *ls, *alpha, *beta, *gamma;
+    int first, last;
+    // last chunk only
+    const float *ztgt;
+    const int32_t *tgt;
+    const float *w;
+    float inv_L;
+    float *lse_out;  // or nullptr
+    float *block_sums;
+    unsigned int *ticket;
+    float *loss;
+    int *status;
+};
+
+// Bookkeeping of one chunk, 32 rows per block (lane = row), log2 units:
+//   warp k reads the chunk's tiles t = k (mod 8) with coalesced loads of
+//   part[t, rows]; per row the chunk max M_c and the chunk's (max, sum) pair,
+//   merged into the running pair (lm, ls);
+//   R = mref, the reference GEMM1 wrote this chunk's E against.  A tile whose
+//   max exceeded R by more than kCeRefJump used its own max, and then
+//   (M_c - R > kCeRefJump) the row is rewritten against M_c tile by tile
+//   (Rp = M_c); otherwise it stays against R (Rp = R);
+//   acc = alpha * acc + beta * (E W_c) with A_new = max(A_old, Rp),
+//   alpha = exp2(A_old - A_new), beta = exp2(Rp - A_new);  mref <- max(R, M_c).
+// Last chunk: lse = ln 2 (lm + log2 ls); the weighted NLL of the block's rows
+// goes to block_sums and the last block (ticket) adds them in block order;
+// alpha and beta take the factor (w/L) exp2(A_new - lse log2 e) and gamma =
+// w/L, so the last GEMM2 writes dh itself.
+__global__ void __launch_bounds__(kChunkWarps * 32) ce_chunk_kernel(const CeChunkArgs a) {
+    __shared__ float s_mc[kChunkWarps][kChunkRows], s_m[kChunkWarps][kChunkRows], s_s[kChunkWarps][kChunkRows];
+    __shared__ float s_r[kChunkRows], s_mcf[kChunkRows];
+    __shared__ int s_rw[kChunkRows];
+    __shared__ bool s_last;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int j0 = blockIdx.x * kChunkRows;
+    const int j = j0 + lane;
+    const int L = a.L;
+    float mc = -INFINITY, m = -INFINITY, s = 0.f;
+    if (j < L) {
+        for (int t = warp; t < a.ntiles; t += kChunkWarps) {
+            const float2 p = __ldcg(a.part + (int64_t)(a.tile0 + t) * L + j);
+            mc = fmaxf(mc, p.x);
+            lse_merge(m, s, p.x, p.y);
+        }
+    }
+    s_mc[warp][lane] = mc;
+    s_m[warp][lane] = m;
+    s_s[warp][lane] = s;
+    __syncthreads();
+    if (warp == 0) {
+        for (int k = 1; k < kChunkWarps; ++k) {
+            mc = fmaxf(mc, s_mc[k][lane]);
+            lse_merge(m, s, s_m[k][lane], s_s[k][lane]);
+        }
+        int rw = 0;
+        float r = 0.f, contrib = 0.f;
+        if (j < L) {
+            if (!a.first) {  // running pair first, then this chunk's
+                float rm = a.lm[j], rs = a.ls[j];
+                lse_merge(rm, rs, m, s);
+                m = rm;
+                s = rs;
+            }
+            a.lm[j] = m;
+            a.ls[j] = s;
+            r = a.mref[j];
+            rw = (mc - r > kCeRefJump) ? 1 : 0;
+            const float rp = rw ? mc : r;
+            const float aold = a.first ? -INFINITY : a.aref[j];
+            const float anew = fmaxf(aold, rp);
+            float al = (aold == -INFINITY) ? 0.f : exp2f(aold - anew);
+            float be = exp2f(rp - anew);
+            a.aref[j] = anew;
+            a.mref[j] = fmaxf(r, mc);
+            if (a.last) {
+                const float lse2 = m + log2f(s);
+                const float lse = lse2 * 0.69314718055994531f;
+                if (a.lse_out) a.lse_out[j] = lse;
+                const int t = a.tgt[j];
+                const float c = a.w[j] * a.inv_L;
+                float nll;
+                if (t < 0 || t >= a.V) {
+                    record_error(a.status, ATTT_ERR_TOKEN_RANGE);
+                    nll = __int_as_float(0x7fc00000);
+                    a.gamma[j] = __int_as_float(0x7fc00000);
+                } else {
+                    nll = lse - __ldcg(a.ztgt + j);
+                    a.gamma[j] = c;
                 }
-                row[t * per_tile + i] = u;
+                contrib = a.w[j] * nll;
+                const float f = c * exp2f(anew - lse2);
+                al *= f;
+                be *= f;
+            }
+            a.alpha[j] = al;
+            a.beta[j] = be;
+        }
+        s_rw[lane] = rw;
+        s_r[lane] = r;
+        s_mcf[lane] = mc;
+        if (a.last) {
+            for (int o = 16; o > 0; o >>= 1) contrib += __shfl_xor_sync(0xffffffffu, contrib, o);
+            if (lane == 0) {
+                a.block_sums[blockIdx.x] = contrib;
+                __threadfence();
+                s_last = atomicAdd(a.ticket, 1u) == gridDim.x - 1;
             }
         }
     }
-    if (lane == 0) {
-        const float aold = first ? -INFINITY : aref[j];
-        const float anew = fmaxf(aold, rp);
-        alpha[j] = (aold == -INFINITY) ? 0.f : exp2f(aold - anew);
-        beta[j] = exp2f(rp - anew);
-        aref[j] = anew;
-        mref[j] = fmaxf(r, mc);
+    __syncthreads();
+    // rows whose tiles used their own max: E against M_c, tile by tile
+    const int per_tile = kCeBN / 8;  // uint4 (8 x bf16) per tile row
+    for (int i = warp; i < kChunkRows; i += kChunkWarps) {
+        if (!s_rw[i]) continue;
+        const int jr = j0 + i;
+        const float r = s_r[i], mcr = s_mcf[i];
+        uint4 *row = reinterpret_cast<uint4 *>(a.G + (int64_t)jr * a.G_ld);
+        for (int t = 0; t < a.ntiles; ++t) {
+            const float mt = __ldcg(&a.part[(int64_t)(a.tile0 + t) * L + jr].x);
+            const float sc = (mt - r > kCeRefJump) ? exp2f(mt - mcr) : exp2f(r - mcr);
+            for (int q = lane; q < per_tile; q += 32) {
+                uint4 u = row[t * per_tile + q];
+                uint32_t *wd = reinterpret_cast<uint32_t *>(&u);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162 *>(&wd[e]);
+                    const float2 v = __bfloat1622float2(b);
+                    b = __floats2bfloat162_rn(v.x * sc, v.y * sc);
+                    wd[e] = *reinterpret_cast<uint32_t *>(&b);
+                }
+                row[t * per_tile + q] = u;
+            }
+        }
     }
-}
-
-// dh_j = (w_j / L) (acc_j exp(A_j - lse_j) - W_{x_j}); one block per row.
-__global__ void __launch_bounds__(256) ce_fixup_kernel(float *dh, int64_t d, const __nv_bfloat16 *__restrict__ W,
-                                                       const int32_t *__restrict__ tgt, const float *__restrict__ w,
-                                                       float inv_L, const float *__restrict__ aref,
-                                                       const float *__restrict__ lse, int V) {
-    const int j = blockIdx.x;
-    const int t = tgt[j];
-    const float c = w[j] * inv_L;
-    const float sc = exp2f(aref[j] - lse[j] * kLog2e);
-    float *row = dh + (int64_t)j * d;
-    if (t < 0 || t >= V) {
-        for (int64_t k = threadIdx.x; k < d; k += blockDim.x) row[k] = __int_as_float(0x7fc00000);
-        return;
-    }
-    const __nv_bfloat16 *wt = W + (int64_t)t * d;
-    // d % 8 == 0: 8 columns per step (one 16-byte load of W, two float4 of dh)
-    for (int64_t k = (int64_t)threadIdx.x * 8; k < d; k += (int64_t)blockDim.x * 8) {
-        const uint4 u = *reinterpret_cast<const uint4 *>(wt + k);
-        const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&u);
-        float4 *o = reinterpret_cast<float4 *>(row + k);
-        float4 a0 = o[0], a1 = o[1];
-        const float2 w0 = __bfloat1622float2(b[0]), w1 = __bfloat1622float2(b[1]);
-        const float2 w2 = __bfloat1622float2(b[2]), w3 = __bfloat1622float2(b[3]);
-        a0.x = c * (a0.x * sc - w0.x); a0.y = c * (a0.y * sc - w0.y);
-        a0.z = c * (a0.z * sc - w1.x); a0.w = c * (a0.w * sc - w1.y);
-        a1.x = c * (a1.x * sc - w2.x); a1.y = c * (a1.y * sc - w2.y);
-        a1.z = c * (a1.z * sc - w3.x); a1.w = c * (a1.w * sc - w3.y);
-        o[0] = a0;
-        o[1] = a1;
+    if (a.last && s_last && threadIdx.x == 0) {
+        __threadfence();
+        float total = 0.f;
+        for (unsigned i = 0; i < gridDim.x; ++i) total += __ldcg(a.block_sums + i);
+        *a.loss = total * a.inv_L;
+        *a.ticket = 0u;
     }
 }
 
@@ -295,15 +337,21 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
     if (!status) return ATTT_ERR_CUDA;
 
     CeLayout c = ce_layout(d_ws, L, d, V);
-    float *lse = d_lse ? d_lse : c.lse_tmp;
     if (cudaMemsetAsync(c.ticket, 0, sizeof(unsigned int) * (4 + (size_t)c.split_regions), stream) != cudaSuccess)
         return ATTT_ERR_CUDA;
+
+    ce_ref_kernel<<<(unsigned)cdiv(L, 8), 256, 0, stream>>>(reinterpret_cast<const __nv_bfloat16 *>(d_h),
+                                                            reinterpret_cast<const __nv_bfloat16 *>(d_W), d_tgt,
+                                                            (int)L, d, (int)V, c.mref);
+    count_launch();
+    if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
 
     const CePlan plan = ce_plan(L, d, V, num_sms(dev));
     for (int64_t v0 = 0, ci = 0; v0 < V; v0 += plan.Vc, ++ci) {
         const int64_t Nc = (V - v0 < plan.Vc) ? V - v0 : plan.Vc;
         const int ntiles = (int)cdiv(Nc, kCeBN);
-        {   // GEMM1: logits of the chunk -> per-tile stats and E = exp(z - m_t)
+        const bool last = v0 + Nc >= V;
+        {   // GEMM1: logits of the chunk -> per-tile stats and E = exp(z - R)
             GemmProblem p{};
             p.a = d_h; p.a_rows_ld = d; p.a_rows = L; p.a_k = d;
             p.b = d_W; p.b_rows_ld = d; p.b_rows = V; p.b_k = d;
@@ -312,13 +360,19 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
             EpiParams ep{};
             ep.tgt = d_tgt; ep.part = c.part; ep.tile0 = (int)(v0 / kCeBN); ep.ztgt = c.ztgt; ep.v0 = (int)v0;
             ep.G = c.G; ep.G_ld = c.Vc;
-            ep.eref = ci == 0 ? nullptr : c.mref;
+            ep.eref = c.mref;
             st = launch_gemm<EPI_CE_EXP, false, false>(p, ep, dev, stream);
             if (st != ATTT_OK) return st;
         }
-        ce_chunk_kernel<<<(unsigned)cdiv(L, 8), 256, 0, stream>>>(c.part, (int)(v0 / kCeBN), ntiles, (int)L, c.G,
-                                                                  c.Vc, c.aref, c.mref, c.alpha, c.beta,
-                                                                  ci == 0 ? 1 : 0);
+        CeChunkArgs ca{};
+        ca.part = c.part; ca.tile0 = (int)(v0 / kCeBN); ca.ntiles = ntiles; ca.L = (int)L; ca.V = (int)V;
+        ca.G = c.G; ca.G_ld = c.Vc;
+        ca.aref = c.aref; ca.mref = c.mref; ca.lm = c.lm; ca.ls = c.ls;
+        ca.alpha = c.alpha; ca.beta = c.beta; ca.gamma = c.gamma;
+        ca.first = ci == 0 ? 1 : 0; ca.last = last ? 1 : 0;
+        ca.ztgt = c.ztgt; ca.tgt = d_tgt; ca.w = d_w; ca.inv_L = 1.0f / (float)L; ca.lse_out = d_lse;
+        ca.block_sums = c.block_sums; ca.ticket = c.ticket; ca.loss = d_loss; ca.status = status;
+        ce_chunk_kernel<<<(unsigned)c.nblk, kChunkWarps * 32, 0, stream>>>(ca);
         count_launch();
         if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
         {   // GEMM2: acc = alpha * acc + beta * (E W_c)
@@ -330,20 +384,15 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
             EpiParams ep{};
             ep.out = d_dh; ep.out_ld = d; ep.accumulate = ci > 0 ? 1 : 0; ep.alpha = 1.0f;
             ep.row_alpha = c.alpha; ep.row_beta = c.beta;
+            if (last) {  // dh = (w/L) (acc exp(A - lse) - W_target), factors folded by the chunk kernel
+                ep.row_gamma = c.gamma; ep.fix_tgt = d_tgt;
+                ep.fix_W = reinterpret_cast<const __nv_bfloat16 *>(d_W); ep.fix_ld = d; ep.fix_V = (int)V;
+            }
             p.split_ws = c.split_ws; p.split_tick = c.split_tick; p.split_regions = c.split_regions;
             st = launch_gemm<EPI_F32_ACC, false, true>(p, ep, dev, stream);
             if (st != ATTT_OK) return st;
         }
     }
-    ce_finalize_kernel<<<(unsigned)c.nblk, kFinThreads, 0, stream>>>(c.part, (int)c.nvt, c.ztgt, d_tgt, d_w, (int)L,
-                                                                     (int)V, lse, 1.0f / (float)L, c.block_sums,
-                                                                     c.ticket, d_loss, status);
-    count_launch();
-    if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
-    ce_fixup_kernel<<<(unsigned)L, 256, 0, stream>>>(d_dh, d, reinterpret_cast<const __nv_bfloat16 *>(d_W), d_tgt,
-                                                     d_w, 1.0f / (float)L, c.aref, lse, (int)V);
-    count_launch();
-    if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
     return ATTT_OK;
 }
 

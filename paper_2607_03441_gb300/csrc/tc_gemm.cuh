@@ -28,7 +28,7 @@ namespace attt {
 
 enum EpiKind : int {
     EPI_CE_EXP = 0,    // per (row, vocab tile): max m, E = exp(z - m) as bf16, sum of E, target logit
-    EPI_F32_ACC = 2,   // out[m, n] = (acc ? alpha_m out[m, n] : 0) + beta_m acc  (fp32, row-major)
+    EPI_F32_ACC = 2,   // out[m, n] = (acc ? alpha_m out[m, n] : 0) + beta_m acc [- gamma_m W[t_m, n]]  (fp32)
     EPI_ATOMIC_T = 3,  // out[n, m] += alpha * acc   (fp32, transposed, split-K)
     EPI_ATOMIC_N = 4,  // out_p[m, c] += alpha * acc for column n = p * rpad + c (split-K)
 };
@@ -52,6 +52,11 @@ struct EpiParams {
     float alpha;
     const float *row_alpha;  // [M] or nullptr (1)
     const float *row_beta;   // [M] or nullptr (1)
+    const float *row_gamma;  // [M] or nullptr (no W term)
+    const int32_t *fix_tgt;  // [M] row of fix_W each output row subtracts (clamped into [0, fix_V))
+    const __nv_bfloat16 *fix_W;
+    int64_t fix_ld;
+    int fix_V;
     __nv_bfloat16 *out16;    // grouped EPI_ATOMIC_T: bf16 copy of out, written by the last split
     unsigned int *tickets;   // grouped EPI_ATOMIC_T: one counter per tile, starts at 0
     float *outp[kMaxProj];
@@ -118,29 +123,76 @@ __device__ __forceinline__ int work_count(const GemmArgs &g, int tiles_m) {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
-// A CE tile whose max exceeds the row reference by more than 2^kCeRefJump
-// (log2 units) writes E against its own max instead, so E <= 2^kCeRefJump.
-constexpr float kCeRefJump = 32.f;
+// A CE tile whose max exceeds the row reference by more than kCeRefJump
+// (log2 units) writes E against its own max instead, so E <= 2^64.  The dh
+// contraction of a chunk sums at most 2^16 such terms times |W|, and the fp32
+// accumulator holds that for |W| up to 2^40.
+constexpr float kCeRefJump = 64.f;
 
-// out[gm, col0 + i] = (accumulate ? ra * out : 0) + rb * v[i] for the 32
-// columns of one TMEM chunk (EPI_F32_ACC), nothing at or past n_end.
-__device__ __forceinline__ void f32_acc_store(const EpiParams &ep, float *orow, int col0, int n_end, float ra,
-                                              float rb, const float (&v)[32]) {
+// Per-row terms of EPI_F32_ACC for output row gm: ra, rb and, when the
+// epilogue subtracts gamma_m W[t_m, :], gamma and that row of W.
+struct AccRow {
+    float ra, rb, gam;
+    const __nv_bfloat16 *wrow;
+};
+
+__device__ __forceinline__ AccRow acc_row(const EpiParams &ep, int gm, bool rv) {
+    AccRow a{1.f, 1.f, 0.f, nullptr};
+    if (rv) {
+        if (ep.row_alpha) a.ra = __ldg(ep.row_alpha + gm);
+        if (ep.row_beta) a.rb = __ldg(ep.row_beta + gm);
+        if (ep.row_gamma) {
+            a.gam = __ldg(ep.row_gamma + gm);
+            int t = __ldg(ep.fix_tgt + gm);
+            if (t < 0 || t >= ep.fix_V) t = 0;
+            a.wrow = ep.fix_W + (int64_t)t * ep.fix_ld;
+        }
+    }
+    return a;
+}
+
+// out[gm, col0 + i] = (accumulate ? ra * out : 0) + rb * v[i] - gam * W[t, col0 + i]
+// for the 32 columns of one TMEM chunk (EPI_F32_ACC), nothing at or past
+// n_end.  The W row (when present) is 16-byte aligned with col0 % 32 == 0.
+__device__ __forceinline__ void f32_acc_store(const EpiParams &ep, float *orow, int col0, int n_end,
+                                              const AccRow &a, const float (&v)[32]) {
     if (col0 + 32 <= n_end) {
+        float wv[32];
+        if (a.wrow) {
+            const uint4 *src = reinterpret_cast<const uint4 *>(a.wrow + col0);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint4 u = __ldg(src + q);
+                const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float2 f = __bfloat1622float2(b[e]);
+                    wv[8 * q + 2 * e] = f.x;
+                    wv[8 * q + 2 * e + 1] = f.y;
+                }
+            }
+        }
         float4 *dst = reinterpret_cast<float4 *>(orow + col0);
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
-            float4 o = make_float4(rb * v[4 * q], rb * v[4 * q + 1], rb * v[4 * q + 2], rb * v[4 * q + 3]);
+            float4 o = make_float4(a.rb * v[4 * q], a.rb * v[4 * q + 1], a.rb * v[4 * q + 2], a.rb * v[4 * q + 3]);
             if (ep.accumulate) {
                 const float4 p = dst[q];
-                o.x = fmaf(ra, p.x, o.x); o.y = fmaf(ra, p.y, o.y);
-                o.z = fmaf(ra, p.z, o.z); o.w = fmaf(ra, p.w, o.w);
+                o.x = fmaf(a.ra, p.x, o.x); o.y = fmaf(a.ra, p.y, o.y);
+                o.z = fmaf(a.ra, p.z, o.z); o.w = fmaf(a.ra, p.w, o.w);
+            }
+            if (a.wrow) {
+                o.x = fmaf(-a.gam, wv[4 * q], o.x); o.y = fmaf(-a.gam, wv[4 * q + 1], o.y);
+                o.z = fmaf(-a.gam, wv[4 * q + 2], o.z); o.w = fmaf(-a.gam, wv[4 * q + 3], o.w);
             }
             dst[q] = o;
         }
     } else {
-        for (int i = 0; i < 32 && col0 + i < n_end; ++i)
-            orow[col0 + i] = ep.accumulate ? fmaf(ra, orow[col0 + i], rb * v[i]) : rb * v[i];
+        for (int i = 0; i < 32 && col0 + i < n_end; ++i) {
+            float o = ep.accumulate ? fmaf(a.ra, orow[col0 + i], a.rb * v[i]) : a.rb * v[i];
+            if (a.wrow) o = fmaf(-a.gam, __bfloat162float(a.wrow[col0 + i]), o);
+            orow[col0 + i] = o;
+        }
     }
 }
 
@@ -224,14 +276,12 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
         }
     } else if constexpr (EPI == EPI_F32_ACC) {
         float *orow = ep.out + (int64_t)gm * ep.out_ld;
-        float ra = 1.f, rb = 1.f;
-        if (rv && ep.row_alpha) ra = __ldg(ep.row_alpha + gm);
-        if (rv && ep.row_beta) rb = __ldg(ep.row_beta + gm);
+        const AccRow a = acc_row(ep, gm, rv);
         for (int c = 0; c < g.BN; c += 32) {
             if (n_base + c >= n_end) break;
             float v[32];
             tmem_ld_x32(taddr + (uint32_t)c, v);
-            if (rv) f32_acc_store(ep, orow, n_base + c, n_end, ra, rb, v);
+            if (rv) f32_acc_store(ep, orow, n_base + c, n_end, a, v);
         }
     } else if constexpr (EPI == EPI_ATOMIC_T) {
         for (int c = 0; c < g.BN; c += 16) {
@@ -301,9 +351,7 @@ __device__ __forceinline__ void epilogue_piece_f32_acc(const GemmArgs &g, const 
     const bool rv = gm < g.M;
     const int n_base = k.tn * BN;
     const int n_end = min(g.N, n_base + BN);
-    float ra = 1.f, rb = 1.f;
-    if (rv && ep.row_alpha) ra = __ldg(ep.row_alpha + gm);
-    if (rv && ep.row_beta) rb = __ldg(ep.row_beta + gm);
+    const AccRow a = acc_row(ep, gm, rv);
     float *orow = ep.out + (int64_t)gm * ep.out_ld;
     for (int c = 0; c < BN; c += 32) {
         if (n_base + c >= n_end) break;
@@ -324,7 +372,7 @@ __device__ __forceinline__ void epilogue_piece_f32_acc(const GemmArgs &g, const 
 #pragma unroll
             for (int i = 0; i < 32; ++i) s[i] = (j == 0) ? v[i] : s[i] + v[i];
         }
-        if (rv) f32_acc_store(ep, orow, n_base + c, n_end, ra, rb, s);
+        if (rv) f32_acc_store(ep, orow, n_base + c, n_end, a, s);
     }
 }
 

@@ -99,6 +99,19 @@ def test_target_out_of_range(attt):
     assert np.isnan(loss.item())
     assert attt.attt_device_status() == 3  # ATTT_ERR_TOKEN_RANGE
     assert attt.attt_device_status() == 0  # read clears it
+    # the row with the bad target is NaN; every other row is still exact
+    w = np.ones(L, np.float32)
+    lse_t = torch.empty(L, dtype=torch.float32, device=DEV)
+    _, dh_t, _ = attt.attt_weighted_ce_fwd_bwd(bf16_dev(h), bf16_dev(W), i32_dev(tgt), f32_dev(w), lse=lse_t)
+    assert attt.attt_device_status() == 3
+    dh = dh_t.cpu().numpy()
+    assert np.all(np.isnan(dh[3]))
+    rows = np.array([j for j in range(L) if j != 3], np.int64)
+    tgt_ok = tgt.copy()
+    tgt_ok[3] = 0
+    rlse, _, rdh = oracle.ce_rows(h, W, tgt_ok, w, rows)
+    np.testing.assert_allclose(lse_t.cpu().numpy()[rows], rlse, atol=LSE_ATOL, rtol=0)
+    assert rel_l2(dh[rows], rdh) < DH_RL2
 
 
 def test_bad_arguments(attt):
@@ -155,18 +168,21 @@ def test_32b_sampled(attt):
 
 
 def test_multichunk_with_reference_jumps(attt):
-    """Several vocab chunks, with rows whose max logit jumps far above the
-    running max of the earlier chunks (2^92 in log2 units) and rows whose
-    later chunks sit far below it; sampled rows against the oracle."""
+    """Several vocab chunks, with rows whose max logit sits far above their
+    reference (the target logit, then the running max): 2^92 in log2 units
+    (E rewritten, in the first chunk for row 1500, the last for row 77) and
+    2^61 (E written up to 2^61, no rewrite: rows 300 and 900); row 5's target
+    is its max, so the chunks before it sit far below the reference; sampled
+    rows against the oracle."""
     L, V, d = 2048, 80000, 64
     rng = wk.rng_for(77, "jump")
     h = wk.normal_bf16(77, "h", (L, d), 0.5)
     W = wk.normal_bf16(77, "W", (V, d), 0.05)
-    hot_rows = [5, 77, 1500]
-    for j, v in zip(hot_rows, [60000, 79999, 30]):
+    hot_rows = [5, 77, 1500, 300, 900]
+    for j, v, x in zip(hot_rows, [60000, 79999, 30, 100, 50000], [8.0, 8.0, 8.0, 6.5, 6.5]):
         h[j] = 0
-        h[j, 0] = wk.bf16_bits(np.array([8.0], np.float32))[0]
-        W[v, 0] = wk.bf16_bits(np.array([8.0], np.float32))[0]  # z[j, v] = 64
+        h[j, 0] = wk.bf16_bits(np.array([x], np.float32))[0]
+        W[v, 0] = wk.bf16_bits(np.array([x], np.float32))[0]  # z[j, v] = x^2 (64 or 42.25)
     tgt = rng.integers(0, V, L).astype(np.int32)
     tgt[5] = 60000
     w = rng.choice(np.array([1.0, 0.5, 0.05], np.float32), L).astype(np.float32)
@@ -207,8 +223,8 @@ def test_tail_pieces_deterministic(attt, L, V, d):
 
 
 def test_launch_counter_counts_every_kernel(attt):
-    """One single-chunk call launches GEMM1, the chunk kernel, GEMM2, the
-    finalize and the fixup kernels: five kernels, all counted."""
+    """One single-chunk call launches the reference kernel, GEMM1, the chunk
+    kernel and GEMM2: four kernels, all counted."""
     L, V, d = 200, 1000, 64
     h = wk.normal_bf16(8, "h", (L, d), 1.0)
     W = wk.normal_bf16(8, "W", (V, d), 0.1)
@@ -217,4 +233,4 @@ def test_launch_counter_counts_every_kernel(attt):
     attt.attt_weighted_ce_fwd_bwd(*args)
     n0 = attt.attt_kernel_launches()
     attt.attt_weighted_ce_fwd_bwd(*args)
-    assert attt.attt_kernel_launches() - n0 == 5
+    assert attt.attt_kernel_launches() - n0 == 4
