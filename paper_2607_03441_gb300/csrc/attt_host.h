@@ -20,11 +20,12 @@ int num_sms(int dev);
 // Per-device status word used by the contraction kernels (lazily allocated).
 int *device_status_word(int dev);
 
-// Encodes a 2-D bf16 tensor map with 128-byte swizzle and zero fill for
-// out-of-range elements.  `inner` is the contiguous extent, `outer` the number
-// of rows, `row_bytes` the row pitch.  Returns false if the driver rejects it.
+// Encodes a 2-D bf16 tensor map with zero fill for out-of-range elements and
+// a shared-memory swizzle of `swizzle_bytes` (128, 64, or 0 for none).
+// `inner` is the contiguous extent, `outer` the number of rows, `row_bytes`
+// the row pitch.  Returns false if the driver rejects it.
 bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
-                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer);
+                    uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle_bytes = 128);
 
 // Counts one kernel launch (attt_kernel_launches).
 void count_launch();

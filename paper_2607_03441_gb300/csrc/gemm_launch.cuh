@@ -49,9 +49,9 @@ inline int tail_pieces(int tiles, int units, int kb_total, int nranks, int regio
 
 constexpr size_t kMaxSmem = 232448;  // 227 KB opt-in per CTA on sm_100-class parts
 
-inline int gemm_stages(int BN) {
+inline int gemm_stages(int BN, uint32_t extra = 0) {
     int s = 8;
-    while (s > 2 && gemm_smem_bytes(BN, s) > kMaxSmem) --s;
+    while (s > 2 && gemm_smem_bytes(BN, s, extra) > kMaxSmem) --s;
     return s;
 }
 
@@ -85,13 +85,20 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     else
         ok = make_tmap_bf16(&tb, p.b, (uint64_t)p.b_rows, (uint64_t)p.b_k, (uint64_t)p.b_rows_ld * 2, 64, 64);
     if (!ok) return ATTT_ERR_INVALID_ARG;
+    // EPI_CE_EXP writes E through TMA stores: [M, G_ld] bf16, 32 x 32 boxes
+    CUtensorMap tc = tb;
+    if (EPI == EPI_CE_EXP) {
+        if (!make_tmap_bf16(&tc, ep.G, (uint64_t)ep.G_ld, (uint64_t)p.M, (uint64_t)ep.G_ld * 2, 32, 32, 64))
+            return ATTT_ERR_INVALID_ARG;
+    }
 
     GemmArgs g{};
     g.M = p.M;
     g.N = p.N;
     g.BN = p.BN;
     const int bn_cta = p.pair ? p.BN / 2 : p.BN;  // B rows one CTA stages
-    g.stages = gemm_stages(bn_cta);
+    g.e_stage_bytes = EPI == EPI_CE_EXP ? kEStageBytes : 0u;
+    g.stages = gemm_stages(bn_cta, g.e_stage_bytes);
     g.tiles_m = (int)cdiv(p.M, 128);
     g.tiles_n = (int)cdiv(p.N, p.BN);
     g.kb_total = (int)cdiv(p.K, 64);
@@ -119,13 +126,13 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.status = status ? status : device_status_word(dev);
     g.ep = ep;
 
-    const size_t smem = gemm_smem_bytes(bn_cta, g.stages);
+    const size_t smem = gemm_smem_bytes(bn_cta, g.stages, g.e_stage_bytes);
     const int ntiles = g.whole_tiles + (tiles - g.whole_tiles) * g.tail_s;  // work items
     if (!p.pair) {
         auto kern = tc_gemm_kernel<EPI, A_MN, B_MN>;
         if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
         const int grid = ntiles < sms ? ntiles : sms;
-        kern<<<grid, kGemmThreads, smem, stream>>>(ta, tb, g);
+        kern<<<grid, kGemmThreads, smem, stream>>>(ta, tb, tc, g);
     } else {
         auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN>;
         if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
@@ -142,7 +149,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
         attr[0].val.clusterDim.z = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        if (cudaLaunchKernelEx(&cfg, kern, ta, tb, g) != cudaSuccess) return ATTT_ERR_CUDA;
+        if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, g) != cudaSuccess) return ATTT_ERR_CUDA;
     }
     count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;

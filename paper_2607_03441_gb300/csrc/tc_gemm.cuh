@@ -72,6 +72,7 @@ struct GemmArgs {
     int a_m_off, a_k_off;  // coordinate offsets into A's tensor map
     int b_n_off, b_k_off;  // coordinate offsets into B's tensor map
     uint32_t tmem_cols;
+    uint32_t e_stage_bytes;  // shared-memory staging of the TMA-stored epilogue output (EPI_CE_EXP), else 0
     int *status;
     EpiParams ep;
     // Tail split (tc_gemm_kernel / tc_gemm_pair_kernel): tiles [0, whole_tiles)
@@ -86,8 +87,36 @@ constexpr int kGemmThreads = 192;
 
 __host__ __device__ inline uint32_t gemm_b_stage_bytes(int BN) { return (uint32_t)BN * 128u; }
 
-__host__ __device__ inline size_t gemm_smem_bytes(int BN, int stages) {
-    return 1024 + (size_t)stages * (kABytes + gemm_b_stage_bytes(BN)) + 8 * (2 * stages + 5) + 16;
+// EPI_CE_EXP stages E through shared memory: per epilogue warp two buffers of
+// 32 rows x 32 bf16 (64-byte swizzle), written out by TMA stores.
+constexpr uint32_t kEStageBytes = 4 * 2 * 32 * 64;
+
+__host__ __device__ inline size_t gemm_smem_bytes(int BN, int stages, uint32_t extra = 0) {
+    return 1024 + (size_t)stages * (kABytes + gemm_b_stage_bytes(BN)) + extra + 8 * (2 * stages + 5) + 16;
+}
+
+// One 32 x 32 bf16 block of E (this warp's 32 rows, 32 columns from x) to
+// global memory through the warp's staging buffer `chunk & 1`: lane = row,
+// 16-byte pieces placed as the 64-byte swizzle expects (piece q of row r at
+// q ^ ((r >> 1) & 3)), so the 8 lanes of each quarter-warp hit distinct banks.
+// Lane 0 owns the bulk group; before a buffer is refilled, the store that used
+// it two blocks ago has finished reading it.
+__device__ __forceinline__ void e_block_store(const CUtensorMap *tm, uint32_t sbuf, int chunk, int lane,
+                                              const uint32_t (&pk)[16], int x, int y) {
+    const uint32_t buf = sbuf + (uint32_t)(chunk & 1) * 2048u;
+    if (lane == 0) bulk_wait_read<1>();
+    __syncwarp();
+    const uint32_t rowp = buf + (uint32_t)lane * 64u;
+    const uint32_t sw = ((uint32_t)lane >> 1) & 3u;
+#pragma unroll
+    for (uint32_t q = 0; q < 4; ++q)
+        st_shared_v4(rowp + ((q ^ sw) << 4), pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+        tma_store_2d(tm, buf, x, y);
+        bulk_commit();
+    }
 }
 
 // One unit of work of tc_gemm_kernel / tc_gemm_pair_kernel: an output tile
@@ -202,8 +231,10 @@ __device__ __forceinline__ void f32_acc_store(const EpiParams &ep, float *orow, 
 // past M (the loads are warp-collective); only stores are predicated.
 // ---------------------------------------------------------------------------
 
+// tmE / sE: the E tensor map and this warp's staging buffers (EPI_CE_EXP).
 template <int EPI>
-__device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, int tn, int row, uint32_t taddr) {
+__device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, int tn, int row, uint32_t taddr,
+                                              const CUtensorMap *tmE = nullptr, uint32_t sE = 0) {
     const int gm = gm_base + row;
     const bool rv = gm < g.M;
     const int n_base = tn * g.BN;
@@ -216,59 +247,96 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
     const EpiParams &ep = g.ep;
 
     if constexpr (EPI == EPI_CE_EXP) {
-        // Pass 1 over the tile's columns: the row max (log2 units) and the
-        // target logit.  Pass 2: E = exp(z - max) rounded to bf16 into the
-        // gradient block (columns past N as zeros), and the sum of the
-        // unrounded exponentials.
+        // One pass over the tile's columns against the row reference R
+        // (log2 units): E = exp2(z2 - R) rounded to bf16 into the gradient
+        // block (columns past N as zeros), the tile max m, the sum of the
+        // unrounded exp2(z2 - R) and the target logit.  The pair stored is
+        // (m, sum of exp2(z2 - m)).  A row whose tile max exceeds R by more
+        // than kCeRefJump (or has no reference) takes a second pass that
+        // writes E = exp2(z2 - m) instead; that pass is warp-wide because TMEM
+        // loads are.
         const int t = rv ? __ldg(ep.tgt + gm) - ep.v0 : -1;
-        float mx = -INFINITY, zt = 0.f;
+        const float R = (ep.eref && rv) ? __ldg(ep.eref + gm) : -INFINITY;
+        const int lane = row & 31, y = gm - lane;
+        float mx = -INFINITY, zt = 0.f, sr = 0.f;
         bool hit = false;
         for (int c = 0; c < g.BN; c += 32) {
-            if (n_base + c >= n_end) break;
             float v[32];
             tmem_ld_x32(taddr + (uint32_t)c, v);
+            const int col0 = n_base + c;
+            const int tc = t - col0;
+            uint32_t pk[16];
+            if (col0 + 32 <= n_end) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                const int col = n_base + c + i;
-                if (col < n_end) {
-                    if (col == t) { zt = v[i]; hit = true; }
-                    mx = fmaxf(mx, v[i] * kLog2e);
+                for (int i = 0; i < 32; i += 2) {
+                    const float z0 = v[i] * kLog2e, z1 = v[i + 1] * kLog2e;
+                    mx = fmaxf(mx, fmaxf(z0, z1));
+                    if (tc == i) { zt = v[i]; hit = true; }
+                    if (tc == i + 1) { zt = v[i + 1]; hit = true; }
+                    const float e0 = exp2f(z0 - R), e1 = exp2f(z1 - R);
+                    sr += e0 + e1;
+                    __nv_bfloat162 b = __floats2bfloat162_rn(e0, e1);
+                    pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; i += 2) {
+                    float e0 = 0.f, e1 = 0.f;
+                    if (col0 + i < n_end) {
+                        const float z0 = v[i] * kLog2e;
+                        mx = fmaxf(mx, z0);
+                        if (tc == i) { zt = v[i]; hit = true; }
+                        e0 = exp2f(z0 - R);
+                    }
+                    if (col0 + i + 1 < n_end) {
+                        const float z1 = v[i + 1] * kLog2e;
+                        mx = fmaxf(mx, z1);
+                        if (tc == i + 1) { zt = v[i + 1]; hit = true; }
+                        e1 = exp2f(z1 - R);
+                    }
+                    sr += e0 + e1;
+                    __nv_bfloat162 b = __floats2bfloat162_rn(e0, e1);
+                    pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
                 }
             }
+            // zeros past N (inside the tile) are stored too: the dh
+            // contraction reads whole 64-column K blocks; rows past M are
+            // clipped by the tensor map
+            e_block_store(tmE, sE, c >> 5, lane, pk, col0, y);
         }
-        float sm = 0.f;
-        // E = exp2(z2 - mx) * sc: against the row reference R given by the
-        // caller (sc = exp2(mx - R)), or against the tile max (sc = 1) when
-        // there is none or mx - R > kCeRefJump.  The sum is always taken
-        // against the tile max.
-        float sc = 1.f;
-        if (ep.eref && rv) {
-            const float jump = mx - __ldg(ep.eref + gm);
-            if (jump <= kCeRefJump) sc = exp2f(jump);
+        const bool own = rv && !(mx - R <= kCeRefJump);
+        float sm;
+        if (!own) {
+            // sum against m from the sum against R; when R - m >= 100 every
+            // term against R may have underflowed, and such a tile is below
+            // 2^-92 of the row's sum (R is at most the row max)
+            const float dd = R - mx;
+            sm = (dd < 100.f) ? sr * exp2f(dd) : (sr > 0.f ? exp2f(log2f(sr) + dd) : 1.f);
         }
-        __nv_bfloat16 *grow = ep.G + (int64_t)gm * ep.G_ld;
-        for (int c = 0; c < g.BN; c += 32) {
-            float v[32];
-            tmem_ld_x32(taddr + (uint32_t)c, v);
-            uint32_t pk[16];
+        if (__any_sync(0xffffffffu, own)) {
+            // the warp's blocks again, after the first pass's stores have
+            // landed: rows against their own max, the others as before
+            if (lane == 0) bulk_wait<0>();
+            __syncwarp();
+            float so = 0.f;
+            for (int c = 0; c < g.BN; c += 32) {
+                float v[32];
+                tmem_ld_x32(taddr + (uint32_t)c, v);
+                const int col0 = n_base + c;
+                uint32_t pk[16];
 #pragma unroll
-            for (int i = 0; i < 32; i += 2) {
-                const int col = n_base + c + i;
-                const float e0 = (col < n_end) ? exp2f(fmaf(v[i], kLog2e, -mx)) : 0.f;
-                const float e1 = (col + 1 < n_end) ? exp2f(fmaf(v[i + 1], kLog2e, -mx)) : 0.f;
-                sm += e0 + e1;
-                __nv_bfloat162 b = __floats2bfloat162_rn(e0 * sc, e1 * sc);
-                pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
+                for (int i = 0; i < 32; i += 2) {
+                    float e0 = 0.f, e1 = 0.f;
+                    if (col0 + i < n_end) e0 = own ? exp2f(fmaf(v[i], kLog2e, -mx)) : exp2f(v[i] * kLog2e - R);
+                    if (col0 + i + 1 < n_end)
+                        e1 = own ? exp2f(fmaf(v[i + 1], kLog2e, -mx)) : exp2f(v[i + 1] * kLog2e - R);
+                    so += e0 + e1;
+                    __nv_bfloat162 b = __floats2bfloat162_rn(e0, e1);
+                    pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
+                }
+                e_block_store(tmE, sE, c >> 5, lane, pk, col0, y);
             }
-            if (rv) {
-                // zeros past N (inside the tile) are stored too: the dh
-                // contraction reads whole 64-column K blocks
-                uint4 *dst = reinterpret_cast<uint4 *>(grow + n_base + c);
-#pragma unroll
-                for (int q = 0; q < 4; ++q)
-                    if (n_base + c + 8 * q < n_tile)
-                        dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-            }
+            if (own) sm = so;
         }
         if (rv) {
             ep.part[(int64_t)(ep.tile0 + tn) * g.M + gm] = make_float2(mx, sm);
@@ -383,14 +451,15 @@ __device__ __forceinline__ void epilogue_piece_f32_acc(const GemmArgs &g, const 
 template <int EPI, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const GemmArgs g) {
+                   const __grid_constant__ CUtensorMap tmC, const GemmArgs g) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = g.stages;
     const uint32_t b_bytes = gemm_b_stage_bytes(g.BN);
     uint8_t *sA = smem;
     uint8_t *sB = smem + (size_t)S * kABytes;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + (size_t)S * b_bytes);
+    uint8_t *sE = sB + (size_t)S * b_bytes;  // 1024-byte aligned: b_bytes is a multiple of 2048
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sE + g.e_stage_bytes);
     const uint32_t full0 = smem_u32(bars);
     const uint32_t empty0 = smem_u32(bars + S);
     const uint32_t tfull0 = smem_u32(bars + 2 * S);
@@ -540,11 +609,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 else
                     epilogue_tile<EPI>(g, wi.tm * 128, wi.tn, row, taddr);
             } else {
-                epilogue_tile<EPI>(g, wi.tm * 128, wi.tn, row, taddr);
+                epilogue_tile<EPI>(g, wi.tm * 128, wi.tn, row, taddr, &tmC, smem_u32(sE) + (uint32_t)q * 4096u);
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
+        }
+        // every TMA store of E has landed before the CTA retires
+        if constexpr (EPI == EPI_CE_EXP) {
+            if (lane == 0) bulk_wait<0>();
         }
     }
 
@@ -567,7 +640,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 template <int EPI, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                        const GemmArgs g) {
+                   const __grid_constant__ CUtensorMap tmC, const GemmArgs g) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = g.stages;
@@ -575,7 +648,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t b_bytes = gemm_b_stage_bytes(BNh);
     uint8_t *sA = smem;
     uint8_t *sB = smem + (size_t)S * kABytes;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + (size_t)S * b_bytes);
+    uint8_t *sE = sB + (size_t)S * b_bytes;  // 1024-byte aligned: b_bytes is a multiple of 2048
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sE + g.e_stage_bytes);
     const uint32_t full0 = smem_u32(bars);
     const uint32_t empty0 = smem_u32(bars + S);
     const uint32_t tfull0 = smem_u32(bars + 2 * S);
@@ -725,11 +799,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 else
                     epilogue_tile<EPI>(g, gm_base, wi.tn, row, taddr);
             } else {
-                epilogue_tile<EPI>(g, gm_base, wi.tn, row, taddr);
+                epilogue_tile<EPI>(g, gm_base, wi.tn, row, taddr, &tmC, smem_u32(sE) + (uint32_t)q * 4096u);
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(lead_tempty0 + 8 * acc);
+        }
+        // every TMA store of E has landed before the CTA retires
+        if constexpr (EPI == EPI_CE_EXP) {
+            if (lane == 0) bulk_wait<0>();
         }
     }
 
