@@ -27,6 +27,10 @@ int *device_status_word(int dev);
 bool make_tmap_bf16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
                     uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle_bytes = 128);
 
+// The same for a 2-D fp32 tensor (128-byte swizzle).
+bool make_tmap_f32(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+                   uint32_t box_inner, uint32_t box_outer);
+
 // Counts one kernel launch (attt_kernel_launches).
 void count_launch();
 

@@ -86,9 +86,13 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
         ok = make_tmap_bf16(&tb, p.b, (uint64_t)p.b_rows, (uint64_t)p.b_k, (uint64_t)p.b_rows_ld * 2, 64, 64);
     if (!ok) return ATTT_ERR_INVALID_ARG;
     // EPI_CE_EXP writes E through TMA stores: [M, G_ld] bf16, 32 x 32 boxes
+    // EPI_F32_ACC reads and writes `out` through TMA: [M, N] fp32 of pitch out_ld, 32 x 32 boxes
     CUtensorMap tc = tb;
     if (EPI == EPI_CE_EXP) {
         if (!make_tmap_bf16(&tc, ep.G, (uint64_t)ep.G_ld, (uint64_t)p.M, (uint64_t)ep.G_ld * 2, 32, 32, 64))
+            return ATTT_ERR_INVALID_ARG;
+    } else if (EPI == EPI_F32_ACC) {
+        if (!make_tmap_f32(&tc, ep.out, (uint64_t)p.N, (uint64_t)p.M, (uint64_t)ep.out_ld * 4, 32, 32))
             return ATTT_ERR_INVALID_ARG;
     }
 
@@ -97,7 +101,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.N = p.N;
     g.BN = p.BN;
     const int bn_cta = p.pair ? p.BN / 2 : p.BN;  // B rows one CTA stages
-    g.e_stage_bytes = EPI == EPI_CE_EXP ? kEStageBytes : 0u;
+    g.e_stage_bytes = EPI == EPI_CE_EXP ? kEStageBytes : EPI == EPI_F32_ACC ? kF32StageBytes : 0u;
     g.stages = gemm_stages(bn_cta, g.e_stage_bytes);
     g.tiles_m = (int)cdiv(p.M, 128);
     g.tiles_n = (int)cdiv(p.N, p.BN);

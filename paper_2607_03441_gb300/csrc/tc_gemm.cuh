@@ -180,56 +180,105 @@ __device__ __forceinline__ AccRow acc_row(const EpiParams &ep, int gm, bool rv) 
     return a;
 }
 
-// out[gm, col0 + i] = (accumulate ? ra * out : 0) + rb * v[i] - gam * W[t, col0 + i]
-// for the 32 columns of one TMEM chunk (EPI_F32_ACC), nothing at or past
-// n_end.  The W row (when present) is 16-byte aligned with col0 % 32 == 0.
-__device__ __forceinline__ void f32_acc_store(const EpiParams &ep, float *orow, int col0, int n_end,
-                                              const AccRow &a, const float (&v)[32]) {
-    if (col0 + 32 <= n_end) {
-        float wv[32];
-        if (a.wrow) {
-            const uint4 *src = reinterpret_cast<const uint4 *>(a.wrow + col0);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint4 u = __ldg(src + q);
-                const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&u);
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float2 f = __bfloat1622float2(b[e]);
-                    wv[8 * q + 2 * e] = f.x;
-                    wv[8 * q + 2 * e + 1] = f.y;
-                }
-            }
-        }
-        float4 *dst = reinterpret_cast<float4 *>(orow + col0);
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            float4 o = make_float4(a.rb * v[4 * q], a.rb * v[4 * q + 1], a.rb * v[4 * q + 2], a.rb * v[4 * q + 3]);
-            if (ep.accumulate) {
-                const float4 p = dst[q];
-                o.x = fmaf(a.ra, p.x, o.x); o.y = fmaf(a.ra, p.y, o.y);
-                o.z = fmaf(a.ra, p.z, o.z); o.w = fmaf(a.ra, p.w, o.w);
-            }
-            if (a.wrow) {
-                o.x = fmaf(-a.gam, wv[4 * q], o.x); o.y = fmaf(-a.gam, wv[4 * q + 1], o.y);
-                o.z = fmaf(-a.gam, wv[4 * q + 2], o.z); o.w = fmaf(-a.gam, wv[4 * q + 3], o.w);
-            }
-            dst[q] = o;
-        }
-    } else {
-        for (int i = 0; i < 32 && col0 + i < n_end; ++i) {
-            float o = ep.accumulate ? fmaf(a.ra, orow[col0 + i], a.rb * v[i]) : a.rb * v[i];
-            if (a.wrow) o = fmaf(-a.gam, __bfloat162float(a.wrow[col0 + i]), o);
-            orow[col0 + i] = o;
-        }
-    }
-}
-
 // ---------------------------------------------------------------------------
 // Epilogues.  Every thread owns accumulator row `row` of the tile; all 32
 // lanes of a warp execute the TMEM loads together even when their row is
 // past M (the loads are warp-collective); only stores are predicated.
 // ---------------------------------------------------------------------------
+
+// EPI_F32_ACC goes through TMA too: per epilogue warp two 32 x 32 fp32 boxes
+// (128-byte swizzle) and one mbarrier each, after the 8 boxes.
+constexpr uint32_t kF32StageBytes = 4 * 2 * 4096 + 64;
+
+struct F32Stage {
+    uint32_t buf0;  // this warp's box 0 (box 1 at +4096)
+    uint32_t bar0;  // its mbarrier 0 (1 at +8)
+    uint32_t ec;    // boxes handled so far: box ec & 1, load parity (ec >> 1) & 1
+};
+
+// TMA load of the old outputs of one box into box `slot`, once the store that
+// last used it has read it (lane 0 owns the bulk group and the barrier).
+__device__ __forceinline__ void f32_box_load(const CUtensorMap *tm, const F32Stage &st, uint32_t slot, int lane,
+                                             int x, int y) {
+    if (lane == 0) {
+        bulk_wait_read<0>();
+        const uint32_t bar = st.bar0 + 8u * slot;
+        mbar_arrive_expect_tx(bar, 4096u);
+        tma_load_2d(st.buf0 + 4096u * slot, tm, bar, x, y);
+    }
+}
+
+// EPI_F32_ACC for this warp's 32 rows (from y; lane = row), box by box over
+// the tile's columns [n_base, n_end): out = (accumulate ? ra out : 0) + rb v
+// - gam W[t, :], where src(c, v) gives the lane's accumulator values of
+// columns n_base + c .. + 31.  The old outputs of the next box load while this
+// one is combined in shared memory; each box goes back by a TMA store (rows
+// past M and columns past N are clipped by the tensor map).
+template <class Src>
+__device__ __forceinline__ void f32_tile_store(const GemmArgs &g, const CUtensorMap *tm, F32Stage &st, int lane,
+                                               int y, const AccRow &a, int n_base, int n_end,
+                                               volatile int *abort_flag, Src &&src) {
+    const EpiParams &ep = g.ep;
+    if (y >= g.M) return;  // every row of this warp lies past M (warp-uniform)
+    const int nch = min(g.BN, n_end - n_base + 31) >> 5;
+    if (ep.accumulate) f32_box_load(tm, st, st.ec & 1u, lane, n_base, y);
+    for (int k = 0; k < nch; ++k, ++st.ec) {
+        const uint32_t slot = st.ec & 1u;
+        const uint32_t buf = st.buf0 + 4096u * slot;
+        const int x = n_base + 32 * k;
+        if (ep.accumulate && k + 1 < nch) f32_box_load(tm, st, slot ^ 1u, lane, x + 32, y);
+        float v[32];
+        src(32 * k, v);
+        float w[32];
+        if (a.wrow) {
+            if (x + 32 <= n_end) {
+                const uint4 *wp = reinterpret_cast<const uint4 *>(a.wrow + x);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint4 u = __ldg(wp + q);
+                    const __nv_bfloat162 *b = reinterpret_cast<const __nv_bfloat162 *>(&u);
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float2 f = __bfloat1622float2(b[e]);
+                        w[8 * q + 2 * e] = f.x;
+                        w[8 * q + 2 * e + 1] = f.y;
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) w[i] = (x + i < n_end) ? __bfloat162float(a.wrow[x + i]) : 0.f;
+            }
+        }
+        if (ep.accumulate) {
+            if (!mbar_wait(st.bar0 + 8u * slot, (st.ec >> 1) & 1u, abort_flag)) record_error(g.status, ATTT_ERR_TIMEOUT);
+        } else if (lane == 0) {
+            bulk_wait_read<1>();  // the store two boxes back has read this box
+        }
+        __syncwarp();
+        const uint32_t rowp = buf + (uint32_t)lane * 128u;
+#pragma unroll
+        for (uint32_t q = 0; q < 8; ++q) {
+            const uint32_t ad = rowp + ((q ^ ((uint32_t)lane & 7u)) << 4);
+            float4 o = make_float4(a.rb * v[4 * q], a.rb * v[4 * q + 1], a.rb * v[4 * q + 2], a.rb * v[4 * q + 3]);
+            if (ep.accumulate) {
+                const float4 p = ld_shared_f4(ad);
+                o.x = fmaf(a.ra, p.x, o.x); o.y = fmaf(a.ra, p.y, o.y);
+                o.z = fmaf(a.ra, p.z, o.z); o.w = fmaf(a.ra, p.w, o.w);
+            }
+            if (a.wrow) {
+                o.x = fmaf(-a.gam, w[4 * q], o.x); o.y = fmaf(-a.gam, w[4 * q + 1], o.y);
+                o.z = fmaf(-a.gam, w[4 * q + 2], o.z); o.w = fmaf(-a.gam, w[4 * q + 3], o.w);
+            }
+            st_shared_f4(ad, o);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+            tma_store_2d(tm, buf, x, y);
+            bulk_commit();
+        }
+    }
+}
 
 // tmE / sE: the E tensor map and this warp's staging buffers (EPI_CE_EXP).
 template <int EPI>
@@ -342,15 +391,6 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
             ep.part[(int64_t)(ep.tile0 + tn) * g.M + gm] = make_float2(mx, sm);
             if (hit) ep.ztgt[gm] = zt;
         }
-    } else if constexpr (EPI == EPI_F32_ACC) {
-        float *orow = ep.out + (int64_t)gm * ep.out_ld;
-        const AccRow a = acc_row(ep, gm, rv);
-        for (int c = 0; c < g.BN; c += 32) {
-            if (n_base + c >= n_end) break;
-            float v[32];
-            tmem_ld_x32(taddr + (uint32_t)c, v);
-            if (rv) f32_acc_store(ep, orow, n_base + c, n_end, a, v);
-        }
     } else if constexpr (EPI == EPI_ATOMIC_T) {
         for (int c = 0; c < g.BN; c += 16) {
             if (n_base + c >= n_end) break;
@@ -391,7 +431,8 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
 // forms the sum P_0 + P_1 + ... in piece order, its own term read back from
 // TMEM, and applies the epilogue to it.  BN is a multiple of 32.
 __device__ __forceinline__ void epilogue_piece_f32_acc(const GemmArgs &g, const Work &k, int gm_base, int rank,
-                                                    int nranks, int row, uint32_t taddr) {
+                                                      int nranks, int row, uint32_t taddr, const CUtensorMap *tm,
+                                                      F32Stage &st, volatile int *abort_flag) {
     const int BN = g.BN;
     const size_t region = (size_t)128 * (size_t)BN;
     const size_t slot0 = (size_t)k.tail * (size_t)g.tail_s;
@@ -414,34 +455,29 @@ __device__ __forceinline__ void epilogue_piece_f32_acc(const GemmArgs &g, const 
     }
     if (!named_barrier_or(1, 128, last)) return;
 
-    const EpiParams &ep = g.ep;
     const int gm = gm_base + row;
-    const bool rv = gm < g.M;
     const int n_base = k.tn * BN;
-    const int n_end = min(g.N, n_base + BN);
-    const AccRow a = acc_row(ep, gm, rv);
-    float *orow = ep.out + (int64_t)gm * ep.out_ld;
-    for (int c = 0; c < BN; c += 32) {
-        if (n_base + c >= n_end) break;
-        float s[32];
-        for (int j = 0; j < g.tail_s; ++j) {
-            float v[32];
-            if (j == k.piece) {
-                tmem_ld_x32(taddr + (uint32_t)c, v);
-            } else {
-                const float4 *src =
-                    reinterpret_cast<const float4 *>(g.split_ws + ((slot0 + j) * nranks + rank) * region) + row;
+    const AccRow a = acc_row(g.ep, gm, gm < g.M);
+    f32_tile_store(g, tm, st, row & 31, gm - (row & 31), a, n_base, min(g.N, n_base + BN), abort_flag,
+                   [&](int c, float(&sm)[32]) {
+                       for (int j = 0; j < g.tail_s; ++j) {
+                           float v[32];
+                           if (j == k.piece) {
+                               tmem_ld_x32(taddr + (uint32_t)c, v);
+                           } else {
+                               const float4 *src = reinterpret_cast<const float4 *>(
+                                                       g.split_ws + ((slot0 + j) * nranks + rank) * region) +
+                                                   row;
 #pragma unroll
-                for (int q = 0; q < 8; ++q) {
-                    const float4 p = __ldcg(src + (size_t)(c / 4 + q) * 128);
-                    v[4 * q] = p.x; v[4 * q + 1] = p.y; v[4 * q + 2] = p.z; v[4 * q + 3] = p.w;
-                }
-            }
+                               for (int q = 0; q < 8; ++q) {
+                                   const float4 p = __ldcg(src + (size_t)(c / 4 + q) * 128);
+                                   v[4 * q] = p.x; v[4 * q + 1] = p.y; v[4 * q + 2] = p.z; v[4 * q + 3] = p.w;
+                               }
+                           }
 #pragma unroll
-            for (int i = 0; i < 32; ++i) s[i] = (j == 0) ? v[i] : s[i] + v[i];
-        }
-        if (rv) f32_acc_store(ep, orow, n_base + c, n_end, a, s);
-    }
+                           for (int i = 0; i < 32; ++i) sm[i] = (j == 0) ? v[i] : sm[i] + v[i];
+                       }
+                   });
 }
 
 // ---------------------------------------------------------------------------
@@ -480,6 +516,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             mbar_init(tempty0 + 8 * a, 4);
         }
         mbar_init(drain0, 1);
+        if (EPI == EPI_F32_ACC)
+            for (int b = 0; b < 8; ++b) mbar_init(smem_u32(sE) + 32768u + 8u * b, 1);
         *abort_flag = 0;
         fence_mbar_init();
         tma_prefetch_desc(&tmA);
@@ -587,6 +625,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         // ---------------- epilogue (warps 2..5) ----------------
         const int q = warp & 3;
         const int row = q * 32 + lane;
+        F32Stage fst{smem_u32(sE) + (uint32_t)q * 8192u, smem_u32(sE) + 32768u + (uint32_t)q * 16u, 0u};
         int it = 0;
         for (int w = blockIdx.x; w < nwork; w += gridDim.x, ++it) {
             const Work wi = work_item(g, w, g.tiles_m);
@@ -604,10 +643,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             tc_fence_after();
             const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * g.BN);
             if constexpr (EPI == EPI_F32_ACC) {
-                if (wi.piece >= 0)
-                    epilogue_piece_f32_acc(g, wi, wi.tm * 128, 0, 1, row, taddr);
-                else
-                    epilogue_tile<EPI>(g, wi.tm * 128, wi.tn, row, taddr);
+                if (wi.piece >= 0) {
+                    epilogue_piece_f32_acc(g, wi, wi.tm * 128, 0, 1, row, taddr, &tmC, fst, abort_flag);
+                } else {
+                    const int gm = wi.tm * 128 + row;
+                    const int n_base = wi.tn * g.BN;
+                    f32_tile_store(g, &tmC, fst, lane, gm - lane, acc_row(g.ep, gm, gm < g.M), n_base,
+                                   min(g.N, n_base + g.BN), abort_flag,
+                                   [&](int c, float(&v)[32]) { tmem_ld_x32(taddr + (uint32_t)c, v); });
+                }
             } else {
                 epilogue_tile<EPI>(g, wi.tm * 128, wi.tn, row, taddr, &tmC, smem_u32(sE) + (uint32_t)q * 4096u);
             }
@@ -615,8 +659,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
         }
-        // every TMA store of E has landed before the CTA retires
-        if constexpr (EPI == EPI_CE_EXP) {
+        // every TMA store of the epilogue has landed before the CTA retires
+        if constexpr (EPI == EPI_CE_EXP || EPI == EPI_F32_ACC) {
             if (lane == 0) bulk_wait<0>();
         }
     }
@@ -672,6 +716,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             mbar_init(tempty0 + 8 * a, 8);
         }
         mbar_init(drain0, 1);
+        if (EPI == EPI_F32_ACC)
+            for (int b = 0; b < 8; ++b) mbar_init(smem_u32(sE) + 32768u + 8u * b, 1);
         *abort_flag = 0;
         fence_mbar_init();
         tma_prefetch_desc(&tmA);
@@ -776,6 +822,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         // ---------------- epilogue (warps 2..5, both CTAs) ----------------
         const int q = warp & 3;
         const int row = q * 32 + lane;
+        F32Stage fst{smem_u32(sE) + (uint32_t)q * 8192u, smem_u32(sE) + 32768u + (uint32_t)q * 16u, 0u};
         int it = 0;
         for (int w = cid; w < nwork; w += ncl, ++it) {
             const Work wi = work_item(g, w, tiles_m2);
@@ -794,10 +841,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * g.BN);
             const int gm_base = wi.tm * 256 + 128 * (int)rank;
             if constexpr (EPI == EPI_F32_ACC) {
-                if (wi.piece >= 0)
-                    epilogue_piece_f32_acc(g, wi, gm_base, (int)rank, 2, row, taddr);
-                else
-                    epilogue_tile<EPI>(g, gm_base, wi.tn, row, taddr);
+                if (wi.piece >= 0) {
+                    epilogue_piece_f32_acc(g, wi, gm_base, (int)rank, 2, row, taddr, &tmC, fst, abort_flag);
+                } else {
+                    const int gm = gm_base + row;
+                    const int n_base = wi.tn * g.BN;
+                    f32_tile_store(g, &tmC, fst, lane, gm - lane, acc_row(g.ep, gm, gm < g.M), n_base,
+                                   min(g.N, n_base + g.BN), abort_flag,
+                                   [&](int c, float(&v)[32]) { tmem_ld_x32(taddr + (uint32_t)c, v); });
+                }
             } else {
                 epilogue_tile<EPI>(g, gm_base, wi.tn, row, taddr, &tmC, smem_u32(sE) + (uint32_t)q * 4096u);
             }
@@ -805,8 +857,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(lead_tempty0 + 8 * acc);
         }
-        // every TMA store of E has landed before the CTA retires
-        if constexpr (EPI == EPI_CE_EXP) {
+        // every TMA store of the epilogue has landed before the CTA retires
+        if constexpr (EPI == EPI_CE_EXP || EPI == EPI_F32_ACC) {
             if (lane == 0) bulk_wait<0>();
         }
     }
