@@ -35,6 +35,18 @@ __device__ __forceinline__ void record_error(int *status, int code) {
     if (status) atomicCAS(status, 0, code);
 }
 
+// Programmatic dependent launch.  griddep_wait: block until the grid launched
+// before this one in the stream has completed and its writes are visible (a
+// no-op when this grid was launched without the programmatic attribute).
+// griddep_launch_dependents: let the next grid launch once every CTA of this
+// one has called it or exited; it still waits for this grid's completion
+// before it reads what this grid writes.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // bar.sync on a named barrier shared by `count` threads (a multiple of 32).
 __device__ __forceinline__ void named_barrier_sync(uint32_t id, uint32_t count) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");

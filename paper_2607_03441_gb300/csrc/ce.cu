@@ -137,6 +137,7 @@ __global__ void __launch_bounds__(256) ce_ref_kernel(const __nv_bfloat16 *__rest
                                                      const __nv_bfloat16 *__restrict__ W,
                                                      const int32_t *__restrict__ tgt, int L, int64_t d, int V,
                                                      float *__restrict__ mref) {
+    griddep_launch_dependents();  // the first logits contraction may start its main loop
     const int j = blockIdx.x * 8 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     if (j >= L) return;
@@ -202,6 +203,8 @@ __global__ void __launch_bounds__(kChunkWarps * 32) ce_chunk_kernel(const CeChun
     __shared__ float s_r[kChunkRows], s_mcf[kChunkRows];
     __shared__ int s_rw[kChunkRows];
     __shared__ bool s_last;
+    griddep_launch_dependents();
+    griddep_wait();  // the chunk's logits contraction has completed
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int j0 = blockIdx.x * kChunkRows;
     const int j = j0 + lane;
@@ -357,6 +360,8 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
             p.b = d_W; p.b_rows_ld = d; p.b_rows = V; p.b_k = d;
             p.M = (int)L; p.N = (int)Nc; p.K = (int)d; p.BN = kCeBN; p.pair = plan.pair;
             p.b_n_off = (int)v0;
+            p.pdl = true;
+            p.operands_ready = true;  // h and W are inputs of the call
             EpiParams ep{};
             ep.tgt = d_tgt; ep.part = c.part; ep.tile0 = (int)(v0 / kCeBN); ep.ztgt = c.ztgt; ep.v0 = (int)v0;
             ep.G = c.G; ep.G_ld = c.Vc;
@@ -372,7 +377,18 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
         ca.first = ci == 0 ? 1 : 0; ca.last = last ? 1 : 0;
         ca.ztgt = c.ztgt; ca.tgt = d_tgt; ca.w = d_w; ca.inv_L = 1.0f / (float)L; ca.lse_out = d_lse;
         ca.block_sums = c.block_sums; ca.ticket = c.ticket; ca.loss = d_loss; ca.status = status;
-        ce_chunk_kernel<<<(unsigned)c.nblk, kChunkWarps * 32, 0, stream>>>(ca);
+        {
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3((unsigned)c.nblk);
+            cfg.blockDim = dim3(kChunkWarps * 32);
+            cfg.stream = stream;
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+            attr[0].val.programmaticStreamSerializationAllowed = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            if (cudaLaunchKernelEx(&cfg, ce_chunk_kernel, ca) != cudaSuccess) return ATTT_ERR_CUDA;
+        }
         count_launch();
         if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
         {   // GEMM2: acc = alpha * acc + beta * (E W_c)
@@ -381,6 +397,7 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
             p.b = d_W; p.b_rows_ld = d; p.b_rows = d; p.b_k = V;
             p.M = (int)L; p.N = (int)d; p.K = (int)round_up(Nc, 64); p.BN = kCeBN; p.pair = plan.pair;
             p.b_k_off = (int)v0;
+            p.pdl = true;  // E may be rewritten by the chunk kernel: the producer waits
             EpiParams ep{};
             ep.out = d_dh; ep.out_ld = d; ep.accumulate = ci > 0 ? 1 : 0; ep.alpha = 1.0f;
             ep.row_alpha = c.alpha; ep.row_beta = c.beta;

@@ -19,6 +19,10 @@ struct GemmProblem {
     int BN;
     int a_m_off = 0, a_k_off = 0, b_n_off = 0, b_k_off = 0;
     bool pair = false;  // run on CTA pairs (256-row tiles, cta_group::2)
+    // Launch as a programmatic dependent of the previous grid in the stream;
+    // operands_ready: A and B do not come from that grid.
+    bool pdl = false;
+    bool operands_ready = false;
     // Tail split (EPI_F32_ACC): workspace for up to `split_regions` partials
     // of 128 x BN fp32 and as many arrival counters (zero on entry).
     float *split_ws = nullptr;
@@ -127,32 +131,42 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.b_n_off = p.b_n_off;
     g.b_k_off = p.b_k_off;
     g.tmem_cols = gemm_tmem_cols(p.BN);
+    g.operands_ready = p.operands_ready ? 1 : 0;
     g.status = status ? status : device_status_word(dev);
     g.ep = ep;
 
     const size_t smem = gemm_smem_bytes(bn_cta, g.stages, g.e_stage_bytes);
     const int ntiles = g.whole_tiles + (tiles - g.whole_tiles) * g.tail_s;  // work items
+    cudaLaunchConfig_t cfg = {};
+    cfg.blockDim = dim3(kGemmThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[2];
+    unsigned na = 0;
+    if (p.pdl) {
+        attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[na].val.programmaticStreamSerializationAllowed = 1;
+        ++na;
+    }
     if (!p.pair) {
         auto kern = tc_gemm_kernel<EPI, A_MN, B_MN>;
         if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
-        const int grid = ntiles < sms ? ntiles : sms;
-        kern<<<grid, kGemmThreads, smem, stream>>>(ta, tb, tc, g);
+        cfg.gridDim = dim3((unsigned)(ntiles < sms ? ntiles : sms));
+        cfg.attrs = attr;
+        cfg.numAttrs = na;
+        if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, g) != cudaSuccess) return ATTT_ERR_CUDA;
     } else {
         auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN>;
         if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
         const int pairs = ntiles < units ? ntiles : units;
-        cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3((unsigned)(2 * pairs));
-        cfg.blockDim = dim3(kGemmThreads);
-        cfg.dynamicSmemBytes = smem;
-        cfg.stream = stream;
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = 2;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
+        attr[na].id = cudaLaunchAttributeClusterDimension;
+        attr[na].val.clusterDim.x = 2;
+        attr[na].val.clusterDim.y = 1;
+        attr[na].val.clusterDim.z = 1;
+        ++na;
         cfg.attrs = attr;
-        cfg.numAttrs = 1;
+        cfg.numAttrs = na;
         if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, g) != cudaSuccess) return ATTT_ERR_CUDA;
     }
     count_launch();

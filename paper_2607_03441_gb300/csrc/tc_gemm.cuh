@@ -72,7 +72,11 @@ struct GemmArgs {
     int a_m_off, a_k_off;  // coordinate offsets into A's tensor map
     int b_n_off, b_k_off;  // coordinate offsets into B's tensor map
     uint32_t tmem_cols;
-    uint32_t e_stage_bytes;  // shared-memory staging of the TMA-stored epilogue output (EPI_CE_EXP), else 0
+    uint32_t e_stage_bytes;  // shared-memory staging of the TMA-stored epilogue output, else 0
+    // Programmatic dependent launch: the A/B operands were complete before the
+    // previous grid in the stream started, so the producer need not wait for it
+    // (the epilogue always does).
+    int operands_ready;
     int *status;
     EpiParams ep;
     // Tail split (tc_gemm_kernel / tc_gemm_pair_kernel): tiles [0, whole_tiles)
@@ -515,6 +519,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             mbar_init(tfull0 + 8 * a, 1);
             mbar_init(tempty0 + 8 * a, 4);
         }
+        griddep_launch_dependents();
         mbar_init(drain0, 1);
         if (EPI == EPI_F32_ACC)
             for (int b = 0; b < 8; ++b) mbar_init(smem_u32(sE) + 32768u + 8u * b, 1);
@@ -537,6 +542,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (warp == 0) {
         if (lane == 0) {
             // ---------------- TMA producer ----------------
+            if (!g.operands_ready) griddep_wait();
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_parity = 0;  // per stage: last issue pending?
@@ -623,6 +629,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
     } else {
         // ---------------- epilogue (warps 2..5) ----------------
+        griddep_wait();  // what the epilogue reads or overwrites may come from the previous grid
         const int q = warp & 3;
         const int row = q * 32 + lane;
         F32Stage fst{smem_u32(sE) + (uint32_t)q * 8192u, smem_u32(sE) + 32768u + (uint32_t)q * 16u, 0u};
@@ -715,6 +722,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             mbar_init(tfull0 + 8 * a, 1);
             mbar_init(tempty0 + 8 * a, 8);
         }
+        griddep_launch_dependents();
         mbar_init(drain0, 1);
         if (EPI == EPI_F32_ACC)
             for (int b = 0; b < 8; ++b) mbar_init(smem_u32(sE) + 32768u + 8u * b, 1);
@@ -742,6 +750,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (warp == 0) {
         if (lane == 0) {
             // ---------------- TMA producer (both CTAs) ----------------
+            if (!g.operands_ready) griddep_wait();
             int stage = 0;
             uint32_t phase = 0;
             bool ok = true;
@@ -820,6 +829,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
     } else {
         // ---------------- epilogue (warps 2..5, both CTAs) ----------------
+        griddep_wait();  // what the epilogue reads or overwrites may come from the previous grid
         const int q = warp & 3;
         const int row = q * 32 + lane;
         F32Stage fst{smem_u32(sE) + (uint32_t)q * 8192u, smem_u32(sE) + 32768u + (uint32_t)q * 16u, 0u};
