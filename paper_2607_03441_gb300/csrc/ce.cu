@@ -45,10 +45,12 @@ struct CeLayout {
     size_t bytes;
 };
 
-// Upper bound of the vocab chunk: the chunk's bf16 gradient block L x Vc is
-// kept near 96 MB (L2 is 129 MB).  The workspace is sized for this bound.
+// Upper bound of the vocab chunk: the chunk's bf16 block E (L x Vc) is kept
+// near 256 MB, so the workspace stays bounded whatever V is.  Each chunk costs
+// about 20 us of launch, ramp and tail on top of its FLOPs, and E is streamed
+// once from L2 or HBM either way, so wider chunks are faster up to this bound.
 static int64_t ce_chunk_max(int64_t L, int64_t V) {
-    int64_t vc = (96ll << 20) / (2 * L);
+    int64_t vc = (256ll << 20) / (2 * L);
     vc = (vc / kCeBN) * kCeBN;
     if (vc < 4096) vc = 4096;
     if (vc > kCeMaxTiles * kCeBN) vc = kCeMaxTiles * kCeBN;
@@ -69,7 +71,7 @@ struct CePlan {
 
 static CePlan ce_plan(int64_t L, int64_t d, int64_t V, int sms) {
     const double rate = 1.0e13;    // bf16 FLOP/s of one SM, order of magnitude
-    const double launch = 5.0e-6;  // seconds per launch, ramp-up and tail included
+    const double launch = 7.0e-6;  // seconds per launch, ramp-up and tail included
     const bool pair = L > 128;
     const int64_t rows = pair ? 256 : 128;       // accumulator rows per tile
     const int64_t units = pair ? sms / 2 : sms;  // tiles in flight

@@ -171,7 +171,8 @@ def test_multichunk_with_reference_jumps(attt):
     """Several vocab chunks, with rows whose max logit sits far above their
     reference (the target logit, then the running max): 2^92 in log2 units
     (E rewritten, in the first chunk for row 1500, the last for row 77) and
-    2^61 (E written up to 2^61, no rewrite: rows 300 and 900); row 5's target
+    2^61 (E written up to 2^61, no rewrite: row 300 in the first chunk, row
+    900 in the last); row 5's target
     is its max, so the chunks before it sit far below the reference; sampled
     rows against the oracle."""
     L, V, d = 2048, 80000, 64
@@ -179,7 +180,7 @@ def test_multichunk_with_reference_jumps(attt):
     h = wk.normal_bf16(77, "h", (L, d), 0.5)
     W = wk.normal_bf16(77, "W", (V, d), 0.05)
     hot_rows = [5, 77, 1500, 300, 900]
-    for j, v, x in zip(hot_rows, [60000, 79999, 30, 100, 50000], [8.0, 8.0, 8.0, 6.5, 6.5]):
+    for j, v, x in zip(hot_rows, [60000, 79999, 30, 100, 79000], [8.0, 8.0, 8.0, 6.5, 6.5]):
         h[j] = 0
         h[j, 0] = wk.bf16_bits(np.array([x], np.float32))[0]
         W[v, 0] = wk.bf16_bits(np.array([x], np.float32))[0]  # z[j, v] = x^2 (64 or 42.25)
