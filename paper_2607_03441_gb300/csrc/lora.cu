@@ -10,24 +10,24 @@
 // Every contraction puts the long dimension (L, din or dout) on the 128-row
 // MMA side and the rank on N, so the tensor core streams x and dy once per
 // pass at HBM rate.  Reductions over L (or din/dout) are split across CTAs
-// and merged with fp32 atomics; u and v are rounded to bf16 in between (by
-// the split that finishes each tile last).  Three launches per call: prep
-// (adapters to K-major, every accumulator zeroed), pass 1 (u and every v_p,
-// grouped), pass 2 (dA and every dB_p, grouped).
+// (stream-K, tc_group.cuh) and summed in a fixed order by the piece that
+// finishes each tile last; u and v go to bf16 in between.  Three launches per
+// call: prep (adapters to K-major), pass 1 (u and every v_p, grouped), pass 2
+// (dA and every dB_p, grouped).
 #include "gemm_launch.cuh"
 #include "tc_group.cuh"
 
 namespace attt {
 
 struct LoraLayout {
-    int rpad, Nu;
+    int rpad, Nu, BN;
     int64_t Lp;
     __nv_bfloat16 *AT;            // [Nu, din]
     __nv_bfloat16 *BT[kMaxProj];  // [rpad, dout_p]
-    float *uT32, *vT32;           // [Nu, Lp] each, contiguous
     __nv_bfloat16 *uT16, *vT16;   // [Nu, Lp] each, contiguous
-    unsigned int *tickets;        // pass-1 tile counters, (1 + nproj) x ntick
-    int64_t ntick;
+    int64_t tiles;                // group-wide tiles of the larger pass
+    unsigned int *tickets;        // [tiles] arrival counters (both passes)
+    float *part;                  // [tiles + kGroupMaxGrid] partial slots of 128 x BN fp32
     size_t bytes;
 };
 
@@ -35,16 +35,22 @@ static LoraLayout lora_layout(void *ws, int64_t L, int64_t din, int nproj, const
     LoraLayout c{};
     c.rpad = (int)round_up(r, 16);
     c.Nu = nproj * c.rpad;
+    c.BN = c.Nu <= 256 ? c.Nu : 256;
     c.Lp = round_up(L, 8);
+    // pass 1: u (L x Nu) and each v_p (L x rpad); pass 2: dA (din x Nu) and each dB_p (dout_p x rpad)
+    int64_t t1 = cdiv(L, 128) * cdiv(c.Nu, c.BN), t2 = cdiv(din, 128) * cdiv(c.Nu, c.BN);
+    for (int p = 0; p < nproj; ++p) {
+        t1 += cdiv(L, 128) * cdiv(c.rpad, c.BN);
+        t2 += cdiv(dout[p], 128) * cdiv(c.rpad, c.BN);
+    }
+    c.tiles = t1 > t2 ? t1 : t2;
     Carve cv{static_cast<char *>(ws), 0};
     c.AT = cv.take<__nv_bfloat16>((size_t)(c.Nu * din));
     for (int p = 0; p < nproj; ++p) c.BT[p] = cv.take<__nv_bfloat16>((size_t)(c.rpad * dout[p]));
-    c.uT32 = cv.take<float>((size_t)(2 * c.Nu * c.Lp));
-    c.vT32 = c.uT32 + (size_t)c.Nu * c.Lp;
     c.uT16 = cv.take<__nv_bfloat16>((size_t)(2 * c.Nu * c.Lp));
     c.vT16 = c.uT16 + (size_t)c.Nu * c.Lp;
-    c.ntick = cdiv(L, 128) * cdiv(c.Nu, 256);
-    c.tickets = cv.take<unsigned int>((size_t)((1 + nproj) * c.ntick));
+    c.tickets = cv.take<unsigned int>((size_t)c.tiles);
+    c.part = cv.take<float>((size_t)(c.tiles + kGroupMaxGrid) * 128 * c.BN);
     c.bytes = (size_t)round_up((int64_t)cv.used, 256);
     return c;
 }
@@ -53,48 +59,48 @@ struct PrepArgs {
     const __nv_bfloat16 *A[kMaxProj];
     const __nv_bfloat16 *B[kMaxProj];
     __nv_bfloat16 *BT[kMaxProj];
-    float *dA[kMaxProj];
-    float *dB[kMaxProj];
     int64_t dout[kMaxProj];
     int nproj, r, rpad;
     int64_t din;
     __nv_bfloat16 *AT;
-    float *acc;           // uT32 and vT32, contiguous
-    int64_t nacc;
     unsigned int *tickets;
     int64_t ntickets;
 };
 
 // AT[p*rpad + c, i] = A_p[i, c] (zero for c >= r); BT_p[c, o] = B_p[c, o]
-// (zero rows for c >= r); and every accumulator of the call set to zero
-// (u^T, v^T, dA_p, dB_p and the tile tickets), block row p of the grid doing
-// projection p's share.
-__global__ void lora_prep_kernel(PrepArgs a) {
+// (zero rows for c >= r); and the tile tickets set to zero, block row p of
+// the grid doing projection p's share.  The transpose goes through shared
+// memory in slabs of 64 rows of A_p (read row-contiguous, written as 128-byte
+// runs of AT).
+constexpr int kPrepRows = 64;
+
+__global__ void __launch_bounds__(256) lora_prep_kernel(PrepArgs a) {
+    __shared__ __nv_bfloat16 slab[kPrepRows][64 + 2];  // [row of A_p][column c], r <= 64
     const int p = blockIdx.y;
-    const int64_t nA = (int64_t)a.rpad * a.din;
-    const int64_t nB = (int64_t)a.rpad * a.dout[p];
-    const int64_t ndA = a.din * a.r, ndB = (int64_t)a.r * a.dout[p];
-    const int64_t zacc = (a.nacc + a.nproj - 1) / a.nproj;   // this row's slice of the u/v accumulators
-    const int64_t ztk = (a.ntickets + a.nproj - 1) / a.nproj;
-    int64_t n = nA > nB ? nA : nB;
-    if (ndA > n) n = ndA;
-    if (ndB > n) n = ndB;
-    if (zacc > n) n = zacc;
-    if (ztk > n) n = ztk;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-        if (i < nA) {
-            const int c = (int)(i / a.din);
-            const int64_t k = i - (int64_t)c * a.din;
-            a.AT[((int64_t)p * a.rpad + c) * a.din + k] =
-                c < a.r ? a.A[p][k * a.r + c] : __float2bfloat16_rn(0.f);
+    const int64_t nslab = (a.din + kPrepRows - 1) / kPrepRows;
+    for (int64_t sb = blockIdx.x; sb < nslab; sb += gridDim.x) {
+        const int64_t k0 = sb * kPrepRows;
+        const int rows = (int)min((int64_t)kPrepRows, a.din - k0);
+        for (int e = threadIdx.x; e < rows * a.r; e += blockDim.x) {
+            const int kk = e / a.r, c = e - kk * a.r;
+            slab[kk][c] = a.A[p][(k0 + kk) * a.r + c];
         }
+        __syncthreads();
+        for (int e = threadIdx.x; e < a.rpad * kPrepRows; e += blockDim.x) {
+            const int c = e / kPrepRows, kk = e - c * kPrepRows;
+            if (kk < rows)
+                a.AT[((int64_t)p * a.rpad + c) * a.din + k0 + kk] = c < a.r ? slab[kk][c] : __float2bfloat16_rn(0.f);
+        }
+        __syncthreads();
+    }
+    const int64_t nB = (int64_t)a.rpad * a.dout[p];
+    const int64_t ztk = (a.ntickets + a.nproj - 1) / a.nproj;  // this row's slice of the tickets
+    const int64_t n = nB > ztk ? nB : ztk;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         if (i < nB) {
             const int c = (int)(i / a.dout[p]);
             a.BT[p][i] = c < a.r ? a.B[p][i] : __float2bfloat16_rn(0.f);
         }
-        if (i < ndA) a.dA[p][i] = 0.f;
-        if (i < ndB) a.dB[p][i] = 0.f;
-        if (i < zacc && p * zacc + i < a.nacc) a.acc[p * zacc + i] = 0.f;
         if (i < ztk && p * ztk + i < a.ntickets) a.tickets[p * ztk + i] = 0u;
     }
 }
@@ -133,20 +139,28 @@ struct GroupSpec {
     int64_t b_rows_ld, b_rows, b_k;
     int M, N, K;
     int b_n_off;
-    int epi;
-    EpiParams ep;
+    int out;  // GroupOut
+    float alpha;
+    int r, rpad;
+    int64_t ld;
+    float *out32;
+    __nv_bfloat16 *out16;
+    float *outp[kMaxProj];
 };
 
-// Launches every problem of `specs` in one grouped kernel.  K is split per
-// problem so that each CTA streams about the same number of K blocks.
+// Launches every problem of `specs` in one grouped kernel; every CTA streams
+// the same number of K stages (stream-K split, tc_group.cuh).
 template <bool A_MN, bool B_MN>
-static attt_status launch_group(const GroupSpec *specs, int n, int BN, int dev, cudaStream_t stream, int *status) {
+static attt_status launch_group(const GroupSpec *specs, int n, int BN, float *part, unsigned int *tickets, int dev,
+                                cudaStream_t stream, int *status) {
     if (n < 1 || n > kMaxGroup || BN < 16 || BN > 256 || BN % 16 != 0) return ATTT_ERR_INVALID_ARG;
     static_assert(!B_MN, "grouped B operands are K-major");
     GroupMaps maps;
     GroupArgs g{};
     g.nprob = n;
     g.BN = BN;
+    g.part = part;
+    g.tickets = tickets;
     // Up to four 64-deep K blocks per stage, so each operand row is fetched in
     // runs of up to 512 bytes (better DRAM locality than one 128-byte piece per
     // row per block), as long as at least two stages fit in shared memory.
@@ -162,12 +176,7 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, int dev, 
     g.tmem_cols = gemm_tmem_cols(BN);
     g.status = status ? status : device_status_word(dev);
     const int sms = num_sms(dev);
-    int64_t work = 0;  // tile x K-block units of the whole group
-    for (int q = 0; q < n; ++q) {
-        const GroupSpec &sp = specs[q];
-        work += cdiv(sp.M, 128) * cdiv(sp.N, BN) * cdiv(sp.K, 64);
-    }
-    const int64_t per_cta = cdiv(work, sms) > 0 ? cdiv(work, sms) : 1;
+    int64_t stages = 0;
     int tiles = 0;
     for (int q = 0; q < n; ++q) {
         const GroupSpec &sp = specs[q];
@@ -189,22 +198,28 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, int dev, 
         pr.tiles_m = (int)cdiv(sp.M, 128);
         pr.tiles_n = (int)cdiv(sp.N, BN);
         pr.kb_total = (int)cdiv(sp.K, 64);
-        int splits = (int)cdiv(pr.kb_total, per_cta);
-        if (splits < 1) splits = 1;
-        pr.kb_per_split = (int)round_up(cdiv(pr.kb_total, splits), g.kbs);  // whole stages per split
-        pr.splits = (int)cdiv(pr.kb_total, pr.kb_per_split);
+        pr.nst = (int)cdiv(pr.kb_total, g.kbs);
         pr.b_n_off = sp.b_n_off;
+        pr.stage_begin = stages;
         pr.tile_begin = tiles;
-        pr.epi = sp.epi;
-        pr.ep = sp.ep;
-        tiles += pr.tiles_m * pr.tiles_n * pr.splits;
+        pr.out = sp.out;
+        pr.alpha = sp.alpha;
+        pr.r = sp.r;
+        pr.rpad = sp.rpad;
+        pr.ld = sp.ld;
+        pr.out32 = sp.out32;
+        pr.out16 = sp.out16;
+        for (int j = 0; j < kMaxProj; ++j) pr.outp[j] = sp.outp[j];
+        stages += (int64_t)pr.tiles_m * pr.tiles_n * pr.nst;
+        tiles += pr.tiles_m * pr.tiles_n;
     }
-    g.total_tiles = tiles;
+    g.total_stages = stages;
     const size_t smem =
         1024 + (size_t)g.stages * g.kbs * (kABytes + gemm_b_stage_bytes(BN)) + 8 * (2 * g.stages + 5) + 16;
     auto kern = tc_gemm_group_kernel<A_MN, B_MN>;
     if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
-    const int grid = tiles < sms ? tiles : sms;
+    int grid = stages < sms ? (int)stages : sms;  // every CTA gets at least one stage
+    if (grid > kGroupMaxGrid) grid = kGroupMaxGrid;
     kern<<<grid, kGemmThreads, smem, stream>>>(maps, g);
     count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
@@ -231,25 +246,22 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
     if (st != ATTT_OK) return st;
 
     LoraLayout c = lora_layout(d_ws, L, din, nproj, dout, r);
-    const int BN = c.Nu <= 256 ? c.Nu : 256;
+    const int BN = c.BN;
 
     // prep: adapters to K-major (rank padded with zeros), accumulators zeroed
     {
         PrepArgs a{};
-        int64_t maxn = c.rpad * din;
+        int64_t maxn = cdiv(din, kPrepRows) * 256;  // the transpose slabs (one block each)
         for (int p = 0; p < nproj; ++p) {
             a.A[p] = reinterpret_cast<const __nv_bfloat16 *>(d_A[p]);
             a.B[p] = reinterpret_cast<const __nv_bfloat16 *>(d_B[p]);
             a.BT[p] = c.BT[p];
-            a.dA[p] = d_dA[p];
-            a.dB[p] = d_dB[p];
             a.dout[p] = dout[p];
             if (c.rpad * dout[p] > maxn) maxn = c.rpad * dout[p];
         }
         a.nproj = nproj; a.r = r; a.rpad = c.rpad; a.din = din; a.AT = c.AT;
-        a.acc = c.uT32; a.nacc = (int64_t)2 * c.Nu * c.Lp;
-        a.tickets = c.tickets; a.ntickets = (1 + nproj) * c.ntick;
-        if (a.nacc / nproj > maxn) maxn = a.nacc / nproj + 1;
+        a.tickets = c.tickets; a.ntickets = c.tiles;
+        if (a.ntickets / nproj > maxn) maxn = a.ntickets / nproj + 1;
         dim3 grid(grid_for(maxn, 256, dev), nproj);
         lora_prep_kernel<<<grid, 256, 0, stream>>>(a);
         count_launch();
@@ -264,20 +276,18 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
         u = GroupSpec{};
         u.a = d_x; u.a_rows_ld = din; u.a_rows = L; u.a_k = din;
         u.b = c.AT; u.b_rows_ld = din; u.b_rows = c.Nu; u.b_k = din;
-        u.M = (int)L; u.N = c.Nu; u.K = (int)din; u.epi = EPI_ATOMIC_T;
-        u.ep.out = c.uT32; u.ep.out_ld = c.Lp; u.ep.alpha = 1.0f; u.ep.r = c.rpad; u.ep.rpad = c.rpad;
-        u.ep.out16 = c.uT16; u.ep.tickets = c.tickets;
+        u.M = (int)L; u.N = c.Nu; u.K = (int)din;
+        u.out = GOUT_T16; u.out16 = c.uT16; u.ld = c.Lp; u.alpha = 1.0f; u.r = c.rpad; u.rpad = c.rpad;
         for (int q = 0; q < nproj; ++q) {
             GroupSpec &v = sp[n++];
             v = GroupSpec{};
             v.a = d_dy[q]; v.a_rows_ld = dout[q]; v.a_rows = L; v.a_k = dout[q];
             v.b = c.BT[q]; v.b_rows_ld = dout[q]; v.b_rows = c.rpad; v.b_k = dout[q];
-            v.M = (int)L; v.N = c.rpad; v.K = (int)dout[q]; v.epi = EPI_ATOMIC_T;
-            v.ep.out = c.vT32 + (size_t)q * c.rpad * c.Lp; v.ep.out_ld = c.Lp; v.ep.alpha = 1.0f;
-            v.ep.r = c.rpad; v.ep.rpad = c.rpad;
-            v.ep.out16 = c.vT16 + (size_t)q * c.rpad * c.Lp; v.ep.tickets = c.tickets + (1 + q) * c.ntick;
+            v.M = (int)L; v.N = c.rpad; v.K = (int)dout[q];
+            v.out = GOUT_T16; v.out16 = c.vT16 + (size_t)q * c.rpad * c.Lp; v.ld = c.Lp; v.alpha = 1.0f;
+            v.r = c.rpad; v.rpad = c.rpad;
         }
-        st = launch_group<false, false>(sp, n, BN, dev, stream, status);
+        st = launch_group<false, false>(sp, n, BN, c.part, c.tickets, dev, stream, status);
         if (st != ATTT_OK) return st;
     }
 
@@ -290,19 +300,20 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
         a = GroupSpec{};
         a.a = d_x; a.a_rows_ld = din; a.a_rows = din; a.a_k = L;
         a.b = c.vT16; a.b_rows_ld = c.Lp; a.b_rows = c.Nu; a.b_k = L;  // padding columns read as zeros
-        a.M = (int)din; a.N = c.Nu; a.K = (int)L; a.epi = EPI_ATOMIC_N;
-        for (int q = 0; q < nproj; ++q) a.ep.outp[q] = d_dA[q];
-        a.ep.alpha = scale; a.ep.r = r; a.ep.rpad = c.rpad;
+        a.M = (int)din; a.N = c.Nu; a.K = (int)L;
+        a.out = GOUT_N32;
+        for (int q = 0; q < nproj; ++q) a.outp[q] = d_dA[q];
+        a.alpha = scale; a.r = r; a.rpad = c.rpad;
         for (int q = 0; q < nproj; ++q) {
             GroupSpec &b = sp[n++];
             b = GroupSpec{};
             b.a = d_dy[q]; b.a_rows_ld = dout[q]; b.a_rows = dout[q]; b.a_k = L;
             b.b = c.uT16; b.b_rows_ld = c.Lp; b.b_rows = c.Nu; b.b_k = L;
             b.b_n_off = q * c.rpad;
-            b.M = (int)dout[q]; b.N = c.rpad; b.K = (int)L; b.epi = EPI_ATOMIC_T;
-            b.ep.out = d_dB[q]; b.ep.out_ld = dout[q]; b.ep.alpha = scale; b.ep.r = r; b.ep.rpad = c.rpad;
+            b.M = (int)dout[q]; b.N = c.rpad; b.K = (int)L;
+            b.out = GOUT_T32; b.out32 = d_dB[q]; b.ld = dout[q]; b.alpha = scale; b.r = r; b.rpad = c.rpad;
         }
-        st = launch_group<true, false>(sp, n, BN, dev, stream, status);
+        st = launch_group<true, false>(sp, n, BN, c.part, c.tickets, dev, stream, status);
         if (st != ATTT_OK) return st;
     }
     return ATTT_OK;

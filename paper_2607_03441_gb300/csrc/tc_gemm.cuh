@@ -415,13 +415,22 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
             float v[16];
             tmem_ld_x16(taddr + (uint32_t)c, v);
             if (rv) {
+                // the 16 columns lie in one projection (rpad is a multiple of
+                // 16); with r % 4 == 0 and an aligned row they go out as four
+                // 16-byte reductions instead of sixteen scalar atomics
+                const int col0 = n_base + c;
+                const int p = col0 / ep.rpad, cc0 = col0 - p * ep.rpad;
+                float *orow = ep.outp[p] + (int64_t)gm * ep.r;
+                if (col0 + 16 <= n_end && (ep.r & 3) == 0 && (reinterpret_cast<uintptr_t>(orow) & 15) == 0) {
 #pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int col = n_base + c + i;
-                    if (col < n_end) {
-                        const int p = col / ep.rpad, cc = col - p * ep.rpad;
-                        if (cc < ep.r) atomicAdd(ep.outp[p] + (int64_t)gm * ep.r + cc, ep.alpha * v[i]);
-                    }
+                    for (int i = 0; i < 16; i += 4)
+                        if (cc0 + i < ep.r)
+                            red_add_v4(orow + cc0 + i, ep.alpha * v[i], ep.alpha * v[i + 1], ep.alpha * v[i + 2],
+                                       ep.alpha * v[i + 3]);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i)
+                        if (col0 + i < n_end && cc0 + i < ep.r) atomicAdd(orow + cc0 + i, ep.alpha * v[i]);
                 }
             }
         }

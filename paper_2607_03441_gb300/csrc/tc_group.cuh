@@ -1,14 +1,24 @@
 // tc_group.cuh -- grouped tcgen05 contractions: several independent problems
-// (own operands, sizes, K split and epilogue) in one persistent launch.
+// (own operands, sizes and output) in one persistent launch.
 //
 // The LoRA gradients are a handful of skinny, HBM-bound contractions (the
 // rank on N); launched one by one, each pays a launch, a ramp and a tail
 // that cost more than streaming its operands.  Grouping runs every
 // contraction of a pass in one launch.  The pipeline is the single-CTA one
 // of tc_gemm.cuh (TMA producer warp, MMA warp, four epilogue warps, two TMEM
-// accumulators); only the tile -> problem decode and the per-problem tensor
-// maps and epilogue differ.  All problems of a group share BN and the operand
-// majors.
+// accumulators); only the work decode, the per-problem tensor maps and the
+// epilogue differ.  All problems of a group share BN and the operand majors.
+//
+// Work is split stream-K style: the K stages of every tile of every problem
+// are laid end to end (problem by problem, tile by tile), and CTA c takes the
+// stages [c S / G, (c + 1) S / G) of the S stages for G CTAs, so every CTA
+// streams the same number of stages.  A CTA's range is a few segments (the
+// end of one tile, whole tiles, the start of another), each one accumulator
+// pass.  A tile that one segment covers is written straight from TMEM; a tile
+// split over several CTAs has each piece store its fp32 partial in a slot,
+// and the piece that arrives last (ticket) sums the partials in CTA order and
+// writes the tile.  No atomics on the outputs, and the result does not depend
+// on which piece finishes last.
 #pragma once
 
 #include "tc_gemm.cuh"
@@ -16,14 +26,30 @@
 namespace attt {
 
 constexpr int kMaxGroup = kMaxProj + 1;
+constexpr int kGroupMaxGrid = 256;  // CTAs of a grouped launch at most: partial slots are CTA + tile
+
+// How a problem writes its result D (fp32 accumulator, rows m < M, columns
+// n < N).
+enum GroupOut : int {
+    GOUT_T16 = 0,  // out16[n * ld + m] = bf16(alpha D[m, n])                          (transposed, bf16)
+    GOUT_N32 = 1,  // outp[n / rpad][m * r + n % rpad] = alpha D[m, n], n % rpad < r   (a row-major block per rpad columns)
+    GOUT_T32 = 2,  // out32[n * ld + m] = alpha D[m, n], n % rpad < r                  (transposed, fp32)
+};
 
 struct GroupProblem {
     int M, N;
-    int tiles_m, tiles_n, splits, kb_per_split, kb_total;
+    int tiles_m, tiles_n, kb_total;
+    int nst;  // K stages per tile (kbs K blocks each)
     int a_m_off, a_k_off, b_n_off, b_k_off;
-    int tile_begin;  // first group-wide tile index of this problem
-    int epi;         // EPI_ATOMIC_T or EPI_ATOMIC_N
-    EpiParams ep;
+    int64_t stage_begin;  // first group-wide stage of this problem
+    int tile_begin;       // first group-wide tile of this problem
+    int out;              // GroupOut
+    float alpha;
+    int r, rpad;
+    int64_t ld;
+    float *out32;
+    __nv_bfloat16 *out16;
+    float *outp[kMaxProj];
 };
 
 struct GroupMaps {
@@ -32,66 +58,140 @@ struct GroupMaps {
 };
 
 struct GroupArgs {
-    int nprob, total_tiles;
+    int nprob;
+    int64_t total_stages;  // S; the grid G is at most S, so no CTA's range is empty
     int BN, stages;
     int kbs;  // 64-deep K blocks per pipeline stage (each row is fetched in kbs x 128 B runs)
     uint32_t tmem_cols;
     int *status;
+    float *part;            // partial slots of 128 x BN fp32, [BN / 4][128] float4 each; CTA + tile slots
+    unsigned int *tickets;  // one arrival counter per group-wide tile, 0 between launches
     GroupProblem prob[kMaxGroup];
 };
 
-__device__ __forceinline__ void decode_group(const GroupArgs &g, int t, int &q, int &tm, int &tn, int &split) {
-    q = 0;
-    while (q + 1 < g.nprob && t >= g.prob[q + 1].tile_begin) ++q;
+// One segment of a CTA's stage range: problem q, tile (tm, tn), K blocks
+// [kb0, kb1); ts / te bound the tile's own stages.
+struct GroupSeg {
+    int q, tm, tn, kb0, kb1;
+    int64_t ts, te;
+};
+
+// The segment that starts at stage x of a range ending at xend; advances x.
+__device__ __forceinline__ bool group_next(const GroupArgs &g, int64_t &x, int64_t xend, GroupSeg &sg) {
+    if (x >= xend) return false;
+    int q = 0;
+    while (q + 1 < g.nprob && x >= g.prob[q + 1].stage_begin) ++q;
     const GroupProblem &p = g.prob[q];
-    const int local = t - p.tile_begin;
-    const int per = p.tiles_m * p.tiles_n;
-    split = local / per;
-    const int rem = local - split * per;
-    tn = rem / p.tiles_m;
-    tm = rem - tn * p.tiles_m;
+    const int64_t loc = x - p.stage_begin;
+    const int tile = (int)(loc / p.nst);
+    const int s0 = (int)(loc - (int64_t)tile * p.nst);
+    sg.ts = p.stage_begin + (int64_t)tile * p.nst;
+    sg.te = sg.ts + p.nst;
+    const int64_t end = xend < sg.te ? xend : sg.te;
+    sg.q = q;
+    sg.tn = tile / p.tiles_m;
+    sg.tm = tile - sg.tn * p.tiles_m;
+    sg.kb0 = s0 * g.kbs;
+    sg.kb1 = min(p.kb_total, (int)(s0 + (end - x)) * g.kbs);
+    x = end;
+    return true;
 }
 
-// A GemmArgs view of one problem, for the shared epilogues.
-__device__ __forceinline__ GemmArgs group_view(const GroupArgs &g, const GroupProblem &p) {
-    GemmArgs v{};
-    v.M = p.M;
-    v.N = p.N;
-    v.BN = g.BN;
-    v.tiles_m = p.tiles_m;
-    v.tiles_n = p.tiles_n;
-    v.splits = p.splits;
-    v.status = g.status;
-    v.ep = p.ep;
-    return v;
+// The CTA whose range holds stage x: the largest c with floor(c S / G) <= x.
+__device__ __forceinline__ int64_t group_owner(const GroupArgs &g, int64_t x, int64_t G) {
+    return ((x + 1) * G - 1) / g.total_stages;
 }
 
-// EPI_ATOMIC_T epilogue with an optional bf16 finalize: after this split's
-// atomics, the split that takes the tile's last ticket converts the tile's
-// fp32 sums (out[n, m]) to bf16 (out16[n, m]).  No CTA waits for another.
-__device__ __forceinline__ void group_atomic_t_tile(const GemmArgs &v, int gm_base, int tm, int tn, int row,
-                                                    uint32_t taddr) {
-    epilogue_tile<EPI_ATOMIC_T>(v, gm_base, tn, row, taddr);
-    const EpiParams &ep = v.ep;
-    if (!ep.out16) return;
-    __threadfence();
-    named_barrier_sync(1, 128);
-    __shared__ int s_last;
-    if (threadIdx.x == 64) {
-        unsigned int *tk = ep.tickets + (tm + tn * v.tiles_m);
-        s_last = atomicAdd(tk, 1u) == (unsigned)(v.splits - 1);
-        if (s_last) *tk = 0u;
+// Writes the 16 columns [col0, col0 + 16) of row m (values already summed
+// over the tile's pieces).
+__device__ __forceinline__ void group_store16(const GroupProblem &p, int m, int col0, int n_end,
+                                              const float (&v)[16]) {
+    if (p.out == GOUT_T16) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+            if (col0 + i < n_end) p.out16[(int64_t)(col0 + i) * p.ld + m] = __float2bfloat16_rn(p.alpha * v[i]);
+    } else if (p.out == GOUT_N32) {
+        // the 16 columns lie in one rpad block (rpad is a multiple of 16)
+        const int blk = col0 / p.rpad, cc0 = col0 - blk * p.rpad;
+        float *orow = p.outp[blk] + (int64_t)m * p.r;
+        if (col0 + 16 <= n_end && (p.r & 3) == 0 && (reinterpret_cast<uintptr_t>(orow) & 15) == 0) {
+#pragma unroll
+            for (int i = 0; i < 16; i += 4)
+                if (cc0 + i < p.r)
+                    *reinterpret_cast<float4 *>(orow + cc0 + i) =
+                        make_float4(p.alpha * v[i], p.alpha * v[i + 1], p.alpha * v[i + 2], p.alpha * v[i + 3]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+                if (col0 + i < n_end && cc0 + i < p.r) orow[cc0 + i] = p.alpha * v[i];
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int col = col0 + i;
+            if (col < n_end && (col % p.rpad) < p.r) p.out32[(int64_t)col * p.ld + m] = p.alpha * v[i];
+        }
     }
-    named_barrier_sync(1, 128);
-    if (!s_last) return;
+}
+
+// Epilogue of one segment, on CTA `cta` of G (four warps, thread = row).
+__device__ __forceinline__ void group_segment_epilogue(const GroupArgs &g, const GroupSeg &sg, int64_t cta, int64_t G,
+                                                       int row, uint32_t taddr) {
+    const GroupProblem &p = g.prob[sg.q];
+    const int gm = sg.tm * 128 + row;
+    const bool rv = gm < p.M;
+    const int n_base = sg.tn * g.BN;
+    const int n_end = min(p.N, n_base + g.BN);
+    const int64_t c0 = group_owner(g, sg.ts, G), c1 = group_owner(g, sg.te - 1, G);
+    if (c0 == c1) {  // the whole tile is this segment
+        for (int c = 0; c < g.BN; c += 16) {
+            if (n_base + c >= n_end) break;
+            float v[16];
+            tmem_ld_x16(taddr + (uint32_t)c, v);
+            if (rv) group_store16(p, gm, n_base + c, n_end, v);
+        }
+        return;
+    }
+    const int64_t gtile = p.tile_begin + sg.tm + (int64_t)sg.tn * p.tiles_m;
+    const size_t slot = (size_t)128 * g.BN;
+    float4 *mine = reinterpret_cast<float4 *>(g.part + (size_t)(cta + gtile) * slot) + row;
+    for (int c = 0; c < g.BN; c += 16) {
+        if (n_base + c >= n_end) break;
+        float v[16];
+        tmem_ld_x16(taddr + (uint32_t)c, v);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            __stcg(mine + (size_t)(c / 4 + q) * 128, make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]));
+    }
     __threadfence();
-    const int gm = gm_base + row;
-    if (gm >= v.M) return;
-    const int n_base = tn * v.BN;
-    const int n_end = min(v.N, n_base + v.BN);
-    for (int col = n_base; col < n_end; ++col) {
-        const float x = __ldcg(ep.out + (int64_t)col * ep.out_ld + gm);
-        ep.out16[(int64_t)col * ep.out_ld + gm] = __float2bfloat16_rn(x);
+    named_barrier_sync(1, 128);
+    int last = 0;
+    if (row == 0) {
+        unsigned int *tk = g.tickets + gtile;
+        last = atomicAdd(tk, 1u) == (unsigned int)(c1 - c0) ? 1 : 0;
+        if (last) atomicExch(tk, 0u);  // every piece has arrived: ready for the next launch
+        __threadfence();
+    }
+    if (!named_barrier_or(1, 128, last)) return;
+    for (int c = 0; c < g.BN; c += 16) {
+        if (n_base + c >= n_end) break;
+        float s[16];
+        for (int64_t j = c0; j <= c1; ++j) {  // pieces in CTA order
+            float v[16];
+            if (j == cta) {
+                tmem_ld_x16(taddr + (uint32_t)c, v);
+            } else {
+                const float4 *src = reinterpret_cast<const float4 *>(g.part + (size_t)(j + gtile) * slot) + row;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 f = __ldcg(src + (size_t)(c / 4 + q) * 128);
+                    v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 16; ++i) s[i] = (j == c0) ? v[i] : s[i] + v[i];
+        }
+        if (rv) group_store16(p, gm, n_base + c, n_end, s);
     }
 }
 
@@ -142,6 +242,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    const int64_t G = gridDim.x;
+    const int64_t x0 = (int64_t)blockIdx.x * g.total_stages / G;
+    const int64_t x1 = ((int64_t)blockIdx.x + 1) * g.total_stages / G;
 
     if (warp == 0) {
         if (lane == 0) {
@@ -149,15 +252,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_parity = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < g.total_tiles && ok; t += gridDim.x) {
-                int q, tm, tn, split;
-                decode_group(g, t, q, tm, tn, split);
-                const GroupProblem &p = g.prob[q];
-                const CUtensorMap *ta = &maps.a[q];
-                const CUtensorMap *tb = &maps.b[q];
-                const int kb0 = split * p.kb_per_split;
-                const int kb1 = min(p.kb_total, kb0 + p.kb_per_split);
-                for (int kb = kb0; kb < kb1; kb += KBS) {
+            GroupSeg sg;
+            for (int64_t x = x0; ok && group_next(g, x, x1, sg);) {
+                const GroupProblem &p = g.prob[sg.q];
+                const CUtensorMap *ta = &maps.a[sg.q];
+                const CUtensorMap *tb = &maps.b[sg.q];
+                const int tm = sg.tm, tn = sg.tn;
+                for (int kb = sg.kb0; kb < sg.kb1; kb += KBS) {
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
                     const uint32_t fb = full0 + 8 * stage;
                     mbar_arrive_expect_tx(fb, kABytesS + b_bytes);  // blocks past K arrive as zeros
@@ -198,12 +299,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             uint32_t phase = 0;
             int it = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < g.total_tiles && ok; t += gridDim.x, ++it) {
-                int q, tm, tn, split;
-                decode_group(g, t, q, tm, tn, split);
-                const GroupProblem &p = g.prob[q];
-                const int kb0 = split * p.kb_per_split;
-                const int kb1 = min(p.kb_total, kb0 + p.kb_per_split);
+            GroupSeg sg;
+            for (int64_t x = x0; ok && group_next(g, x, x1, sg); ++it) {
+                const int kb0 = sg.kb0, kb1 = sg.kb1;
                 const int acc = it & 1;
                 if (!mbar_wait(tempty0 + 8 * acc, (((uint32_t)it >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
                 tc_fence_after();
@@ -241,9 +339,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int qw = warp & 3;
         const int row = qw * 32 + lane;
         int it = 0;
-        for (int t = blockIdx.x; t < g.total_tiles; t += gridDim.x, ++it) {
-            int q, tm, tn, split;
-            decode_group(g, t, q, tm, tn, split);
+        GroupSeg sg;
+        for (int64_t x = x0; group_next(g, x, x1, sg); ++it) {
             const int acc = it & 1;
             const uint32_t par = ((uint32_t)it >> 1) & 1u;
             int ok = 1;
@@ -256,11 +353,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             (void)mbar_try_wait(tfull0 + 8 * acc, par);
             tc_fence_after();
             const uint32_t taddr = tmem_base + ((uint32_t)(qw * 32) << 16) + (uint32_t)(acc * g.BN);
-            const GemmArgs v = group_view(g, g.prob[q]);
-            if (g.prob[q].epi == EPI_ATOMIC_N)
-                epilogue_tile<EPI_ATOMIC_N>(v, tm * 128, tn, row, taddr);
-            else
-                group_atomic_t_tile(v, tm * 128, tm, tn, row, taddr);
+            group_segment_epilogue(g, sg, (int64_t)blockIdx.x, G, row, taddr);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
