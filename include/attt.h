@@ -90,7 +90,7 @@ typedef struct attt_history attt_history;
  * Creates an empty history for n-grams of size n (1 <= n <= 16) that can
  * hold up to max_tokens tokens (0 <= max_tokens <= 16,777,214 = 2^24 - 2) on
  * the current device.  The library allocates the token stream (4 B/token)
- * and an exact n-gram count table of 8 B slots, at least twice as many slots
+ * and an exact n-gram count table of 8 B slots, at least four times as many slots
  * as max_tokens.  *out is set on success.  Allocation failure returns
  * ATTT_ERR_CUDA.
  */

@@ -3,8 +3,9 @@
 // count table over it, and the per-token loss weights of an update.
 //
 // Table design (GB300-first):
-//   * open addressing, linear probing, power-of-two capacity >= 2 * max_tokens
-//     (load factor <= 1/2) of 8-byte slots, one 64-bit word each:
+//   * open addressing, linear probing, power-of-two capacity >= 4 * max_tokens
+//     (load factor <= 1/4: a new n-gram then takes ~1.4 probes, against ~2.5
+//     at 1/2) of 8-byte slots, one 64-bit word each:
 //       [63:48] 16-bit hash tag | [47:24] history position + 1 of the
 //       n-gram's first occurrence | [23:0] count
 //     (0 = empty).  A new n-gram costs one CAS that claims the slot with its
@@ -45,10 +46,12 @@ __device__ __forceinline__ unsigned long long mix64(unsigned long long h) {
     return h;
 }
 
-// Hash of n consecutive tokens.
+// Hash of n consecutive tokens: one odd 64-bit multiply per token (each step
+// a bijection of the state), then one finalizer so that the low bits (the
+// slot) and the top 16 bits (the tag) depend on every token.
 __device__ __forceinline__ unsigned long long ngram_hash(const int32_t *t, int n) {
     unsigned long long h = 0x9e3779b97f4a7c15ull * (unsigned long long)(n + 1);
-    for (int i = 0; i < n; ++i) h = mix64(h ^ (unsigned long long)(uint32_t)t[i]) + 0x632be59bd9b4e019ull;
+    for (int i = 0; i < n; ++i) h = (h ^ (unsigned long long)(uint32_t)t[i]) * 0xbf58476d1ce4e5b9ull;
     return mix64(h);
 }
 
@@ -74,34 +77,66 @@ __device__ __forceinline__ unsigned int table_lookup(const Slot *table, unsigned
     return 0u;
 }
 
-// One thread per new n-gram start position p in [p_begin, p_begin + count).
-// (Aggregating equal n-grams inside a warp with match_any was measured to
-// cost more than the atomics it saves on Zipf text, so every thread inserts
-// its own occurrence.)
+// Inserts one occurrence (at history position p) of the n-gram g with hash
+// hsh, starting from the result k of the optimistic claim of slot idx.
+__device__ __forceinline__ bool insert_rest(Slot *table, unsigned long long mask, const int32_t *hist,
+                                            const int32_t *g, int n, unsigned long long hsh, Slot claim,
+                                            unsigned long long idx, Slot k) {
+    const unsigned int tag = slot_tag(hsh);
+    for (int probe = 0; probe < kMaxProbe; ++probe) {
+        if (k == 0ull) return true;  // claimed with count 1
+        if ((unsigned int)(k >> 48) == tag && ngram_equal(hist + slot_pos(k), g, n)) {
+            atomicAdd(table + idx, 1ull);  // count lives in the low 24 bits
+            return true;
+        }
+        idx = (idx + 1) & mask;
+        k = atomicCAS(table + idx, 0ull, claim);
+    }
+    return false;
+}
+
+// kInsPer new n-gram start positions per thread, p = p_begin + blockIdx.x *
+// kInsTile + k * blockDim.x + threadIdx.x.  The block's tokens are staged in
+// shared memory (coalesced); each thread hashes its n-gram there and makes
+// the optimistic claim (atomicCAS of an empty slot with count 1); an occupied
+// slot returns its word, which is then compared.  Measured on the 1 M-token
+// stress history: 2, 4 or 8 n-grams per thread (their claims in flight
+// together) were slower than one (the insert is bound by L2 atomic throughput,
+// ~88 G random 64-bit CAS/s measured alone, not by a thread's latency), and a
+// load factor of 1/4 instead of 1/2 took it from 42-51 to 32-35 us.
+// (Aggregating equal n-grams inside a warp with match_any cost more than the
+// atomics it saves on Zipf text, so every occurrence is inserted.)
+constexpr int kInsPer = 1;
+constexpr int kInsTile = 256 * kInsPer;
+
 __global__ void __launch_bounds__(256) history_insert_kernel(const int32_t *__restrict__ hist, int64_t p_begin,
                                                              int64_t count, int n, Slot *table,
                                                              unsigned long long mask, int *status) {
-    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= count) return;
-    const int64_t p = p_begin + i;
-    const int32_t *g = hist + p;
-    const unsigned long long hsh = ngram_hash(g, n);
-    const unsigned int tag = slot_tag(hsh);
-    const Slot claim = ((unsigned long long)tag << 48) | ((unsigned long long)(uint32_t)(p + 1) << 24) | 1ull;
-    unsigned long long idx = hsh & mask;
-    for (int probe = 0; probe < kMaxProbe; ++probe) {
-        Slot *s = table + idx;
-        // Optimistic claim: one round trip for a new n-gram; an occupied slot
-        // returns its word, which is then compared.
-        const Slot k = atomicCAS(s, 0ull, claim);
-        if (k == 0ull) return;  // claimed with count 1
-        if ((unsigned int)(k >> 48) == tag && ngram_equal(hist + slot_pos(k), g, n)) {
-            atomicAdd(s, 1ull);  // count lives in the low 24 bits
-            return;
+    __shared__ int32_t tok[kInsTile + kMaxN];
+    const int64_t i0 = (int64_t)blockIdx.x * kInsTile;
+    const int64_t rem = count - i0;
+    const int nt = (int)(rem < kInsTile ? rem : kInsTile) + n - 1;  // tokens of this block's n-grams
+    for (int t = threadIdx.x; t < nt; t += blockDim.x) tok[t] = hist[p_begin + i0 + t];
+    __syncthreads();
+    unsigned long long hsh[kInsPer], idx[kInsPer];
+    Slot claim[kInsPer], k[kInsPer];
+#pragma unroll
+    for (int q = 0; q < kInsPer; ++q) {
+        const int li = q * blockDim.x + threadIdx.x;
+        if (i0 + li < count) {
+            hsh[q] = ngram_hash(tok + li, n);
+            idx[q] = hsh[q] & mask;
+            claim[q] = ((unsigned long long)slot_tag(hsh[q]) << 48) |
+                       ((unsigned long long)(uint32_t)(p_begin + i0 + li + 1) << 24) | 1ull;
+            k[q] = atomicCAS(table + idx[q], 0ull, claim[q]);
         }
-        idx = (idx + 1) & mask;
     }
-    record_error(status, ATTT_ERR_TABLE_FULL);
+#pragma unroll
+    for (int q = 0; q < kInsPer; ++q) {
+        const int li = q * blockDim.x + threadIdx.x;
+        if (i0 + li < count && !insert_rest(table, mask, hist, tok + li, n, hsh[q], claim[q], idx[q], k[q]))
+            record_error(status, ATTT_ERR_TABLE_FULL);
+    }
 }
 
 // count(g, H) for m query n-grams stored row-major [m, n].
@@ -179,7 +214,7 @@ attt_status attt_history_create(int n, int64_t max_tokens, attt_history **out) {
     attt_status st = attt::current_device(&dev);
     if (st != ATTT_OK) return st;
     unsigned long long cap = 1024;
-    while (cap < 2ull * (unsigned long long)max_tokens) cap <<= 1;
+    while (cap < 4ull * (unsigned long long)max_tokens) cap <<= 1;
     attt_history *h = new (std::nothrow) attt_history();
     if (!h) return ATTT_ERR_CUDA;
     h->n = n;
@@ -251,7 +286,7 @@ attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_
     if (p_end < p_begin) return ATTT_OK;
     const int64_t count = p_end - p_begin + 1;
     const int threads = 256;
-    const int64_t blocks = (count + threads - 1) / threads;
+    const int64_t blocks = (count + attt::kInsTile - 1) / attt::kInsTile;
     attt::history_insert_kernel<<<(unsigned)blocks, threads, 0, stream>>>(h->d_tokens, p_begin, count, h->n,
                                                                           h->d_table, h->capacity - 1, h->d_status);
     attt::count_launch();
