@@ -76,6 +76,7 @@ constexpr int kPrepRows = 64;
 
 __global__ void __launch_bounds__(256) lora_prep_kernel(PrepArgs a) {
     __shared__ __nv_bfloat16 slab[kPrepRows][64 + 2];  // [row of A_p][column c], r <= 64
+    griddep_launch_dependents();  // pass 1 may launch; it waits for this grid before reading AT, BT
     const int p = blockIdx.y;
     const int64_t nslab = (a.din + kPrepRows - 1) / kPrepRows;
     for (int64_t sb = blockIdx.x; sb < nslab; sb += gridDim.x) {
@@ -148,6 +149,8 @@ struct GroupSpec {
     float *outp[kMaxProj];
 };
 
+constexpr int kGroupMinStages = 2;
+
 // Launches every problem of `specs` in one grouped kernel; every CTA streams
 // the same number of K stages (stream-K split, tc_group.cuh).
 template <bool A_MN, bool B_MN>
@@ -218,9 +221,24 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, float *pa
         1024 + (size_t)g.stages * g.kbs * (kABytes + gemm_b_stage_bytes(BN)) + 8 * (2 * g.stages + 5) + 16;
     auto kern = tc_gemm_group_kernel<A_MN, B_MN>;
     if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
-    int grid = stages < sms ? (int)stages : sms;  // every CTA gets at least one stage
+    // every CTA gets at least kGroupMinStages stages (at least one), so that a
+    // tile is not cut into more pieces than its final sum can afford
+    int64_t gmax = stages / kGroupMinStages;
+    if (gmax < 1) gmax = 1;
+    int grid = gmax < sms ? (int)gmax : sms;
     if (grid > kGroupMaxGrid) grid = kGroupMaxGrid;
-    kern<<<grid, kGemmThreads, smem, stream>>>(maps, g);
+    // a programmatic dependent of the previous kernel of the call (prep, or pass 1)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kGemmThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, kern, maps, g) != cudaSuccess) return ATTT_ERR_CUDA;
     count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }

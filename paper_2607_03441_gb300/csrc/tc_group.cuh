@@ -175,21 +175,37 @@ __device__ __forceinline__ void group_segment_epilogue(const GroupArgs &g, const
     if (!named_barrier_or(1, 128, last)) return;
     for (int c = 0; c < g.BN; c += 16) {
         if (n_base + c >= n_end) break;
+        float own[16];
+        tmem_ld_x16(taddr + (uint32_t)c, own);
         float s[16];
-        for (int64_t j = c0; j <= c1; ++j) {  // pieces in CTA order
-            float v[16];
-            if (j == cta) {
-                tmem_ld_x16(taddr + (uint32_t)c, v);
-            } else {
-                const float4 *src = reinterpret_cast<const float4 *>(g.part + (size_t)(j + gtile) * slot) + row;
+        // pieces in CTA order, four partials loaded together (their loads in
+        // flight at once), summed in order after they land
+        for (int64_t j0 = c0; j0 <= c1; j0 += 4) {
+            float4 f[4][4];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float4 f = __ldcg(src + (size_t)(c / 4 + q) * 128);
-                    v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
+            for (int b = 0; b < 4; ++b) {
+                const int64_t j = j0 + b;
+                if (j <= c1 && j != cta) {
+                    const float4 *src = reinterpret_cast<const float4 *>(g.part + (size_t)(j + gtile) * slot) + row;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) f[b][q] = __ldcg(src + (size_t)(c / 4 + q) * 128);
                 }
             }
 #pragma unroll
-            for (int i = 0; i < 16; ++i) s[i] = (j == c0) ? v[i] : s[i] + v[i];
+            for (int b = 0; b < 4; ++b) {
+                const int64_t j = j0 + b;
+                if (j > c1) break;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 x = (j == cta) ? make_float4(own[4 * q], own[4 * q + 1], own[4 * q + 2], own[4 * q + 3])
+                                                : f[b][q];
+                    if (j == c0) {
+                        s[4 * q] = x.x; s[4 * q + 1] = x.y; s[4 * q + 2] = x.z; s[4 * q + 3] = x.w;
+                    } else {
+                        s[4 * q] += x.x; s[4 * q + 1] += x.y; s[4 * q + 2] += x.z; s[4 * q + 3] += x.w;
+                    }
+                }
+            }
         }
         if (rv) group_store16(p, gm, n_base + c, n_end, s);
     }
@@ -226,6 +242,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             mbar_init(tfull0 + 8 * a, 1);
             mbar_init(tempty0 + 8 * a, 4);
         }
+        griddep_launch_dependents();  // the next grid may launch; it waits for this one before reading its results
         mbar_init(drain0, 1);
         *abort_flag = 0;
         fence_mbar_init();
@@ -248,6 +265,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
     if (warp == 0) {
         if (lane == 0) {
+            griddep_wait();  // the B operands (adapters, u, v) come from the previous grid
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_parity = 0;
@@ -336,6 +354,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (!mbar_wait(drain0, 0u, &no_abort)) record_error(g.status, ATTT_ERR_TIMEOUT);
         }
     } else {
+        griddep_wait();  // tickets, slots and outputs follow the previous grid
         const int qw = warp & 3;
         const int row = qw * 32 + lane;
         int it = 0;
