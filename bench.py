@@ -17,7 +17,6 @@ host cores instead (rank 0 only).
 from __future__ import annotations
 
 import argparse
-import glob
 import hashlib
 import json
 import os
@@ -243,11 +242,16 @@ def row_report(wl, events, peaks):
     return out
 
 
+# The sources the Eq. 10 call is built from (its kernels, the contraction
+# engine they share, the PTX wrappers and the host-side helpers).
+CE_SOURCES = ("ce.cu", "tc_gemm.cuh", "gemm_launch.cuh", "attt_common.cuh", "attt_host.h", "api.cu")
+
+
 def _sources_sha256() -> str:
-    """Hash of the CUDA sources and the C header, to tell whether a stored
-    ncu capture still describes the kernels that run."""
+    """Hash of the sources of the Eq. 10 call and the C header, to tell whether
+    a stored ncu capture of that call still describes the kernels that run."""
     h = hashlib.sha256()
-    files = sorted(glob.glob(os.path.join(ROOT, "paper_2607_03441_gb300", "csrc", "*")))
+    files = [os.path.join(ROOT, "paper_2607_03441_gb300", "csrc", f) for f in CE_SOURCES]
     files.append(os.path.join(ROOT, "include", "attt.h"))
     for f in files:
         h.update(os.path.basename(f).encode())
