@@ -149,10 +149,12 @@ __global__ void __launch_bounds__(256) history_count_kernel(const int32_t *__res
     out[i] = table_lookup(table, mask, hist, g, n, ngram_hash(g, n));
 }
 
-constexpr int kWTile = 256;  // positions j per block
+constexpr int kWTile = 256;                 // positions j per block
+constexpr int kWThreads = kWTile + kMaxN;  // one thread per candidate window (at most kWTile + n - 1)
 
-// Eq. 8 then Eq. 9 for positions [j0, j0 + kWTile) of the update.
-__global__ void __launch_bounds__(kWTile) ngram_weights_kernel(const int32_t *__restrict__ x, int64_t L, int n,
+// Eq. 8 then Eq. 9 for positions [j0, j0 + kWTile) of the update.  Each
+// window has its own thread, so a block's critical path is one lookup.
+__global__ void __launch_bounds__(kWThreads) ngram_weights_kernel(const int32_t *__restrict__ x, int64_t L, int n,
                                                                const int32_t *__restrict__ hist, int64_t hist_len,
                                                                const Slot *table, unsigned long long mask,
                                                                float w_min, float *__restrict__ w) {
@@ -178,7 +180,7 @@ __global__ void __launch_bounds__(kWTile) ngram_weights_kernel(const int32_t *__
     }
     __syncthreads();
     const int64_t j = j0 + threadIdx.x;
-    if (j >= L) return;
+    if (threadIdx.x >= kWTile || j >= L) return;
     // windows covering j: s in [j-n+1, j], i.e. indices [threadIdx.x, threadIdx.x + n - 1];
     // invalid windows (s < 0 or s > L-n) hold count 0, which never changes the max.
     unsigned int f = 0u;
@@ -319,7 +321,7 @@ attt_status attt_ngram_weights(const attt_history *h, const int32_t *d_tokens, i
         return ATTT_ERR_INVALID_ARG;
     if (L == 0) return ATTT_OK;
     const int64_t blocks = (L + attt::kWTile - 1) / attt::kWTile;
-    attt::ngram_weights_kernel<<<(unsigned)blocks, attt::kWTile, 0, stream>>>(
+    attt::ngram_weights_kernel<<<(unsigned)blocks, attt::kWThreads, 0, stream>>>(
         d_tokens, L, h->n, h->d_tokens, h->len, h->d_table, h->capacity - 1, w_min, d_w);
     attt::count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
