@@ -65,6 +65,10 @@ def _load():
         lib.oracle_lora_grad.argtypes = [P, P, P, P, i64, i64, i64, ctypes.c_int,
                                          ctypes.c_double, P, P]
         lib.oracle_sgd_step.restype = None
+        lib.oracle_lora_forward.argtypes = [P, P, P, P, i64, i64, i64, ctypes.c_int, ctypes.c_double, P]
+        lib.oracle_lora_forward.restype = None
+        lib.oracle_lora_input_grad.argtypes = [P, P, P, P, i64, i64, i64, ctypes.c_int, ctypes.c_double, P]
+        lib.oracle_lora_input_grad.restype = None
         lib.oracle_sgd_step.argtypes = [P, P, i64, ctypes.c_float]
         lib.oracle_to_bf16.restype = None
         lib.oracle_to_bf16.argtypes = [P, P, i64]
@@ -188,6 +192,37 @@ def lora_grad(x_bf16, dy_bf16, A_bf16, B_bf16, scale: float):
                              dA.ctypes.data_as(ctypes.c_void_p),
                              dB.ctypes.data_as(ctypes.c_void_p))
     return dA, dB
+
+
+def lora_forward(x_bf16, W0_bf16, A_bf16, B_bf16, scale: float):
+    """h = x W0 + s (x A) B in fp64 [L, dout] (the adapted projection)."""
+    x, px = _c(x_bf16, np.uint16)
+    W0, pW = _c(W0_bf16, np.uint16)
+    A, pA = _c(A_bf16, np.uint16)
+    B, pB = _c(B_bf16, np.uint16)
+    L, din = x.shape
+    dout = W0.shape[1]
+    r = A.shape[1]
+    assert W0.shape[0] == din and A.shape[0] == din and B.shape == (r, dout)
+    h = np.zeros((L, dout), dtype=np.float64)
+    _load().oracle_lora_forward(px, pW, pA, pB, L, din, dout, r, float(scale), h.ctypes.data_as(ctypes.c_void_p))
+    return h
+
+
+def lora_input_grad(dy_bf16, W0_bf16, A_bf16, B_bf16, scale: float):
+    """dx = dy W0^T + s (dy B^T) A^T in fp64 [L, din]."""
+    dy, pdy = _c(dy_bf16, np.uint16)
+    W0, pW = _c(W0_bf16, np.uint16)
+    A, pA = _c(A_bf16, np.uint16)
+    B, pB = _c(B_bf16, np.uint16)
+    L, dout = dy.shape
+    din = W0.shape[0]
+    r = A.shape[1]
+    assert W0.shape[1] == dout and A.shape[0] == din and B.shape == (r, dout)
+    dx = np.zeros((L, din), dtype=np.float64)
+    _load().oracle_lora_input_grad(pdy, pW, pA, pB, L, din, dout, r, float(scale),
+                                   dx.ctypes.data_as(ctypes.c_void_p))
+    return dx
 
 
 def sgd_step(p32, g32, lr: float):

@@ -22,6 +22,9 @@
  *           dB = s (xA)^T dy,  dA = s x^T (dy B^T);
  *           then plain SGD  theta <- theta - lr * grad  on fp32 masters and a
  *           round-to-nearest-even refresh of the bf16 copies.
+ *   For an update chained through the adapted projection (its output is the
+ *           LM head's input): the forward h = x W0 + s (x A) B and the input
+ *           gradient dx = dy W0^T + s (dy B^T) A^T.
  *
  * Floating point: all sums in fp64 over the bf16 inputs exactly as stored;
  * Eq. 9 and the SGD step in fp32 exactly as the formulas read (this file is
@@ -275,6 +278,68 @@ void oracle_lora_grad(const uint16_t *x, const uint16_t *dy, const uint16_t *A, 
     }
     free(u);
     free(v);
+}
+
+/* ------------------------------------------------------------------------ */
+/* The adapted projection of a chained update (Appendix C adapter)          */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * x [L, din], W0 [din, dout], A [din, r], B [r, dout] (bf16, row-major):
+ *   h = x W0 + s (x A) B        [L, dout], fp64
+ */
+void oracle_lora_forward(const uint16_t *x, const uint16_t *W0, const uint16_t *A, const uint16_t *B,
+                         int64_t L, int64_t din, int64_t dout, int r, double s, double *h)
+{
+#pragma omp parallel
+    {
+        double *u = (double *)calloc((size_t)(r > 0 ? r : 1), sizeof(double));
+#pragma omp for schedule(static)
+        for (int64_t l = 0; l < L; ++l) {
+            for (int c = 0; c < r; ++c) {
+                double a = 0.0;
+                for (int64_t i = 0; i < din; ++i) a += bf16_value(x[l * din + i]) * bf16_value(A[i * r + c]);
+                u[c] = a;
+            }
+            for (int64_t o = 0; o < dout; ++o) {
+                double a = 0.0;
+                for (int64_t i = 0; i < din; ++i) a += bf16_value(x[l * din + i]) * bf16_value(W0[i * dout + o]);
+                double b = 0.0;
+                for (int c = 0; c < r; ++c) b += u[c] * bf16_value(B[(int64_t)c * dout + o]);
+                h[l * dout + o] = a + s * b;
+            }
+        }
+        free(u);
+    }
+}
+
+/*
+ * The gradient of the projection's input, dy [L, dout] being the gradient of
+ * its output:  dx = dy W0^T + s (dy B^T) A^T        [L, din], fp64
+ */
+void oracle_lora_input_grad(const uint16_t *dy, const uint16_t *W0, const uint16_t *A, const uint16_t *B,
+                            int64_t L, int64_t din, int64_t dout, int r, double s, double *dx)
+{
+#pragma omp parallel
+    {
+        double *v = (double *)calloc((size_t)(r > 0 ? r : 1), sizeof(double));
+#pragma omp for schedule(static)
+        for (int64_t l = 0; l < L; ++l) {
+            for (int c = 0; c < r; ++c) {
+                double a = 0.0;
+                for (int64_t o = 0; o < dout; ++o) a += bf16_value(dy[l * dout + o]) * bf16_value(B[(int64_t)c * dout + o]);
+                v[c] = a;
+            }
+            for (int64_t i = 0; i < din; ++i) {
+                double a = 0.0;
+                for (int64_t o = 0; o < dout; ++o) a += bf16_value(dy[l * dout + o]) * bf16_value(W0[i * dout + o]);
+                double b = 0.0;
+                for (int c = 0; c < r; ++c) b += v[c] * bf16_value(A[i * r + c]);
+                dx[l * din + i] = a + s * b;
+            }
+        }
+        free(v);
+    }
 }
 
 /* ------------------------------------------------------------------------ */
