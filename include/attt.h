@@ -13,6 +13,9 @@
  *                           gradient step, given the upstream gradient dy of
  *                           each adapted projection.
  *   attt_lora_step          the Eq. 2 SGD step on the adapter parameters.
+ *   attt_lora_forward,      the adapted projection of a chained update (its
+ *   attt_lora_input_grad    output feeds the LM head): forward and the
+ *                           gradient of its input.
  *   attt_history_insert     Algorithm 1's last line: append x_k to the token
  *                           history H (a concatenation, Sec. 3.3).
  *
@@ -255,6 +258,45 @@ ATTT_API attt_status attt_lora_grad_noalloc(const attt_bf16 *d_x, int64_t L, int
 ATTT_API attt_status attt_lora_step(float *d_A32, float *d_B32, const float *d_dA, const float *d_dB,
                            int64_t din, int64_t dout, int r, float lr,
                            attt_bf16 *d_A16, attt_bf16 *d_B16, attt_stream stream);
+
+/* ------------------------------------------------------------------------ */
+/* The adapted projection of a chained update: the LoRA-adapted linear map   */
+/* y = x W0 + s (x A) B (Appendix C adapter; W0 frozen) whose output is the  */
+/* LM head's input h, so that the second gradient step of an update         */
+/* (Appendix C: two steps per update) sees the adapter the first one moved. */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Workspace bytes attt_lora_forward / attt_lora_input_grad need.
+ */
+ATTT_API size_t attt_lora_forward_workspace_bytes(int64_t L, int64_t din, int64_t dout, int r);
+ATTT_API size_t attt_lora_input_grad_workspace_bytes(int64_t L, int64_t din, int64_t dout, int r);
+
+/*
+ * h = x W0 + s (x A) B with x = d_x (bf16 [L, din]), W0 = d_W0 (bf16
+ * [din, dout], frozen), A = d_A (bf16 [din, r]), B = d_B (bf16 [r, dout]),
+ * s = scale; h = d_h (bf16 [L, dout], round to nearest even).  s (x A) is
+ * rounded to bf16 once; products are bf16, sums fp32.  Requirements:
+ * L >= 1, din and dout multiples of 8 (>= 8), 1 <= r <= 64, every pointer
+ * 16-byte aligned, d_ws at least attt_lora_forward_workspace_bytes(L, din,
+ * dout, r) bytes and 256-byte aligned.  Three launches.
+ */
+ATTT_API attt_status attt_lora_forward(const attt_bf16 *d_x, const attt_bf16 *d_W0, const attt_bf16 *d_A,
+                                       const attt_bf16 *d_B, int64_t L, int64_t din, int64_t dout, int r,
+                                       float scale, attt_bf16 *d_h, void *d_ws, size_t ws_bytes,
+                                       attt_stream stream);
+
+/*
+ * The gradient of the projection's input from the gradient dy = d_dy (bf16
+ * [L, dout]) of its output:  dx = dy W0^T + s (dy B^T) A^T  (fp32 [L, din]
+ * into d_dx).  Shapes and alignment as attt_lora_forward; r must be a
+ * multiple of 8 (A is read in place; ATTT_ERR_UNSUPPORTED otherwise).
+ * s (dy B^T) is rounded to bf16 once.  Two launches.
+ */
+ATTT_API attt_status attt_lora_input_grad(const attt_bf16 *d_dy, const attt_bf16 *d_W0, const attt_bf16 *d_A,
+                                          const attt_bf16 *d_B, int64_t L, int64_t din, int64_t dout, int r,
+                                          float scale, float *d_dx, void *d_ws, size_t ws_bytes,
+                                          attt_stream stream);
 
 #ifdef __cplusplus
 }

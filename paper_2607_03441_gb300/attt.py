@@ -66,6 +66,10 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_lora_grad": (i32, [P, i64, i64, i32, P, P, P, P, i32, f32, P, P, P, sz, P]),
             "attt_lora_step": (i32, [P, P, P, P, i64, i64, i32, f32, P, P, P]),
             "attt_lora_grad_noalloc": (i32, [P, i64, i64, i32, P, P, P, P, i32, f32, P, P, P]),
+            "attt_lora_forward_workspace_bytes": (sz, [i64, i64, i64, i32]),
+            "attt_lora_input_grad_workspace_bytes": (sz, [i64, i64, i64, i32]),
+            "attt_lora_forward": (i32, [P, P, P, P, i64, i64, i64, i32, f32, P, P, sz, P]),
+            "attt_lora_input_grad": (i32, [P, P, P, P, i64, i64, i64, i32, f32, P, P, sz, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -300,3 +304,51 @@ def attt_lora_step(A32: torch.Tensor, B32: torch.Tensor, dA: torch.Tensor, dB: t
         _ptr(A32), _ptr(B32), _ptr(dA), _ptr(dB), din, dout, r, float(lr),
         _bf16(A16) if A16 is not None else None, _bf16(B16) if B16 is not None else None, _stream(stream)),
         "attt_lora_step")
+
+
+# --------------------------------------------------------------------------
+# the adapted projection of a chained update
+# --------------------------------------------------------------------------
+
+def attt_lora_forward_workspace_bytes(L: int, din: int, dout: int, r: int) -> int:
+    return int(load_library().attt_lora_forward_workspace_bytes(int(L), int(din), int(dout), int(r)))
+
+
+def attt_lora_input_grad_workspace_bytes(L: int, din: int, dout: int, r: int) -> int:
+    return int(load_library().attt_lora_input_grad_workspace_bytes(int(L), int(din), int(dout), int(r)))
+
+
+def attt_lora_forward(x: torch.Tensor, W0: torch.Tensor, A: torch.Tensor, B: torch.Tensor, scale: float,
+                      h: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
+                      stream=None) -> torch.Tensor:
+    """h = x W0 + s (x A) B (bf16).  Returns h."""
+    L, din = x.shape
+    dout = W0.shape[1]
+    r = A.shape[1]
+    if h is None:
+        h = torch.empty(L, dout, dtype=torch.bfloat16, device=x.device)
+    if workspace is None:
+        workspace = torch.empty(attt_lora_forward_workspace_bytes(L, din, dout, r), dtype=torch.uint8,
+                                device=x.device)
+    _check(load_library().attt_lora_forward(
+        _bf16(x), _bf16(W0), _bf16(A), _bf16(B), L, din, dout, int(r), float(scale), _bf16(h), _ptr(workspace),
+        workspace.numel(), _stream(stream)), "attt_lora_forward")
+    return h
+
+
+def attt_lora_input_grad(dy: torch.Tensor, W0: torch.Tensor, A: torch.Tensor, B: torch.Tensor, scale: float,
+                         dx: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None,
+                         stream=None) -> torch.Tensor:
+    """dx = dy W0^T + s (dy B^T) A^T (fp32).  Returns dx."""
+    L, dout = dy.shape
+    din = W0.shape[0]
+    r = A.shape[1]
+    if dx is None:
+        dx = torch.empty(L, din, dtype=torch.float32, device=dy.device)
+    if workspace is None:
+        workspace = torch.empty(attt_lora_input_grad_workspace_bytes(L, din, dout, r), dtype=torch.uint8,
+                                device=dy.device)
+    _check(load_library().attt_lora_input_grad(
+        _bf16(dy), _bf16(W0), _bf16(A), _bf16(B), L, din, dout, int(r), float(scale), _ptr(dx), _ptr(workspace),
+        workspace.numel(), _stream(stream)), "attt_lora_input_grad")
+    return dx

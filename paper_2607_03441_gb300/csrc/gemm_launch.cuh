@@ -16,6 +16,13 @@ struct GemmProblem {
     int64_t b_rows_ld;
     int64_t b_rows, b_k;
     int M, N, K;
+    // optional second operand pair over K2 more K (same majors, no offsets):
+    // D = A B^T + A2 B2^T
+    const void *a2 = nullptr;
+    int64_t a2_rows_ld = 0, a2_rows = 0, a2_k = 0;
+    const void *b2 = nullptr;
+    int64_t b2_rows_ld = 0, b2_rows = 0, b2_k = 0;
+    int K2 = 0;
     int BN;
     int a_m_off = 0, a_k_off = 0, b_n_off = 0, b_k_off = 0;
     bool pair = false;  // run on CTA pairs (256-row tiles, cta_group::2)
@@ -89,6 +96,21 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     else
         ok = make_tmap_bf16(&tb, p.b, (uint64_t)p.b_rows, (uint64_t)p.b_k, (uint64_t)p.b_rows_ld * 2, 64, 64);
     if (!ok) return ATTT_ERR_INVALID_ARG;
+    CUtensorMap ta2 = ta, tb2 = tb;
+    if (p.K2 > 0) {
+        if (!p.a2 || !p.b2) return ATTT_ERR_INVALID_ARG;
+        if (!A_MN)
+            ok = make_tmap_bf16(&ta2, p.a2, (uint64_t)p.a2_k, (uint64_t)p.a2_rows, (uint64_t)p.a2_rows_ld * 2, 64, 128);
+        else
+            ok = make_tmap_bf16(&ta2, p.a2, (uint64_t)p.a2_rows, (uint64_t)p.a2_k, (uint64_t)p.a2_rows_ld * 2, 64, 64);
+        if (!ok) return ATTT_ERR_INVALID_ARG;
+        if (!B_MN)
+            ok = make_tmap_bf16(&tb2, p.b2, (uint64_t)p.b2_k, (uint64_t)p.b2_rows, (uint64_t)p.b2_rows_ld * 2, 64,
+                                (uint32_t)(p.pair ? p.BN / 2 : p.BN));
+        else
+            ok = make_tmap_bf16(&tb2, p.b2, (uint64_t)p.b2_rows, (uint64_t)p.b2_k, (uint64_t)p.b2_rows_ld * 2, 64, 64);
+        if (!ok) return ATTT_ERR_INVALID_ARG;
+    }
     // EPI_CE_EXP writes E through TMA stores: [M, G_ld] bf16, 32 x 32 boxes
     // EPI_F32_ACC reads and writes `out` through TMA: [M, N] fp32 of pitch out_ld, 32 x 32 boxes
     CUtensorMap tc = tb;
@@ -98,6 +120,9 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     } else if (EPI == EPI_F32_ACC) {
         if (!make_tmap_f32(&tc, ep.out, (uint64_t)p.N, (uint64_t)p.M, (uint64_t)ep.out_ld * 4, 32, 32))
             return ATTT_ERR_INVALID_ARG;
+    } else if (EPI == EPI_BF16) {
+        if (!make_tmap_bf16(&tc, ep.out16, (uint64_t)p.N, (uint64_t)p.M, (uint64_t)ep.out_ld * 2, 32, 32, 64))
+            return ATTT_ERR_INVALID_ARG;
     }
 
     GemmArgs g{};
@@ -105,11 +130,12 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.N = p.N;
     g.BN = p.BN;
     const int bn_cta = p.pair ? p.BN / 2 : p.BN;  // B rows one CTA stages
-    g.e_stage_bytes = EPI == EPI_CE_EXP ? kEStageBytes : EPI == EPI_F32_ACC ? kF32StageBytes : 0u;
+    g.e_stage_bytes = (EPI == EPI_CE_EXP || EPI == EPI_BF16) ? kEStageBytes : EPI == EPI_F32_ACC ? kF32StageBytes : 0u;
     g.stages = gemm_stages(bn_cta, g.e_stage_bytes);
     g.tiles_m = (int)cdiv(p.M, 128);
     g.tiles_n = (int)cdiv(p.N, p.BN);
-    g.kb_total = (int)cdiv(p.K, 64);
+    g.kb_split = (int)cdiv(p.K, 64);
+    g.kb_total = g.kb_split + (p.K2 > 0 ? (int)cdiv(p.K2, 64) : 0);
     const int sms = num_sms(dev);
     const int units = p.pair ? sms / 2 : sms;  // concurrent tiles
     const int tiles = (p.pair ? (g.tiles_m + 1) / 2 : g.tiles_m) * g.tiles_n;
@@ -154,7 +180,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
         cfg.gridDim = dim3((unsigned)(ntiles < sms ? ntiles : sms));
         cfg.attrs = attr;
         cfg.numAttrs = na;
-        if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, g) != cudaSuccess) return ATTT_ERR_CUDA;
+        if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, ta2, tb2, g) != cudaSuccess) return ATTT_ERR_CUDA;
     } else {
         auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN>;
         if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
@@ -167,7 +193,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
         ++na;
         cfg.attrs = attr;
         cfg.numAttrs = na;
-        if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, g) != cudaSuccess) return ATTT_ERR_CUDA;
+        if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, ta2, tb2, g) != cudaSuccess) return ATTT_ERR_CUDA;
     }
     count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;

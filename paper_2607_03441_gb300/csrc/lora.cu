@@ -14,6 +14,12 @@
 // finishes each tile last; u and v go to bf16 in between.  Three launches per
 // call: prep (adapters to K-major), pass 1 (u and every v_p, grouped), pass 2
 // (dA and every dB_p, grouped).
+//
+// The adapted projection itself (for a chained update, where the projection
+// feeds the LM head): the forward h = x W0 + s (x A) B and the input gradient
+// dx = dy W0^T + s (dy B^T) A^T.  Each is one tcgen05 contraction whose K runs
+// over two operand pairs, [x | s u] [W0 ; B] and [dy | s v] [W0^T ; A^T], after
+// a skinny grouped launch that forms s u = s x A or s v = s dy B^T in bf16.
 #include "gemm_launch.cuh"
 #include "tc_group.cuh"
 
@@ -337,9 +343,159 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
     return ATTT_OK;
 }
 
+
+// ---------------------------------------------------------------------------
+// The adapted projection: forward and input gradient
+// ---------------------------------------------------------------------------
+
+// Split slots of the dx contraction's tail split (as for the CE's dh).
+constexpr int kDxSplitRegions = 160;
+
+struct ProjLayout {
+    int rpad;
+    __nv_bfloat16 *AT, *BT;  // forward: A^T padded [rpad, din]; B padded [rpad, dout] (written by the prep)
+    __nv_bfloat16 *s16;      // s u or s v, [L, rpad] bf16 row-major
+    unsigned int *tickets;   // the skinny launch's tiles, then the tail split's counters
+    float *part;             // the skinny launch's partial slots
+    float *split_ws;         // input gradient: tail-split partials
+    int64_t tiles;
+    size_t bytes;
+};
+
+static ProjLayout proj_layout(void *ws, int64_t L, int64_t din, int64_t dout, int r, bool fwd) {
+    ProjLayout c{};
+    c.rpad = (int)round_up(r, 16);
+    c.tiles = cdiv(L, 128);
+    Carve cv{static_cast<char *>(ws), 0};
+    if (fwd) {
+        c.AT = cv.take<__nv_bfloat16>((size_t)(c.rpad * din));
+        c.BT = cv.take<__nv_bfloat16>((size_t)(c.rpad * dout));
+    }
+    c.s16 = cv.take<__nv_bfloat16>((size_t)(L * c.rpad));
+    c.tickets = cv.take<unsigned int>((size_t)(c.tiles + kDxSplitRegions));
+    c.part = cv.take<float>((size_t)(c.tiles + kGroupMaxGrid) * 128 * c.rpad);
+    if (!fwd) c.split_ws = cv.take<float>((size_t)kDxSplitRegions * 128 * 256);
+    c.bytes = (size_t)round_up((int64_t)cv.used, 256);
+    return c;
+}
+
+static attt_status proj_check(const void *a, const void *b, const void *c, const void *d, const void *out,
+                              int64_t L, int64_t din, int64_t dout, int r) {
+    if (!a || !b || !c || !d || !out) return ATTT_ERR_INVALID_ARG;
+    if (L < 1 || din < 8 || dout < 8 || din % 8 != 0 || dout % 8 != 0 || r < 1 || r > 64) return ATTT_ERR_INVALID_ARG;
+    if (L > (1ll << 30) || din > (1ll << 30) || dout > (1ll << 30)) return ATTT_ERR_UNSUPPORTED;
+    if (!aligned16(a) || !aligned16(b) || !aligned16(c) || !aligned16(d) || !aligned16(out)) return ATTT_ERR_INVALID_ARG;
+    return ATTT_OK;
+}
+
 }  // namespace attt
 
 extern "C" {
+
+size_t attt_lora_forward_workspace_bytes(int64_t L, int64_t din, int64_t dout, int r) {
+    if (L < 1 || din < 1 || dout < 1 || r < 1 || r > 64) return 0;
+    return attt::proj_layout(nullptr, L, din, dout, r, true).bytes;
+}
+
+size_t attt_lora_input_grad_workspace_bytes(int64_t L, int64_t din, int64_t dout, int r) {
+    if (L < 1 || din < 1 || dout < 1 || r < 1 || r > 64) return 0;
+    return attt::proj_layout(nullptr, L, din, dout, r, false).bytes;
+}
+
+attt_status attt_lora_forward(const attt_bf16 *d_x, const attt_bf16 *d_W0, const attt_bf16 *d_A, const attt_bf16 *d_B,
+                              int64_t L, int64_t din, int64_t dout, int r, float scale, attt_bf16 *d_h, void *d_ws,
+                              size_t ws_bytes, attt_stream stream) {
+    using namespace attt;
+    attt_status st = proj_check(d_x, d_W0, d_A, d_B, d_h, L, din, dout, r);
+    if (st != ATTT_OK) return st;
+    if (!d_ws || !aligned256(d_ws) || ws_bytes < attt_lora_forward_workspace_bytes(L, din, dout, r))
+        return ATTT_ERR_WORKSPACE;
+    int dev;
+    st = current_device(&dev);
+    if (st != ATTT_OK) return st;
+    ProjLayout c = proj_layout(d_ws, L, din, dout, r, true);
+    {   // A^T (and B) padded to rpad rows, tickets zeroed
+        PrepArgs a{};
+        a.A[0] = reinterpret_cast<const __nv_bfloat16 *>(d_A);
+        a.B[0] = reinterpret_cast<const __nv_bfloat16 *>(d_B);
+        a.BT[0] = c.BT;
+        a.dout[0] = dout;
+        a.nproj = 1; a.r = r; a.rpad = c.rpad; a.din = din; a.AT = c.AT;
+        a.tickets = c.tickets; a.ntickets = c.tiles;
+        int64_t maxn = cdiv(din, kPrepRows) * 256;
+        if (c.rpad * dout > maxn) maxn = c.rpad * dout;
+        lora_prep_kernel<<<dim3(grid_for(maxn, 256, dev), 1), 256, 0, stream>>>(a);
+        count_launch();
+        if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
+    }
+    {   // s u = s x A, bf16 [L, rpad]
+        GroupSpec u{};
+        u.a = d_x; u.a_rows_ld = din; u.a_rows = L; u.a_k = din;
+        u.b = c.AT; u.b_rows_ld = din; u.b_rows = c.rpad; u.b_k = din;
+        u.M = (int)L; u.N = c.rpad; u.K = (int)din;
+        u.out = GOUT_N16; u.out16 = c.s16; u.ld = c.rpad; u.alpha = scale; u.r = c.rpad; u.rpad = c.rpad;
+        st = launch_group<false, false>(&u, 1, c.rpad, c.part, c.tickets, dev, stream, nullptr);
+        if (st != ATTT_OK) return st;
+    }
+    {   // h = [x | s u] [W0 ; B]: W0 [din, dout] and B [r, dout] are read MN-major
+        GemmProblem p{};
+        p.a = d_x; p.a_rows_ld = din; p.a_rows = L; p.a_k = din;
+        p.b = d_W0; p.b_rows_ld = dout; p.b_rows = dout; p.b_k = din;
+        p.a2 = c.s16; p.a2_rows_ld = c.rpad; p.a2_rows = L; p.a2_k = c.rpad;
+        p.b2 = d_B; p.b2_rows_ld = dout; p.b2_rows = dout; p.b2_k = r;
+        p.M = (int)L; p.N = (int)dout; p.K = (int)din; p.K2 = c.rpad; p.BN = 256; p.pair = L > 128;
+        p.pdl = true;
+        EpiParams ep{};
+        ep.out16 = reinterpret_cast<__nv_bfloat16 *>(d_h); ep.out_ld = dout; ep.alpha = 1.0f;
+        st = launch_gemm<EPI_BF16, false, true>(p, ep, dev, stream);
+        if (st != ATTT_OK) return st;
+    }
+    return ATTT_OK;
+}
+
+attt_status attt_lora_input_grad(const attt_bf16 *d_dy, const attt_bf16 *d_W0, const attt_bf16 *d_A,
+                                 const attt_bf16 *d_B, int64_t L, int64_t din, int64_t dout, int r, float scale,
+                                 float *d_dx, void *d_ws, size_t ws_bytes, attt_stream stream) {
+    using namespace attt;
+    attt_status st = proj_check(d_dy, d_W0, d_A, d_B, d_dx, L, din, dout, r);
+    if (st != ATTT_OK) return st;
+    if (r % 8 != 0) return ATTT_ERR_UNSUPPORTED;  // A [din, r] is read in place: rows of 16-byte multiples
+    if (!d_ws || !aligned256(d_ws) || ws_bytes < attt_lora_input_grad_workspace_bytes(L, din, dout, r))
+        return ATTT_ERR_WORKSPACE;
+    int dev;
+    st = current_device(&dev);
+    if (st != ATTT_OK) return st;
+    ProjLayout c = proj_layout(d_ws, L, din, dout, r, false);
+    if (cudaMemsetAsync(c.tickets, 0, sizeof(unsigned int) * (size_t)(c.tiles + kDxSplitRegions), stream) !=
+        cudaSuccess)
+        return ATTT_ERR_CUDA;
+    {   // s v = s dy B^T, bf16 [L, rpad]; B [r, dout] is the K-major operand (rows past r read as zeros)
+        GroupSpec v{};
+        v.a = d_dy; v.a_rows_ld = dout; v.a_rows = L; v.a_k = dout;
+        v.b = d_B; v.b_rows_ld = dout; v.b_rows = r; v.b_k = dout;
+        v.M = (int)L; v.N = c.rpad; v.K = (int)dout;
+        v.out = GOUT_N16; v.out16 = c.s16; v.ld = c.rpad; v.alpha = scale; v.r = c.rpad; v.rpad = c.rpad;
+        st = launch_group<false, false>(&v, 1, c.rpad, c.part, c.tickets, dev, stream, nullptr);
+        if (st != ATTT_OK) return st;
+    }
+    {   // dx = [dy | s v] [W0^T ; A^T]: W0 [din, dout] and A [din, r] are read K-major
+        GemmProblem p{};
+        p.a = d_dy; p.a_rows_ld = dout; p.a_rows = L; p.a_k = dout;
+        p.b = d_W0; p.b_rows_ld = dout; p.b_rows = din; p.b_k = dout;
+        p.a2 = c.s16; p.a2_rows_ld = c.rpad; p.a2_rows = L; p.a2_k = c.rpad;
+        p.b2 = d_A; p.b2_rows_ld = r; p.b2_rows = din; p.b2_k = r;
+        p.M = (int)L; p.N = (int)din; p.K = (int)dout; p.K2 = c.rpad; p.BN = 256; p.pair = L > 128;
+        p.pdl = true;
+        p.split_ws = c.split_ws; p.split_tick = c.tickets + c.tiles; p.split_regions = kDxSplitRegions;
+        EpiParams ep{};
+        ep.out = d_dx; ep.out_ld = din; ep.accumulate = 0; ep.alpha = 1.0f;
+        st = launch_gemm<EPI_F32_ACC, false, false>(p, ep, dev, stream);
+        if (st != ATTT_OK) return st;
+    }
+    return ATTT_OK;
+}
+
+
 
 size_t attt_lora_workspace_bytes(int64_t L, int64_t din, int nproj, const int64_t *dout, int r) {
     if (L < 1 || din < 1 || nproj < 1 || nproj > attt::kMaxProj || !dout || r < 1 || r > 64) return 0;

@@ -2,6 +2,8 @@
 // kernels and the LoRA adapter-gradient kernels.
 //
 // D[M x N] = A[M x K] * B[N x K]^T with bf16 operands and fp32 accumulation.
+// K may run over two operand pairs, D = A B^T + A2 B2^T (the K blocks of A2 /
+// B2 follow those of A / B; both pairs share the operand majors).
 //   * one CTA per SM, persistent over output tiles of 128 x BN (BN <= 256);
 //   * warp 0: TMA producer (one thread) filling a ring of `stages` shared-
 //     memory stages of 64-deep K blocks, 128-byte swizzled;
@@ -29,8 +31,7 @@ namespace attt {
 enum EpiKind : int {
     EPI_CE_EXP = 0,    // per (row, vocab tile): max m, E = exp(z - m) as bf16, sum of E, target logit
     EPI_F32_ACC = 2,   // out[m, n] = (acc ? alpha_m out[m, n] : 0) + beta_m acc [- gamma_m W[t_m, n]]  (fp32)
-    EPI_ATOMIC_T = 3,  // out[n, m] += alpha * acc   (fp32, transposed, split-K)
-    EPI_ATOMIC_N = 4,  // out_p[m, c] += alpha * acc for column n = p * rpad + c (split-K)
+    EPI_BF16 = 5,      // out16[m, n] = bf16(alpha * acc)  (row-major, through TMA boxes)
 };
 
 constexpr int kMaxProj = 8;
@@ -57,11 +58,7 @@ struct EpiParams {
     const __nv_bfloat16 *fix_W;
     int64_t fix_ld;
     int fix_V;
-    __nv_bfloat16 *out16;    // grouped EPI_ATOMIC_T: bf16 copy of out, written by the last split
-    unsigned int *tickets;   // grouped EPI_ATOMIC_T: one counter per tile, starts at 0
-    float *outp[kMaxProj];
-    int r;     // valid columns per projection block
-    int rpad;  // column block width per projection
+    __nv_bfloat16 *out16;    // EPI_BF16 output, row pitch out_ld
 };
 
 struct GemmArgs {
@@ -77,6 +74,7 @@ struct GemmArgs {
     // previous grid in the stream started, so the producer need not wait for it
     // (the epilogue always does).
     int operands_ready;
+    int kb_split;  // K blocks of the first operand pair; later ones come from A2 / B2
     int *status;
     EpiParams ep;
     // Tail split (tc_gemm_kernel / tc_gemm_pair_kernel): tiles [0, whole_tiles)
@@ -284,6 +282,26 @@ __device__ __forceinline__ void f32_tile_store(const GemmArgs &g, const CUtensor
     }
 }
 
+// EPI_BF16 for this warp's 32 rows (from y; lane = row): out16 = bf16(alpha
+// acc) for the tile's columns [n_base, n_end), box by box through the warp's
+// staging buffers; the running box count `ec` picks the buffer.
+__device__ __forceinline__ void bf16_tile_store(const GemmArgs &g, const CUtensorMap *tm, uint32_t sE, uint32_t &ec,
+                                                int lane, int y, int n_base, int n_end, uint32_t taddr) {
+    if (y >= g.M) return;  // every row of this warp lies past M (warp-uniform)
+    for (int c = 0; c < g.BN; c += 32) {
+        if (n_base + c >= n_end) break;
+        float v[32];
+        tmem_ld_x32(taddr + (uint32_t)c, v);
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+            __nv_bfloat162 b = __floats2bfloat162_rn(g.ep.alpha * v[i], g.ep.alpha * v[i + 1]);
+            pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
+        }
+        e_block_store(tm, sE, (int)(ec++), lane, pk, n_base + c, y);
+    }
+}
+
 // tmE / sE: the E tensor map and this warp's staging buffers (EPI_CE_EXP).
 template <int EPI>
 __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, int tn, int row, uint32_t taddr,
@@ -395,45 +413,6 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
             ep.part[(int64_t)(ep.tile0 + tn) * g.M + gm] = make_float2(mx, sm);
             if (hit) ep.ztgt[gm] = zt;
         }
-    } else if constexpr (EPI == EPI_ATOMIC_T) {
-        for (int c = 0; c < g.BN; c += 16) {
-            if (n_base + c >= n_end) break;
-            float v[16];
-            tmem_ld_x16(taddr + (uint32_t)c, v);
-            if (rv) {
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int col = n_base + c + i;
-                    if (col < n_end && (col % ep.rpad) < ep.r)
-                        atomicAdd(ep.out + (int64_t)col * ep.out_ld + gm, ep.alpha * v[i]);
-                }
-            }
-        }
-    } else if constexpr (EPI == EPI_ATOMIC_N) {
-        for (int c = 0; c < g.BN; c += 16) {
-            if (n_base + c >= n_end) break;
-            float v[16];
-            tmem_ld_x16(taddr + (uint32_t)c, v);
-            if (rv) {
-                // the 16 columns lie in one projection (rpad is a multiple of
-                // 16); with r % 4 == 0 and an aligned row they go out as four
-                // 16-byte reductions instead of sixteen scalar atomics
-                const int col0 = n_base + c;
-                const int p = col0 / ep.rpad, cc0 = col0 - p * ep.rpad;
-                float *orow = ep.outp[p] + (int64_t)gm * ep.r;
-                if (col0 + 16 <= n_end && (ep.r & 3) == 0 && (reinterpret_cast<uintptr_t>(orow) & 15) == 0) {
-#pragma unroll
-                    for (int i = 0; i < 16; i += 4)
-                        if (cc0 + i < ep.r)
-                            red_add_v4(orow + cc0 + i, ep.alpha * v[i], ep.alpha * v[i + 1], ep.alpha * v[i + 2],
-                                       ep.alpha * v[i + 3]);
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 16; ++i)
-                        if (col0 + i < n_end && cc0 + i < ep.r) atomicAdd(orow + cc0 + i, ep.alpha * v[i]);
-                }
-            }
-        }
     }
 }
 
@@ -500,7 +479,8 @@ __device__ __forceinline__ void epilogue_piece_f32_acc(const GemmArgs &g, const 
 template <int EPI, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const __grid_constant__ CUtensorMap tmC, const GemmArgs g) {
+                   const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmA2,
+                   const __grid_constant__ CUtensorMap tmB2, const GemmArgs g) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = g.stages;
@@ -536,6 +516,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         fence_mbar_init();
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
+        if (g.kb_split < g.kb_total) {
+            tma_prefetch_desc(&tmA2);
+            tma_prefetch_desc(&tmB2);
+        }
     }
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), g.tmem_cols);
@@ -565,18 +549,24 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     mbar_arrive_expect_tx(fb, kABytes + b_bytes);
                     const uint32_t a_dst = smem_u32(sA + (size_t)stage * kABytes);
                     const uint32_t b_dst = smem_u32(sB + (size_t)stage * b_bytes);
-                    const int k = kb * 64;
+                    // K block kb of the first pair, or K block kb - kb_split of the second
+                    const bool sec = kb >= g.kb_split;
+                    const CUtensorMap *pa = sec ? &tmA2 : &tmA;
+                    const CUtensorMap *pb = sec ? &tmB2 : &tmB;
+                    const int ka = sec ? (kb - g.kb_split) * 64 : g.a_k_off + kb * 64;
+                    const int kbk = sec ? (kb - g.kb_split) * 64 : g.b_k_off + kb * 64;
+                    const int am = (sec ? 0 : g.a_m_off) + tm * 128;
+                    const int bn = (sec ? 0 : g.b_n_off) + tn * g.BN;
                     if (!A_MN) {
-                        tma_load_2d(a_dst, &tmA, fb, g.a_k_off + k, g.a_m_off + tm * 128);
+                        tma_load_2d(a_dst, pa, fb, ka, am);
                     } else {
-                        tma_load_2d(a_dst, &tmA, fb, g.a_m_off + tm * 128, g.a_k_off + k);
-                        tma_load_2d(a_dst + 8192, &tmA, fb, g.a_m_off + tm * 128 + 64, g.a_k_off + k);
+                        tma_load_2d(a_dst, pa, fb, am, ka);
+                        tma_load_2d(a_dst + 8192, pa, fb, am + 64, ka);
                     }
                     if (!B_MN) {
-                        tma_load_2d(b_dst, &tmB, fb, g.b_k_off + k, g.b_n_off + tn * g.BN);
+                        tma_load_2d(b_dst, pb, fb, kbk, bn);
                     } else {
-                        for (int b = 0; b < g.BN / 64; ++b)
-                            tma_load_2d(b_dst + 8192 * b, &tmB, fb, g.b_n_off + tn * g.BN + 64 * b, g.b_k_off + k);
+                        for (int b = 0; b < g.BN / 64; ++b) tma_load_2d(b_dst + 8192 * b, pb, fb, bn + 64 * b, kbk);
                     }
                     issued_mask |= 1u << stage;
                     issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
@@ -642,6 +632,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int q = warp & 3;
         const int row = q * 32 + lane;
         F32Stage fst{smem_u32(sE) + (uint32_t)q * 8192u, smem_u32(sE) + 32768u + (uint32_t)q * 16u, 0u};
+        uint32_t bec = 0;  // EPI_BF16 boxes stored by this warp
         int it = 0;
         for (int w = blockIdx.x; w < nwork; w += gridDim.x, ++it) {
             const Work wi = work_item(g, w, g.tiles_m);
@@ -668,6 +659,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                                    min(g.N, n_base + g.BN), abort_flag,
                                    [&](int c, float(&v)[32]) { tmem_ld_x32(taddr + (uint32_t)c, v); });
                 }
+            } else if constexpr (EPI == EPI_BF16) {
+                const int gm = wi.tm * 128 + row;
+                bf16_tile_store(g, &tmC, smem_u32(sE) + (uint32_t)q * 4096u, bec, lane, gm - lane, wi.tn * g.BN,
+                                min(g.N, (wi.tn + 1) * g.BN), taddr);
             } else {
                 epilogue_tile<EPI>(g, wi.tm * 128, wi.tn, row, taddr, &tmC, smem_u32(sE) + (uint32_t)q * 4096u);
             }
@@ -676,7 +671,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
         }
         // every TMA store of the epilogue has landed before the CTA retires
-        if constexpr (EPI == EPI_CE_EXP || EPI == EPI_F32_ACC) {
+        if constexpr (EPI == EPI_CE_EXP || EPI == EPI_F32_ACC || EPI == EPI_BF16) {
             if (lane == 0) bulk_wait<0>();
         }
     }
@@ -700,7 +695,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 template <int EPI, bool A_MN, bool B_MN>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const __grid_constant__ CUtensorMap tmC, const GemmArgs g) {
+                   const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmA2,
+                   const __grid_constant__ CUtensorMap tmB2, const GemmArgs g) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = g.stages;
@@ -739,6 +735,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         fence_mbar_init();
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
+        if (g.kb_split < g.kb_total) {
+            tma_prefetch_desc(&tmA2);
+            tma_prefetch_desc(&tmB2);
+        }
     }
     cluster_sync();  // both CTAs' barriers exist before any cross-CTA signal
     if (warp == 1) {
@@ -765,26 +765,32 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bool ok = true;
             for (int w = cid; w < nwork && ok; w += ncl) {
                 const Work wi = work_item(g, w, tiles_m2);
-                const int arow = g.a_m_off + wi.tm * 256 + 128 * (int)rank;
-                const int brow = g.b_n_off + wi.tn * g.BN + BNh * (int)rank;
+                const int arow0 = wi.tm * 256 + 128 * (int)rank;
+                const int brow0 = wi.tn * g.BN + BNh * (int)rank;
                 for (int kb = wi.kb0; kb < wi.kb1; ++kb) {
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
                     if (leader) mbar_arrive_expect_tx(full0 + 8 * stage, 2u * (kABytes + b_bytes));
                     const uint32_t fb = lead_full0 + 8 * stage;
                     const uint32_t a_dst = smem_u32(sA + (size_t)stage * kABytes);
                     const uint32_t b_dst = smem_u32(sB + (size_t)stage * b_bytes);
-                    const int k = kb * 64;
+                    // K block kb of the first pair, or K block kb - kb_split of the second
+                    const bool sec = kb >= g.kb_split;
+                    const CUtensorMap *pa = sec ? &tmA2 : &tmA;
+                    const CUtensorMap *pb = sec ? &tmB2 : &tmB;
+                    const int ka = sec ? (kb - g.kb_split) * 64 : g.a_k_off + kb * 64;
+                    const int kbk = sec ? (kb - g.kb_split) * 64 : g.b_k_off + kb * 64;
+                    const int arow = (sec ? 0 : g.a_m_off) + arow0;
+                    const int brow = (sec ? 0 : g.b_n_off) + brow0;
                     if (!A_MN) {
-                        tma_load_2d_pair(a_dst, &tmA, fb, g.a_k_off + k, arow);
+                        tma_load_2d_pair(a_dst, pa, fb, ka, arow);
                     } else {
-                        tma_load_2d_pair(a_dst, &tmA, fb, arow, g.a_k_off + k);
-                        tma_load_2d_pair(a_dst + 8192, &tmA, fb, arow + 64, g.a_k_off + k);
+                        tma_load_2d_pair(a_dst, pa, fb, arow, ka);
+                        tma_load_2d_pair(a_dst + 8192, pa, fb, arow + 64, ka);
                     }
                     if (!B_MN) {
-                        tma_load_2d_pair(b_dst, &tmB, fb, g.b_k_off + k, brow);
+                        tma_load_2d_pair(b_dst, pb, fb, kbk, brow);
                     } else {
-                        for (int b = 0; b < BNh / 64; ++b)
-                            tma_load_2d_pair(b_dst + 8192 * b, &tmB, fb, brow + 64 * b, g.b_k_off + k);
+                        for (int b = 0; b < BNh / 64; ++b) tma_load_2d_pair(b_dst + 8192 * b, pb, fb, brow + 64 * b, kbk);
                     }
                     if (++stage == S) { stage = 0; phase ^= 1u; }
                 }
@@ -842,6 +848,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int q = warp & 3;
         const int row = q * 32 + lane;
         F32Stage fst{smem_u32(sE) + (uint32_t)q * 8192u, smem_u32(sE) + 32768u + (uint32_t)q * 16u, 0u};
+        uint32_t bec = 0;  // EPI_BF16 boxes stored by this warp
         int it = 0;
         for (int w = cid; w < nwork; w += ncl, ++it) {
             const Work wi = work_item(g, w, tiles_m2);
@@ -869,6 +876,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                                    min(g.N, n_base + g.BN), abort_flag,
                                    [&](int c, float(&v)[32]) { tmem_ld_x32(taddr + (uint32_t)c, v); });
                 }
+            } else if constexpr (EPI == EPI_BF16) {
+                bf16_tile_store(g, &tmC, smem_u32(sE) + (uint32_t)q * 4096u, bec, lane, gm_base + 32 * q,
+                                wi.tn * g.BN, min(g.N, (wi.tn + 1) * g.BN), taddr);
             } else {
                 epilogue_tile<EPI>(g, gm_base, wi.tn, row, taddr, &tmC, smem_u32(sE) + (uint32_t)q * 4096u);
             }
@@ -877,7 +887,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (lane == 0) mbar_arrive_cluster(lead_tempty0 + 8 * acc);
         }
         // every TMA store of the epilogue has landed before the CTA retires
-        if constexpr (EPI == EPI_CE_EXP || EPI == EPI_F32_ACC) {
+        if constexpr (EPI == EPI_CE_EXP || EPI == EPI_F32_ACC || EPI == EPI_BF16) {
             if (lane == 0) bulk_wait<0>();
         }
     }

@@ -34,6 +34,7 @@ enum GroupOut : int {
     GOUT_T16 = 0,  // out16[n * ld + m] = bf16(alpha D[m, n])                          (transposed, bf16)
     GOUT_N32 = 1,  // outp[n / rpad][m * r + n % rpad] = alpha D[m, n], n % rpad < r   (a row-major block per rpad columns)
     GOUT_T32 = 2,  // out32[n * ld + m] = alpha D[m, n], n % rpad < r                  (transposed, fp32)
+    GOUT_N16 = 3,  // out16[m * ld + n] = bf16(alpha D[m, n])                          (row-major, bf16)
 };
 
 struct GroupProblem {
@@ -125,11 +126,27 @@ __device__ __forceinline__ void group_store16(const GroupProblem &p, int m, int 
             for (int i = 0; i < 16; ++i)
                 if (col0 + i < n_end && cc0 + i < p.r) orow[cc0 + i] = p.alpha * v[i];
         }
-    } else {
+    } else if (p.out == GOUT_T32) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
             const int col = col0 + i;
             if (col < n_end && (col % p.rpad) < p.r) p.out32[(int64_t)col * p.ld + m] = p.alpha * v[i];
+        }
+    } else {
+        __nv_bfloat16 *o = p.out16 + (int64_t)m * p.ld + col0;
+        if (col0 + 16 <= n_end && (reinterpret_cast<uintptr_t>(o) & 15) == 0) {
+            uint32_t pk[8];
+#pragma unroll
+            for (int i = 0; i < 16; i += 2) {
+                __nv_bfloat162 b = __floats2bfloat162_rn(p.alpha * v[i], p.alpha * v[i + 1]);
+                pk[i / 2] = *reinterpret_cast<uint32_t *>(&b);
+            }
+            reinterpret_cast<uint4 *>(o)[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            reinterpret_cast<uint4 *>(o)[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+                if (col0 + i < n_end) o[i] = __float2bfloat16_rn(p.alpha * v[i]);
         }
     }
 }
