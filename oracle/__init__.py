@@ -243,3 +243,42 @@ def to_bf16(p32) -> np.ndarray:
     b = np.zeros(p.shape, dtype=np.uint16)
     _load().oracle_to_bf16(pp, b.ctypes.data_as(ctypes.c_void_p), p.size)
     return b
+
+
+# --------------------------------------------------------------------------
+# One update of Algorithm 1, chained through the adapted projection
+# --------------------------------------------------------------------------
+
+def episode_update(H, tokens, x_bf16, W0_bf16, Wlm_bf16, A32, B32, *, n: int, w_min: float, scale: float,
+                   lr: float, grad_steps: int = 2, want_dx: bool = True):
+    """Algorithm 1 for update x_k (= `tokens`, also the Eq. 10 targets) with
+    the adapter on the projection whose output is the LM head's input:
+
+      w = Eq. 9(Eq. 8(x_k, H))                       (once per update)
+      grad_steps times (Appendix C: two):
+        h = x W0 + s (x A) B, stored as bf16          (A, B: bf16 copies)
+        loss, dh = Eq. 10(h, W_lm, x_k, w)
+        dy = bf16(fp32(dh))
+        dA, dB = the adapter gradients; dx = dy W0^T + s (dy B^T) A^T
+        A, B <- A - lr dA, B - lr dB (Eq. 2, fp32) and refresh the bf16 copies
+      H <- H || x_k
+
+    Returns a dict with w, losses [grad_steps], dx (list, or None), A32, B32
+    (fp32 after the update) and H (the new history)."""
+    w = ngram_weights(H, tokens, n, w_min)
+    A = np.array(A32, dtype=np.float32, copy=True)
+    B = np.array(B32, dtype=np.float32, copy=True)
+    A16, B16 = to_bf16(A), to_bf16(B)
+    losses, dxs = [], []
+    for _ in range(int(grad_steps)):
+        h16 = to_bf16(lora_forward(x_bf16, W0_bf16, A16, B16, scale).astype(np.float32))
+        loss, _, _, dh = ce_loss(h16, Wlm_bf16, tokens, w)
+        dy = to_bf16(dh.astype(np.float32))
+        dA, dB = lora_grad(x_bf16, dy, A16, B16, scale)
+        if want_dx:
+            dxs.append(lora_input_grad(dy, W0_bf16, A16, B16, scale))
+        A, A16 = sgd_step(A, dA.astype(np.float32), lr)
+        B, B16 = sgd_step(B, dB.astype(np.float32), lr)
+        losses.append(loss)
+    H = np.concatenate([np.asarray(H, dtype=np.int32), np.asarray(tokens, dtype=np.int32)])
+    return {"w": w, "losses": np.array(losses), "dx": dxs if want_dx else None, "A32": A, "B32": B, "H": H}

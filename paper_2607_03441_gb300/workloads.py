@@ -19,6 +19,11 @@ Qwen / Gemma weights, none of which are available here):
 * Dense tensors: fp32 normal samples rounded once to bf16 (round to nearest
   even); hidden ~ N(0, 1), LM head ~ N(0, 0.02), LoRA A ~ N(0, 0.02),
   B = 0.01 * N(0, 1), activations x and upstream grads dy ~ N(0, 1).
+* Chained episodes (the adapted projection's output is the LM head's input):
+  the frozen projection W0 [din, d] ~ N(0, 1/din), so that h = x W0 has unit
+  variance like the hidden states above; one x ~ N(0, 1) per update; update
+  texts copy spans from the episode's history so far, with the repeat
+  fraction rising like the long episode's.
 
 Every array comes from its own numpy PCG64 stream keyed by (seed, name).
 """
@@ -228,3 +233,83 @@ def dense_inputs(wl: Workload, with_lm_head: bool = True) -> Dict[str, np.ndarra
         out[f"B/{p.name}"] = normal_bf16(s, f"B/{p.name}", (wl.r, p.dout), 0.01)
         out[f"dy/{p.name}"] = normal_bf16(s, f"dy/{p.name}", (wl.L, p.dout), 1.0)
     return out
+
+
+# --------------------------------------------------------------------------
+# chained episodes: the adapted projection feeds the LM head
+# --------------------------------------------------------------------------
+
+@dataclasses.dataclass
+class EpisodeWorkload:
+    name: str
+    seed: int
+    L: int                # update tokens
+    V: int
+    n: int
+    din: int              # adapted projection input width
+    d: int                # its output width = LM head input
+    r: int
+    updates: int          # updates per episode
+    hist_len: int = 0     # prior history before the first update
+    grad_steps: int = 2   # Appendix C
+    cadence: int = 5      # Sec. 4 default K
+    frac_first: float = 0.05
+    frac_last: float = 0.80
+    w_min: float = W_MIN
+    lr: float = LORA_LR
+
+    @property
+    def scale(self) -> float:
+        return 2.0
+
+
+EPISODES: Dict[str, EpisodeWorkload] = {
+    # Tiny shapes (512 x 512 projection, vocab 8192), three updates after the
+    # 2,048-token prior history.
+    "tiny-episode": EpisodeWorkload("tiny-episode", 0, L=256, V=8192, n=4, din=512, d=512, r=8, updates=3,
+                                    hist_len=2048),
+    # 7B-class shapes (hidden 3584, vocab 152064, rank 16): 16 updates of
+    # 2,048 tokens from an empty history.
+    "7b-episode": EpisodeWorkload("7b-episode", 1, L=2048, V=152064, n=4, din=3584, d=3584, r=16, updates=16),
+}
+
+
+def episode_frac(ew: EpisodeWorkload, k: int) -> float:
+    """Repeat fraction of update k (1-based), linear from first to last."""
+    if ew.updates <= 1:
+        return ew.frac_first
+    return ew.frac_first + (ew.frac_last - ew.frac_first) * (k - 1) / (ew.updates - 1)
+
+
+def episode_history(ew: EpisodeWorkload) -> np.ndarray:
+    return zipf_ids(rng_for(ew.seed, "episode/history"), ew.hist_len, ew.V)
+
+
+def episode_texts(ew: EpisodeWorkload) -> List[np.ndarray]:
+    """Update texts of one episode; update k copies spans from the prior
+    history and the updates before it."""
+    out: List[np.ndarray] = []
+    H = episode_history(ew)
+    for k in range(1, ew.updates + 1):
+        x = zipf_ids(rng_for(ew.seed, f"episode/ids{k}"), ew.L, ew.V)
+        x = copy_spans(rng_for(ew.seed, f"episode/spans{k}"), x, H, episode_frac(ew, k))
+        out.append(x)
+        H = np.concatenate([H, x])
+    return out
+
+
+def episode_dense(ew: EpisodeWorkload) -> Dict[str, np.ndarray]:
+    """bf16 bits of W0 [din, d] and the LM head [V, d]; fp32 A0 [din, r] and
+    B0 [r, d] (the bf16-rounded draws, so both copies start equal)."""
+    s = ew.seed
+    return {
+        "W0": normal_bf16(s, "episode/W0", (ew.din, ew.d), float(1.0 / np.sqrt(ew.din))),
+        "W": normal_bf16(s, "episode/lm_head", (ew.V, ew.d), 0.02),
+        "A0": bf16_to_f32(normal_bf16(s, "episode/A0", (ew.din, ew.r), 0.02)),
+        "B0": bf16_to_f32(normal_bf16(s, "episode/B0", (ew.r, ew.d), 0.01)),
+    }
+
+
+def episode_x(ew: EpisodeWorkload, k: int) -> np.ndarray:
+    """bf16 bits of the projection inputs [L, din] of update k (1-based)."""
+    return normal_bf16(ew.seed, f"episode/x{k}", (ew.L, ew.din), 1.0)
