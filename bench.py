@@ -248,11 +248,10 @@ CE_SOURCES = ("ce.cu", "tc_gemm.cuh", "gemm_launch.cuh", "attt_common.cuh", "att
 
 
 def _sources_sha256() -> str:
-    """Hash of the sources of the Eq. 10 call and the C header, to tell whether
-    a stored ncu capture of that call still describes the kernels that run."""
+    """Hash of the sources of the Eq. 10 call, to tell whether a stored ncu
+    capture of that call still describes the kernels that run."""
     h = hashlib.sha256()
     files = [os.path.join(ROOT, "paper_2607_03441_gb300", "csrc", f) for f in CE_SOURCES]
-    files.append(os.path.join(ROOT, "include", "attt.h"))
     for f in files:
         h.update(os.path.basename(f).encode())
         with open(f, "rb") as fh:
@@ -570,6 +569,186 @@ def run_stress(args):
 
 
 # ---------------------------------------------------------------------------
+# chained episodes: Algorithm 1 with the Sec. 4 / Appendix C schedule, the
+# adapted projection feeding the LM head (attt_episode_*)
+# ---------------------------------------------------------------------------
+
+def _agent_cuts(L, K):
+    """Split an update text of L tokens into the texts of K agent steps."""
+    return [round(i * L / K) for i in range(K + 1)]
+
+
+def episode_flops(ew):
+    """Tensor FLOPs of one update: per gradient step the Eq. 10 pair (4 L V d),
+    the projection forward and input gradient (2 L din d each, plus the
+    rank-r terms) and the adapter gradients (4 L r (din + d))."""
+    L, V, din, d, r = ew.L, ew.V, ew.din, ew.d, ew.r
+    per_step = 4.0 * L * V * d + 2 * (2.0 * L * din * d + 2.0 * L * r * (din + d)) + 4.0 * L * r * (din + d)
+    return ew.grad_steps * per_step
+
+
+def run_episode(args):
+    import torch
+    from paper_2607_03441_gb300 import attt
+    from paper_2607_03441_gb300 import build
+    ws, rank, local = _dist()
+    build.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+    ew = wk.EPISODES[args.workload]
+    peaks = _peaks()
+    texts = wk.episode_texts(ew)
+    dense = wk.episode_dense(ew)
+    xs_host = [wk.episode_x(ew, k) for k in range(1, ew.updates + 1)]
+
+    def bf(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    W0, Wlm = bf(dense["W0"]), bf(dense["W"])
+    ep = attt.Episode(W0, Wlm, torch.from_numpy(dense["A0"]).to(dev), torch.from_numpy(dense["B0"]).to(dev),
+                      n=ew.n, max_history=ew.hist_len + ew.L * ew.updates, max_update=ew.L, scale=ew.scale,
+                      lr=ew.lr, w_min=ew.w_min, grad_steps=ew.grad_steps, cadence=ew.cadence)
+    H0 = torch.from_numpy(wk.episode_history(ew)).to(dev)
+    tok = [torch.from_numpy(t).to(dev) for t in texts]
+    xs = [bf(x) for x in xs_host]
+    cuts = _agent_cuts(ew.L, ew.cadence)
+    losses = torch.empty(ew.grad_steps, dtype=torch.float32, device=dev)
+    dx = torch.empty(ew.grad_steps, ew.L, ew.din, dtype=torch.float32, device=dev)
+    state = {"k": 0}
+
+    def start_episode():
+        ep.reset()
+        if ew.hist_len:
+            attt.attt_history_insert(ep.history(), H0)
+
+    def step(tok_k=None, x_k=None):
+        """One update: K agent steps, the last of which trains; a new episode
+        (reset + prior history) starts after the last update of one."""
+        k = state["k"]
+        if k == 0:
+            start_episode()
+        t, x = (tok[k], xs[k]) if tok_k is None else (tok_k, x_k)
+        fired = False
+        for i in range(ew.cadence):
+            fired = ep.agent_step(t[cuts[i]:cuts[i + 1]], x[cuts[i]:cuts[i + 1]], losses=losses, dx=dx)
+        assert fired
+        state["k"] = (k + 1) % ew.updates
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if attt.attt_device_status() != 0 or attt.attt_history_status(ep.history()) != 0:
+        raise RuntimeError("device status error after warm-up")
+
+    def barrier():
+        if pg is not None:
+            pg.barrier()
+
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    n0 = attt.attt_kernel_launches()
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    n1 = attt.attt_kernel_launches()
+    barrier()
+    clk = clocks.stop()
+    t_ms = e0.elapsed_time(e1)
+    if attt.attt_device_status() != 0 or attt.attt_history_status(ep.history()) != 0:
+        raise RuntimeError("device status error in the timed region")
+
+    # end to end: each update's text and projection inputs copied from pinned
+    # host memory every step (on the same stream, before its agent steps), the
+    # losses read back every step
+    tok_h = [torch.from_numpy(t).pin_memory() for t in texts]
+    xs_h = [torch.from_numpy(x.view(np.int16)).pin_memory() for x in xs_host]
+    tok_d = torch.empty(ew.L, dtype=torch.int32, device=dev)
+    x_d = torch.empty(ew.L, ew.din, dtype=torch.int16, device=dev)
+    loss_host = torch.empty(ew.grad_steps, dtype=torch.float32).pin_memory()
+    h2d = tok_d.numel() * 4 + x_d.numel() * 2
+    d2h = loss_host.numel() * 4
+    state["k"] = 0
+    barrier()
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    f0.record()
+    for _ in range(args.steps):
+        k = state["k"]
+        tok_d.copy_(tok_h[k], non_blocking=True)
+        x_d.copy_(xs_h[k], non_blocking=True)
+        step(tok_d, x_d.view(torch.bfloat16))
+        loss_host.copy_(losses, non_blocking=True)
+    f1.record()
+    torch.cuda.synchronize()
+    barrier()
+    t_e2e = f0.elapsed_time(f1)
+    if pg is not None:
+        t_ms, t_e2e = max_over_ranks([t_ms, t_e2e], pg, dev)
+
+    value = replica_throughput(ew.L, args.steps, ws, t_ms)
+    e2e_value = replica_throughput(ew.L, args.steps, ws, t_e2e)
+    out = None
+    if rank == 0:
+        flops = episode_flops(ew)
+        ach = flops / (t_ms / args.steps * 1e-3) / 1e12
+        cpu = None
+        if ws == 1 and args.cpu_rows > 0:
+            cpu = _episode_oracle_sample(ew, texts, dense, xs_host, min(args.cpu_rows, 16))[1]
+        out = {
+            "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(t_ms / args.steps, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": (f"{ew.name}: chained aTTT updates, L={ew.L} tokens in {ew.cadence} agent steps "
+                                    f"per update, {ew.updates} updates per episode (reset between episodes), "
+                                    f"V={ew.V}, adapter r={ew.r} on a {ew.din}x{ew.d} projection feeding the LM "
+                                    f"head, {ew.grad_steps} SGD steps per update with dx, n={ew.n}"),
+                       "global_batch": ew.L * ws, "seq_len": ew.L, "parallelism": f"replicas{ws}",
+                       "l2": f"inputs larger than L2 (LM head {2 * ew.V * ew.d / 1e9:.2f} GB streamed twice per step)"},
+            "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": int(n1 - n0),
+            "roofline": {"bound": "tensor", "achieved": round(ach, 1), "peak": peaks["bf16_sustained"],
+                         "unit": "TFLOP/s", "frac": round(ach / peaks["bf16_sustained"], 4), "traffic": None,
+                         "kernel": "whole update (two Eq. 10 calls, projection forward and dx, adapter grads)",
+                         "peak_kind": f"bf16 sustained, {peaks['src']}"},
+            "clocks": clk,
+            "cpu_baseline": cpu,
+        }
+    if pg is not None:
+        pg.barrier()
+        pg.destroy_process_group()
+    ep.close()
+    return out
+
+
+def _episode_oracle_sample(ew, texts, dense, xs_host, rows):
+    """The oracle's chained update on the first `rows` tokens of the first
+    update (all V vocabulary rows, both gradient steps, dx)."""
+    import oracle
+    oracle.build()
+    H = wk.episode_history(ew)
+    t0 = time.perf_counter()
+    oracle.episode_update(H, texts[0][:rows], xs_host[0][:rows], dense["W0"], dense["W"], dense["A0"],
+                          dense["B0"], n=ew.n, w_min=ew.w_min, scale=ew.scale, lr=ew.lr,
+                          grad_steps=ew.grad_steps)
+    dt = time.perf_counter() - t0
+    return dt, {"value": round(rows / dt, 3), "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+                "sample": (f"an update of the first {rows} tokens of the {ew.name} workload's first update: Eq. 8/9 "
+                           f"weights, {ew.grad_steps} chained gradient steps over all {ew.V} vocab entries with dx; "
+                           f"fp64 C oracle with OpenMP, {dt:.1f} s")}
+
+
+# ---------------------------------------------------------------------------
 # the reference arm: the CPU oracle on the host cores
 # ---------------------------------------------------------------------------
 
@@ -577,7 +756,7 @@ def run_reference(args):
     ws, rank, _ = _dist()
     if rank != 0:
         return None
-    wl = wk.WORKLOADS[args.workload if args.workload != "stress" else WORKLOAD]
+    wl = wk.WORKLOADS[args.workload if args.workload in wk.WORKLOADS and args.workload != "stress" else WORKLOAD]
     sample = OracleSample(wl)
     for _ in range(args.warmup):
         sample.run(1)
@@ -603,8 +782,10 @@ def main():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["attt", "reference"], default="attt")
-    ap.add_argument("--workload", default=WORKLOAD, choices=["tiny", "7b", "long", "32b", "stress"],
-                    help="'stress' times the n-gram insert and weights on the 1M-token history")
+    ap.add_argument("--workload", default=WORKLOAD,
+                    choices=["tiny", "7b", "long", "32b", "stress"] + sorted(wk.EPISODES),
+                    help="'stress' times the n-gram insert and weights on the 1M-token history; "
+                         "'*-episode' runs chained updates through attt_episode_*")
     ap.add_argument("--part", default="all", choices=["all", "ce", "lora", "ngram"],
                     help="time one stage alone (profiling aid); 'all' is the benchmark")
     ap.add_argument("--cpu-rows", type=int, default=64, help="rows of the oracle CPU-baseline sample (0: skip)")
@@ -616,6 +797,8 @@ def main():
         out = run_reference(args)
     elif args.workload == "stress":
         out = run_stress(args)
+    elif args.workload in wk.EPISODES:
+        out = run_episode(args)
     else:
         out = run_gpu(args)
     if out is not None:

@@ -298,6 +298,101 @@ ATTT_API attt_status attt_lora_input_grad(const attt_bf16 *d_dy, const attt_bf16
                                           float scale, float *d_dx, void *d_ws, size_t ws_bytes,
                                           attt_stream stream);
 
+/*
+ * d_dst[i] = bf16(d_src[i]) (round to nearest even) for i < n: the gradient
+ * of the LM head's input (fp32 dh of attt_weighted_ce_fwd_bwd) as the bf16
+ * upstream gradient dy of the adapted projection in a chained update.
+ */
+ATTT_API attt_status attt_cast_bf16(const float *d_src, attt_bf16 *d_dst, int64_t n, attt_stream stream);
+
+/* ------------------------------------------------------------------------ */
+/* The episode: Algorithm 1 run end to end with the schedule of Sec. 4 and  */
+/* Appendix C -- an update every K agent steps, two gradient steps per      */
+/* update, the adapter persisting within an episode and reset between       */
+/* episodes.  The adapted projection's output is the LM head's input.       */
+/* ------------------------------------------------------------------------ */
+
+typedef struct attt_episode attt_episode;
+
+typedef struct attt_episode_config {
+    int n;               /* n-gram size of Eq. 8 (1..16)                        */
+    float w_min;         /* Eq. 9 floor, 0 < w_min <= 1                         */
+    int64_t max_history; /* tokens the history may hold over the episode        */
+    int64_t max_update;  /* largest update text L (<= max_history)              */
+    int64_t din;         /* adapted projection: input width  (multiple of 8)    */
+    int64_t d;           /*   output width = LM head input   (multiple of 8)    */
+    int64_t V;           /* vocabulary (LM head rows)                           */
+    int r;               /* adapter rank, 1..64 (a multiple of 8 for dx)        */
+    float scale;         /* s = alpha / r                                       */
+    float lr;            /* SGD learning rate of Eq. 2                          */
+    int grad_steps;      /* gradient steps per update (Appendix C: 2), 1..64    */
+    int cadence;         /* K: agent steps per update (Sec. 4 default 5), >= 1  */
+} attt_episode_config;
+
+/*
+ * Creates an episode on the current device.  d_W0 (bf16 [din, d]) and d_Wlm
+ * (bf16 [V, d]) are the frozen projection and LM head: borrowed, they must
+ * stay valid and unchanged while the episode lives.  d_A0 (fp32 [din, r]) and
+ * d_B0 (fp32 [r, d]) are the adapter's initial value, copied at create and
+ * restored by every reset.  The episode allocates its history, adapter,
+ * activations and one shared workspace up front (the update path allocates
+ * nothing) and synchronises the device once.  *out is set on success.
+ */
+ATTT_API attt_status attt_episode_create(const attt_episode_config *cfg, const attt_bf16 *d_W0,
+                                         const attt_bf16 *d_Wlm, const float *d_A0, const float *d_B0,
+                                         attt_episode **out);
+
+/* Frees the episode and everything it allocated (synchronises the device). */
+ATTT_API attt_status attt_episode_destroy(attt_episode *e);
+
+/*
+ * The episode boundary: the adapter returns to (A0, B0), the history is
+ * emptied and pending agent-step text is dropped.  Async on `stream`.
+ */
+ATTT_API attt_status attt_episode_reset(attt_episode *e, attt_stream stream);
+
+/*
+ * One update (Algorithm 1) on the update text x_k = d_tokens (int32 [L], the
+ * targets of Eq. 10, each in [0, V)) whose rows of the adapted projection's
+ * input are d_x (bf16 [L, din]):
+ *   w = Eq. 9(Eq. 8(x_k, H))
+ *   grad_steps times:  h = x W0 + s (x A) B  (bf16);  loss_g, dh = Eq. 10;
+ *     dy = bf16(dh);  dA, dB of h;  dx_g = dy W0^T + s (dy B^T) A^T when d_dx
+ *     is not NULL;  A -= lr dA, B -= lr dB
+ *   H <- H || x_k
+ * d_losses (fp32 [grad_steps]) receives each step's Eq. 10 loss (NULL: kept
+ * internally).  d_dx (fp32 [grad_steps, L, din], 16-byte aligned) receives the
+ * gradient of each step's projection input, or NULL to skip it.  The caller's
+ * buffers must stay valid until the stream reaches the end of the update.
+ * 1 <= L <= max_update; ATTT_ERR_CAPACITY (nothing launched) if the history
+ * would exceed max_history.  Async on `stream`.
+ */
+ATTT_API attt_status attt_episode_update(attt_episode *e, const int32_t *d_tokens, const attt_bf16 *d_x, int64_t L,
+                                         float *d_losses, float *d_dx, attt_stream stream);
+
+/*
+ * One agent step: appends its text (d_tokens int32 [len], d_x bf16 [len, din];
+ * len may be 0) to the pending update text.  Every cadence-th call runs
+ * attt_episode_update on the text of the last `cadence` steps (if it is not
+ * empty), clears it and sets *updated (may be NULL) to 1, else 0.  Text of
+ * fewer than `cadence` steps at the end of an episode is not trained on.
+ * ATTT_ERR_CAPACITY (nothing launched, nothing appended) if the pending text
+ * would exceed max_update or the history max_history.  Async on `stream`.
+ */
+ATTT_API attt_status attt_episode_agent_step(attt_episode *e, const int32_t *d_tokens, const attt_bf16 *d_x,
+                                             int64_t len, float *d_losses, float *d_dx, int *updated,
+                                             attt_stream stream);
+
+/* Copies the adapter's fp32 values (A [din, r], B [r, d]) out.  Async. */
+ATTT_API attt_status attt_episode_read_adapter(const attt_episode *e, float *d_A32, float *d_B32,
+                                               attt_stream stream);
+
+/* The episode's history (owned by the episode; do not destroy it). */
+ATTT_API attt_history *attt_episode_history(attt_episode *e);
+
+/* Tokens of pending agent-step text not yet trained on. */
+ATTT_API int64_t attt_episode_pending_tokens(const attt_episode *e);
+
 #ifdef __cplusplus
 }
 #endif

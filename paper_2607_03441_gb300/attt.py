@@ -11,7 +11,7 @@ from __future__ import annotations
 import ctypes
 import os
 import threading
-from typing import Optional, Sequence
+from typing import Optional, Sequence, Tuple
 
 import torch
 
@@ -19,6 +19,14 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libattt.so")
 
 ATTT_OK = 0
+ATTT_ERR_INVALID_ARG = 1
+ATTT_ERR_TABLE_FULL = 2
+ATTT_ERR_TOKEN_RANGE = 3
+ATTT_ERR_TIMEOUT = 4
+ATTT_ERR_WORKSPACE = 5
+ATTT_ERR_CUDA = 6
+ATTT_ERR_UNSUPPORTED = 7
+ATTT_ERR_CAPACITY = 8
 STATUS_NAMES = {
     0: "ATTT_OK", 1: "ATTT_ERR_INVALID_ARG", 2: "ATTT_ERR_TABLE_FULL", 3: "ATTT_ERR_TOKEN_RANGE",
     4: "ATTT_ERR_TIMEOUT", 5: "ATTT_ERR_WORKSPACE", 6: "ATTT_ERR_CUDA", 7: "ATTT_ERR_UNSUPPORTED",
@@ -33,6 +41,14 @@ class AtttError(RuntimeError):
     def __init__(self, code: int, where: str):
         self.code = int(code)
         super().__init__(f"{where}: {STATUS_NAMES.get(int(code), code)}")
+
+
+class EpisodeConfig(ctypes.Structure):
+    """attt_episode_config (field order and types as in attt.h)."""
+    _fields_ = [("n", ctypes.c_int), ("w_min", ctypes.c_float), ("max_history", ctypes.c_int64),
+                ("max_update", ctypes.c_int64), ("din", ctypes.c_int64), ("d", ctypes.c_int64),
+                ("V", ctypes.c_int64), ("r", ctypes.c_int), ("scale", ctypes.c_float), ("lr", ctypes.c_float),
+                ("grad_steps", ctypes.c_int), ("cadence", ctypes.c_int)]
 
 
 def load_library(path: Optional[str] = None) -> ctypes.CDLL:
@@ -70,6 +86,15 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_lora_input_grad_workspace_bytes": (sz, [i64, i64, i64, i32]),
             "attt_lora_forward": (i32, [P, P, P, P, i64, i64, i64, i32, f32, P, P, sz, P]),
             "attt_lora_input_grad": (i32, [P, P, P, P, i64, i64, i64, i32, f32, P, P, sz, P]),
+            "attt_cast_bf16": (i32, [P, P, i64, P]),
+            "attt_episode_create": (i32, [ctypes.POINTER(EpisodeConfig), P, P, P, P, ctypes.POINTER(P)]),
+            "attt_episode_destroy": (i32, [P]),
+            "attt_episode_reset": (i32, [P, P]),
+            "attt_episode_update": (i32, [P, P, P, i64, P, P, P]),
+            "attt_episode_agent_step": (i32, [P, P, P, i64, P, P, ctypes.POINTER(i32), P]),
+            "attt_episode_read_adapter": (i32, [P, P, P, P]),
+            "attt_episode_history": (P, [P]),
+            "attt_episode_pending_tokens": (i64, [P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -141,10 +166,24 @@ class History:
         self.handle = h
         self.n = int(n)
         self.max_tokens = int(max_tokens)
+        self._owned = True
+
+    @classmethod
+    def _view(cls, handle: int, n: int, max_tokens: int, owner) -> "History":
+        """Non-owning handle of a history that another object owns."""
+        self = cls.__new__(cls)
+        self._lib = load_library()
+        self.handle = ctypes.c_void_p(handle)
+        self.n = int(n)
+        self.max_tokens = int(max_tokens)
+        self._owned = False
+        self._owner = owner
+        return self
 
     def close(self) -> None:
         if getattr(self, "handle", None):
-            self._lib.attt_history_destroy(self.handle)
+            if self._owned:
+                self._lib.attt_history_destroy(self.handle)
             self.handle = None
 
     def __del__(self):
@@ -352,3 +391,114 @@ def attt_lora_input_grad(dy: torch.Tensor, W0: torch.Tensor, A: torch.Tensor, B:
         _bf16(dy), _bf16(W0), _bf16(A), _bf16(B), L, din, dout, int(r), float(scale), _ptr(dx), _ptr(workspace),
         workspace.numel(), _stream(stream)), "attt_lora_input_grad")
     return dx
+
+
+def attt_cast_bf16(src: torch.Tensor, dst: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """dst = bf16(src) (round to nearest even).  Returns dst."""
+    if src.dtype != torch.float32:
+        raise ValueError(f"expected float32, got {src.dtype}")
+    if dst is None:
+        dst = torch.empty(src.shape, dtype=torch.bfloat16, device=src.device)
+    _check(load_library().attt_cast_bf16(_ptr(src), _bf16(dst), src.numel(), _stream(stream)), "attt_cast_bf16")
+    return dst
+
+
+# --------------------------------------------------------------------------
+# the episode (Algorithm 1 with the Sec. 4 / Appendix C schedule)
+# --------------------------------------------------------------------------
+
+class Episode:
+    """Owning handle of an attt_episode.
+
+    W0 (bf16 [din, d]) and Wlm (bf16 [V, d]) are borrowed by the library: this
+    object keeps references to them so they outlive the episode.  A0 / B0
+    (fp32) are the adapter's initial value, restored by reset().
+    """
+
+    def __init__(self, W0: torch.Tensor, Wlm: torch.Tensor, A0: torch.Tensor, B0: torch.Tensor, *, n: int,
+                 max_history: int, max_update: int, scale: float, lr: float, w_min: float = 0.05,
+                 grad_steps: int = 2, cadence: int = 5):
+        self._lib = load_library()
+        din, d = W0.shape
+        V = Wlm.shape[0]
+        r = A0.shape[1]
+        if Wlm.shape[1] != d or A0.shape[0] != din or tuple(B0.shape) != (r, d):
+            raise ValueError("shape mismatch between W0, Wlm, A0, B0")
+        if A0.dtype != torch.float32 or B0.dtype != torch.float32:
+            raise ValueError("A0 and B0 must be float32")
+        self.cfg = EpisodeConfig(n=int(n), w_min=float(w_min), max_history=int(max_history),
+                                 max_update=int(max_update), din=int(din), d=int(d), V=int(V), r=int(r),
+                                 scale=float(scale), lr=float(lr), grad_steps=int(grad_steps),
+                                 cadence=int(cadence))
+        e = ctypes.c_void_p()
+        _check(self._lib.attt_episode_create(ctypes.byref(self.cfg), _bf16(W0), _bf16(Wlm), _ptr(A0), _ptr(B0),
+                                             ctypes.byref(e)), "attt_episode_create")
+        self.handle = e
+        self._keep = (W0, Wlm)
+        self.device = W0.device
+
+    def close(self) -> None:
+        if getattr(self, "handle", None):
+            self._lib.attt_episode_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def _out(self, losses, dx, L):
+        c = self.cfg
+        if losses is not None and (losses.dtype != torch.float32 or losses.numel() < c.grad_steps):
+            raise ValueError("losses must be float32 with grad_steps entries")
+        if dx is not None and (dx.dtype != torch.float32 or dx.numel() < c.grad_steps * L * c.din):
+            raise ValueError("dx must be float32 [grad_steps, L, din]")
+        return _ptr(losses), _ptr(dx)
+
+    def update(self, tokens: torch.Tensor, x: torch.Tensor, losses: Optional[torch.Tensor] = None,
+               dx: Optional[torch.Tensor] = None, stream=None) -> None:
+        """One update on `tokens` (int32 [L]) with projection inputs `x` (bf16 [L, din])."""
+        if tokens.dtype != torch.int32:
+            raise ValueError("tokens must be int32")
+        L = tokens.numel()
+        if tuple(x.shape) != (L, self.cfg.din):
+            raise ValueError("x must be [L, din]")
+        pl, pd = self._out(losses, dx, L)
+        _check(self._lib.attt_episode_update(self.handle, _ptr(tokens), _bf16(x), L, pl, pd, _stream(stream)),
+               "attt_episode_update")
+
+    def agent_step(self, tokens: torch.Tensor, x: torch.Tensor, losses: Optional[torch.Tensor] = None,
+                   dx: Optional[torch.Tensor] = None, stream=None) -> bool:
+        """Appends one agent step's text; returns True if it triggered an update."""
+        if tokens.dtype != torch.int32:
+            raise ValueError("tokens must be int32")
+        n = tokens.numel()
+        if tuple(x.shape) != (n, self.cfg.din):
+            raise ValueError("x must be [len, din]")
+        pending = self.pending_tokens()
+        pl, pd = self._out(losses, dx, pending + n)
+        up = ctypes.c_int(0)
+        _check(self._lib.attt_episode_agent_step(self.handle, _ptr(tokens) if n else None,
+                                                 _bf16(x) if n else None, n, pl, pd, ctypes.byref(up),
+                                                 _stream(stream)), "attt_episode_agent_step")
+        return bool(up.value)
+
+    def reset(self, stream=None) -> None:
+        _check(self._lib.attt_episode_reset(self.handle, _stream(stream)), "attt_episode_reset")
+
+    def read_adapter(self, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+        """(A [din, r], B [r, d]) fp32 copies of the current adapter."""
+        c = self.cfg
+        A = torch.empty((c.din, c.r), dtype=torch.float32, device=self.device)
+        B = torch.empty((c.r, c.d), dtype=torch.float32, device=self.device)
+        _check(self._lib.attt_episode_read_adapter(self.handle, _ptr(A), _ptr(B), _stream(stream)),
+               "attt_episode_read_adapter")
+        return A, B
+
+    def history(self) -> History:
+        h = self._lib.attt_episode_history(self.handle)
+        return History._view(h, self.cfg.n, self.cfg.max_history, self)
+
+    def pending_tokens(self) -> int:
+        return int(self._lib.attt_episode_pending_tokens(self.handle))

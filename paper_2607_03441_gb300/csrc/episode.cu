@@ -1,0 +1,235 @@
+// episode.cu -- the in-episode update driver: Algorithm 1 run end to end on
+// one stream, with the schedule of Sec. 4 / Appendix C (an update every K
+// agent steps, two gradient steps per update, the adapter persisting within
+// an episode and reset between episodes).
+//
+// One update k (attt_episode_update):
+//   w = Eq. 9(Eq. 8(x_k, H_k))                        attt_ngram_weights
+//   repeat grad_steps times (Eq. 2 / Algorithm 1's gradient step):
+//     h  = x W0 + s (x A) B                           attt_lora_forward
+//     loss, dh = Eq. 10(h, W_lm, targets x_k, w)      attt_weighted_ce_fwd_bwd
+//     dy = bf16(dh)                                   attt_cast_bf16
+//     dA, dB = adapter gradients of h                 attt_lora_grad
+//     dx = dy W0^T + s (dy B^T) A^T  (if requested)   attt_lora_input_grad
+//     A, B <- A - lr dA, B - lr dB                    attt_lora_step
+//   H_{k+1} = H_k || x_k                              attt_history_insert
+//
+// Everything is host code that issues the library's own calls; the episode
+// owns its device buffers (allocated once at create) and one workspace that
+// the calls share, since they run one after another on the caller's stream
+// and the first kernel of each call waits for the previous call to finish.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <new>
+
+#include "attt.h"
+#include "attt_host.h"
+
+struct attt_episode {
+    attt_episode_config cfg;
+    const attt_bf16 *W0;   // [din, d] frozen projection (borrowed)
+    const attt_bf16 *Wlm;  // [V, d] frozen LM head (borrowed)
+    attt_history *hist;
+    // adapter: fp32 masters, bf16 copies, initial values, gradients
+    float *A32, *B32, *A0, *B0, *dA, *dB;
+    attt_bf16 *A16, *B16;
+    // per-update activations
+    float *w, *dh, *losses;
+    attt_bf16 *h, *dy;
+    // pending update text (agent steps since the last update)
+    int32_t *pend_tok;
+    attt_bf16 *pend_x;
+    int64_t pend_len;
+    int pend_steps;
+    void *ws;
+    size_t ws_bytes;
+};
+
+namespace {
+
+using attt::cdiv;
+
+template <class T>
+bool dev_alloc(T **p, size_t count) {
+    *p = nullptr;
+    return cudaMalloc(reinterpret_cast<void **>(p), (count > 0 ? count : 1) * sizeof(T)) == cudaSuccess;
+}
+
+void free_all(attt_episode *e) {
+    if (e->hist) attt_history_destroy(e->hist);
+    void *bufs[] = {e->A32, e->B32, e->A0, e->B0, e->dA, e->dB, e->A16, e->B16, e->w,
+                    e->dh,  e->losses, e->h, e->dy, e->pend_tok, e->pend_x, e->ws};
+    for (void *b : bufs) cudaFree(b);
+}
+
+bool config_ok(const attt_episode_config *c) {
+    return c && c->n >= 1 && c->n <= 16 && c->w_min > 0.0f && c->w_min <= 1.0f && c->max_history >= 0 &&
+           c->max_history <= 16777214 && c->max_update >= 1 && c->max_update <= c->max_history &&
+           c->din >= 8 && c->din % 8 == 0 && c->d >= 8 && c->d % 8 == 0 && c->V >= 1 && c->r >= 1 && c->r <= 64 &&
+           std::isfinite(c->scale) && std::isfinite(c->lr) && c->grad_steps >= 1 && c->grad_steps <= 64 &&
+           c->cadence >= 1;
+}
+
+// Workspace that every call of an update of up to max_update tokens fits in.
+// The Eq. 10 workspace is not monotone in L (its vocabulary chunk depends on
+// L), so the bound takes the maximum over every L.
+size_t workspace_bound(const attt_episode_config &c) {
+    size_t ws = 0;
+    auto upd = [&](size_t b) { if (b > ws) ws = b; };
+    for (int64_t L = 1; L <= c.max_update; ++L) upd(attt_ce_workspace_bytes(L, c.d, c.V));
+    const int64_t L = c.max_update;
+    upd(attt_lora_workspace_bytes(L, c.din, 1, &c.d, c.r));
+    upd(attt_lora_forward_workspace_bytes(L, c.din, c.d, c.r));
+    upd(attt_lora_input_grad_workspace_bytes(L, c.din, c.d, c.r));
+    return ws;
+}
+
+attt_status load_adapter(attt_episode *e, cudaStream_t s) {
+    const size_t nA = (size_t)e->cfg.din * e->cfg.r, nB = (size_t)e->cfg.r * e->cfg.d;
+    if (cudaMemcpyAsync(e->A32, e->A0, nA * sizeof(float), cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
+        cudaMemcpyAsync(e->B32, e->B0, nB * sizeof(float), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+        return ATTT_ERR_CUDA;
+    attt_status st = attt_cast_bf16(e->A32, e->A16, (int64_t)nA, s);
+    if (st != ATTT_OK) return st;
+    return attt_cast_bf16(e->B32, e->B16, (int64_t)nB, s);
+}
+
+}  // namespace
+
+extern "C" {
+
+attt_status attt_episode_create(const attt_episode_config *cfg, const attt_bf16 *d_W0, const attt_bf16 *d_Wlm,
+                                const float *d_A0, const float *d_B0, attt_episode **out) {
+    using namespace attt;
+    if (!out) return ATTT_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!config_ok(cfg) || !d_W0 || !d_Wlm || !d_A0 || !d_B0 || !aligned16(d_W0) || !aligned16(d_Wlm))
+        return ATTT_ERR_INVALID_ARG;
+    int dev;
+    attt_status st = current_device(&dev);
+    if (st != ATTT_OK) return st;
+
+    attt_episode *e = new (std::nothrow) attt_episode{};
+    if (!e) return ATTT_ERR_CUDA;
+    e->cfg = *cfg;
+    e->W0 = d_W0;
+    e->Wlm = d_Wlm;
+    const attt_episode_config &c = e->cfg;
+    const size_t nA = (size_t)c.din * c.r, nB = (size_t)c.r * c.d, Ld = (size_t)c.max_update * c.d;
+    e->ws_bytes = workspace_bound(c);
+    bool ok = attt_history_create(c.n, c.max_history, &e->hist) == ATTT_OK;
+    ok = ok && dev_alloc(&e->A32, nA) && dev_alloc(&e->B32, nB) && dev_alloc(&e->A0, nA) && dev_alloc(&e->B0, nB) &&
+         dev_alloc(&e->dA, nA) && dev_alloc(&e->dB, nB) && dev_alloc(&e->A16, nA) && dev_alloc(&e->B16, nB) &&
+         dev_alloc(&e->w, (size_t)c.max_update) && dev_alloc(&e->dh, Ld) && dev_alloc(&e->losses, (size_t)c.grad_steps) &&
+         dev_alloc(&e->h, Ld) && dev_alloc(&e->dy, Ld) && dev_alloc(&e->pend_tok, (size_t)c.max_update) &&
+         dev_alloc(&e->pend_x, (size_t)c.max_update * c.din) &&
+         dev_alloc(reinterpret_cast<char **>(&e->ws), e->ws_bytes);
+    if (ok) {
+        // The initial adapter is copied once; later resets restore it.
+        ok = cudaMemcpy(e->A0, d_A0, nA * sizeof(float), cudaMemcpyDeviceToDevice) == cudaSuccess &&
+             cudaMemcpy(e->B0, d_B0, nB * sizeof(float), cudaMemcpyDeviceToDevice) == cudaSuccess &&
+             load_adapter(e, nullptr) == ATTT_OK && cudaDeviceSynchronize() == cudaSuccess;
+    }
+    if (!ok) {
+        free_all(e);
+        delete e;
+        return ATTT_ERR_CUDA;
+    }
+    *out = e;
+    return ATTT_OK;
+}
+
+attt_status attt_episode_destroy(attt_episode *e) {
+    if (!e) return ATTT_ERR_INVALID_ARG;
+    cudaDeviceSynchronize();
+    free_all(e);
+    delete e;
+    return ATTT_OK;
+}
+
+attt_status attt_episode_reset(attt_episode *e, attt_stream stream) {
+    if (!e) return ATTT_ERR_INVALID_ARG;
+    attt_status st = attt_history_reset(e->hist, stream);
+    if (st != ATTT_OK) return st;
+    e->pend_len = 0;
+    e->pend_steps = 0;
+    return load_adapter(e, stream);
+}
+
+attt_status attt_episode_update(attt_episode *e, const int32_t *d_tokens, const attt_bf16 *d_x, int64_t L,
+                                float *d_losses, float *d_dx, attt_stream stream) {
+    using namespace attt;
+    if (!e || L < 1 || !d_tokens || !d_x || !aligned16(d_x) || (d_dx && !aligned16(d_dx)))
+        return ATTT_ERR_INVALID_ARG;
+    const attt_episode_config &c = e->cfg;
+    if (L > c.max_update) return ATTT_ERR_INVALID_ARG;
+    if (attt_history_length(e->hist) + L > c.max_history) return ATTT_ERR_CAPACITY;
+    if (d_dx && c.r % 8 != 0) return ATTT_ERR_UNSUPPORTED;
+    float *losses = d_losses ? d_losses : e->losses;
+
+    attt_status st = attt_ngram_weights(e->hist, d_tokens, L, c.w_min, e->w, stream);
+    for (int g = 0; g < c.grad_steps && st == ATTT_OK; ++g) {
+        st = attt_lora_forward(d_x, e->W0, e->A16, e->B16, L, c.din, c.d, c.r, c.scale, e->h, e->ws, e->ws_bytes,
+                               stream);
+        if (st == ATTT_OK)
+            st = attt_weighted_ce_fwd_bwd(e->h, e->Wlm, d_tokens, e->w, L, c.d, c.V, losses + g, e->dh, nullptr,
+                                          e->ws, e->ws_bytes, stream);
+        if (st == ATTT_OK) st = attt_cast_bf16(e->dh, e->dy, L * c.d, stream);
+        if (st == ATTT_OK) {
+            const attt_bf16 *dys[1] = {e->dy}, *As[1] = {e->A16}, *Bs[1] = {e->B16};
+            float *dAs[1] = {e->dA}, *dBs[1] = {e->dB};
+            st = attt_lora_grad(d_x, L, c.din, 1, dys, &c.d, As, Bs, c.r, c.scale, dAs, dBs, e->ws, e->ws_bytes,
+                                stream);
+        }
+        if (st == ATTT_OK && d_dx)
+            st = attt_lora_input_grad(e->dy, e->W0, e->A16, e->B16, L, c.din, c.d, c.r, c.scale,
+                                      d_dx + (size_t)g * L * c.din, e->ws, e->ws_bytes, stream);
+        if (st == ATTT_OK) st = attt_lora_step(e->A32, e->B32, e->dA, e->dB, c.din, c.d, c.r, c.lr, e->A16, e->B16, stream);
+    }
+    if (st == ATTT_OK) st = attt_history_insert(e->hist, d_tokens, L, stream);
+    return st;
+}
+
+attt_status attt_episode_agent_step(attt_episode *e, const int32_t *d_tokens, const attt_bf16 *d_x, int64_t len,
+                                    float *d_losses, float *d_dx, int *updated, attt_stream stream) {
+    if (!e || len < 0 || (len > 0 && (!d_tokens || !d_x))) return ATTT_ERR_INVALID_ARG;
+    const attt_episode_config &c = e->cfg;
+    if (updated) *updated = 0;
+    if (e->pend_len + len > c.max_update) return ATTT_ERR_CAPACITY;
+    const bool fire = e->pend_steps + 1 >= c.cadence;
+    if (fire && e->pend_len + len > 0 && attt_history_length(e->hist) + e->pend_len + len > c.max_history)
+        return ATTT_ERR_CAPACITY;
+    if (len > 0) {
+        if (cudaMemcpyAsync(e->pend_tok + e->pend_len, d_tokens, (size_t)len * sizeof(int32_t),
+                            cudaMemcpyDeviceToDevice, stream) != cudaSuccess ||
+            cudaMemcpyAsync(e->pend_x + (size_t)e->pend_len * c.din, d_x, (size_t)len * c.din * sizeof(attt_bf16),
+                            cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
+            return ATTT_ERR_CUDA;
+    }
+    e->pend_len += len;
+    e->pend_steps += 1;
+    if (!fire) return ATTT_OK;
+    const int64_t L = e->pend_len;
+    e->pend_len = 0;
+    e->pend_steps = 0;
+    if (L == 0) return ATTT_OK;  // K steps without update text: nothing to train on
+    attt_status st = attt_episode_update(e, e->pend_tok, e->pend_x, L, d_losses, d_dx, stream);
+    if (st == ATTT_OK && updated) *updated = 1;
+    return st;
+}
+
+attt_status attt_episode_read_adapter(const attt_episode *e, float *d_A32, float *d_B32, attt_stream stream) {
+    if (!e || !d_A32 || !d_B32) return ATTT_ERR_INVALID_ARG;
+    const size_t nA = (size_t)e->cfg.din * e->cfg.r, nB = (size_t)e->cfg.r * e->cfg.d;
+    if (cudaMemcpyAsync(d_A32, e->A32, nA * sizeof(float), cudaMemcpyDeviceToDevice, stream) != cudaSuccess ||
+        cudaMemcpyAsync(d_B32, e->B32, nB * sizeof(float), cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
+        return ATTT_ERR_CUDA;
+    return ATTT_OK;
+}
+
+attt_history *attt_episode_history(attt_episode *e) { return e ? e->hist : nullptr; }
+
+int64_t attt_episode_pending_tokens(const attt_episode *e) { return e ? e->pend_len : -1; }
+
+}  // extern "C"

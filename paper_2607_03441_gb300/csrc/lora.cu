@@ -130,6 +130,23 @@ __global__ void lora_step_kernel(float *A32, const float *dA, __nv_bfloat16 *A16
     }
 }
 
+// dst = bf16(src), round to nearest even; 8 elements per thread per step
+// (two 16-byte loads, one 16-byte store) when both are 16-byte aligned.
+__global__ void cast_bf16_kernel(const float *__restrict__ src, __nv_bfloat16 *__restrict__ dst, int64_t n) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const bool vec = ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15) == 0;
+    const int64_t n8 = vec ? n / 8 : 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n8; i += stride) {
+        const float4 a = reinterpret_cast<const float4 *>(src)[2 * i];
+        const float4 b = reinterpret_cast<const float4 *>(src)[2 * i + 1];
+        __nv_bfloat162 o[4] = {__floats2bfloat162_rn(a.x, a.y), __floats2bfloat162_rn(a.z, a.w),
+                               __floats2bfloat162_rn(b.x, b.y), __floats2bfloat162_rn(b.z, b.w)};
+        reinterpret_cast<uint4 *>(dst)[i] = *reinterpret_cast<uint4 *>(o);
+    }
+    for (int64_t i = 8 * n8 + (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride)
+        dst[i] = __float2bfloat16_rn(src[i]);
+}
+
 static unsigned grid_for(int64_t n, int threads, int dev) {
     int64_t b = cdiv(n, threads);
     const int64_t cap = (int64_t)num_sms(dev) * 8;
@@ -521,6 +538,19 @@ attt_status attt_lora_step(float *d_A32, float *d_B32, const float *d_dA, const 
     lora_step_kernel<<<grid_for(nA + nB, 256, dev), 256, 0, stream>>>(
         d_A32, d_dA, reinterpret_cast<__nv_bfloat16 *>(d_A16), nA, d_B32, d_dB,
         reinterpret_cast<__nv_bfloat16 *>(d_B16), nB, lr);
+    count_launch();
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+attt_status attt_cast_bf16(const float *d_src, attt_bf16 *d_dst, int64_t n, attt_stream stream) {
+    using namespace attt;
+    if (n < 0 || (n > 0 && (!d_src || !d_dst))) return ATTT_ERR_INVALID_ARG;
+    if (n == 0) return ATTT_OK;
+    int dev;
+    attt_status st = current_device(&dev);
+    if (st != ATTT_OK) return st;
+    cast_bf16_kernel<<<grid_for(cdiv(n, 8), 256, dev), 256, 0, stream>>>(
+        d_src, reinterpret_cast<__nv_bfloat16 *>(d_dst), n);
     count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
