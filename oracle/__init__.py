@@ -282,3 +282,44 @@ def episode_update(H, tokens, x_bf16, W0_bf16, Wlm_bf16, A32, B32, *, n: int, w_
         losses.append(loss)
     H = np.concatenate([np.asarray(H, dtype=np.int32), np.asarray(tokens, dtype=np.int32)])
     return {"w": w, "losses": np.array(losses), "dx": dxs if want_dx else None, "A32": A, "B32": B, "H": H}
+
+
+# --------------------------------------------------------------------------
+# Eq. 6 / Eq. 7: update-text repetition and the sequence-level filter
+# --------------------------------------------------------------------------
+
+def words(text: bytes) -> set:
+    """W(x): the set of whitespace-separated words of the update text, split
+    on runs of the ASCII whitespace bytes (space, tab, LF, VT, FF, CR), the
+    words compared byte for byte."""
+    return set(bytes(text).split())
+
+
+def jaccard(a: set, b: set) -> np.float32:
+    """J(a, b) = |a & b| / |a | b| as one fp32 division of the two integer
+    sizes; 0 when both sets are empty."""
+    union = len(a | b)
+    if union == 0:
+        return np.float32(0.0)
+    return np.float32(len(a & b)) / np.float32(union)
+
+
+def repetition(previous, text: bytes):
+    """Eq. 6 and Eq. 7: (rho, nu) of update text `text` given the episode's
+    previous update texts; rho = 0 for the first update, nu = 1 - rho (fp32)."""
+    cur = words(text)
+    rho = np.float32(0.0)
+    for prev in previous:
+        rho = max(rho, jaccard(cur, words(prev)))
+    return rho, np.float32(1.0) - rho
+
+
+def sequence_filter(texts, tau: float):
+    """The sequence-level filter over an episode's candidate update texts in
+    order: [(rho, nu, keep)] with keep = not (nu < tau).  Every candidate text
+    joins the previous texts of the later ones, kept or not."""
+    out = []
+    for k, text in enumerate(texts):
+        rho, nu = repetition(texts[:k], text)
+        out.append((rho, nu, not bool(nu < np.float32(tau))))
+    return out
