@@ -749,6 +749,92 @@ def _episode_oracle_sample(ew, texts, dense, xs_host, rows):
 
 
 # ---------------------------------------------------------------------------
+# update-text repetition (Eq. 6), novelty (Eq. 7) and the sequence filter
+# ---------------------------------------------------------------------------
+
+def run_texts(args):
+    """One step = one episode of update texts through attt_repetition (a reset,
+    then one call per update), replayed from a CUDA graph.  Algorithmic bytes
+    per call: the text once, plus per word occurrence its key probe (8 B) and
+    its mask word read and written (16 B)."""
+    import torch
+    from paper_2607_03441_gb300 import attt
+    from paper_2607_03441_gb300 import build
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peaks = _peaks()
+    tw = wk.TEXT_WORKLOADS[args.workload]
+    texts = wk.episode_update_texts(tw)
+    nbytes = sum(len(t) for t in texts)
+    nwords = sum(len(t.split()) for t in texts)
+    dtexts = [torch.frombuffer(bytearray(t), dtype=torch.uint8).to(dev) for t in texts]
+    ws = attt.WordSets(tw.updates, nbytes)
+    out = torch.empty(tw.updates, 2, dtype=torch.float32, device=dev)
+    keep = torch.empty(tw.updates, dtype=torch.int32, device=dev)
+    outs = [out[k] for k in range(tw.updates)]
+    keeps = [keep[k:k + 1] for k in range(tw.updates)]
+
+    def episode():
+        attt.attt_wordsets_reset(ws)
+        for k, t in enumerate(dtexts):
+            attt.attt_repetition(ws, t, tw.tau, out=outs[k], keep=keeps[k])
+
+    def timed(fn):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record()
+        for _ in range(args.steps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / args.steps
+
+    for _ in range(args.warmup):
+        episode()
+    # the host issues a call in a few microseconds, about as long as a call
+    # runs on the device: the device time is taken from a CUDA graph of one
+    # episode (the reset and every call, replayed as captured), the
+    # host-issued time alongside it
+    ms_host = timed(episode)
+    graph = torch.cuda.CUDAGraph()
+    cap = torch.cuda.Stream(device=dev)
+    cap.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(cap):
+        with torch.cuda.graph(graph, stream=cap):
+            episode()
+    torch.cuda.current_stream().wait_stream(cap)
+    for _ in range(args.warmup):
+        graph.replay()
+    clocks = ClockSampler(0)
+    clocks.start()
+    ms = timed(graph.replay)
+    clk = clocks.stop()
+    if attt.attt_wordsets_status(ws) != 0:
+        raise RuntimeError("word-set status error")
+    alg = nbytes + 24 * nwords
+    ach = alg / (ms * 1e-3) / 1e9
+    res = {"metric": "Eq. 6/7 update-text repetition and the sequence filter: update texts/s, GB/s of "
+                     "algorithmic bytes vs HBM",
+           "value": round(tw.updates / (ms * 1e-3), 1), "unit": "update texts/s", "n_gpus": 1, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True, "data": "synthetic",
+           "dtype": "u8",
+           "config": {"workload": (f"{tw.name}: {tw.updates} update texts of {tw.words} Zipf(1.1) words over a "
+                                   f"{tw.vocab}-word vocabulary, spans copied from the previous text at "
+                                   f"{tw.frac_first:.0%}->{tw.frac_last:.0%}, tau {tw.tau}; one step = one episode "
+                                   f"(reset + {tw.updates} calls), {nbytes} text bytes, {nwords} words")},
+           "gpu_launches": tw.updates * args.steps,  # one repetition_kernel per update, replayed
+           "host_issued_ms_per_step": round(ms_host, 4),
+           "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                        "frac": round(ach / peaks["hbm_gbs"], 4), "traffic": None,
+                        "kernel": "attt_repetition (repetition_kernel, one launch per update), per episode"},
+           "clocks": clk,
+           "kept": int(keep.sum().item())}
+    ws.close()
+    return res
+
+
+# ---------------------------------------------------------------------------
 # the reference arm: the CPU oracle on the host cores
 # ---------------------------------------------------------------------------
 
@@ -783,7 +869,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["attt", "reference"], default="attt")
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=["tiny", "7b", "long", "32b", "stress"] + sorted(wk.EPISODES),
+                    choices=["tiny", "7b", "long", "32b", "stress"] + sorted(wk.EPISODES) + sorted(wk.TEXT_WORKLOADS),
                     help="'stress' times the n-gram insert and weights on the 1M-token history; "
                          "'*-episode' runs chained updates through attt_episode_*")
     ap.add_argument("--part", default="all", choices=["all", "ce", "lora", "ngram"],
@@ -799,6 +885,8 @@ def main():
         out = run_stress(args)
     elif args.workload in wk.EPISODES:
         out = run_episode(args)
+    elif args.workload in wk.TEXT_WORKLOADS:
+        out = run_texts(args)
     else:
         out = run_gpu(args)
     if out is not None:

@@ -306,6 +306,53 @@ ATTT_API attt_status attt_lora_input_grad(const attt_bf16 *d_dy, const attt_bf16
 ATTT_API attt_status attt_cast_bf16(const float *d_src, attt_bf16 *d_dst, int64_t n, attt_stream stream);
 
 /* ------------------------------------------------------------------------ */
+/* Update-text repetition (Eq. 6), novelty (Eq. 7) and the sequence-level   */
+/* filter of Sec. 4 (skip an update whose novelty is below tau; Appendix C: */
+/* tau = 0.5), over the episode's word sets.                                */
+/* ------------------------------------------------------------------------ */
+
+typedef struct attt_wordsets attt_wordsets;
+
+/*
+ * Creates an empty set of update texts for an episode of up to max_updates
+ * (1..4096) updates whose texts total at most max_bytes bytes, on the current
+ * device.  The library allocates a byte arena for the texts and an exact word
+ * index (hash table of 8 B keys plus one bit per update and word).
+ */
+ATTT_API attt_status attt_wordsets_create(int max_updates, int64_t max_bytes, attt_wordsets **out);
+
+/* Frees the sets and their device memory (synchronises the device). */
+ATTT_API attt_status attt_wordsets_destroy(attt_wordsets *s);
+
+/* Forgets every text (an episode boundary).  Async on `stream`. */
+ATTT_API attt_status attt_wordsets_reset(attt_wordsets *s, attt_stream stream);
+
+/*
+ * For the update text d_text (nbytes bytes, any values) of update k = the
+ * number of texts recorded so far, with W(x) the set of words of x (maximal
+ * runs of bytes other than the ASCII whitespace space, tab, LF, VT, FF, CR,
+ * compared byte for byte):
+ *   J_i   = |W(x_k) & W(x_i)| / |W(x_k) | W(x_i)|   (one fp32 division; 0 when
+ *           both sets are empty)
+ *   *d_rho  = max_{i<k} J_i  (0 for k = 0)                         (Eq. 6)
+ *   *d_nu   = 1 - rho in fp32                                      (Eq. 7)
+ *   *d_keep = 0 if nu < tau (the filter skips the update), else 1
+ * then records x_k as update k (every candidate text counts for the later
+ * ones, kept or not).  Outputs may be NULL.  Bit-exact.  ATTT_ERR_CAPACITY
+ * (nothing launched) if max_updates texts are recorded or the texts would
+ * exceed max_bytes.  A full probe sequence sets ATTT_ERR_TABLE_FULL in the
+ * status word read by attt_wordsets_status.  Async on `stream`.
+ */
+ATTT_API attt_status attt_repetition(attt_wordsets *s, const uint8_t *d_text, int64_t nbytes, float tau,
+                                     float *d_rho, float *d_nu, int32_t *d_keep, attt_stream stream);
+
+/* Number of update texts recorded (host-side bookkeeping, no sync). */
+ATTT_API int attt_wordsets_updates(const attt_wordsets *s);
+
+/* Synchronises `stream`, then reads and clears the sets' status word. */
+ATTT_API attt_status attt_wordsets_status(attt_wordsets *s, attt_stream stream);
+
+/* ------------------------------------------------------------------------ */
 /* The episode: Algorithm 1 run end to end with the schedule of Sec. 4 and  */
 /* Appendix C -- an update every K agent steps, two gradient steps per      */
 /* update, the adapter persisting within an episode and reset between       */

@@ -95,6 +95,12 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_episode_read_adapter": (i32, [P, P, P, P]),
             "attt_episode_history": (P, [P]),
             "attt_episode_pending_tokens": (i64, [P]),
+            "attt_wordsets_create": (i32, [i32, i64, ctypes.POINTER(P)]),
+            "attt_wordsets_destroy": (i32, [P]),
+            "attt_wordsets_reset": (i32, [P, P]),
+            "attt_repetition": (i32, [P, P, i64, f32, P, P, P, P]),
+            "attt_wordsets_updates": (i32, [P]),
+            "attt_wordsets_status": (i32, [P, P]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -502,3 +508,70 @@ class Episode:
 
     def pending_tokens(self) -> int:
         return int(self._lib.attt_episode_pending_tokens(self.handle))
+
+
+# --------------------------------------------------------------------------
+# update-text repetition (Eq. 6), novelty (Eq. 7), the sequence filter
+# --------------------------------------------------------------------------
+
+class WordSets:
+    """Owning handle of an attt_wordsets (the episode's update texts)."""
+
+    def __init__(self, max_updates: int, max_bytes: int):
+        self._lib = load_library()
+        s = ctypes.c_void_p()
+        _check(self._lib.attt_wordsets_create(int(max_updates), int(max_bytes), ctypes.byref(s)),
+               "attt_wordsets_create")
+        self.handle = s
+
+    def close(self) -> None:
+        if getattr(self, "handle", None):
+            self._lib.attt_wordsets_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __len__(self) -> int:
+        return int(self._lib.attt_wordsets_updates(self.handle))
+
+
+def attt_wordsets_create(max_updates: int, max_bytes: int) -> WordSets:
+    return WordSets(max_updates, max_bytes)
+
+
+def attt_wordsets_destroy(s: WordSets) -> None:
+    s.close()
+
+
+def attt_wordsets_reset(s: WordSets, stream=None) -> None:
+    _check(load_library().attt_wordsets_reset(s.handle, _stream(stream)), "attt_wordsets_reset")
+
+
+def attt_wordsets_updates(s: WordSets) -> int:
+    return int(load_library().attt_wordsets_updates(s.handle))
+
+
+def attt_wordsets_status(s: WordSets, stream=None) -> int:
+    return int(load_library().attt_wordsets_status(s.handle, _stream(stream)))
+
+
+def attt_repetition(s: WordSets, text: torch.Tensor, tau: float = 0.5, out: Optional[torch.Tensor] = None,
+                    keep: Optional[torch.Tensor] = None, stream=None):
+    """Eq. 6 / Eq. 7 for the update text `text` (uint8 bytes on the device):
+    returns (out, keep) with out = float32 [2] (rho, nu) and keep = int32 [1]."""
+    if text.dtype != torch.uint8:
+        raise ValueError("text must be uint8 bytes")
+    dev = text.device
+    if out is None:
+        out = torch.empty(2, dtype=torch.float32, device=dev)
+    if keep is None:
+        keep = torch.empty(1, dtype=torch.int32, device=dev)
+    n = text.numel()
+    base = _ptr(out)
+    _check(load_library().attt_repetition(s.handle, _ptr(text) if n else None, n, float(tau), base, base + 4,
+                                          _ptr(keep), _stream(stream)), "attt_repetition")
+    return out, keep

@@ -19,6 +19,12 @@ Qwen / Gemma weights, none of which are available here):
 * Dense tensors: fp32 normal samples rounded once to bf16 (round to nearest
   even); hidden ~ N(0, 1), LM head ~ N(0, 0.02), LoRA A ~ N(0, 0.02),
   B = 0.01 * N(0, 1), activations x and upstream grads dy ~ N(0, 1).
+* Update texts as bytes (Eq. 6 works on whitespace-separated words): a
+  synthetic vocabulary of words (1-12 characters over lowercase letters,
+  digits and ``._/()-:``), Zipf(1.1) word ids, joined by a space (80%), a
+  newline (10%), a tab (4%), two spaces (4%) or CR LF (2%); spans of words
+  copied from the previous update's text at a fraction rising linearly from
+  5% to 95% (an episode drifting into the repetitive, stuck regime).
 * Chained episodes (the adapted projection's output is the LM head's input):
   the frozen projection W0 [din, d] ~ N(0, 1/din), so that h = x W0 has unit
   variance like the hidden states above; one x ~ N(0, 1) per update; update
@@ -313,3 +319,69 @@ def episode_dense(ew: EpisodeWorkload) -> Dict[str, np.ndarray]:
 def episode_x(ew: EpisodeWorkload, k: int) -> np.ndarray:
     """bf16 bits of the projection inputs [L, din] of update k (1-based)."""
     return normal_bf16(ew.seed, f"episode/x{k}", (ew.L, ew.din), 1.0)
+
+
+# --------------------------------------------------------------------------
+# update texts as bytes (Eq. 6 / Eq. 7)
+# --------------------------------------------------------------------------
+
+_WORD_ALPHABET = np.frombuffer(b"abcdefghijklmnopqrstuvwxyzabcdefghijklmnopqrstuvwxyz0123456789._/()-:", dtype=np.uint8)
+_SEPS = (b" ", b"\n", b"\t", b"  ", b"\r\n")
+_SEP_P = np.array([0.80, 0.10, 0.04, 0.04, 0.02])
+
+
+@functools.lru_cache(maxsize=4)
+def word_vocab(seed: int, size: int) -> Tuple[bytes, ...]:
+    """`size` distinct synthetic words (1-12 characters)."""
+    rng = rng_for(seed, "words/vocab")
+    out, seen = [], set()
+    while len(out) < size:
+        n = int(rng.integers(1, 13))
+        w = bytes(_WORD_ALPHABET[rng.integers(0, _WORD_ALPHABET.size, n)])
+        if w not in seen:
+            seen.add(w)
+            out.append(w)
+    return tuple(out)
+
+
+def text_bytes(rng: np.random.Generator, ids: np.ndarray, vocab: Tuple[bytes, ...]) -> bytes:
+    """Words `ids` of `vocab` joined by random whitespace separators."""
+    seps = rng.choice(len(_SEPS), size=len(ids), p=_SEP_P)
+    return b"".join(vocab[int(i)] + _SEPS[int(j)] for i, j in zip(ids, seps))
+
+
+@dataclasses.dataclass
+class TextWorkload:
+    name: str
+    seed: int
+    updates: int
+    words: int            # words per update text
+    vocab: int            # synthetic word vocabulary
+    frac_first: float = 0.05
+    frac_last: float = 0.95
+    tau: float = 0.5      # Appendix C
+
+
+TEXT_WORKLOADS: Dict[str, TextWorkload] = {
+    # a long-episode-shaped run of update texts: 32 updates of ~1,536 words
+    # (a 2,048-token update at ~1.33 tokens per word)
+    "texts": TextWorkload("texts", 5, updates=32, words=1536, vocab=50000),
+    # larger texts for throughput: 64 updates of 131,072 words (~0.8 MB each)
+    "texts-stress": TextWorkload("texts-stress", 6, updates=64, words=131072, vocab=200000),
+}
+
+
+def episode_update_texts(tw: TextWorkload) -> List[bytes]:
+    """The update texts of one episode: Zipf words, with spans of words
+    copied from the previous update's text at a fraction rising linearly."""
+    vocab = word_vocab(tw.seed, tw.vocab)
+    texts: List[bytes] = []
+    prev = np.zeros(0, dtype=np.int32)
+    for k in range(1, tw.updates + 1):
+        frac = tw.frac_first if tw.updates <= 1 else \
+            tw.frac_first + (tw.frac_last - tw.frac_first) * (k - 1) / (tw.updates - 1)
+        ids = zipf_ids(rng_for(tw.seed, f"texts/ids{k}"), tw.words, tw.vocab)
+        ids = copy_spans(rng_for(tw.seed, f"texts/spans{k}"), ids, prev, frac)
+        texts.append(text_bytes(rng_for(tw.seed, f"texts/seps{k}"), ids, vocab))
+        prev = ids
+    return texts
