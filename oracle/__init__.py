@@ -57,6 +57,8 @@ def _load():
         lib.oracle_exposure_sorted.argtypes = [P, i64, P, i64, ctypes.c_int, P]
         lib.oracle_weights_from_exposure.restype = None
         lib.oracle_weights_from_exposure.argtypes = [P, i64, ctypes.c_float, P]
+        lib.oracle_kl_rows.restype = None
+        lib.oracle_kl_rows.argtypes = [P, P, P, i64, i64, P, i64, P]
         lib.oracle_ce_rows.restype = None
         lib.oracle_ce_rows.argtypes = [P, P, P, P, i64, i64, i64, P, i64, P, P, P]
         lib.oracle_ce_loss.restype = ctypes.c_double
@@ -322,4 +324,23 @@ def sequence_filter(texts, tau: float):
     for k, text in enumerate(texts):
         rho, nu = repetition(texts[:k], text)
         out.append((rho, nu, not bool(nu < np.float32(tau))))
+    return out
+
+
+# --------------------------------------------------------------------------
+# Adapter drift: KL of the adapted from the base next-token distribution
+# --------------------------------------------------------------------------
+
+def kl_rows(hp_bf16, hq_bf16, W_bf16, rows=None):
+    """KL(softmax(h_p W^T) || softmax(h_q W^T)) per row (fp64), for `rows`
+    (all rows when None)."""
+    hp, php = _c(hp_bf16, np.uint16)
+    hq, phq = _c(hq_bf16, np.uint16)
+    W, pW = _c(W_bf16, np.uint16)
+    L, d = hp.shape
+    assert hq.shape == (L, d) and W.shape[1] == d
+    rows = np.arange(L, dtype=np.int64) if rows is None else rows
+    rows, pr = _c(rows, np.int64)
+    out = np.zeros(rows.size, dtype=np.float64)
+    _load().oracle_kl_rows(php, phq, pW, d, W.shape[0], pr, rows.size, out.ctypes.data_as(ctypes.c_void_p))
     return out

@@ -347,6 +347,60 @@ void oracle_lora_input_grad(const uint16_t *dy, const uint16_t *W0, const uint16
 /* ------------------------------------------------------------------------ */
 
 /* p <- p - lr * g, in fp32, multiply then subtract (no fused multiply-add). */
+/*
+ * Adapter drift (Sec. 4, Fig. 6): per row j, the KL divergence of the
+ * adapted model's next-token distribution p_j = softmax(h_p[j] W^T) from the
+ * base model's q_j = softmax(h_q[j] W^T):
+ *   KL_j = sum_v p_jv (log p_jv - log q_jv)
+ * with log p_jv = z_p,jv - lse_p,j (fp64 logits over the bf16 inputs).
+ */
+void oracle_kl_rows(const uint16_t *hp, const uint16_t *hq, const uint16_t *W, int64_t d, int64_t V,
+                    const int64_t *rows, int64_t nrows, double *kl)
+{
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t i = 0; i < nrows; ++i) {
+        int64_t j = rows[i];
+        double *a = (double *)malloc((size_t)d * sizeof(double));
+        double *b = (double *)malloc((size_t)d * sizeof(double));
+        double *zp = (double *)malloc((size_t)V * sizeof(double));
+        double *zq = (double *)malloc((size_t)V * sizeof(double));
+        for (int64_t k = 0; k < d; ++k) {
+            a[k] = bf16_value(hp[j * d + k]);
+            b[k] = bf16_value(hq[j * d + k]);
+        }
+        double mp = -INFINITY, mq = -INFINITY;
+        for (int64_t v = 0; v < V; ++v) {
+            const uint16_t *Wv = W + v * d;
+            double sp = 0.0, sq = 0.0;
+            for (int64_t k = 0; k < d; ++k) {
+                double wv = bf16_value(Wv[k]);
+                sp += a[k] * wv;
+                sq += b[k] * wv;
+            }
+            zp[v] = sp;
+            zq[v] = sq;
+            if (sp > mp) mp = sp;
+            if (sq > mq) mq = sq;
+        }
+        double ep = 0.0, eq = 0.0;
+        for (int64_t v = 0; v < V; ++v) {
+            ep += exp(zp[v] - mp);
+            eq += exp(zq[v] - mq);
+        }
+        double lp = mp + log(ep), lq = mq + log(eq);
+        double acc = 0.0;
+        for (int64_t v = 0; v < V; ++v) {
+            double logp = zp[v] - lp, logq = zq[v] - lq;
+            acc += exp(logp) * (logp - logq);
+        }
+        kl[i] = acc;
+        free(zq);
+        free(zp);
+        free(b);
+        free(a);
+    }
+}
+
 void oracle_sgd_step(float *p, const float *g, int64_t n, float lr)
 {
     for (int64_t i = 0; i < n; ++i) {
