@@ -692,6 +692,22 @@ def run_episode(args):
     torch.cuda.synchronize()
     barrier()
     t_e2e = f0.elapsed_time(f1)
+    # the adapter-drift diagnostic (Sec. 4, Fig. 6) on the last update's rows:
+    # 4 L V d algorithmic FLOPs per call (both logit sets once)
+    kl = torch.empty(ew.L, dtype=torch.float32, device=dev)
+    kl_mean = torch.empty(1, dtype=torch.float32, device=dev)
+    x_last = xs[(state["k"] - 1) % ew.updates]
+    for _ in range(3):
+        ep.drift(x_last, kl, kl_mean)
+    torch.cuda.synchronize()
+    g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g0.record()
+    for _ in range(args.steps):
+        ep.drift(x_last, kl, kl_mean)
+    g1.record()
+    torch.cuda.synchronize()
+    t_kl = g0.elapsed_time(g1) / args.steps
+    kl_flops = 4.0 * ew.L * ew.V * ew.d + 2 * 2.0 * ew.L * ew.din * ew.d
     if pg is not None:
         t_ms, t_e2e = max_over_ranks([t_ms, t_e2e], pg, dev)
 
@@ -723,6 +739,11 @@ def run_episode(args):
                          "peak_kind": f"bf16 sustained, {peaks['src']}"},
             "clocks": clk,
             "cpu_baseline": cpu,
+            "kl_drift": {"ms": round(t_kl, 4), "kl_mean": round(kl_mean.item(), 6),
+                         "achieved_tflops": round(kl_flops / (t_kl * 1e-3) / 1e12, 1),
+                         "frac": round(kl_flops / (t_kl * 1e-3) / 1e12 / peaks["bf16_sustained"], 4),
+                         "work": "attt_episode_drift: adapted and base projection forward, then the KL through "
+                                 "the LM head (4 L V d + 4 L din d FLOPs)"},
         }
     if pg is not None:
         pg.barrier()

@@ -306,6 +306,30 @@ ATTT_API attt_status attt_lora_input_grad(const attt_bf16 *d_dy, const attt_bf16
 ATTT_API attt_status attt_cast_bf16(const float *d_src, attt_bf16 *d_dst, int64_t n, attt_stream stream);
 
 /* ------------------------------------------------------------------------ */
+/* Adapter drift (Sec. 4, Fig. 6): the KL divergence of the adapted model's */
+/* next-token distribution from the base model's, through the frozen LM     */
+/* head, without the [L, V] logits in HBM.                                  */
+/* ------------------------------------------------------------------------ */
+
+/* Workspace bytes attt_kl_drift needs for (L, d, V). */
+ATTT_API size_t attt_kl_workspace_bytes(int64_t L, int64_t d, int64_t V);
+
+/*
+ * With p_j = softmax(h_p[j] W^T) (the adapted model) and q_j =
+ * softmax(h_q[j] W^T) (the base model), h_p = d_hp and h_q = d_hq (bf16
+ * [L, d]), W = d_W (bf16 [V, d]):
+ *   d_kl[j]    = KL(p_j || q_j) = sum_v p_jv (log p_jv - log q_jv)   (fp32 [L])
+ *   *d_kl_mean = (1/L) sum_j KL(p_j || q_j)    (summed in a fixed order)
+ * Either output may be NULL (not both).  bf16 products, fp32 accumulation;
+ * every logit is computed once (4 L V d FLOPs).  Requirements: L >= 1,
+ * V >= 1, d >= 8 and d % 8 == 0, d_hp / d_hq / d_W 16-byte aligned, d_ws at
+ * least attt_kl_workspace_bytes(L, d, V) bytes and 256-byte aligned.
+ */
+ATTT_API attt_status attt_kl_drift(const attt_bf16 *d_hp, const attt_bf16 *d_hq, const attt_bf16 *d_W,
+                                   int64_t L, int64_t d, int64_t V, float *d_kl, float *d_kl_mean,
+                                   void *d_ws, size_t ws_bytes, attt_stream stream);
+
+/* ------------------------------------------------------------------------ */
 /* Update-text repetition (Eq. 6), novelty (Eq. 7) and the sequence-level   */
 /* filter of Sec. 4 (skip an update whose novelty is below tau; Appendix C: */
 /* tau = 0.5), over the episode's word sets.                                */
@@ -429,6 +453,16 @@ ATTT_API attt_status attt_episode_update(attt_episode *e, const int32_t *d_token
 ATTT_API attt_status attt_episode_agent_step(attt_episode *e, const int32_t *d_tokens, const attt_bf16 *d_x,
                                              int64_t len, float *d_losses, float *d_dx, int *updated,
                                              attt_stream stream);
+
+/*
+ * The adapter-drift diagnostic (Sec. 4, Fig. 6) on the projection inputs d_x
+ * (bf16 [L, din], 1 <= L <= max_update): attt_kl_drift between the adapted
+ * model's hidden states x W0 + s (x A) B (the current adapter) and the base
+ * model's x W0 (no adapter), through the LM head; d_kl (fp32 [L]) and / or
+ * d_kl_mean (fp32 [1]).  Does not change the episode.  Async on `stream`.
+ */
+ATTT_API attt_status attt_episode_drift(attt_episode *e, const attt_bf16 *d_x, int64_t L, float *d_kl,
+                                        float *d_kl_mean, attt_stream stream);
 
 /* Copies the adapter's fp32 values (A [din, r], B [r, d]) out.  Async. */
 ATTT_API attt_status attt_episode_read_adapter(const attt_episode *e, float *d_A32, float *d_B32,

@@ -93,8 +93,11 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_episode_update": (i32, [P, P, P, i64, P, P, P]),
             "attt_episode_agent_step": (i32, [P, P, P, i64, P, P, ctypes.POINTER(i32), P]),
             "attt_episode_read_adapter": (i32, [P, P, P, P]),
+            "attt_episode_drift": (i32, [P, P, i64, P, P, P]),
             "attt_episode_history": (P, [P]),
             "attt_episode_pending_tokens": (i64, [P]),
+            "attt_kl_workspace_bytes": (sz, [i64, i64, i64]),
+            "attt_kl_drift": (i32, [P, P, P, i64, i64, i64, P, P, P, sz, P]),
             "attt_wordsets_create": (i32, [i32, i64, ctypes.POINTER(P)]),
             "attt_wordsets_destroy": (i32, [P]),
             "attt_wordsets_reset": (i32, [P, P]),
@@ -493,6 +496,21 @@ class Episode:
     def reset(self, stream=None) -> None:
         _check(self._lib.attt_episode_reset(self.handle, _stream(stream)), "attt_episode_reset")
 
+    def drift(self, x: torch.Tensor, kl: Optional[torch.Tensor] = None, kl_mean: Optional[torch.Tensor] = None,
+              stream=None):
+        """KL of the adapted from the base next-token distribution on the rows
+        of x (bf16 [L, din]).  Returns (kl [L], kl_mean [1])."""
+        L = x.shape[0]
+        if tuple(x.shape) != (L, self.cfg.din):
+            raise ValueError("x must be [L, din]")
+        if kl is None:
+            kl = torch.empty(L, dtype=torch.float32, device=x.device)
+        if kl_mean is None:
+            kl_mean = torch.empty(1, dtype=torch.float32, device=x.device)
+        _check(self._lib.attt_episode_drift(self.handle, _bf16(x), L, _ptr(kl), _ptr(kl_mean), _stream(stream)),
+               "attt_episode_drift")
+        return kl, kl_mean
+
     def read_adapter(self, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
         """(A [din, r], B [r, d]) fp32 copies of the current adapter."""
         c = self.cfg
@@ -508,6 +526,34 @@ class Episode:
 
     def pending_tokens(self) -> int:
         return int(self._lib.attt_episode_pending_tokens(self.handle))
+
+
+# --------------------------------------------------------------------------
+# adapter drift (Sec. 4, Fig. 6)
+# --------------------------------------------------------------------------
+
+def attt_kl_workspace_bytes(L: int, d: int, V: int) -> int:
+    return int(load_library().attt_kl_workspace_bytes(L, d, V))
+
+
+def attt_kl_drift(hp: torch.Tensor, hq: torch.Tensor, W: torch.Tensor, kl: Optional[torch.Tensor] = None,
+                  kl_mean: Optional[torch.Tensor] = None, workspace: Optional[torch.Tensor] = None, stream=None):
+    """KL(softmax(h_p W^T) || softmax(h_q W^T)) per row (fp32 [L]) and its
+    mean (fp32 [1]).  Returns (kl, kl_mean)."""
+    L, d = hp.shape
+    V = W.shape[0]
+    if tuple(hq.shape) != (L, d) or W.shape[1] != d:
+        raise ValueError("shape mismatch")
+    dev = hp.device
+    if kl is None:
+        kl = torch.empty(L, dtype=torch.float32, device=dev)
+    if kl_mean is None:
+        kl_mean = torch.empty(1, dtype=torch.float32, device=dev)
+    if workspace is None:
+        workspace = torch.empty(attt_kl_workspace_bytes(L, d, V), dtype=torch.uint8, device=dev)
+    _check(load_library().attt_kl_drift(_bf16(hp), _bf16(hq), _bf16(W), L, d, V, _ptr(kl), _ptr(kl_mean),
+                                        _ptr(workspace), workspace.numel(), _stream(stream)), "attt_kl_drift")
+    return kl, kl_mean
 
 
 # --------------------------------------------------------------------------

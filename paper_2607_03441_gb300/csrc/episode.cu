@@ -36,7 +36,7 @@ struct attt_episode {
     attt_bf16 *A16, *B16;
     // per-update activations
     float *w, *dh, *losses;
-    attt_bf16 *h, *dy;
+    attt_bf16 *h, *dy, *h_base;
     // pending update text (agent steps since the last update)
     int32_t *pend_tok;
     attt_bf16 *pend_x;
@@ -59,7 +59,7 @@ bool dev_alloc(T **p, size_t count) {
 void free_all(attt_episode *e) {
     if (e->hist) attt_history_destroy(e->hist);
     void *bufs[] = {e->A32, e->B32, e->A0, e->B0, e->dA, e->dB, e->A16, e->B16, e->w,
-                    e->dh,  e->losses, e->h, e->dy, e->pend_tok, e->pend_x, e->ws};
+                    e->dh,  e->losses, e->h, e->dy, e->h_base, e->pend_tok, e->pend_x, e->ws};
     for (void *b : bufs) cudaFree(b);
 }
 
@@ -82,6 +82,7 @@ size_t workspace_bound(const attt_episode_config &c) {
     upd(attt_lora_workspace_bytes(L, c.din, 1, &c.d, c.r));
     upd(attt_lora_forward_workspace_bytes(L, c.din, c.d, c.r));
     upd(attt_lora_input_grad_workspace_bytes(L, c.din, c.d, c.r));
+    upd(attt_kl_workspace_bytes(L, c.d, c.V));  // grows with L
     return ws;
 }
 
@@ -122,7 +123,8 @@ attt_status attt_episode_create(const attt_episode_config *cfg, const attt_bf16 
     ok = ok && dev_alloc(&e->A32, nA) && dev_alloc(&e->B32, nB) && dev_alloc(&e->A0, nA) && dev_alloc(&e->B0, nB) &&
          dev_alloc(&e->dA, nA) && dev_alloc(&e->dB, nB) && dev_alloc(&e->A16, nA) && dev_alloc(&e->B16, nB) &&
          dev_alloc(&e->w, (size_t)c.max_update) && dev_alloc(&e->dh, Ld) && dev_alloc(&e->losses, (size_t)c.grad_steps) &&
-         dev_alloc(&e->h, Ld) && dev_alloc(&e->dy, Ld) && dev_alloc(&e->pend_tok, (size_t)c.max_update) &&
+         dev_alloc(&e->h, Ld) && dev_alloc(&e->dy, Ld) && dev_alloc(&e->h_base, Ld) &&
+         dev_alloc(&e->pend_tok, (size_t)c.max_update) &&
          dev_alloc(&e->pend_x, (size_t)c.max_update * c.din) &&
          dev_alloc(reinterpret_cast<char **>(&e->ws), e->ws_bytes);
     if (ok) {
@@ -216,6 +218,23 @@ attt_status attt_episode_agent_step(attt_episode *e, const int32_t *d_tokens, co
     if (L == 0) return ATTT_OK;  // K steps without update text: nothing to train on
     attt_status st = attt_episode_update(e, e->pend_tok, e->pend_x, L, d_losses, d_dx, stream);
     if (st == ATTT_OK && updated) *updated = 1;
+    return st;
+}
+
+attt_status attt_episode_drift(attt_episode *e, const attt_bf16 *d_x, int64_t L, float *d_kl, float *d_kl_mean,
+                               attt_stream stream) {
+    using namespace attt;
+    if (!e || L < 1 || L > e->cfg.max_update || !d_x || !aligned16(d_x) || (!d_kl && !d_kl_mean))
+        return ATTT_ERR_INVALID_ARG;
+    const attt_episode_config &c = e->cfg;
+    // the adapted model (current adapter) and the base model (no adapter: s = 0)
+    attt_status st = attt_lora_forward(d_x, e->W0, e->A16, e->B16, L, c.din, c.d, c.r, c.scale, e->h, e->ws,
+                                       e->ws_bytes, stream);
+    if (st == ATTT_OK)
+        st = attt_lora_forward(d_x, e->W0, e->A16, e->B16, L, c.din, c.d, c.r, 0.0f, e->h_base, e->ws,
+                               e->ws_bytes, stream);
+    if (st == ATTT_OK)
+        st = attt_kl_drift(e->h, e->h_base, e->Wlm, L, c.d, c.V, d_kl, d_kl_mean, e->ws, e->ws_bytes, stream);
     return st;
 }
 

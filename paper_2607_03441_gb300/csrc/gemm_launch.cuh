@@ -60,9 +60,9 @@ inline int tail_pieces(int tiles, int units, int kb_total, int nranks, int regio
 
 constexpr size_t kMaxSmem = 232448;  // 227 KB opt-in per CTA on sm_100-class parts
 
-inline int gemm_stages(int BN, uint32_t extra = 0) {
+inline int gemm_stages(int BN, uint32_t extra = 0, int a_tiles = 1) {
     int s = 8;
-    while (s > 2 && gemm_smem_bytes(BN, s, extra) > kMaxSmem) --s;
+    while (s > 2 && gemm_smem_bytes(BN, s, extra, a_tiles) > kMaxSmem) --s;
     return s;
 }
 
@@ -97,7 +97,12 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
         ok = make_tmap_bf16(&tb, p.b, (uint64_t)p.b_rows, (uint64_t)p.b_k, (uint64_t)p.b_rows_ld * 2, 64, 64);
     if (!ok) return ATTT_ERR_INVALID_ARG;
     CUtensorMap ta2 = ta, tb2 = tb;
-    if (p.K2 > 0) {
+    if (EPI == EPI_KL) {
+        // the second A operand (same shape as A) shares every B tile
+        if (!p.a2 || !p.pair || A_MN || B_MN) return ATTT_ERR_INVALID_ARG;
+        if (!make_tmap_bf16(&ta2, p.a2, (uint64_t)p.a_k, (uint64_t)p.a_rows, (uint64_t)p.a2_rows_ld * 2, 64, 128))
+            return ATTT_ERR_INVALID_ARG;
+    } else if (p.K2 > 0) {
         if (!p.a2 || !p.b2) return ATTT_ERR_INVALID_ARG;
         if (!A_MN)
             ok = make_tmap_bf16(&ta2, p.a2, (uint64_t)p.a2_k, (uint64_t)p.a2_rows, (uint64_t)p.a2_rows_ld * 2, 64, 128);
@@ -131,7 +136,8 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.BN = p.BN;
     const int bn_cta = p.pair ? p.BN / 2 : p.BN;  // B rows one CTA stages
     g.e_stage_bytes = (EPI == EPI_CE_EXP || EPI == EPI_BF16) ? kEStageBytes : EPI == EPI_F32_ACC ? kF32StageBytes : 0u;
-    g.stages = gemm_stages(bn_cta, g.e_stage_bytes);
+    const int a_tiles = EPI == EPI_KL ? 2 : 1;
+    g.stages = gemm_stages(bn_cta, g.e_stage_bytes, a_tiles);
     g.tiles_m = (int)cdiv(p.M, 128);
     g.tiles_n = (int)cdiv(p.N, p.BN);
     g.kb_split = (int)cdiv(p.K, 64);
@@ -156,12 +162,12 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.a_k_off = p.a_k_off;
     g.b_n_off = p.b_n_off;
     g.b_k_off = p.b_k_off;
-    g.tmem_cols = gemm_tmem_cols(p.BN);
+    g.tmem_cols = gemm_tmem_cols(p.BN * a_tiles);
     g.operands_ready = p.operands_ready ? 1 : 0;
     g.status = status ? status : device_status_word(dev);
     g.ep = ep;
 
-    const size_t smem = gemm_smem_bytes(bn_cta, g.stages, g.e_stage_bytes);
+    const size_t smem = gemm_smem_bytes(bn_cta, g.stages, g.e_stage_bytes, a_tiles);
     const int ntiles = g.whole_tiles + (tiles - g.whole_tiles) * g.tail_s;  // work items
     cudaLaunchConfig_t cfg = {};
     cfg.blockDim = dim3(kGemmThreads);
@@ -175,12 +181,14 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
         ++na;
     }
     if (!p.pair) {
-        auto kern = tc_gemm_kernel<EPI, A_MN, B_MN>;
-        if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
-        cfg.gridDim = dim3((unsigned)(ntiles < sms ? ntiles : sms));
-        cfg.attrs = attr;
-        cfg.numAttrs = na;
-        if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, ta2, tb2, g) != cudaSuccess) return ATTT_ERR_CUDA;
+        if constexpr (EPI != EPI_KL) {  // EPI_KL runs on CTA pairs only
+            auto kern = tc_gemm_kernel<EPI, A_MN, B_MN>;
+            if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
+            cfg.gridDim = dim3((unsigned)(ntiles < sms ? ntiles : sms));
+            cfg.attrs = attr;
+            cfg.numAttrs = na;
+            if (cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, ta2, tb2, g) != cudaSuccess) return ATTT_ERR_CUDA;
+        }
     } else {
         auto kern = tc_gemm_pair_kernel<EPI, A_MN, B_MN>;
         if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;

@@ -32,6 +32,7 @@ enum EpiKind : int {
     EPI_CE_EXP = 0,    // per (row, vocab tile): max m, E = exp(z - m) as bf16, sum of E, target logit
     EPI_F32_ACC = 2,   // out[m, n] = (acc ? alpha_m out[m, n] : 0) + beta_m acc [- gamma_m W[t_m, n]]  (fp32)
     EPI_BF16 = 5,      // out16[m, n] = bf16(alpha * acc)  (row-major, through TMA boxes)
+    EPI_KL = 6,        // two accumulators z = A B^T, z2 = A2 B^T: per (row, tile) max, sum of exp, cross term
 };
 
 constexpr int kMaxProj = 8;
@@ -59,6 +60,9 @@ struct EpiParams {
     int64_t fix_ld;
     int fix_V;
     __nv_bfloat16 *out16;    // EPI_BF16 output, row pitch out_ld
+    // EPI_KL: five planes of [tiles, M] fp32 (m_p, s_p, m_q, s_q, x), kl_plane apart
+    float *kl_part;
+    int64_t kl_plane;
 };
 
 struct GemmArgs {
@@ -93,8 +97,9 @@ __host__ __device__ inline uint32_t gemm_b_stage_bytes(int BN) { return (uint32_
 // 32 rows x 32 bf16 (64-byte swizzle), written out by TMA stores.
 constexpr uint32_t kEStageBytes = 4 * 2 * 32 * 64;
 
-__host__ __device__ inline size_t gemm_smem_bytes(int BN, int stages, uint32_t extra = 0) {
-    return 1024 + (size_t)stages * (kABytes + gemm_b_stage_bytes(BN)) + extra + 8 * (2 * stages + 5) + 16;
+// a_tiles: A tiles per stage (2 for EPI_KL, whose two accumulators share B).
+__host__ __device__ inline size_t gemm_smem_bytes(int BN, int stages, uint32_t extra = 0, int a_tiles = 1) {
+    return 1024 + (size_t)stages * (a_tiles * kABytes + gemm_b_stage_bytes(BN)) + extra + 8 * (2 * stages + 5) + 16;
 }
 
 // One 32 x 32 bf16 block of E (this warp's 32 rows, 32 columns from x) to
@@ -416,6 +421,55 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
     }
 }
 
+// EPI_KL, one accumulator row per thread: z_p = h_p W^T at taddr and z_q =
+// h_q W^T at taddr + BN.  Over the tile's columns: the maxima m_p, m_q and the
+// sums s = sum exp2(z log2e - m) (log2 units), and the cross term
+// x = sum exp2(z_p log2e - m_p) (z_p - z_q) (nats), all in fp32 from the fp32
+// accumulators.  TMEM loads are warp-wide, so rows past M load and skip the
+// store.
+__device__ __forceinline__ void epilogue_kl(const GemmArgs &g, int gm_base, int tn, int row, uint32_t taddr) {
+    const int gm = gm_base + row;
+    const int n_base = tn * g.BN;
+    const int nv = min(g.N, n_base + g.BN) - n_base;  // valid columns of the tile
+    float mp = -INFINITY, mq = -INFINITY;
+    for (int c = 0; c < g.BN; c += 32) {
+        float vp[32], vq[32];
+        tmem_ld_x32(taddr + (uint32_t)c, vp);
+        tmem_ld_x32(taddr + (uint32_t)(g.BN + c), vq);
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+            if (c + i < nv) {
+                mp = fmaxf(mp, vp[i]);
+                mq = fmaxf(mq, vq[i]);
+            }
+    }
+    mp *= kLog2e;
+    mq *= kLog2e;
+    float sp = 0.f, sq = 0.f, x = 0.f;
+    for (int c = 0; c < g.BN; c += 32) {
+        float vp[32], vq[32];
+        tmem_ld_x32(taddr + (uint32_t)c, vp);
+        tmem_ld_x32(taddr + (uint32_t)(g.BN + c), vq);
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+            if (c + i < nv) {
+                const float ep = exp2f(fmaf(vp[i], kLog2e, -mp));
+                sp += ep;
+                sq += exp2f(fmaf(vq[i], kLog2e, -mq));
+                x = fmaf(ep, vp[i] - vq[i], x);
+            }
+    }
+    if (gm < g.M) {
+        const EpiParams &ep = g.ep;
+        const int64_t o = (int64_t)(ep.tile0 + tn) * g.M + gm, P = ep.kl_plane;
+        ep.kl_part[o] = mp;
+        ep.kl_part[P + o] = sp;
+        ep.kl_part[2 * P + o] = mq;
+        ep.kl_part[3 * P + o] = sq;
+        ep.kl_part[4 * P + o] = x;
+    }
+}
+
 // EPI_F32_ACC for K piece k.piece of tail tile k.tail, on the 128 accumulator
 // rows this CTA holds (CTA `rank` of `nranks`).  The four epilogue warps store
 // the piece's partial (column-quad major: a warp writes 512 contiguous bytes
@@ -702,8 +756,13 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int S = g.stages;
     const int BNh = g.BN / 2;  // B rows held by this CTA
     const uint32_t b_bytes = gemm_b_stage_bytes(BNh);
+    // EPI_KL stages two A tiles (h_p, h_q) against one B tile and keeps two
+    // accumulators per tile
+    constexpr int kAT = EPI == EPI_KL ? 2 : 1;
+    static_assert(EPI != EPI_KL || (!A_MN && !B_MN), "EPI_KL: K-major operands");
+    constexpr uint32_t a_bytes = kAT * kABytes;
     uint8_t *sA = smem;
-    uint8_t *sB = smem + (size_t)S * kABytes;
+    uint8_t *sB = smem + (size_t)S * a_bytes;
     uint8_t *sE = sB + (size_t)S * b_bytes;  // 1024-byte aligned: b_bytes is a multiple of 2048
     uint64_t *bars = reinterpret_cast<uint64_t *>(sE + g.e_stage_bytes);
     const uint32_t full0 = smem_u32(bars);
@@ -769,9 +828,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const int brow0 = wi.tn * g.BN + BNh * (int)rank;
                 for (int kb = wi.kb0; kb < wi.kb1; ++kb) {
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
-                    if (leader) mbar_arrive_expect_tx(full0 + 8 * stage, 2u * (kABytes + b_bytes));
+                    if (leader) mbar_arrive_expect_tx(full0 + 8 * stage, 2u * (a_bytes + b_bytes));
                     const uint32_t fb = lead_full0 + 8 * stage;
-                    const uint32_t a_dst = smem_u32(sA + (size_t)stage * kABytes);
+                    const uint32_t a_dst = smem_u32(sA + (size_t)stage * a_bytes);
                     const uint32_t b_dst = smem_u32(sB + (size_t)stage * b_bytes);
                     // K block kb of the first pair, or K block kb - kb_split of the second
                     const bool sec = kb >= g.kb_split;
@@ -783,6 +842,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     const int brow = (sec ? 0 : g.b_n_off) + brow0;
                     if (!A_MN) {
                         tma_load_2d_pair(a_dst, pa, fb, ka, arow);
+                        if constexpr (kAT == 2) tma_load_2d_pair(a_dst + kABytes, &tmA2, fb, ka, arow);
                     } else {
                         tma_load_2d_pair(a_dst, pa, fb, arow, ka);
                         tma_load_2d_pair(a_dst + 8192, pa, fb, arow + 64, ka);
@@ -814,11 +874,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const int acc = it & 1;
                 if (!mbar_wait(tempty0 + 8 * acc, (((uint32_t)it >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * g.BN);
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * kAT * g.BN);
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) { ok = false; break; }
                     tc_fence_after();
-                    const uint32_t a_addr = smem_u32(sA + (size_t)stage * kABytes);
+                    const uint32_t a_addr = smem_u32(sA + (size_t)stage * a_bytes);
                     const uint32_t b_addr = smem_u32(sB + (size_t)stage * b_bytes);
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk) {
@@ -827,6 +887,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         const uint64_t bd = B_MN ? smem_desc_sw128(b_addr + kk * 2048, 8192, 1024)
                                                  : smem_desc_sw128(b_addr + kk * 32, 16, 1024);
                         umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+                        if constexpr (kAT == 2) {
+                            const uint64_t ad2 = smem_desc_sw128(a_addr + kABytes + kk * 32, 16, 1024);
+                            umma_bf16_pair(d_tmem + (uint32_t)g.BN, ad2, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+                        }
                     }
                     umma_commit_pair(empty0 + 8 * stage, 3);
                     if (++stage == S) { stage = 0; phase ^= 1u; }
@@ -864,9 +928,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             }
             (void)mbar_try_wait(tfull0 + 8 * acc, par);
             tc_fence_after();
-            const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * g.BN);
+            const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kAT * g.BN);
             const int gm_base = wi.tm * 256 + 128 * (int)rank;
-            if constexpr (EPI == EPI_F32_ACC) {
+            if constexpr (EPI == EPI_KL) {
+                epilogue_kl(g, gm_base, wi.tn, row, taddr);
+            } else if constexpr (EPI == EPI_F32_ACC) {
                 if (wi.piece >= 0) {
                     epilogue_piece_f32_acc(g, wi, gm_base, (int)rank, 2, row, taddr, &tmC, fst, abort_flag);
                 } else {

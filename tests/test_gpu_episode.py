@@ -234,3 +234,33 @@ def test_7b_update_is_the_composition_of_its_calls(attt):
     assert attt.attt_device_status() == 0
     ep.close()
     attt.attt_history_destroy(hist)
+
+
+def test_drift_is_the_kl_of_adapted_and_base_states(attt, tiny):
+    """attt_episode_drift = attt_kl_drift of the adapted projection's output
+    (current adapter) and the base one's (no adapter), bit for bit; that KL
+    against the oracle on the same hidden states."""
+    ew, texts, dense, xs = tiny
+    ep = _episode(attt, ew, dense, 20.0)
+    for k in range(2):
+        ep.update(i32_dev(texts[k]), bf16_dev(xs[k]))
+    x = bf16_dev(xs[2])
+    kl, mean = ep.drift(x)
+    A32, B32 = ep.read_adapter()
+    A16, B16 = attt.attt_cast_bf16(A32), attt.attt_cast_bf16(B32)
+    W0, W = bf16_dev(dense["W0"]), bf16_dev(dense["W"])
+    hp = attt.attt_lora_forward(x, W0, A16, B16, ew.scale)
+    hq = attt.attt_lora_forward(x, W0, A16, B16, 0.0)
+    kl2, mean2 = attt.attt_kl_drift(hp, hq, W)
+    assert torch.equal(kl, kl2) and torch.equal(mean, mean2)
+    hp_b = hp.view(torch.int16).cpu().numpy().view(np.uint16)
+    hq_b = hq.view(torch.int16).cpu().numpy().view(np.uint16)
+    ref = oracle.kl_rows(hp_b, hq_b, dense["W"])
+    got = kl.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(got - ref) <= 5e-5 + 1e-3 * np.abs(ref))
+    assert ref.mean() > 1e-4   # the adapter moved the model
+    # a fresh episode's adapter (the initial one) drifts less than the trained one
+    fresh = _episode(attt, ew, dense, 20.0)
+    assert fresh.drift(x)[1].item() < mean.item()
+    ep.close()
+    fresh.close()
