@@ -770,6 +770,101 @@ def _episode_oracle_sample(ew, texts, dense, xs_host, rows):
 
 
 # ---------------------------------------------------------------------------
+# a batch of concurrent episodes updated together (attt_batch_*)
+# ---------------------------------------------------------------------------
+
+BATCH_EPISODES = 16  # Sec. 4: 16 episodes run concurrently
+
+
+def run_batch(args):
+    """One step = one batched update of 16 episodes (the 7B-class episode's
+    shapes): every episode updates on its own 2,048-token text (episode e takes
+    text (k + e) mod 16 of the episode workload at step k), two gradient steps
+    with dx, one history per episode; all histories and adapters are reset
+    after 16 steps."""
+    import torch
+    from paper_2607_03441_gb300 import attt
+    from paper_2607_03441_gb300 import build
+    build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peaks = _peaks()
+    ew = wk.EPISODES["7b-episode"]
+    E = BATCH_EPISODES
+    texts = wk.episode_texts(ew)
+    dense = wk.episode_dense(ew)
+    xs_host = [wk.episode_x(ew, k) for k in range(1, ew.updates + 1)]
+
+    def bf(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
+
+    W0, Wlm = bf(dense["W0"]), bf(dense["W"])
+    b = attt.Batch(W0, Wlm, torch.from_numpy(dense["A0"]).to(dev), torch.from_numpy(dense["B0"]).to(dev),
+                   episodes=E, n=ew.n, max_history=ew.L * ew.updates, max_update=ew.L, scale=ew.scale, lr=ew.lr,
+                   w_min=ew.w_min, grad_steps=ew.grad_steps)
+    xs = [bf(x) for x in xs_host]
+    toks = [torch.from_numpy(t).to(dev) for t in texts]
+    # the stacked inputs of each step index, resident before timing
+    stacked = []
+    for k in range(ew.updates):
+        order = [(k + e) % ew.updates for e in range(E)]
+        stacked.append((torch.cat([toks[i] for i in order]), torch.cat([xs[i] for i in order])))
+    lens = [ew.L] * E
+    R = ew.L * E
+    losses = torch.empty(E, ew.grad_steps, dtype=torch.float32, device=dev)
+    dx = torch.empty(ew.grad_steps, R, ew.din, dtype=torch.float32, device=dev)
+    state = {"k": 0}
+
+    def step():
+        k = state["k"]
+        if k == 0:
+            b.reset(-1)
+        t, x = stacked[k]
+        b.update(t, x, lens, losses=losses, dx=dx)
+        state["k"] = (k + 1) % ew.updates
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if attt.attt_device_status() != 0:
+        raise RuntimeError("device status error after warm-up")
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(0)
+    clocks.start()
+    n0 = attt.attt_kernel_launches()
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    n1 = attt.attt_kernel_launches()
+    clk = clocks.stop()
+    if attt.attt_device_status() != 0:
+        raise RuntimeError("device status error in the timed region")
+    t_ms = e0.elapsed_time(e1)
+    value = R * args.steps / (t_ms * 1e-3)
+    flops = E * episode_flops(ew)
+    ach = flops / (t_ms / args.steps * 1e-3) / 1e12
+    out = {"metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": round(t_ms / args.steps, 4), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+           "config": {"workload": (f"7b-batch: {E} concurrent episodes updated together (attt_batch_update), each "
+                                   f"L={ew.L} tokens, V={ew.V}, adapter r={ew.r} on a {ew.din}x{ew.d} projection "
+                                   f"feeding the LM head, {ew.grad_steps} SGD steps with dx, n={ew.n}; "
+                                   f"reset after {ew.updates} steps"),
+                      "global_batch": R, "seq_len": ew.L, "parallelism": "replicas1",
+                      "l2": "inputs larger than L2 (LM head streamed by every Eq. 10 chunk)"},
+           "gpu_launches": int(n1 - n0),
+           "roofline": {"bound": "tensor", "achieved": round(ach, 1), "peak": peaks["bf16_sustained"],
+                        "unit": "TFLOP/s", "frac": round(ach / peaks["bf16_sustained"], 4), "traffic": None,
+                        "kernel": "whole batched update (Eq. 10 over all rows twice, projection forward and dx, "
+                                  "adapter grads)", "peak_kind": f"bf16 sustained, {peaks['src']}"},
+           "clocks": clk}
+    b.close()
+    return out
+
+
+# ---------------------------------------------------------------------------
 # update-text repetition (Eq. 6), novelty (Eq. 7) and the sequence filter
 # ---------------------------------------------------------------------------
 
@@ -890,7 +985,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["attt", "reference"], default="attt")
     ap.add_argument("--workload", default=WORKLOAD,
-                    choices=["tiny", "7b", "long", "32b", "stress"] + sorted(wk.EPISODES) + sorted(wk.TEXT_WORKLOADS),
+                    choices=["tiny", "7b", "long", "32b", "stress", "7b-batch"] + sorted(wk.EPISODES)
+                    + sorted(wk.TEXT_WORKLOADS),
                     help="'stress' times the n-gram insert and weights on the 1M-token history; "
                          "'*-episode' runs chained updates through attt_episode_*")
     ap.add_argument("--part", default="all", choices=["all", "ce", "lora", "ngram"],
@@ -908,6 +1004,8 @@ def main():
         out = run_episode(args)
     elif args.workload in wk.TEXT_WORKLOADS:
         out = run_texts(args)
+    elif args.workload == "7b-batch":
+        out = run_batch(args)
     else:
         out = run_gpu(args)
     if out is not None:

@@ -474,6 +474,65 @@ ATTT_API attt_history *attt_episode_history(attt_episode *e);
 /* Tokens of pending agent-step text not yet trained on. */
 ATTT_API int64_t attt_episode_pending_tokens(const attt_episode *e);
 
+/* ------------------------------------------------------------------------ */
+/* A batch of concurrent episodes (Sec. 4 runs 16 at once, each with a      */
+/* private adapter and history) updated together.                           */
+/* ------------------------------------------------------------------------ */
+
+typedef struct attt_batch attt_batch;
+
+typedef struct attt_batch_config {
+    int episodes;        /* E, 1..32                                            */
+    int n;               /* n-gram size of Eq. 8 (1..16)                        */
+    float w_min;         /* Eq. 9 floor                                         */
+    int64_t max_history; /* tokens each episode's history may hold              */
+    int64_t max_update;  /* largest update text of one episode (<= max_history) */
+    int64_t din, d, V;   /* adapted projection [din, d], LM head [V, d]         */
+    int r;               /* adapter rank, 1..64 (a multiple of 8 for dx)        */
+    float scale, lr;     /* s = alpha / r; SGD rate of Eq. 2                    */
+    int grad_steps;      /* gradient steps per update (Appendix C: 2)           */
+} attt_batch_config;
+
+/*
+ * Creates E episodes on the current device sharing the frozen d_W0 (bf16
+ * [din, d]) and d_Wlm (bf16 [V, d]) (borrowed, as for attt_episode_create);
+ * every episode's adapter starts at d_A0 (fp32 [din, r]) / d_B0 (fp32 [r, d])
+ * (copied).  Everything the updates need is allocated here.
+ */
+ATTT_API attt_status attt_batch_create(const attt_batch_config *cfg, const attt_bf16 *d_W0, const attt_bf16 *d_Wlm,
+                                       const float *d_A0, const float *d_B0, attt_batch **out);
+
+/* Frees the batch and everything it allocated (synchronises the device). */
+ATTT_API attt_status attt_batch_destroy(attt_batch *b);
+
+/* Episode boundary for episode e (-1: every episode): its adapter returns to
+ * (A0, B0) and its history is emptied.  Async on `stream`. */
+ATTT_API attt_status attt_batch_reset(attt_batch *b, int e, attt_stream stream);
+
+/*
+ * One update (Algorithm 1, as attt_episode_update) for every episode e with
+ * lens[e] > 0 (lens: HOST array of E lengths, 0 <= lens[e] <= max_update; an
+ * episode with lens[e] = 0 is left unchanged).  The update texts are stacked:
+ * d_tokens (int32 [sum lens]) and d_x (bf16 [sum lens, din]) hold episode 0's
+ * rows, then episode 1's, and so on.  d_losses (fp32 [E, grad_steps], or
+ * NULL) receives each episode's Eq. 10 loss per step (0 for an episode
+ * without rows); d_dx (fp32 [grad_steps, sum lens, din], 16-byte aligned, or
+ * NULL) the projection-input gradients.  Eq. 8/9, the dh -> dy cast, the SGD
+ * step and the history append each run as one launch for the whole batch
+ * and Eq. 10 as one call over every row; the adapter contractions run per
+ * episode.  ATTT_ERR_CAPACITY (nothing launched) if an episode's history
+ * would exceed max_history.  Async on `stream`.
+ */
+ATTT_API attt_status attt_batch_update(attt_batch *b, const int32_t *d_tokens, const attt_bf16 *d_x,
+                                       const int64_t *lens, float *d_losses, float *d_dx, attt_stream stream);
+
+/* Copies episode e's adapter (fp32 A [din, r], B [r, d]) out.  Async. */
+ATTT_API attt_status attt_batch_read_adapter(const attt_batch *b, int e, float *d_A32, float *d_B32,
+                                             attt_stream stream);
+
+/* Episode e's history (owned by the batch). */
+ATTT_API attt_history *attt_batch_history(attt_batch *b, int e);
+
 #ifdef __cplusplus
 }
 #endif

@@ -51,6 +51,14 @@ class EpisodeConfig(ctypes.Structure):
                 ("grad_steps", ctypes.c_int), ("cadence", ctypes.c_int)]
 
 
+class BatchConfig(ctypes.Structure):
+    """attt_batch_config (field order and types as in attt.h)."""
+    _fields_ = [("episodes", ctypes.c_int), ("n", ctypes.c_int), ("w_min", ctypes.c_float),
+                ("max_history", ctypes.c_int64), ("max_update", ctypes.c_int64), ("din", ctypes.c_int64),
+                ("d", ctypes.c_int64), ("V", ctypes.c_int64), ("r", ctypes.c_int), ("scale", ctypes.c_float),
+                ("lr", ctypes.c_float), ("grad_steps", ctypes.c_int)]
+
+
 def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     """Loads libattt.so (raises if it has not been built)."""
     global _lib
@@ -98,6 +106,12 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_episode_pending_tokens": (i64, [P]),
             "attt_kl_workspace_bytes": (sz, [i64, i64, i64]),
             "attt_kl_drift": (i32, [P, P, P, i64, i64, i64, P, P, P, sz, P]),
+            "attt_batch_create": (i32, [ctypes.POINTER(BatchConfig), P, P, P, P, ctypes.POINTER(P)]),
+            "attt_batch_destroy": (i32, [P]),
+            "attt_batch_reset": (i32, [P, i32, P]),
+            "attt_batch_update": (i32, [P, P, P, P, P, P, P]),
+            "attt_batch_read_adapter": (i32, [P, i32, P, P, P]),
+            "attt_batch_history": (P, [P, i32]),
             "attt_wordsets_create": (i32, [i32, i64, ctypes.POINTER(P)]),
             "attt_wordsets_destroy": (i32, [P]),
             "attt_wordsets_reset": (i32, [P, P]),
@@ -621,3 +635,74 @@ def attt_repetition(s: WordSets, text: torch.Tensor, tau: float = 0.5, out: Opti
     _check(load_library().attt_repetition(s.handle, _ptr(text) if n else None, n, float(tau), base, base + 4,
                                           _ptr(keep), _stream(stream)), "attt_repetition")
     return out, keep
+
+
+# --------------------------------------------------------------------------
+# a batch of concurrent episodes
+# --------------------------------------------------------------------------
+
+class Batch:
+    """Owning handle of an attt_batch: E episodes sharing W0 and the LM head
+    (borrowed: kept referenced here), each adapter starting at (A0, B0)."""
+
+    def __init__(self, W0: torch.Tensor, Wlm: torch.Tensor, A0: torch.Tensor, B0: torch.Tensor, *, episodes: int,
+                 n: int, max_history: int, max_update: int, scale: float, lr: float, w_min: float = 0.05,
+                 grad_steps: int = 2):
+        self._lib = load_library()
+        din, d = W0.shape
+        r = A0.shape[1]
+        if Wlm.shape[1] != d or A0.shape[0] != din or tuple(B0.shape) != (r, d):
+            raise ValueError("shape mismatch between W0, Wlm, A0, B0")
+        self.cfg = BatchConfig(episodes=int(episodes), n=int(n), w_min=float(w_min), max_history=int(max_history),
+                               max_update=int(max_update), din=int(din), d=int(d), V=int(Wlm.shape[0]), r=int(r),
+                               scale=float(scale), lr=float(lr), grad_steps=int(grad_steps))
+        b = ctypes.c_void_p()
+        _check(self._lib.attt_batch_create(ctypes.byref(self.cfg), _bf16(W0), _bf16(Wlm), _ptr(A0), _ptr(B0),
+                                           ctypes.byref(b)), "attt_batch_create")
+        self.handle = b
+        self._keep = (W0, Wlm)
+        self.device = W0.device
+
+    def close(self) -> None:
+        if getattr(self, "handle", None):
+            self._lib.attt_batch_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def update(self, tokens: torch.Tensor, x: torch.Tensor, lens: Sequence[int],
+               losses: Optional[torch.Tensor] = None, dx: Optional[torch.Tensor] = None, stream=None) -> None:
+        """One update of every episode with lens[e] > 0; tokens (int32) and x
+        (bf16 [sum lens, din]) hold the episodes' rows one after another."""
+        c = self.cfg
+        if len(lens) != c.episodes:
+            raise ValueError("one length per episode")
+        R = int(sum(lens))
+        if tokens.dtype != torch.int32 or tokens.numel() != R or tuple(x.shape) != (R, c.din):
+            raise ValueError("tokens must be int32 [sum lens] and x [sum lens, din]")
+        if losses is not None and (losses.dtype != torch.float32 or losses.numel() < c.episodes * c.grad_steps):
+            raise ValueError("losses must be float32 [E, grad_steps]")
+        if dx is not None and (dx.dtype != torch.float32 or dx.numel() < c.grad_steps * R * c.din):
+            raise ValueError("dx must be float32 [grad_steps, sum lens, din]")
+        arr = (ctypes.c_int64 * c.episodes)(*[int(v) for v in lens])
+        _check(self._lib.attt_batch_update(self.handle, _ptr(tokens), _bf16(x), arr, _ptr(losses), _ptr(dx),
+                                           _stream(stream)), "attt_batch_update")
+
+    def reset(self, e: int = -1, stream=None) -> None:
+        _check(self._lib.attt_batch_reset(self.handle, int(e), _stream(stream)), "attt_batch_reset")
+
+    def read_adapter(self, e: int, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+        c = self.cfg
+        A = torch.empty((c.din, c.r), dtype=torch.float32, device=self.device)
+        B = torch.empty((c.r, c.d), dtype=torch.float32, device=self.device)
+        _check(self._lib.attt_batch_read_adapter(self.handle, int(e), _ptr(A), _ptr(B), _stream(stream)),
+               "attt_batch_read_adapter")
+        return A, B
+
+    def history(self, e: int) -> History:
+        h = self._lib.attt_batch_history(self.handle, int(e))
+        return History._view(h, self.cfg.n, self.cfg.max_history, self)

@@ -44,6 +44,20 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
                           float scale, float *const *d_dA, float *const *d_dB, void *d_ws, size_t ws_bytes,
                           int *status, cudaStream_t stream);
 
+// Batched n-gram work over E histories (ngram.cu): rows [off[e], off[e+1])
+// of d_tokens are episode e's update (off: host array of E + 1 offsets).
+attt_status ngram_weights_batch(attt_history *const *hs, int E, const int32_t *d_tokens, const int64_t *off,
+                                float w_min, float *d_w, float *d_rowscale, cudaStream_t stream);
+attt_status history_insert_batch(attt_history *const *hs, int E, const int32_t *d_tokens, const int64_t *off,
+                                 cudaStream_t stream);
+
+// Eq. 10 as attt_weighted_ce_fwd_bwd, with per-row normalisers `row_scale`
+// (dh_j = w_j row_scale_j (...); nullptr: 1/L for every row) and the per-row
+// NLL lse_j - z_{j,t_j} into `nll` (nullptr: not written) (ce.cu).
+attt_status ce_fwd_bwd_run(const attt_bf16 *d_h, const attt_bf16 *d_W, const int32_t *d_tgt, const float *d_w,
+                           const float *row_scale, int64_t L, int64_t d, int64_t V, float *d_loss, float *d_dh,
+                           float *d_lse, float *d_nll, void *d_ws, size_t ws_bytes, cudaStream_t stream);
+
 // Device address of attt_lora_grad_noalloc's static status word on `dev`, or
 // nullptr if that entry point has not been set up on the device.
 int *noalloc_status_word(int dev);

@@ -179,7 +179,9 @@ struct CeChunkArgs {
     const int32_t *tgt;
     const float *w;
     float inv_L;
+    const float *row_scale;  // per-row normaliser, or nullptr (inv_L)
     float *lse_out;  // or nullptr
+    float *nll_out;  // or nullptr
     float *block_sums;
     unsigned int *ticket;
     float *loss;
@@ -253,7 +255,7 @@ __global__ void __launch_bounds__(kChunkWarps * 32) ce_chunk_kernel(const CeChun
                 const float lse = lse2 * 0.69314718055994531f;
                 if (a.lse_out) a.lse_out[j] = lse;
                 const int t = a.tgt[j];
-                const float c = a.w[j] * a.inv_L;
+                const float c = a.w[j] * (a.row_scale ? a.row_scale[j] : a.inv_L);
                 float nll;
                 if (t < 0 || t >= a.V) {
                     record_error(a.status, ATTT_ERR_TOKEN_RANGE);
@@ -264,6 +266,7 @@ __global__ void __launch_bounds__(kChunkWarps * 32) ce_chunk_kernel(const CeChun
                     a.gamma[j] = c;
                 }
                 contrib = a.w[j] * nll;
+                if (a.nll_out) a.nll_out[j] = nll;
                 const float f = c * exp2f(anew - lse2);
                 al *= f;
                 be *= f;
@@ -329,7 +332,17 @@ size_t attt_ce_workspace_bytes(int64_t L, int64_t d, int64_t V) {
 attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W, const int32_t *d_tgt,
                                      const float *d_w, int64_t L, int64_t d, int64_t V, float *d_loss,
                                      float *d_dh, float *d_lse, void *d_ws, size_t ws_bytes, attt_stream stream) {
-    using namespace attt;
+    return attt::ce_fwd_bwd_run(d_h, d_W, d_tgt, d_w, nullptr, L, d, V, d_loss, d_dh, d_lse, nullptr, d_ws, ws_bytes,
+                                stream);
+}
+
+}  // extern "C"
+
+namespace attt {
+
+attt_status ce_fwd_bwd_run(const attt_bf16 *d_h, const attt_bf16 *d_W, const int32_t *d_tgt, const float *d_w,
+                           const float *row_scale, int64_t L, int64_t d, int64_t V, float *d_loss, float *d_dh,
+                           float *d_lse, float *d_nll, void *d_ws, size_t ws_bytes, cudaStream_t stream) {
     if (!d_h || !d_W || !d_tgt || !d_w || !d_loss || !d_dh) return ATTT_ERR_INVALID_ARG;
     if (L < 1 || V < 1 || d < 8 || d % 8 != 0) return ATTT_ERR_INVALID_ARG;
     if (L > (1ll << 30) || V > (1ll << 30) || d > (1ll << 20)) return ATTT_ERR_UNSUPPORTED;
@@ -378,6 +391,7 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
         ca.alpha = c.alpha; ca.beta = c.beta; ca.gamma = c.gamma;
         ca.first = ci == 0 ? 1 : 0; ca.last = last ? 1 : 0;
         ca.ztgt = c.ztgt; ca.tgt = d_tgt; ca.w = d_w; ca.inv_L = 1.0f / (float)L; ca.lse_out = d_lse;
+        ca.row_scale = row_scale; ca.nll_out = d_nll;
         ca.block_sums = c.block_sums; ca.ticket = c.ticket; ca.loss = d_loss; ca.status = status;
         {
             cudaLaunchConfig_t cfg = {};
@@ -415,4 +429,4 @@ attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W,
     return ATTT_OK;
 }
 
-}  // extern "C"
+}  // namespace attt

@@ -109,11 +109,12 @@ __device__ __forceinline__ bool insert_rest(Slot *table, unsigned long long mask
 constexpr int kInsPer = 1;
 constexpr int kInsTile = 256 * kInsPer;
 
-__global__ void __launch_bounds__(256) history_insert_kernel(const int32_t *__restrict__ hist, int64_t p_begin,
-                                                             int64_t count, int n, Slot *table,
-                                                             unsigned long long mask, int *status) {
+// One block of history_insert_kernel's work: new n-gram starts
+// p = p_begin + blk * kInsTile + threadIdx.x, p - p_begin < count.
+__device__ __forceinline__ void insert_block(const int32_t *__restrict__ hist, int64_t p_begin, int64_t count, int n,
+                                             Slot *table, unsigned long long mask, int *status, int64_t blk) {
     __shared__ int32_t tok[kInsTile + kMaxN];
-    const int64_t i0 = (int64_t)blockIdx.x * kInsTile;
+    const int64_t i0 = blk * kInsTile;
     const int64_t rem = count - i0;
     const int nt = (int)(rem < kInsTile ? rem : kInsTile) + n - 1;  // tokens of this block's n-grams
     for (int t = threadIdx.x; t < nt; t += blockDim.x) tok[t] = hist[p_begin + i0 + t];
@@ -139,6 +140,29 @@ __global__ void __launch_bounds__(256) history_insert_kernel(const int32_t *__re
     }
 }
 
+__global__ void __launch_bounds__(256) history_insert_kernel(const int32_t *__restrict__ hist, int64_t p_begin,
+                                                             int64_t count, int n, Slot *table,
+                                                             unsigned long long mask, int *status) {
+    insert_block(hist, p_begin, count, n, table, mask, status, blockIdx.x);
+}
+
+// The histories of a batch of episodes (one per blockIdx.y).
+constexpr int kMaxBatch = 32;
+struct InsertBatch {
+    const int32_t *hist[kMaxBatch];
+    Slot *table[kMaxBatch];
+    unsigned long long mask[kMaxBatch];
+    int *status[kMaxBatch];
+    int64_t p_begin[kMaxBatch], count[kMaxBatch];
+    int n;
+};
+
+__global__ void __launch_bounds__(256) history_insert_batch_kernel(const __grid_constant__ InsertBatch b) {
+    const int e = blockIdx.y;
+    if ((int64_t)blockIdx.x * kInsTile >= b.count[e]) return;
+    insert_block(b.hist[e], b.p_begin[e], b.count[e], b.n, b.table[e], b.mask[e], b.status[e], blockIdx.x);
+}
+
 // count(g, H) for m query n-grams stored row-major [m, n].
 __global__ void __launch_bounds__(256) history_count_kernel(const int32_t *__restrict__ hist, const Slot *table,
                                                             unsigned long long mask, const int32_t *__restrict__ q,
@@ -154,13 +178,13 @@ constexpr int kWThreads = kWTile + kMaxN;  // one thread per candidate window (a
 
 // Eq. 8 then Eq. 9 for positions [j0, j0 + kWTile) of the update.  Each
 // window has its own thread, so a block's critical path is one lookup.
-__global__ void __launch_bounds__(kWThreads) ngram_weights_kernel(const int32_t *__restrict__ x, int64_t L, int n,
-                                                               const int32_t *__restrict__ hist, int64_t hist_len,
-                                                               const Slot *table, unsigned long long mask,
-                                                               float w_min, float *__restrict__ w) {
+// rowscale (may be null) receives `scale` at every position written.
+__device__ __forceinline__ void weights_block(const int32_t *__restrict__ x, int64_t L, int n,
+                                              const int32_t *__restrict__ hist, int64_t hist_len, const Slot *table,
+                                              unsigned long long mask, float w_min, float *__restrict__ w,
+                                              float *__restrict__ rowscale, float scale, int64_t j0) {
     __shared__ int32_t tok[kWTile + 2 * kMaxN];
     __shared__ unsigned int cnt[kWTile + kMaxN];
-    const int64_t j0 = (int64_t)blockIdx.x * kWTile;
     // Window starts s that cover some j in the tile: s in [j0-n+1, j0+kWTile-1]
     // clipped to [0, L-n].  Tokens needed: x[s0 .. s1+n-1].
     const int64_t s_lo = j0 - (n - 1);
@@ -187,6 +211,38 @@ __global__ void __launch_bounds__(kWThreads) ngram_weights_kernel(const int32_t 
     for (int k = 0; k < n; ++k) f = max(f, cnt[threadIdx.x + k]);
     const float q = __fdiv_rn(1.0f, __fadd_rn(1.0f, __uint2float_rn(f)));
     w[j] = fmaxf(w_min, q);
+    if (rowscale) rowscale[j] = scale;
+}
+
+__global__ void __launch_bounds__(kWThreads) ngram_weights_kernel(const int32_t *__restrict__ x, int64_t L, int n,
+                                                               const int32_t *__restrict__ hist, int64_t hist_len,
+                                                               const Slot *table, unsigned long long mask,
+                                                               float w_min, float *__restrict__ w) {
+    weights_block(x, L, n, hist, hist_len, table, mask, w_min, w, nullptr, 0.0f, (int64_t)blockIdx.x * kWTile);
+}
+
+// The updates of a batch of episodes (one per blockIdx.y), each against its
+// own history; rowscale[j] = 1 / L_e for every row of episode e.
+struct WeightsBatch {
+    const int32_t *x[kMaxBatch];
+    int64_t L[kMaxBatch];
+    const int32_t *hist[kMaxBatch];
+    int64_t hist_len[kMaxBatch];
+    const Slot *table[kMaxBatch];
+    unsigned long long mask[kMaxBatch];
+    float *w[kMaxBatch];
+    float *rowscale[kMaxBatch];
+    float inv_L[kMaxBatch];
+    int n;
+    float w_min;
+};
+
+__global__ void __launch_bounds__(kWThreads) ngram_weights_batch_kernel(const __grid_constant__ WeightsBatch b) {
+    const int e = blockIdx.y;
+    const int64_t j0 = (int64_t)blockIdx.x * kWTile;
+    if (j0 >= b.L[e]) return;
+    weights_block(b.x[e], b.L[e], b.n, b.hist[e], b.hist_len[e], b.table[e], b.mask[e], b.w_min, b.w[e],
+                  b.rowscale[e], b.inv_L[e], j0);
 }
 
 }  // namespace attt
@@ -314,6 +370,84 @@ attt_status attt_history_count(const attt_history *h, const int32_t *d_ngrams, i
     attt::count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
+
+}  // extern "C"
+
+namespace attt {
+
+// Eq. 8 / Eq. 9 weights of E updates (rows [off[e], off[e+1]) of d_tokens,
+// against history hs[e]) in one launch; rowscale[j] = 1/L_e (fp32 round to
+// nearest of 1.0f / L_e) for every row of episode e.
+attt_status ngram_weights_batch(attt_history *const *hs, int E, const int32_t *d_tokens, const int64_t *off,
+                                float w_min, float *d_w, float *d_rowscale, cudaStream_t stream) {
+    if (E < 1 || E > kMaxBatch || !(w_min > 0.0f) || !(w_min <= 1.0f)) return ATTT_ERR_INVALID_ARG;
+    WeightsBatch b{};
+    b.n = hs[0]->n;
+    b.w_min = w_min;
+    int64_t maxL = 0;
+    for (int e = 0; e < E; ++e) {
+        const attt_history *h = hs[e];
+        if (h->n != b.n) return ATTT_ERR_INVALID_ARG;
+        const int64_t L = off[e + 1] - off[e];
+        b.x[e] = d_tokens + off[e];
+        b.L[e] = L;
+        b.hist[e] = h->d_tokens;
+        b.hist_len[e] = h->len;
+        b.table[e] = h->d_table;
+        b.mask[e] = h->capacity - 1;
+        b.w[e] = d_w + off[e];
+        b.rowscale[e] = d_rowscale ? d_rowscale + off[e] : nullptr;
+        b.inv_L[e] = L > 0 ? 1.0f / (float)L : 0.0f;
+        if (L > maxL) maxL = L;
+    }
+    if (maxL == 0) return ATTT_OK;
+    ngram_weights_batch_kernel<<<dim3((unsigned)cdiv(maxL, kWTile), (unsigned)E), kWThreads, 0, stream>>>(b);
+    count_launch();
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+// Algorithm 1's append for E histories (rows [off[e], off[e+1]) of d_tokens
+// to hs[e]): one copy per history, then one insert launch for all.
+attt_status history_insert_batch(attt_history *const *hs, int E, const int32_t *d_tokens, const int64_t *off,
+                                 cudaStream_t stream) {
+    if (E < 1 || E > kMaxBatch) return ATTT_ERR_INVALID_ARG;
+    for (int e = 0; e < E; ++e)
+        if (hs[e]->len + (off[e + 1] - off[e]) > hs[e]->max_tokens) return ATTT_ERR_CAPACITY;
+    InsertBatch b{};
+    b.n = hs[0]->n;
+    int64_t maxc = 0;
+    for (int e = 0; e < E; ++e) {
+        attt_history *h = hs[e];
+        const int64_t len = off[e + 1] - off[e];
+        b.hist[e] = h->d_tokens;
+        b.table[e] = h->d_table;
+        b.mask[e] = h->capacity - 1;
+        b.status[e] = h->d_status;
+        b.count[e] = 0;
+        if (len == 0) continue;
+        if (cudaMemcpyAsync(h->d_tokens + h->len, d_tokens + off[e], (size_t)len * sizeof(int32_t),
+                            cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
+            return ATTT_ERR_CUDA;
+        const int64_t new_len = h->len + len;
+        int64_t p_begin = h->len - (h->n - 1);
+        if (p_begin < 0) p_begin = 0;
+        const int64_t p_end = new_len - h->n;
+        h->len = new_len;
+        if (p_end >= p_begin) {
+            b.p_begin[e] = p_begin;
+            b.count[e] = p_end - p_begin + 1;
+            if (b.count[e] > maxc) maxc = b.count[e];
+        }
+    }
+    if (maxc == 0) return ATTT_OK;
+    history_insert_batch_kernel<<<dim3((unsigned)cdiv(maxc, kInsTile), (unsigned)E), 256, 0, stream>>>(b);
+    count_launch();
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+}  // namespace attt
+
+extern "C" {
 
 attt_status attt_ngram_weights(const attt_history *h, const int32_t *d_tokens, int64_t L, float w_min, float *d_w,
                                attt_stream stream) {
