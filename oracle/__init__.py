@@ -252,7 +252,7 @@ def to_bf16(p32) -> np.ndarray:
 # --------------------------------------------------------------------------
 
 def episode_update(H, tokens, x_bf16, W0_bf16, Wlm_bf16, A32, B32, *, n: int, w_min: float, scale: float,
-                   lr: float, grad_steps: int = 2, want_dx: bool = True):
+                   lr: float, grad_steps: int = 2, want_dx: bool = True, adamw=None):
     """Algorithm 1 for update x_k (= `tokens`, also the Eq. 10 targets) with
     the adapter on the projection whose output is the LM head's input:
 
@@ -266,7 +266,11 @@ def episode_update(H, tokens, x_bf16, W0_bf16, Wlm_bf16, A32, B32, *, n: int, w_
       H <- H || x_k
 
     Returns a dict with w, losses [grad_steps], dx (list, or None), A32, B32
-    (fp32 after the update) and H (the new history)."""
+    (fp32 after the update) and H (the new history).
+
+    adamw: None for the paper's SGD, else a dict {"t", "mA", "vA", "mB", "vB",
+    "beta1", "beta2", "eps", "weight_decay"} of AdamW's state and settings,
+    advanced in place (t counts the steps taken so far)."""
     w = ngram_weights(H, tokens, n, w_min)
     A = np.array(A32, dtype=np.float32, copy=True)
     B = np.array(B32, dtype=np.float32, copy=True)
@@ -279,8 +283,16 @@ def episode_update(H, tokens, x_bf16, W0_bf16, Wlm_bf16, A32, B32, *, n: int, w_
         dA, dB = lora_grad(x_bf16, dy, A16, B16, scale)
         if want_dx:
             dxs.append(lora_input_grad(dy, W0_bf16, A16, B16, scale))
-        A, A16 = sgd_step(A, dA.astype(np.float32), lr)
-        B, B16 = sgd_step(B, dB.astype(np.float32), lr)
+        if adamw is None:
+            A, A16 = sgd_step(A, dA.astype(np.float32), lr)
+            B, B16 = sgd_step(B, dB.astype(np.float32), lr)
+        else:
+            o = adamw
+            o["t"] += 1
+            kw = dict(beta1=o["beta1"], beta2=o["beta2"], eps=o["eps"], weight_decay=o["weight_decay"])
+            A, o["mA"], o["vA"] = adamw_step(A, dA.astype(np.float32), o["mA"], o["vA"], o["t"], lr, **kw)
+            B, o["mB"], o["vB"] = adamw_step(B, dB.astype(np.float32), o["mB"], o["vB"], o["t"], lr, **kw)
+            A16, B16 = to_bf16(A), to_bf16(B)
         losses.append(loss)
     H = np.concatenate([np.asarray(H, dtype=np.int32), np.asarray(tokens, dtype=np.int32)])
     return {"w": w, "losses": np.array(losses), "dx": dxs if want_dx else None, "A32": A, "B32": B, "H": H}
@@ -344,3 +356,27 @@ def kl_rows(hp_bf16, hq_bf16, W_bf16, rows=None):
     out = np.zeros(rows.size, dtype=np.float64)
     _load().oracle_kl_rows(php, phq, pW, d, W.shape[0], pr, rows.size, out.ctypes.data_as(ctypes.c_void_p))
     return out
+
+
+# --------------------------------------------------------------------------
+# AdamW (an optional optimizer for the update; the paper's is SGD, Eq. 2)
+# --------------------------------------------------------------------------
+
+def adamw_step(p32, g32, m, v, t: int, lr: float, beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8,
+               weight_decay: float = 0.01):
+    """One AdamW step (Adam with decoupled weight decay, Loshchilov and
+    Hutter), in fp64 on fp32 inputs: step t (1-based),
+      p <- p (1 - lr wd);  m <- b1 m + (1 - b1) g;  v <- b2 v + (1 - b2) g^2
+      p <- p - (lr / (1 - b1^t)) m / (sqrt(v) / sqrt(1 - b2^t) + eps)
+    Returns (p as fp32, m, v) with m, v in fp64."""
+    p = np.asarray(p32, dtype=np.float32).astype(np.float64)
+    g = np.asarray(g32, dtype=np.float32).astype(np.float64)
+    m = np.asarray(m, dtype=np.float64)
+    v = np.asarray(v, dtype=np.float64)
+    p = p * (1.0 - lr * weight_decay)
+    m = beta1 * m + (1.0 - beta1) * g
+    v = beta2 * v + (1.0 - beta2) * g * g
+    step_size = lr / (1.0 - beta1 ** t)
+    denom = np.sqrt(v) / np.sqrt(1.0 - beta2 ** t) + eps
+    p = p - step_size * m / denom
+    return p.astype(np.float32), m, v
