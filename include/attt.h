@@ -259,6 +259,24 @@ ATTT_API attt_status attt_lora_step(float *d_A32, float *d_B32, const float *d_d
                            int64_t din, int64_t dout, int r, float lr,
                            attt_bf16 *d_A16, attt_bf16 *d_B16, attt_stream stream);
 
+/*
+ * AdamW (Adam with decoupled weight decay) as an alternative to the paper's
+ * SGD step, on the same adapter layout, with the first and second moments
+ * d_mA, d_vA ([din, r]) and d_mB, d_vB ([r, dout]) (fp32, caller-owned,
+ * zero before the first step) and `step` = 1 for the first step:
+ *   p <- p (1 - lr wd);  m <- b1 m + (1 - b1) g;  v <- b2 v + (1 - b2) g^2
+ *   p <- p - (lr / (1 - b1^step)) m / (sqrt(v) / sqrt(1 - b2^step) + eps)
+ * fp32, every operation rounded on its own, the scalars (1 - lr wd, b1,
+ * 1 - b1, b2, 1 - b2, lr / (1 - b1^step), sqrt(1 - b2^step), eps) formed in
+ * double from the double settings and rounded once; the bf16 copies are
+ * refreshed when not NULL.  0 <= b1, b2 < 1, eps > 0, wd >= 0, step >= 1.
+ */
+ATTT_API attt_status attt_lora_adamw_step(float *d_A32, float *d_B32, const float *d_dA, const float *d_dB,
+                                          float *d_mA, float *d_vA, float *d_mB, float *d_vB, int64_t din,
+                                          int64_t dout, int r, float lr, double beta1, double beta2, double eps,
+                                          double weight_decay, int step, attt_bf16 *d_A16, attt_bf16 *d_B16,
+                                          attt_stream stream);
+
 /* ------------------------------------------------------------------------ */
 /* The adapted projection of a chained update: the LoRA-adapted linear map   */
 /* y = x W0 + s (x A) B (Appendix C adapter; W0 frozen) whose output is the  */
@@ -398,6 +416,8 @@ typedef struct attt_episode_config {
     float lr;            /* SGD learning rate of Eq. 2                          */
     int grad_steps;      /* gradient steps per update (Appendix C: 2), 1..64    */
     int cadence;         /* K: agent steps per update (Sec. 4 default 5), >= 1  */
+    int optimizer;       /* 0: SGD (Eq. 2, the paper's); 1: AdamW               */
+    double beta1, beta2, eps, weight_decay; /* AdamW settings (optimizer 1)     */
 } attt_episode_config;
 
 /*
@@ -418,7 +438,8 @@ ATTT_API attt_status attt_episode_destroy(attt_episode *e);
 
 /*
  * The episode boundary: the adapter returns to (A0, B0), the history is
- * emptied and pending agent-step text is dropped.  Async on `stream`.
+ * emptied, pending agent-step text is dropped and AdamW's moments and step
+ * count (optimizer 1) return to zero.  Async on `stream`.
  */
 ATTT_API attt_status attt_episode_reset(attt_episode *e, attt_stream stream);
 

@@ -48,7 +48,9 @@ class EpisodeConfig(ctypes.Structure):
     _fields_ = [("n", ctypes.c_int), ("w_min", ctypes.c_float), ("max_history", ctypes.c_int64),
                 ("max_update", ctypes.c_int64), ("din", ctypes.c_int64), ("d", ctypes.c_int64),
                 ("V", ctypes.c_int64), ("r", ctypes.c_int), ("scale", ctypes.c_float), ("lr", ctypes.c_float),
-                ("grad_steps", ctypes.c_int), ("cadence", ctypes.c_int)]
+                ("grad_steps", ctypes.c_int), ("cadence", ctypes.c_int), ("optimizer", ctypes.c_int),
+                ("beta1", ctypes.c_double), ("beta2", ctypes.c_double), ("eps", ctypes.c_double),
+                ("weight_decay", ctypes.c_double)]
 
 
 class BatchConfig(ctypes.Structure):
@@ -70,6 +72,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             raise RuntimeError(f"libattt.so not found at {p}; run paper_2607_03441_gb300.build.build()")
         lib = ctypes.CDLL(p)
         P, i64, i32, f32, sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+        f64 = ctypes.c_double
         sig = {
             "attt_status_string": (ctypes.c_char_p, [i32]),
             "attt_abi_version": (i32, []),
@@ -95,6 +98,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_lora_forward": (i32, [P, P, P, P, i64, i64, i64, i32, f32, P, P, sz, P]),
             "attt_lora_input_grad": (i32, [P, P, P, P, i64, i64, i64, i32, f32, P, P, sz, P]),
             "attt_cast_bf16": (i32, [P, P, i64, P]),
+            "attt_lora_adamw_step": (i32, [P, P, P, P, P, P, P, P, i64, i64, i32, f32, f64, f64, f64, f64, i32, P,
+                                           P, P]),
             "attt_episode_create": (i32, [ctypes.POINTER(EpisodeConfig), P, P, P, P, ctypes.POINTER(P)]),
             "attt_episode_destroy": (i32, [P]),
             "attt_episode_reset": (i32, [P, P]),
@@ -440,7 +445,8 @@ class Episode:
 
     def __init__(self, W0: torch.Tensor, Wlm: torch.Tensor, A0: torch.Tensor, B0: torch.Tensor, *, n: int,
                  max_history: int, max_update: int, scale: float, lr: float, w_min: float = 0.05,
-                 grad_steps: int = 2, cadence: int = 5):
+                 grad_steps: int = 2, cadence: int = 5, optimizer: str = "sgd", betas=(0.9, 0.999),
+                 eps: float = 1e-8, weight_decay: float = 0.01):
         self._lib = load_library()
         din, d = W0.shape
         V = Wlm.shape[0]
@@ -452,7 +458,9 @@ class Episode:
         self.cfg = EpisodeConfig(n=int(n), w_min=float(w_min), max_history=int(max_history),
                                  max_update=int(max_update), din=int(din), d=int(d), V=int(V), r=int(r),
                                  scale=float(scale), lr=float(lr), grad_steps=int(grad_steps),
-                                 cadence=int(cadence))
+                                 cadence=int(cadence), optimizer={"sgd": 0, "adamw": 1}[optimizer],
+                                 beta1=float(betas[0]), beta2=float(betas[1]), eps=float(eps),
+                                 weight_decay=float(weight_decay))
         e = ctypes.c_void_p()
         _check(self._lib.attt_episode_create(ctypes.byref(self.cfg), _bf16(W0), _bf16(Wlm), _ptr(A0), _ptr(B0),
                                              ctypes.byref(e)), "attt_episode_create")
@@ -706,3 +714,17 @@ class Batch:
     def history(self, e: int) -> History:
         h = self._lib.attt_batch_history(self.handle, int(e))
         return History._view(h, self.cfg.n, self.cfg.max_history, self)
+
+
+def attt_lora_adamw_step(A32: torch.Tensor, B32: torch.Tensor, dA: torch.Tensor, dB: torch.Tensor,
+                         mA: torch.Tensor, vA: torch.Tensor, mB: torch.Tensor, vB: torch.Tensor, lr: float, step: int,
+                         betas=(0.9, 0.999), eps: float = 1e-8, weight_decay: float = 0.01,
+                         A16: Optional[torch.Tensor] = None, B16: Optional[torch.Tensor] = None, stream=None) -> None:
+    """In-place AdamW step on the fp32 masters (moments mA, vA, mB, vB), bf16 refresh."""
+    din, r = A32.shape
+    dout = B32.shape[1]
+    _check(load_library().attt_lora_adamw_step(
+        _ptr(A32), _ptr(B32), _ptr(dA), _ptr(dB), _ptr(mA), _ptr(vA), _ptr(mB), _ptr(vB), din, dout, r, float(lr),
+        float(betas[0]), float(betas[1]), float(eps), float(weight_decay), int(step),
+        _bf16(A16) if A16 is not None else None, _bf16(B16) if B16 is not None else None, _stream(stream)),
+        "attt_lora_adamw_step")

@@ -12,6 +12,7 @@
 //     dA, dB = adapter gradients of h                 attt_lora_grad
 //     dx = dy W0^T + s (dy B^T) A^T  (if requested)   attt_lora_input_grad
 //     A, B <- A - lr dA, B - lr dB                    attt_lora_step
+//       (or AdamW, optimizer 1)                       attt_lora_adamw_step
 //   H_{k+1} = H_k || x_k                              attt_history_insert
 //
 // Everything is host code that issues the library's own calls; the episode
@@ -33,6 +34,8 @@ struct attt_episode {
     attt_history *hist;
     // adapter: fp32 masters, bf16 copies, initial values, gradients
     float *A32, *B32, *A0, *B0, *dA, *dB;
+    float *mA, *vA, *mB, *vB;  // AdamW moments (optimizer 1)
+    int adam_t;                // AdamW steps taken
     attt_bf16 *A16, *B16;
     // per-update activations
     float *w, *dh, *losses;
@@ -58,7 +61,7 @@ bool dev_alloc(T **p, size_t count) {
 
 void free_all(attt_episode *e) {
     if (e->hist) attt_history_destroy(e->hist);
-    void *bufs[] = {e->A32, e->B32, e->A0, e->B0, e->dA, e->dB, e->A16, e->B16, e->w,
+    void *bufs[] = {e->A32, e->B32, e->A0, e->B0, e->dA, e->dB, e->mA, e->vA, e->mB, e->vB, e->A16, e->B16, e->w,
                     e->dh,  e->losses, e->h, e->dy, e->h_base, e->pend_tok, e->pend_x, e->ws};
     for (void *b : bufs) cudaFree(b);
 }
@@ -68,7 +71,9 @@ bool config_ok(const attt_episode_config *c) {
            c->max_history <= 16777214 && c->max_update >= 1 && c->max_update <= c->max_history &&
            c->din >= 8 && c->din % 8 == 0 && c->d >= 8 && c->d % 8 == 0 && c->V >= 1 && c->r >= 1 && c->r <= 64 &&
            std::isfinite(c->scale) && std::isfinite(c->lr) && c->grad_steps >= 1 && c->grad_steps <= 64 &&
-           c->cadence >= 1;
+           c->cadence >= 1 &&
+           (c->optimizer == 0 || (c->optimizer == 1 && c->beta1 >= 0.0 && c->beta1 < 1.0 && c->beta2 >= 0.0 &&
+                                  c->beta2 < 1.0 && c->eps > 0.0 && c->weight_decay >= 0.0));
 }
 
 // Workspace that every call of an update of up to max_update tokens fits in.
@@ -91,6 +96,14 @@ attt_status load_adapter(attt_episode *e, cudaStream_t s) {
     if (cudaMemcpyAsync(e->A32, e->A0, nA * sizeof(float), cudaMemcpyDeviceToDevice, s) != cudaSuccess ||
         cudaMemcpyAsync(e->B32, e->B0, nB * sizeof(float), cudaMemcpyDeviceToDevice, s) != cudaSuccess)
         return ATTT_ERR_CUDA;
+    if (e->cfg.optimizer == 1) {
+        e->adam_t = 0;
+        if (cudaMemsetAsync(e->mA, 0, nA * sizeof(float), s) != cudaSuccess ||
+            cudaMemsetAsync(e->vA, 0, nA * sizeof(float), s) != cudaSuccess ||
+            cudaMemsetAsync(e->mB, 0, nB * sizeof(float), s) != cudaSuccess ||
+            cudaMemsetAsync(e->vB, 0, nB * sizeof(float), s) != cudaSuccess)
+            return ATTT_ERR_CUDA;
+    }
     attt_status st = attt_cast_bf16(e->A32, e->A16, (int64_t)nA, s);
     if (st != ATTT_OK) return st;
     return attt_cast_bf16(e->B32, e->B16, (int64_t)nB, s);
@@ -127,6 +140,8 @@ attt_status attt_episode_create(const attt_episode_config *cfg, const attt_bf16 
          dev_alloc(&e->pend_tok, (size_t)c.max_update) &&
          dev_alloc(&e->pend_x, (size_t)c.max_update * c.din) &&
          dev_alloc(reinterpret_cast<char **>(&e->ws), e->ws_bytes);
+    if (ok && c.optimizer == 1)
+        ok = dev_alloc(&e->mA, nA) && dev_alloc(&e->vA, nA) && dev_alloc(&e->mB, nB) && dev_alloc(&e->vB, nB);
     if (ok) {
         // The initial adapter is copied once; later resets restore it.
         ok = cudaMemcpy(e->A0, d_A0, nA * sizeof(float), cudaMemcpyDeviceToDevice) == cudaSuccess &&
@@ -187,7 +202,16 @@ attt_status attt_episode_update(attt_episode *e, const int32_t *d_tokens, const 
         if (st == ATTT_OK && d_dx)
             st = attt_lora_input_grad(e->dy, e->W0, e->A16, e->B16, L, c.din, c.d, c.r, c.scale,
                                       d_dx + (size_t)g * L * c.din, e->ws, e->ws_bytes, stream);
-        if (st == ATTT_OK) st = attt_lora_step(e->A32, e->B32, e->dA, e->dB, c.din, c.d, c.r, c.lr, e->A16, e->B16, stream);
+        if (st == ATTT_OK) {
+            if (c.optimizer == 0) {
+                st = attt_lora_step(e->A32, e->B32, e->dA, e->dB, c.din, c.d, c.r, c.lr, e->A16, e->B16, stream);
+            } else {
+                st = attt_lora_adamw_step(e->A32, e->B32, e->dA, e->dB, e->mA, e->vA, e->mB, e->vB, c.din, c.d, c.r,
+                                          c.lr, c.beta1, c.beta2, c.eps, c.weight_decay, e->adam_t + 1, e->A16,
+                                          e->B16, stream);
+                if (st == ATTT_OK) ++e->adam_t;
+            }
+        }
     }
     if (st == ATTT_OK) st = attt_history_insert(e->hist, d_tokens, L, stream);
     return st;

@@ -20,6 +20,8 @@
 // dx = dy W0^T + s (dy B^T) A^T.  Each is one tcgen05 contraction whose K runs
 // over two operand pairs, [x | s u] [W0 ; B] and [dy | s v] [W0^T ; A^T], after
 // a skinny grouped launch that forms s u = s x A or s v = s dy B^T in bf16.
+#include <cmath>
+
 #include "gemm_launch.cuh"
 #include "tc_group.cuh"
 
@@ -127,6 +129,39 @@ __global__ void lora_step_kernel(float *A32, const float *dA, __nv_bfloat16 *A16
             B32[k] = v;
             if (B16) B16[k] = __float2bfloat16_rn(v);
         }
+    }
+}
+
+// AdamW (decoupled weight decay) on the fp32 masters of A and B, with the
+// moments m, v (fp32) and the bf16 refresh; every product and sum rounded on
+// its own (no FMA):
+//   p <- p (1 - lr wd);  m <- b1 m + (1 - b1) g;  v <- b2 v + (1 - b2) g^2
+//   p <- p - step_size m / (sqrt(v) / bc2_sqrt + eps)
+// with step_size = lr / (1 - b1^t) and bc2_sqrt = sqrt(1 - b2^t) from the host.
+struct AdamWArgs {
+    float *p[2];
+    const float *g[2];
+    float *m[2], *v[2];
+    __nv_bfloat16 *p16[2];
+    int64_t n[2];
+    float decay, b1, one_b1, b2, one_b2, step_size, bc2_sqrt, eps;
+};
+
+__global__ void lora_adamw_kernel(const AdamWArgs a) {
+    const int64_t total = a.n[0] + a.n[1];
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int t = i < a.n[0] ? 0 : 1;
+        const int64_t k = t == 0 ? i : i - a.n[0];
+        const float g = a.g[t][k];
+        const float m = __fadd_rn(__fmul_rn(a.b1, a.m[t][k]), __fmul_rn(a.one_b1, g));
+        const float v = __fadd_rn(__fmul_rn(a.b2, a.v[t][k]), __fmul_rn(a.one_b2, __fmul_rn(g, g)));
+        a.m[t][k] = m;
+        a.v[t][k] = v;
+        const float denom = __fadd_rn(__fdiv_rn(__fsqrt_rn(v), a.bc2_sqrt), a.eps);
+        const float p = __fsub_rn(__fmul_rn(a.p[t][k], a.decay), __fdiv_rn(__fmul_rn(a.step_size, m), denom));
+        a.p[t][k] = p;
+        if (a.p16[t]) a.p16[t][k] = __float2bfloat16_rn(p);
     }
 }
 
@@ -538,6 +573,39 @@ attt_status attt_lora_step(float *d_A32, float *d_B32, const float *d_dA, const 
     lora_step_kernel<<<grid_for(nA + nB, 256, dev), 256, 0, stream>>>(
         d_A32, d_dA, reinterpret_cast<__nv_bfloat16 *>(d_A16), nA, d_B32, d_dB,
         reinterpret_cast<__nv_bfloat16 *>(d_B16), nB, lr);
+    count_launch();
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+attt_status attt_lora_adamw_step(float *d_A32, float *d_B32, const float *d_dA, const float *d_dB, float *d_mA,
+                                 float *d_vA, float *d_mB, float *d_vB, int64_t din, int64_t dout, int r, float lr,
+                                 double beta1, double beta2, double eps, double weight_decay, int step,
+                                 attt_bf16 *d_A16, attt_bf16 *d_B16, attt_stream stream) {
+    using namespace attt;
+    if (!d_A32 || !d_B32 || !d_dA || !d_dB || !d_mA || !d_vA || !d_mB || !d_vB) return ATTT_ERR_INVALID_ARG;
+    if (din < 1 || dout < 1 || r < 1 || step < 1 || !(beta1 >= 0.0 && beta1 < 1.0) || !(beta2 >= 0.0 && beta2 < 1.0) ||
+        !(eps > 0.0) || !(weight_decay >= 0.0) || !(lr == lr))
+        return ATTT_ERR_INVALID_ARG;
+    int dev;
+    attt_status st = current_device(&dev);
+    if (st != ATTT_OK) return st;
+    AdamWArgs a{};
+    a.p[0] = d_A32; a.p[1] = d_B32;
+    a.g[0] = d_dA; a.g[1] = d_dB;
+    a.m[0] = d_mA; a.m[1] = d_mB;
+    a.v[0] = d_vA; a.v[1] = d_vB;
+    a.p16[0] = reinterpret_cast<__nv_bfloat16 *>(d_A16);
+    a.p16[1] = reinterpret_cast<__nv_bfloat16 *>(d_B16);
+    a.n[0] = din * r;
+    a.n[1] = (int64_t)r * dout;
+    // the step's scalars in double, rounded once to fp32
+    a.decay = (float)(1.0 - (double)lr * weight_decay);
+    a.b1 = (float)beta1; a.one_b1 = (float)(1.0 - beta1);
+    a.b2 = (float)beta2; a.one_b2 = (float)(1.0 - beta2);
+    a.step_size = (float)((double)lr / (1.0 - std::pow(beta1, (double)step)));
+    a.bc2_sqrt = (float)std::sqrt(1.0 - std::pow(beta2, (double)step));
+    a.eps = (float)eps;
+    lora_adamw_kernel<<<grid_for(a.n[0] + a.n[1], 256, dev), 256, 0, stream>>>(a);
     count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
