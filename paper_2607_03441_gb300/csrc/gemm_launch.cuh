@@ -60,9 +60,9 @@ inline int tail_pieces(int tiles, int units, int kb_total, int nranks, int regio
 
 constexpr size_t kMaxSmem = 232448;  // 227 KB opt-in per CTA on sm_100-class parts
 
-inline int gemm_stages(int BN, uint32_t extra = 0, int a_tiles = 1) {
+inline int gemm_stages(int BN, uint32_t extra = 0) {
     int s = 8;
-    while (s > 2 && gemm_smem_bytes(BN, s, extra, a_tiles) > kMaxSmem) --s;
+    while (s > 2 && gemm_smem_bytes(BN, s, extra) > kMaxSmem) --s;
     return s;
 }
 
@@ -85,8 +85,10 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     // K-major operand: storage [rows, K] (K contiguous), box 64 x rows_tile.
     // MN-major operand: storage [K, rows] (rows contiguous), box 64 x 64.
     bool ok;
+    // EPI_KL loads 64 rows of A and 64 of A2 into one 128-row tile
+    const uint32_t a_box_rows = EPI == EPI_KL ? 64u : 128u;
     if (!A_MN)
-        ok = make_tmap_bf16(&ta, p.a, (uint64_t)p.a_k, (uint64_t)p.a_rows, (uint64_t)p.a_rows_ld * 2, 64, 128);
+        ok = make_tmap_bf16(&ta, p.a, (uint64_t)p.a_k, (uint64_t)p.a_rows, (uint64_t)p.a_rows_ld * 2, 64, a_box_rows);
     else
         ok = make_tmap_bf16(&ta, p.a, (uint64_t)p.a_rows, (uint64_t)p.a_k, (uint64_t)p.a_rows_ld * 2, 64, 64);
     if (!ok) return ATTT_ERR_INVALID_ARG;
@@ -100,7 +102,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     if (EPI == EPI_KL) {
         // the second A operand (same shape as A) shares every B tile
         if (!p.a2 || !p.pair || A_MN || B_MN) return ATTT_ERR_INVALID_ARG;
-        if (!make_tmap_bf16(&ta2, p.a2, (uint64_t)p.a_k, (uint64_t)p.a_rows, (uint64_t)p.a2_rows_ld * 2, 64, 128))
+        if (!make_tmap_bf16(&ta2, p.a2, (uint64_t)p.a_k, (uint64_t)p.a_rows, (uint64_t)p.a2_rows_ld * 2, 64, 64))
             return ATTT_ERR_INVALID_ARG;
     } else if (p.K2 > 0) {
         if (!p.a2 || !p.b2) return ATTT_ERR_INVALID_ARG;
@@ -135,10 +137,14 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.N = p.N;
     g.BN = p.BN;
     const int bn_cta = p.pair ? p.BN / 2 : p.BN;  // B rows one CTA stages
-    g.e_stage_bytes = (EPI == EPI_CE_EXP || EPI == EPI_BF16) ? kEStageBytes : EPI == EPI_F32_ACC ? kF32StageBytes : 0u;
-    const int a_tiles = EPI == EPI_KL ? 2 : 1;
-    g.stages = gemm_stages(bn_cta, g.e_stage_bytes, a_tiles);
-    g.tiles_m = (int)cdiv(p.M, 128);
+    g.e_stage_bytes = (EPI == EPI_CE_EXP || EPI == EPI_BF16) ? kEStageBytes
+                      : EPI == EPI_F32_ACC                   ? kF32StageBytes
+                      : EPI == EPI_KL                        ? kKlXBytes
+                                                             : 0u;
+    g.stages = gemm_stages(bn_cta, g.e_stage_bytes);
+    // tiles_m counts tiles of 128 accumulator rows; an EPI_KL tile holds 64
+    // rows of the problem (the other 64 are A2's)
+    g.tiles_m = (int)cdiv(p.M, EPI == EPI_KL ? 64 : 128);
     g.tiles_n = (int)cdiv(p.N, p.BN);
     g.kb_split = (int)cdiv(p.K, 64);
     g.kb_total = g.kb_split + (p.K2 > 0 ? (int)cdiv(p.K2, 64) : 0);
@@ -162,12 +168,12 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     g.a_k_off = p.a_k_off;
     g.b_n_off = p.b_n_off;
     g.b_k_off = p.b_k_off;
-    g.tmem_cols = gemm_tmem_cols(p.BN * a_tiles);
+    g.tmem_cols = gemm_tmem_cols(p.BN);
     g.operands_ready = p.operands_ready ? 1 : 0;
     g.status = status ? status : device_status_word(dev);
     g.ep = ep;
 
-    const size_t smem = gemm_smem_bytes(bn_cta, g.stages, g.e_stage_bytes, a_tiles);
+    const size_t smem = gemm_smem_bytes(bn_cta, g.stages, g.e_stage_bytes);
     const int ntiles = g.whole_tiles + (tiles - g.whole_tiles) * g.tail_s;  // work items
     cudaLaunchConfig_t cfg = {};
     cfg.blockDim = dim3(kGemmThreads);

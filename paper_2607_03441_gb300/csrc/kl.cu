@@ -3,10 +3,11 @@
 // p_j = softmax(h_p[j] W^T) from the base model's q_j = softmax(h_q[j] W^T),
 // through the frozen LM head, without the [L, V] logits in HBM.
 //
-// One contraction over the whole vocabulary with two A operands: each W tile
-// staged in shared memory feeds two tcgen05 MMAs, z_p = h_p W^T and
-// z_q = h_q W^T, into two TMEM accumulators (4 L V d FLOPs: each logit once).
-// The epilogue reduces each (row, 128-column tile) to five fp32 numbers: the
+// One contraction over the whole vocabulary: each CTA's 128-row A tile is 64
+// rows of h_p over the same 64 rows of h_q, so one tcgen05 MMA per K step
+// gives both z_p = h_p W^T and z_q = h_q W^T for those rows (4 L V d FLOPs:
+// each logit once).  The epilogue reduces each (row, 256-column tile) to five
+// fp32 numbers: the
 // maxima m_p, m_q (log2 units), s_p = sum exp2(z_p log2e - m_p), s_q alike,
 // and the cross term x = sum exp2(z_p log2e - m_p) (z_p - z_q).  The reduce
 // kernel merges the tiles of a row like an online logsumexp (rescaling s_p and
@@ -18,7 +19,7 @@
 
 namespace attt {
 
-constexpr int kKlBN = 128;  // two accumulators of 256 x 128 per tile, double-buffered: 512 TMEM columns
+constexpr int kKlBN = 256;  // 256-column tiles (the accumulator double-buffered: 512 TMEM columns)
 constexpr int kKlRows = 32;
 constexpr int kKlWarps = 8;
 

@@ -32,7 +32,7 @@ enum EpiKind : int {
     EPI_CE_EXP = 0,    // per (row, vocab tile): max m, E = exp(z - m) as bf16, sum of E, target logit
     EPI_F32_ACC = 2,   // out[m, n] = (acc ? alpha_m out[m, n] : 0) + beta_m acc [- gamma_m W[t_m, n]]  (fp32)
     EPI_BF16 = 5,      // out16[m, n] = bf16(alpha * acc)  (row-major, through TMA boxes)
-    EPI_KL = 6,        // two accumulators z = A B^T, z2 = A2 B^T: per (row, tile) max, sum of exp, cross term
+    EPI_KL = 6,        // A tile = 64 rows of A over the same 64 rows of A2: per (row, tile) max, sum of exp, cross term
 };
 
 constexpr int kMaxProj = 8;
@@ -97,10 +97,13 @@ __host__ __device__ inline uint32_t gemm_b_stage_bytes(int BN) { return (uint32_
 // 32 rows x 32 bf16 (64-byte swizzle), written out by TMA stores.
 constexpr uint32_t kEStageBytes = 4 * 2 * 32 * 64;
 
-// a_tiles: A tiles per stage (2 for EPI_KL, whose two accumulators share B).
-__host__ __device__ inline size_t gemm_smem_bytes(int BN, int stages, uint32_t extra = 0, int a_tiles = 1) {
-    return 1024 + (size_t)stages * (a_tiles * kABytes + gemm_b_stage_bytes(BN)) + extra + 8 * (2 * stages + 5) + 16;
+__host__ __device__ inline size_t gemm_smem_bytes(int BN, int stages, uint32_t extra = 0) {
+    return 1024 + (size_t)stages * (kABytes + gemm_b_stage_bytes(BN)) + extra + 8 * (2 * stages + 5) + 16;
 }
+
+// EPI_KL hands z_q from the warps holding it to the warps holding z_p through
+// shared memory: per warp pair two buffers of 32 columns x 32 rows fp32.
+constexpr uint32_t kKlXBytes = 2 * 2 * 32 * 32 * 4;
 
 // One 32 x 32 bf16 block of E (this warp's 32 rows, 32 columns from x) to
 // global memory through the warp's staging buffer `chunk & 1`: lane = row,
@@ -421,52 +424,67 @@ __device__ __forceinline__ void epilogue_tile(const GemmArgs &g, int gm_base, in
     }
 }
 
-// EPI_KL, one accumulator row per thread: z_p = h_p W^T at taddr and z_q =
-// h_q W^T at taddr + BN.  Over the tile's columns: the maxima m_p, m_q and the
-// sums s = sum exp2(z log2e - m) (log2 units), and the cross term
-// x = sum exp2(z_p log2e - m_p) (z_p - z_q) (nats), all in fp32 from the fp32
-// accumulators.  TMEM loads are warp-wide, so rows past M load and skip the
-// store.
-__device__ __forceinline__ void epilogue_kl(const GemmArgs &g, int gm_base, int tn, int row, uint32_t taddr) {
-    const int gm = gm_base + row;
+// EPI_KL.  The CTA's 128 accumulator rows are 64 rows of z_p = h_p W^T
+// (TMEM lanes 0-63: warp quarters 0, 1) over the same 64 rows of z_q =
+// h_q W^T (lanes 64-127: quarters 2, 3), so quarter q and quarter q + 2 hold
+// one row's two logit sets.  Each warp takes its rows' max over the tile's
+// columns; then, 32 columns at a time, the z_q warp adds its exp2(z log2e -
+// m_q) and hands the chunk to its partner through shared memory (column-major,
+// so both sides are conflict-free; two buffers, one 64-thread named barrier
+// per chunk), and the z_p warp adds exp2(z_p log2e - m_p) and the cross term
+// x = sum exp2(z_p log2e - m_p) (z_p - z_q).  All from fp32 accumulators.
+// `ck` counts the chunks handed over so far (the buffer parity).
+__device__ __forceinline__ void epilogue_kl(const GemmArgs &g, int gm_base, int tn, int q, int lane, uint32_t taddr,
+                                            float *xbuf, uint32_t &ck) {
+    const bool isp = q < 2;
+    const int gm = gm_base + (q & 1) * 32 + lane;
     const int n_base = tn * g.BN;
     const int nv = min(g.N, n_base + g.BN) - n_base;  // valid columns of the tile
-    float mp = -INFINITY, mq = -INFINITY;
+    const uint32_t bar = 2u + (uint32_t)(q & 1);
+    float *const pair_buf = xbuf + (q & 1) * 2 * 32 * 32;
+    float mx = -INFINITY;
     for (int c = 0; c < g.BN; c += 32) {
-        float vp[32], vq[32];
-        tmem_ld_x32(taddr + (uint32_t)c, vp);
-        tmem_ld_x32(taddr + (uint32_t)(g.BN + c), vq);
+        float v[32];
+        tmem_ld_x32(taddr + (uint32_t)c, v);
 #pragma unroll
         for (int i = 0; i < 32; ++i)
-            if (c + i < nv) {
-                mp = fmaxf(mp, vp[i]);
-                mq = fmaxf(mq, vq[i]);
-            }
+            if (c + i < nv) mx = fmaxf(mx, v[i]);
     }
-    mp *= kLog2e;
-    mq *= kLog2e;
-    float sp = 0.f, sq = 0.f, x = 0.f;
-    for (int c = 0; c < g.BN; c += 32) {
-        float vp[32], vq[32];
-        tmem_ld_x32(taddr + (uint32_t)c, vp);
-        tmem_ld_x32(taddr + (uint32_t)(g.BN + c), vq);
+    const float m2 = mx * kLog2e;
+    float sm = 0.f, x = 0.f;
+    for (int c = 0; c < g.BN; c += 32, ++ck) {
+        float v[32];
+        tmem_ld_x32(taddr + (uint32_t)c, v);
+        float *buf = pair_buf + (ck & 1u) * 32 * 32;
+        if (!isp) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
-            if (c + i < nv) {
-                const float ep = exp2f(fmaf(vp[i], kLog2e, -mp));
-                sp += ep;
-                sq += exp2f(fmaf(vq[i], kLog2e, -mq));
-                x = fmaf(ep, vp[i] - vq[i], x);
+            for (int i = 0; i < 32; ++i) {
+                if (c + i < nv) sm += exp2f(fmaf(v[i], kLog2e, -m2));
+                buf[i * 32 + lane] = v[i];
             }
+        }
+        named_barrier_sync(bar, 64);
+        if (isp) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+                if (c + i < nv) {
+                    const float e = exp2f(fmaf(v[i], kLog2e, -m2));
+                    sm += e;
+                    x = fmaf(e, v[i] - buf[i * 32 + lane], x);
+                }
+        }
     }
     if (gm < g.M) {
         const EpiParams &ep = g.ep;
         const int64_t o = (int64_t)(ep.tile0 + tn) * g.M + gm, P = ep.kl_plane;
-        ep.kl_part[o] = mp;
-        ep.kl_part[P + o] = sp;
-        ep.kl_part[2 * P + o] = mq;
-        ep.kl_part[3 * P + o] = sq;
-        ep.kl_part[4 * P + o] = x;
+        if (isp) {
+            ep.kl_part[o] = m2;
+            ep.kl_part[P + o] = sm;
+            ep.kl_part[4 * P + o] = x;
+        } else {
+            ep.kl_part[2 * P + o] = m2;
+            ep.kl_part[3 * P + o] = sm;
+        }
     }
 }
 
@@ -756,11 +774,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int S = g.stages;
     const int BNh = g.BN / 2;  // B rows held by this CTA
     const uint32_t b_bytes = gemm_b_stage_bytes(BNh);
-    // EPI_KL stages two A tiles (h_p, h_q) against one B tile and keeps two
-    // accumulators per tile
-    constexpr int kAT = EPI == EPI_KL ? 2 : 1;
     static_assert(EPI != EPI_KL || (!A_MN && !B_MN), "EPI_KL: K-major operands");
-    constexpr uint32_t a_bytes = kAT * kABytes;
+    constexpr uint32_t a_bytes = kABytes;
     uint8_t *sA = smem;
     uint8_t *sB = smem + (size_t)S * a_bytes;
     uint8_t *sE = sB + (size_t)S * b_bytes;  // 1024-byte aligned: b_bytes is a multiple of 2048
@@ -824,7 +839,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             bool ok = true;
             for (int w = cid; w < nwork && ok; w += ncl) {
                 const Work wi = work_item(g, w, tiles_m2);
-                const int arow0 = wi.tm * 256 + 128 * (int)rank;
+                // EPI_KL: 64 rows of A and the same 64 rows of A2 per CTA
+                const int arow0 = EPI == EPI_KL ? wi.tm * 128 + 64 * (int)rank : wi.tm * 256 + 128 * (int)rank;
                 const int brow0 = wi.tn * g.BN + BNh * (int)rank;
                 for (int kb = wi.kb0; kb < wi.kb1; ++kb) {
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
@@ -840,9 +856,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     const int kbk = sec ? (kb - g.kb_split) * 64 : g.b_k_off + kb * 64;
                     const int arow = (sec ? 0 : g.a_m_off) + arow0;
                     const int brow = (sec ? 0 : g.b_n_off) + brow0;
-                    if (!A_MN) {
+                    if constexpr (EPI == EPI_KL) {
+                        tma_load_2d_pair(a_dst, &tmA, fb, ka, arow0);          // rows 0-63: h_p
+                        tma_load_2d_pair(a_dst + 8192, &tmA2, fb, ka, arow0);  // rows 64-127: h_q
+                    } else if (!A_MN) {
                         tma_load_2d_pair(a_dst, pa, fb, ka, arow);
-                        if constexpr (kAT == 2) tma_load_2d_pair(a_dst + kABytes, &tmA2, fb, ka, arow);
                     } else {
                         tma_load_2d_pair(a_dst, pa, fb, arow, ka);
                         tma_load_2d_pair(a_dst + 8192, pa, fb, arow + 64, ka);
@@ -874,7 +892,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const int acc = it & 1;
                 if (!mbar_wait(tempty0 + 8 * acc, (((uint32_t)it >> 1) & 1u) ^ 1u, abort_flag)) { ok = false; break; }
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * kAT * g.BN);
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * g.BN);
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!mbar_wait(full0 + 8 * stage, phase, abort_flag)) { ok = false; break; }
                     tc_fence_after();
@@ -887,10 +905,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         const uint64_t bd = B_MN ? smem_desc_sw128(b_addr + kk * 2048, 8192, 1024)
                                                  : smem_desc_sw128(b_addr + kk * 32, 16, 1024);
                         umma_bf16_pair(d_tmem, ad, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
-                        if constexpr (kAT == 2) {
-                            const uint64_t ad2 = smem_desc_sw128(a_addr + kABytes + kk * 32, 16, 1024);
-                            umma_bf16_pair(d_tmem + (uint32_t)g.BN, ad2, bd, idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
-                        }
                     }
                     umma_commit_pair(empty0 + 8 * stage, 3);
                     if (++stage == S) { stage = 0; phase ^= 1u; }
@@ -913,6 +927,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int row = q * 32 + lane;
         F32Stage fst{smem_u32(sE) + (uint32_t)q * 8192u, smem_u32(sE) + 32768u + (uint32_t)q * 16u, 0u};
         uint32_t bec = 0;  // EPI_BF16 boxes stored by this warp
+        uint32_t kl_ck = 0;  // EPI_KL chunks handed over by this warp pair
         int it = 0;
         for (int w = cid; w < nwork; w += ncl, ++it) {
             const Work wi = work_item(g, w, tiles_m2);
@@ -928,10 +943,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             }
             (void)mbar_try_wait(tfull0 + 8 * acc, par);
             tc_fence_after();
-            const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kAT * g.BN);
+            const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * g.BN);
             const int gm_base = wi.tm * 256 + 128 * (int)rank;
             if constexpr (EPI == EPI_KL) {
-                epilogue_kl(g, gm_base, wi.tn, row, taddr);
+                epilogue_kl(g, wi.tm * 128 + 64 * (int)rank, wi.tn, q, lane, taddr, reinterpret_cast<float *>(sE),
+                            kl_ck);
             } else if constexpr (EPI == EPI_F32_ACC) {
                 if (wi.piece >= 0) {
                     epilogue_piece_f32_acc(g, wi, gm_base, (int)rank, 2, row, taddr, &tmC, fst, abort_flag);
