@@ -58,6 +58,9 @@ attt_status ce_fwd_bwd_run(const attt_bf16 *d_h, const attt_bf16 *d_W, const int
                            const float *row_scale, int64_t L, int64_t d, int64_t V, float *d_loss, float *d_dh,
                            float *d_lse, float *d_nll, void *d_ws, size_t ws_bytes, cudaStream_t stream);
 
+// The largest Eq. 10 workspace over every row count up to Lmax (ce.cu).
+size_t ce_workspace_bound(int64_t Lmax, int64_t d, int64_t V);
+
 // Device address of attt_lora_grad_noalloc's static status word on `dev`, or
 // nullptr if that entry point has not been set up on the device.
 int *noalloc_status_word(int dev);

@@ -133,11 +133,7 @@ attt_status attt_batch_create(const attt_batch_config *cfg, const attt_bf16 *d_W
     // stream): Eq. 10 over up to E max_update rows (its bound taken over every
     // row count, since its vocabulary chunk depends on it), the per-episode
     // adapter calls over up to max_update rows
-    size_t ws = 0;
-    for (int64_t L = 1; L <= rows; ++L) {
-        const size_t v = attt_ce_workspace_bytes(L, c.d, c.V);
-        if (v > ws) ws = v;
-    }
+    size_t ws = ce_workspace_bound(rows, c.d, c.V);
     const size_t per_ep[] = {attt_lora_workspace_bytes(c.max_update, c.din, 1, &c.d, c.r),
                              attt_lora_forward_workspace_bytes(c.max_update, c.din, c.d, c.r),
                              attt_lora_input_grad_workspace_bytes(c.max_update, c.din, c.d, c.r)};

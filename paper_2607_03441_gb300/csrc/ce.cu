@@ -329,6 +329,34 @@ size_t attt_ce_workspace_bytes(int64_t L, int64_t d, int64_t V) {
     return attt::ce_layout(nullptr, L, d, V).bytes;
 }
 
+}  // extern "C"
+
+namespace attt {
+
+// The largest attt_ce_workspace_bytes(L, d, V) over 1 <= L <= Lmax.  The
+// workspace grows with L while the vocabulary chunk Vc stays the same, and Vc
+// (a multiple of kCeBN, clamped to [4096, kCeMaxTiles kCeBN] and to V) only
+// changes where 256 MB / (2 L) crosses a multiple of kCeBN, so the maximum is
+// at Lmax or at the last L of one of those ranges.
+size_t ce_workspace_bound(int64_t Lmax, int64_t d, int64_t V) {
+    if (Lmax < 1) return 0;
+    size_t best = attt_ce_workspace_bytes(Lmax, d, V);
+    const int64_t budget = (256ll << 20) / 2;
+    for (int64_t vc = kCeBN; vc <= kCeMaxTiles * kCeBN; vc += kCeBN) {
+        const int64_t L = budget / vc;  // the last L whose unclamped chunk is at least vc
+        for (int64_t c = L - 1; c <= L + 1; ++c)
+            if (c >= 1 && c <= Lmax) {
+                const size_t b = attt_ce_workspace_bytes(c, d, V);
+                if (b > best) best = b;
+            }
+    }
+    return best;
+}
+
+}  // namespace attt
+
+extern "C" {
+
 attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W, const int32_t *d_tgt,
                                      const float *d_w, int64_t L, int64_t d, int64_t V, float *d_loss,
                                      float *d_dh, float *d_lse, void *d_ws, size_t ws_bytes, attt_stream stream) {

@@ -78,11 +78,11 @@ bool config_ok(const attt_episode_config *c) {
 
 // Workspace that every call of an update of up to max_update tokens fits in.
 // The Eq. 10 workspace is not monotone in L (its vocabulary chunk depends on
-// L), so the bound takes the maximum over every L.
+// L): its bound is the maximum over every L.
 size_t workspace_bound(const attt_episode_config &c) {
     size_t ws = 0;
     auto upd = [&](size_t b) { if (b > ws) ws = b; };
-    for (int64_t L = 1; L <= c.max_update; ++L) upd(attt_ce_workspace_bytes(L, c.d, c.V));
+    upd(attt::ce_workspace_bound(c.max_update, c.d, c.V));
     const int64_t L = c.max_update;
     upd(attt_lora_workspace_bytes(L, c.din, 1, &c.d, c.r));
     upd(attt_lora_forward_workspace_bytes(L, c.din, c.d, c.r));
