@@ -42,7 +42,6 @@ struct attt_batch {
 
 namespace {
 
-using attt::cdiv;
 
 constexpr int kMaxEpisodes = 32;
 

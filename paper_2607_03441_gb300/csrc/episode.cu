@@ -51,7 +51,6 @@ struct attt_episode {
 
 namespace {
 
-using attt::cdiv;
 
 template <class T>
 bool dev_alloc(T **p, size_t count) {

@@ -139,3 +139,34 @@ def test_batch_errors_launch_nothing(attt):
     b.update(t[:0], x[:0], [0, 0])               # nobody has text: nothing happens
     assert attt.attt_kernel_launches() == n0
     b.close()
+
+
+@pytest.mark.slow
+def test_7b_shapes_batch_equals_episodes(attt):
+    """Two 7B-class episodes (2,048-token updates, 152,064-entry head,
+    3,584 x 3,584 projection, rank 16) updated as a batch equal the same
+    episodes updated one by one: losses to 1e-5, adapter changes to 1e-3
+    relative L2 (Eq. 10 over 4,096 rows takes other vocabulary chunks than
+    over 2,048, so only rounding differs)."""
+    ew = wk.EPISODES["7b-episode"]
+    dense = wk.episode_dense(ew)
+    texts = wk.episode_texts(ew)[:2]
+    xs = [wk.episode_x(ew, k) for k in (1, 2)]
+    W0, W = bf16_dev(dense["W0"]), bf16_dev(dense["W"])
+    A0, B0 = f32_dev(dense["A0"]), f32_dev(dense["B0"])
+    kw = dict(n=ew.n, max_history=4 * ew.L, max_update=ew.L, scale=ew.scale, lr=0.5, w_min=ew.w_min,
+              grad_steps=ew.grad_steps)
+    b = attt.Batch(W0, W, A0, B0, episodes=2, **kw)
+    lb = torch.empty(2, ew.grad_steps, dtype=torch.float32, device=DEV)
+    b.update(i32_dev(np.concatenate(texts)), bf16_dev(np.concatenate(xs)), [ew.L, ew.L], losses=lb)
+    for e in range(2):
+        ep = attt.Episode(W0, W, A0, B0, cadence=1, **kw)
+        le = torch.empty(ew.grad_steps, dtype=torch.float32, device=DEV)
+        ep.update(i32_dev(texts[e]), bf16_dev(xs[e]), losses=le)
+        np.testing.assert_allclose(lb[e].cpu().numpy(), le.cpu().numpy(), rtol=1e-5)
+        (Ab, Bb), (Ae, Be) = b.read_adapter(e), ep.read_adapter()
+        assert rel_l2(Ab.cpu().numpy() - dense["A0"], Ae.cpu().numpy() - dense["A0"]) < 1e-3
+        assert rel_l2(Bb.cpu().numpy() - dense["B0"], Be.cpu().numpy() - dense["B0"]) < 1e-3
+        ep.close()
+    assert attt.attt_device_status() == 0
+    b.close()

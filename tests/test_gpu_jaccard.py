@@ -124,3 +124,16 @@ def test_capacity_errors_launch_nothing(attt):
     ws.close()
     with pytest.raises(attt.AtttError):
         attt.WordSets(0, 10)
+
+
+@pytest.mark.slow
+def test_stress_texts_first_updates(attt):
+    """The stress texts (~1 MB, 131,072 words each): the first eight updates
+    of the episode, bit-exact with the oracle, through the launch the bench
+    times (chunks of 2,048 bytes, every SM)."""
+    tw = wk.TEXT_WORKLOADS["texts-stress"]
+    texts = wk.episode_update_texts(tw)[:8]
+    ws = attt.WordSets(tw.updates, sum(len(t) for t in texts))
+    _check(_run(attt, ws, texts, tw.tau), oracle.sequence_filter(texts, tw.tau))
+    assert attt.attt_wordsets_status(ws) == 0
+    ws.close()
