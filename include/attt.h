@@ -82,6 +82,15 @@ ATTT_API uint64_t attt_kernel_launches(void);
  */
 ATTT_API attt_status attt_device_status(attt_stream stream);
 
+/*
+ * Failure-detection self-test: launches one kernel whose only wait (on an
+ * mbarrier that nothing completes) runs out after the library's wall-clock
+ * limit of 2 s, as any device-side wait of the library would, so the device
+ * status word then reads ATTT_ERR_TIMEOUT (attt_device_status) and the
+ * context stays usable.  No fault, trap or hang.  Async on `stream`.
+ */
+ATTT_API attt_status attt_selftest_wait_timeout(attt_stream stream);
+
 /* ------------------------------------------------------------------------ */
 /* Token history H (Sec. 3.3: every earlier update's tokens of the episode, */
 /* joined end to end) and its exact n-gram count table.                     */

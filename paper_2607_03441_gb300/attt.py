@@ -78,6 +78,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_abi_version": (i32, []),
             "attt_kernel_launches": (ctypes.c_uint64, []),
             "attt_device_status": (i32, [P]),
+            "attt_selftest_wait_timeout": (i32, [P]),
             "attt_history_create": (i32, [i32, i64, ctypes.POINTER(P)]),
             "attt_history_destroy": (i32, [P]),
             "attt_history_reset": (i32, [P, P]),
@@ -173,6 +174,11 @@ def attt_abi_version() -> int:
 def attt_kernel_launches() -> int:
     """Kernels launched by libattt in this process so far."""
     return int(load_library().attt_kernel_launches())
+
+
+def attt_selftest_wait_timeout(stream=None) -> None:
+    """Launches the bounded-wait self-test (a wait that runs out after 2 s)."""
+    _check(load_library().attt_selftest_wait_timeout(_stream(stream)), "attt_selftest_wait_timeout")
 
 
 def attt_device_status(stream=None) -> int:
