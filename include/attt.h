@@ -129,6 +129,22 @@ ATTT_API attt_status attt_history_reset(attt_history *h, attt_stream stream);
 ATTT_API attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_t len,
                                 attt_stream stream);
 
+/*
+ * Checkpoint of a history: copies its token stream (attt_history_length
+ * tokens, int32) to host_tokens and synchronises `stream`.  The counts need
+ * no copy: attt_history_restore rebuilds them exactly from the stream.
+ */
+ATTT_API attt_status attt_history_save(const attt_history *h, int32_t *host_tokens, attt_stream stream);
+
+/*
+ * Empties the history, then makes it the history of the len tokens in
+ * host_tokens (as one insert from empty: every count exact, so weights after
+ * a save and restore are bit-identical).  Synchronises `stream` once the
+ * tokens are on the device.  ATTT_ERR_CAPACITY if len > max_tokens.
+ */
+ATTT_API attt_status attt_history_restore(attt_history *h, const int32_t *host_tokens, int64_t len,
+                                          attt_stream stream);
+
 /* Current history length in tokens (host-side bookkeeping, no sync). */
 ATTT_API int64_t attt_history_length(const attt_history *h);
 
@@ -497,6 +513,21 @@ ATTT_API attt_status attt_episode_drift(attt_episode *e, const attt_bf16 *d_x, i
 /* Copies the adapter's fp32 values (A [din, r], B [r, d]) out.  Async. */
 ATTT_API attt_status attt_episode_read_adapter(const attt_episode *e, float *d_A32, float *d_B32,
                                                attt_stream stream);
+
+/*
+ * Checkpoint and resume of an episode (the adapter persists within an
+ * episode, Sec. 4): attt_episode_save writes into host_buf (at least
+ * attt_episode_checkpoint_bytes(e) bytes) the configuration, the fp32
+ * adapter, AdamW's moments and step count (optimizer 1), the history's token
+ * stream and the pending agent-step text, and synchronises `stream`.
+ * attt_episode_load restores all of it into an episode created with the same
+ * configuration (ATTT_ERR_INVALID_ARG otherwise, or for a buffer that is not
+ * such a checkpoint); the episode then continues bit for bit as the saved
+ * one would.  The frozen W0, LM head and initial adapter are not saved.
+ */
+ATTT_API size_t attt_episode_checkpoint_bytes(const attt_episode *e);
+ATTT_API attt_status attt_episode_save(attt_episode *e, void *host_buf, size_t bytes, attt_stream stream);
+ATTT_API attt_status attt_episode_load(attt_episode *e, const void *host_buf, size_t bytes, attt_stream stream);
 
 /* The episode's history (owned by the episode; do not destroy it). */
 ATTT_API attt_history *attt_episode_history(attt_episode *e);

@@ -108,6 +108,11 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_episode_agent_step": (i32, [P, P, P, i64, P, P, ctypes.POINTER(i32), P]),
             "attt_episode_read_adapter": (i32, [P, P, P, P]),
             "attt_episode_drift": (i32, [P, P, i64, P, P, P]),
+            "attt_episode_checkpoint_bytes": (sz, [P]),
+            "attt_episode_save": (i32, [P, P, sz, P]),
+            "attt_episode_load": (i32, [P, P, sz, P]),
+            "attt_history_save": (i32, [P, P, P]),
+            "attt_history_restore": (i32, [P, P, i64, P]),
             "attt_episode_history": (P, [P]),
             "attt_episode_pending_tokens": (i64, [P]),
             "attt_kl_workspace_bytes": (sz, [i64, i64, i64]),
@@ -247,6 +252,24 @@ def attt_history_insert(h: History, tokens: torch.Tensor, stream=None) -> None:
         raise ValueError("tokens must be int32")
     _check(load_library().attt_history_insert(h.handle, _ptr(tokens), tokens.numel(), _stream(stream)),
            "attt_history_insert")
+
+
+def attt_history_save(h: History, stream=None):
+    """The history's token stream (int32 numpy array), for a checkpoint."""
+    import numpy as np
+    n = len(h)
+    out = np.empty(n, dtype=np.int32)
+    _check(load_library().attt_history_save(h.handle, out.ctypes.data_as(ctypes.c_void_p) if n else None,
+                                            _stream(stream)), "attt_history_save")
+    return out
+
+
+def attt_history_restore(h: History, tokens, stream=None) -> None:
+    """Makes h the history of `tokens` (int32 numpy array), counts rebuilt exactly."""
+    import numpy as np
+    t = np.ascontiguousarray(tokens, dtype=np.int32)
+    _check(load_library().attt_history_restore(h.handle, t.ctypes.data_as(ctypes.c_void_p) if t.size else None,
+                                               t.size, _stream(stream)), "attt_history_restore")
 
 
 def attt_history_length(h: History) -> int:
@@ -554,6 +577,18 @@ class Episode:
 
     def pending_tokens(self) -> int:
         return int(self._lib.attt_episode_pending_tokens(self.handle))
+
+    def save(self, stream=None) -> bytes:
+        """A checkpoint of the episode (adapter, optimizer state, history, pending text)."""
+        n = int(self._lib.attt_episode_checkpoint_bytes(self.handle))
+        buf = ctypes.create_string_buffer(n)
+        _check(self._lib.attt_episode_save(self.handle, buf, n, _stream(stream)), "attt_episode_save")
+        return buf.raw
+
+    def load(self, blob: bytes, stream=None) -> None:
+        """Restores a checkpoint made by save() of an episode with the same configuration."""
+        buf = ctypes.create_string_buffer(bytes(blob), len(blob))
+        _check(self._lib.attt_episode_load(self.handle, buf, len(blob), _stream(stream)), "attt_episode_load")
 
 
 # --------------------------------------------------------------------------

@@ -22,6 +22,7 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <cstring>
 #include <new>
 
 #include "attt.h"
@@ -268,6 +269,96 @@ attt_status attt_episode_read_adapter(const attt_episode *e, float *d_A32, float
         cudaMemcpyAsync(d_B32, e->B32, nB * sizeof(float), cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
         return ATTT_ERR_CUDA;
     return ATTT_OK;
+}
+
+// Checkpoint layout (host bytes, native endianness): a header, then the
+// arrays in this order, each as stored on the device.
+struct EpisodeCkptHeader {
+    char magic[8];  // "ATTTEPC1"
+    attt_episode_config cfg;
+    int64_t hist_len, pend_len;
+    int32_t pend_steps, adam_t;
+};
+
+static size_t ckpt_bytes(const attt_episode *e, int64_t hist_len, int64_t pend_len) {
+    const attt_episode_config &c = e->cfg;
+    const size_t nA = (size_t)c.din * c.r, nB = (size_t)c.r * c.d;
+    size_t b = sizeof(EpisodeCkptHeader) + (nA + nB) * sizeof(float);
+    if (c.optimizer == 1) b += 2 * (nA + nB) * sizeof(float);
+    b += (size_t)hist_len * sizeof(int32_t) + (size_t)pend_len * (sizeof(int32_t) + c.din * sizeof(attt_bf16));
+    return b;
+}
+
+size_t attt_episode_checkpoint_bytes(const attt_episode *e) {
+    return e ? ckpt_bytes(e, attt_history_length(e->hist), e->pend_len) : 0;
+}
+
+attt_status attt_episode_save(attt_episode *e, void *host_buf, size_t bytes, attt_stream stream) {
+    if (!e || !host_buf) return ATTT_ERR_INVALID_ARG;
+    const int64_t hl = attt_history_length(e->hist);
+    if (bytes < ckpt_bytes(e, hl, e->pend_len)) return ATTT_ERR_INVALID_ARG;
+    const attt_episode_config &c = e->cfg;
+    const size_t nA = (size_t)c.din * c.r, nB = (size_t)c.r * c.d;
+    char *p = static_cast<char *>(host_buf);
+    EpisodeCkptHeader hdr{};
+    memcpy(hdr.magic, "ATTTEPC1", 8);
+    hdr.cfg = c;
+    hdr.hist_len = hl;
+    hdr.pend_len = e->pend_len;
+    hdr.pend_steps = e->pend_steps;
+    hdr.adam_t = e->adam_t;
+    memcpy(p, &hdr, sizeof hdr);
+    p += sizeof hdr;
+    struct Piece { const void *src; size_t n; };
+    Piece pieces[] = {{e->A32, nA * sizeof(float)}, {e->B32, nB * sizeof(float)},
+                      {c.optimizer == 1 ? e->mA : nullptr, nA * sizeof(float)},
+                      {c.optimizer == 1 ? e->vA : nullptr, nA * sizeof(float)},
+                      {c.optimizer == 1 ? e->mB : nullptr, nB * sizeof(float)},
+                      {c.optimizer == 1 ? e->vB : nullptr, nB * sizeof(float)},
+                      {e->pend_tok, (size_t)e->pend_len * sizeof(int32_t)},
+                      {e->pend_x, (size_t)e->pend_len * c.din * sizeof(attt_bf16)}};
+    for (const Piece &q : pieces) {
+        if (!q.src || q.n == 0) continue;
+        if (cudaMemcpyAsync(p, q.src, q.n, cudaMemcpyDeviceToHost, stream) != cudaSuccess) return ATTT_ERR_CUDA;
+        p += q.n;
+    }
+    attt_status st = attt_history_save(e->hist, reinterpret_cast<int32_t *>(p), stream);  // synchronises
+    if (st != ATTT_OK) return st;
+    return cudaStreamSynchronize(stream) == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+attt_status attt_episode_load(attt_episode *e, const void *host_buf, size_t bytes, attt_stream stream) {
+    if (!e || !host_buf || bytes < sizeof(EpisodeCkptHeader)) return ATTT_ERR_INVALID_ARG;
+    EpisodeCkptHeader hdr;
+    memcpy(&hdr, host_buf, sizeof hdr);
+    const attt_episode_config &c = e->cfg;
+    if (memcmp(hdr.magic, "ATTTEPC1", 8) != 0 || memcmp(&hdr.cfg, &c, sizeof c) != 0) return ATTT_ERR_INVALID_ARG;
+    if (hdr.hist_len < 0 || hdr.hist_len > c.max_history || hdr.pend_len < 0 || hdr.pend_len > c.max_update ||
+        bytes < ckpt_bytes(e, hdr.hist_len, hdr.pend_len))
+        return ATTT_ERR_INVALID_ARG;
+    const size_t nA = (size_t)c.din * c.r, nB = (size_t)c.r * c.d;
+    const char *p = static_cast<const char *>(host_buf) + sizeof hdr;
+    struct Piece { void *dst; size_t n; };
+    Piece pieces[] = {{e->A32, nA * sizeof(float)}, {e->B32, nB * sizeof(float)},
+                      {c.optimizer == 1 ? e->mA : nullptr, nA * sizeof(float)},
+                      {c.optimizer == 1 ? e->vA : nullptr, nA * sizeof(float)},
+                      {c.optimizer == 1 ? e->mB : nullptr, nB * sizeof(float)},
+                      {c.optimizer == 1 ? e->vB : nullptr, nB * sizeof(float)},
+                      {e->pend_tok, (size_t)hdr.pend_len * sizeof(int32_t)},
+                      {e->pend_x, (size_t)hdr.pend_len * c.din * sizeof(attt_bf16)}};
+    for (const Piece &q : pieces) {
+        if (!q.dst || q.n == 0) continue;
+        if (cudaMemcpyAsync(q.dst, p, q.n, cudaMemcpyHostToDevice, stream) != cudaSuccess) return ATTT_ERR_CUDA;
+        p += q.n;
+    }
+    attt_status st = attt_cast_bf16(e->A32, e->A16, (int64_t)nA, stream);
+    if (st == ATTT_OK) st = attt_cast_bf16(e->B32, e->B16, (int64_t)nB, stream);
+    if (st == ATTT_OK) st = attt_history_restore(e->hist, reinterpret_cast<const int32_t *>(p), hdr.hist_len, stream);
+    if (st != ATTT_OK) return st;
+    e->pend_len = hdr.pend_len;
+    e->pend_steps = hdr.pend_steps;
+    e->adam_t = hdr.adam_t;
+    return cudaStreamSynchronize(stream) == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
 
 attt_history *attt_episode_history(attt_episode *e) { return e ? e->hist : nullptr; }

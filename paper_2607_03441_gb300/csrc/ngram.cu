@@ -351,6 +351,35 @@ attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
 
+attt_status attt_history_save(const attt_history *h, int32_t *host_tokens, attt_stream stream) {
+    if (!h || (h->len > 0 && !host_tokens)) return ATTT_ERR_INVALID_ARG;
+    if (h->len == 0) return ATTT_OK;
+    if (cudaMemcpyAsync(host_tokens, h->d_tokens, (size_t)h->len * sizeof(int32_t), cudaMemcpyDeviceToHost,
+                        stream) != cudaSuccess ||
+        cudaStreamSynchronize(stream) != cudaSuccess)
+        return ATTT_ERR_CUDA;
+    return ATTT_OK;
+}
+
+attt_status attt_history_restore(attt_history *h, const int32_t *host_tokens, int64_t len, attt_stream stream) {
+    if (!h || len < 0 || (len > 0 && !host_tokens)) return ATTT_ERR_INVALID_ARG;
+    if (len > h->max_tokens) return ATTT_ERR_CAPACITY;
+    attt_status st = attt_history_reset(h, stream);
+    if (st != ATTT_OK || len == 0) return st;
+    if (cudaMemcpyAsync(h->d_tokens, host_tokens, (size_t)len * sizeof(int32_t), cudaMemcpyHostToDevice, stream) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(stream) != cudaSuccess)  // the host buffer may go once this returns
+        return ATTT_ERR_CUDA;
+    // every n-gram of the restored stream, as one insert from an empty history
+    h->len = len;
+    const int64_t count = len - h->n + 1;
+    if (count <= 0) return ATTT_OK;
+    attt::history_insert_kernel<<<(unsigned)((count + attt::kInsTile - 1) / attt::kInsTile), 256, 0, stream>>>(
+        h->d_tokens, 0, count, h->n, h->d_table, h->capacity - 1, h->d_status);
+    attt::count_launch();
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
 attt_status attt_history_status(attt_history *h, attt_stream stream) {
     if (!h) return ATTT_ERR_INVALID_ARG;
     if (cudaStreamSynchronize(stream) != cudaSuccess) return ATTT_ERR_CUDA;
