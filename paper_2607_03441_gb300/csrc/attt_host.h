@@ -3,6 +3,7 @@
 
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 #include <stddef.h>
 #include <stdint.h>
 
@@ -64,6 +65,16 @@ size_t ce_workspace_bound(int64_t Lmax, int64_t d, int64_t V);
 // Device address of attt_lora_grad_noalloc's static status word on `dev`, or
 // nullptr if that entry point has not been set up on the device.
 int *noalloc_status_word(int dev);
+
+// A named NVTX range over one C-ABI call, so that a timeline shows which
+// call each kernel belongs to (nearly free when no tool is attached).
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange &) = delete;
+    NvtxRange &operator=(const NvtxRange &) = delete;
+};
+#define ATTT_NVTX_RANGE() ::attt::NvtxRange attt_nvtx_range_(__func__)
 
 inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 inline bool aligned256(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 255u) == 0; }

@@ -171,6 +171,7 @@ attt_status attt_batch_destroy(attt_batch *b) {
 }
 
 attt_status attt_batch_reset(attt_batch *b, int e, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     if (!b || e < -1 || e >= b->cfg.episodes) return ATTT_ERR_INVALID_ARG;
     const int e0 = e < 0 ? 0 : e, e1 = e < 0 ? b->cfg.episodes : e + 1;
     for (int i = e0; i < e1; ++i) {
@@ -182,6 +183,7 @@ attt_status attt_batch_reset(attt_batch *b, int e, attt_stream stream) {
 
 attt_status attt_batch_update(attt_batch *b, const int32_t *d_tokens, const attt_bf16 *d_x, const int64_t *lens,
                               float *d_losses, float *d_dx, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     if (!b || !lens) return ATTT_ERR_INVALID_ARG;
     const attt_batch_config &c = b->cfg;

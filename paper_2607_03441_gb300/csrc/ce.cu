@@ -360,6 +360,7 @@ extern "C" {
 attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W, const int32_t *d_tgt,
                                      const float *d_w, int64_t L, int64_t d, int64_t V, float *d_loss,
                                      float *d_dh, float *d_lse, void *d_ws, size_t ws_bytes, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     return attt::ce_fwd_bwd_run(d_h, d_W, d_tgt, d_w, nullptr, L, d, V, d_loss, d_dh, d_lse, nullptr, d_ws, ws_bytes,
                                 stream);
 }

@@ -166,6 +166,7 @@ attt_status attt_episode_destroy(attt_episode *e) {
 }
 
 attt_status attt_episode_reset(attt_episode *e, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     if (!e) return ATTT_ERR_INVALID_ARG;
     attt_status st = attt_history_reset(e->hist, stream);
     if (st != ATTT_OK) return st;
@@ -176,6 +177,7 @@ attt_status attt_episode_reset(attt_episode *e, attt_stream stream) {
 
 attt_status attt_episode_update(attt_episode *e, const int32_t *d_tokens, const attt_bf16 *d_x, int64_t L,
                                 float *d_losses, float *d_dx, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     if (!e || L < 1 || !d_tokens || !d_x || !aligned16(d_x) || (d_dx && !aligned16(d_dx)))
         return ATTT_ERR_INVALID_ARG;
@@ -219,6 +221,7 @@ attt_status attt_episode_update(attt_episode *e, const int32_t *d_tokens, const 
 
 attt_status attt_episode_agent_step(attt_episode *e, const int32_t *d_tokens, const attt_bf16 *d_x, int64_t len,
                                     float *d_losses, float *d_dx, int *updated, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     if (!e || len < 0 || (len > 0 && (!d_tokens || !d_x))) return ATTT_ERR_INVALID_ARG;
     const attt_episode_config &c = e->cfg;
     if (updated) *updated = 0;
@@ -247,6 +250,7 @@ attt_status attt_episode_agent_step(attt_episode *e, const int32_t *d_tokens, co
 
 attt_status attt_episode_drift(attt_episode *e, const attt_bf16 *d_x, int64_t L, float *d_kl, float *d_kl_mean,
                                attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     if (!e || L < 1 || L > e->cfg.max_update || !d_x || !aligned16(d_x) || (!d_kl && !d_kl_mean))
         return ATTT_ERR_INVALID_ARG;

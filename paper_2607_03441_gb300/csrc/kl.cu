@@ -133,6 +133,7 @@ size_t attt_kl_workspace_bytes(int64_t L, int64_t d, int64_t V) {
 attt_status attt_kl_drift(const attt_bf16 *d_hp, const attt_bf16 *d_hq, const attt_bf16 *d_W, int64_t L, int64_t d,
                           int64_t V, float *d_kl, float *d_kl_mean, void *d_ws, size_t ws_bytes,
                           attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     if (!d_hp || !d_hq || !d_W || (!d_kl && !d_kl_mean)) return ATTT_ERR_INVALID_ARG;
     if (L < 1 || V < 1 || d < 8 || d % 8 != 0) return ATTT_ERR_INVALID_ARG;

@@ -457,6 +457,7 @@ size_t attt_lora_input_grad_workspace_bytes(int64_t L, int64_t din, int64_t dout
 attt_status attt_lora_forward(const attt_bf16 *d_x, const attt_bf16 *d_W0, const attt_bf16 *d_A, const attt_bf16 *d_B,
                               int64_t L, int64_t din, int64_t dout, int r, float scale, attt_bf16 *d_h, void *d_ws,
                               size_t ws_bytes, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     attt_status st = proj_check(d_x, d_W0, d_A, d_B, d_h, L, din, dout, r);
     if (st != ATTT_OK) return st;
@@ -508,6 +509,7 @@ attt_status attt_lora_forward(const attt_bf16 *d_x, const attt_bf16 *d_W0, const
 attt_status attt_lora_input_grad(const attt_bf16 *d_dy, const attt_bf16 *d_W0, const attt_bf16 *d_A,
                                  const attt_bf16 *d_B, int64_t L, int64_t din, int64_t dout, int r, float scale,
                                  float *d_dx, void *d_ws, size_t ws_bytes, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     attt_status st = proj_check(d_dy, d_W0, d_A, d_B, d_dx, L, din, dout, r);
     if (st != ATTT_OK) return st;
@@ -558,12 +560,14 @@ attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int npr
                            const int64_t *dout, const attt_bf16 *const *d_A, const attt_bf16 *const *d_B, int r,
                            float scale, float *const *d_dA, float *const *d_dB, void *d_ws, size_t ws_bytes,
                            attt_stream stream) {
+    ATTT_NVTX_RANGE();
     return attt::lora_grad_run(d_x, L, din, nproj, d_dy, dout, d_A, d_B, r, scale, d_dA, d_dB, d_ws, ws_bytes,
                                nullptr, stream);
 }
 
 attt_status attt_lora_step(float *d_A32, float *d_B32, const float *d_dA, const float *d_dB, int64_t din,
                            int64_t dout, int r, float lr, attt_bf16 *d_A16, attt_bf16 *d_B16, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     if (!d_A32 || !d_B32 || !d_dA || !d_dB || din < 1 || dout < 1 || r < 1) return ATTT_ERR_INVALID_ARG;
     int dev;
@@ -581,6 +585,7 @@ attt_status attt_lora_adamw_step(float *d_A32, float *d_B32, const float *d_dA, 
                                  float *d_vA, float *d_mB, float *d_vB, int64_t din, int64_t dout, int r, float lr,
                                  double beta1, double beta2, double eps, double weight_decay, int step,
                                  attt_bf16 *d_A16, attt_bf16 *d_B16, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     if (!d_A32 || !d_B32 || !d_dA || !d_dB || !d_mA || !d_vA || !d_mB || !d_vB) return ATTT_ERR_INVALID_ARG;
     if (din < 1 || dout < 1 || r < 1 || step < 1 || !(beta1 >= 0.0 && beta1 < 1.0) || !(beta2 >= 0.0 && beta2 < 1.0) ||
@@ -611,6 +616,7 @@ attt_status attt_lora_adamw_step(float *d_A32, float *d_B32, const float *d_dA, 
 }
 
 attt_status attt_cast_bf16(const float *d_src, attt_bf16 *d_dst, int64_t n, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     if (n < 0 || (n > 0 && (!d_src || !d_dst))) return ATTT_ERR_INVALID_ARG;
     if (n == 0) return ATTT_OK;

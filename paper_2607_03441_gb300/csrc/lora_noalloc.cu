@@ -67,6 +67,7 @@ extern "C" attt_status attt_lora_grad_noalloc(const attt_bf16 *d_x, int64_t L, i
                                               const attt_bf16 *const *d_A, const attt_bf16 *const *d_B, int r,
                                               float scale, float *const *d_dA, float *const *d_dB,
                                               attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     // 0 for an invalid shape (nproj, r, sizes or a null dout array)
     const size_t need = attt_lora_workspace_bytes(L, din, nproj, dout, r);

@@ -316,6 +316,7 @@ attt_status attt_history_destroy(attt_history *h) {
 }
 
 attt_status attt_history_reset(attt_history *h, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     if (!h) return ATTT_ERR_INVALID_ARG;
     if (cudaMemsetAsync(h->d_table, 0, h->capacity * sizeof(attt::Slot), stream) != cudaSuccess)
         return ATTT_ERR_CUDA;
@@ -328,6 +329,7 @@ int64_t attt_history_length(const attt_history *h) { return h ? h->len : -1; }
 int attt_history_ngram(const attt_history *h) { return h ? h->n : -1; }
 
 attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_t len, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     if (!h || len < 0 || (len > 0 && !d_tokens)) return ATTT_ERR_INVALID_ARG;
     if (len == 0) return ATTT_OK;
     if (h->len + len > h->max_tokens) return ATTT_ERR_CAPACITY;
@@ -362,6 +364,7 @@ attt_status attt_history_save(const attt_history *h, int32_t *host_tokens, attt_
 }
 
 attt_status attt_history_restore(attt_history *h, const int32_t *host_tokens, int64_t len, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     if (!h || len < 0 || (len > 0 && !host_tokens)) return ATTT_ERR_INVALID_ARG;
     if (len > h->max_tokens) return ATTT_ERR_CAPACITY;
     attt_status st = attt_history_reset(h, stream);
@@ -391,6 +394,7 @@ attt_status attt_history_status(attt_history *h, attt_stream stream) {
 
 attt_status attt_history_count(const attt_history *h, const int32_t *d_ngrams, int64_t m, uint32_t *d_counts,
                                attt_stream stream) {
+    ATTT_NVTX_RANGE();
     if (!h || m < 0 || (m > 0 && (!d_ngrams || !d_counts))) return ATTT_ERR_INVALID_ARG;
     if (m == 0) return ATTT_OK;
     const int threads = 256;
@@ -480,6 +484,7 @@ extern "C" {
 
 attt_status attt_ngram_weights(const attt_history *h, const int32_t *d_tokens, int64_t L, float w_min, float *d_w,
                                attt_stream stream) {
+    ATTT_NVTX_RANGE();
     if (!h || L < 0 || (L > 0 && (!d_tokens || !d_w)) || !(w_min > 0.0f) || !(w_min <= 1.0f))
         return ATTT_ERR_INVALID_ARG;
     if (L == 0) return ATTT_OK;

@@ -27,6 +27,7 @@ __global__ void wait_selftest_kernel(int *status) {
 }  // namespace
 
 extern "C" attt_status attt_selftest_wait_timeout(attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     int dev;
     attt_status st = current_device(&dev);

@@ -307,6 +307,7 @@ attt_status attt_wordsets_destroy(attt_wordsets *s) {
 }
 
 attt_status attt_wordsets_reset(attt_wordsets *s, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     if (!s) return ATTT_ERR_INVALID_ARG;
     if (cudaMemsetAsync(s->d_keys, 0, s->capacity * sizeof(unsigned long long), stream) != cudaSuccess ||
         cudaMemsetAsync(s->d_masks, 0, s->capacity * s->W * sizeof(unsigned long long), stream) != cudaSuccess)
@@ -330,6 +331,7 @@ attt_status attt_wordsets_status(attt_wordsets *s, attt_stream stream) {
 
 attt_status attt_repetition(attt_wordsets *s, const uint8_t *d_text, int64_t nbytes, float tau, float *d_rho,
                             float *d_nu, int32_t *d_keep, attt_stream stream) {
+    ATTT_NVTX_RANGE();
     using namespace attt;
     if (!s || nbytes < 0 || (nbytes > 0 && !d_text) || !(tau == tau)) return ATTT_ERR_INVALID_ARG;
     if (s->count >= s->max_updates || s->len + nbytes + 1 > s->arena_cap) return ATTT_ERR_CAPACITY;
