@@ -91,6 +91,20 @@ ATTT_API attt_status attt_device_status(attt_stream stream);
  */
 ATTT_API attt_status attt_selftest_wait_timeout(attt_stream stream);
 
+/*
+ * Host fault injection, for tests of the error paths: makes one pending
+ * fault, taken by the first place of its kind that reaches it --
+ *   "alloc"       the next device allocation of a create call fails (the call
+ *                 frees what it had allocated and returns ATTT_ERR_CUDA);
+ *   "table_full"  the next attt_history_insert that has n-grams to record
+ *                 records none and sets ATTT_ERR_TABLE_FULL in the history's
+ *                 status word, as a full probe sequence would;
+ *   "none"        clears a pending fault.
+ * The environment variable ATTT_FAULT=<site> sets one at the library's first
+ * use.  ATTT_ERR_INVALID_ARG for another name.  Nothing runs on the GPU.
+ */
+ATTT_API attt_status attt_fault_inject(const char *site);
+
 /* ------------------------------------------------------------------------ */
 /* Token history H (Sec. 3.3: every earlier update's tokens of the episode, */
 /* joined end to end) and its exact n-gram count table.                     */

@@ -79,6 +79,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_kernel_launches": (ctypes.c_uint64, []),
             "attt_device_status": (i32, [P]),
             "attt_selftest_wait_timeout": (i32, [P]),
+            "attt_fault_inject": (i32, [ctypes.c_char_p]),
             "attt_history_create": (i32, [i32, i64, ctypes.POINTER(P)]),
             "attt_history_destroy": (i32, [P]),
             "attt_history_reset": (i32, [P, P]),
@@ -184,6 +185,11 @@ def attt_kernel_launches() -> int:
 def attt_selftest_wait_timeout(stream=None) -> None:
     """Launches the bounded-wait self-test (a wait that runs out after 2 s)."""
     _check(load_library().attt_selftest_wait_timeout(_stream(stream)), "attt_selftest_wait_timeout")
+
+
+def attt_fault_inject(site: str) -> None:
+    """One pending host-side fault: "alloc", "table_full" or "none"."""
+    _check(load_library().attt_fault_inject(site.encode()), "attt_fault_inject")
 
 
 def attt_device_status(stream=None) -> int:

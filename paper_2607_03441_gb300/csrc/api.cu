@@ -4,6 +4,8 @@
 #include <cudaTypedefs.h>
 
 #include <atomic>
+#include <cstdlib>
+#include <cstring>
 #include <map>
 #include <mutex>
 #include <utility>
@@ -20,6 +22,26 @@ std::map<int, int *> g_status_words;
 std::map<std::pair<const void *, int>, size_t> g_smem_set;
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::atomic<unsigned long long> g_launches{0};
+// The pending injected fault (FaultSite), or -1 before ATTT_FAULT was read.
+std::atomic<int> g_fault{-1};
+
+int fault_site(const char *s) {
+    if (!s || !*s || strcmp(s, "none") == 0) return FAULT_NONE;
+    if (strcmp(s, "alloc") == 0) return FAULT_ALLOC;
+    if (strcmp(s, "table_full") == 0) return FAULT_TABLE_FULL;
+    return -1;
+}
+
+int pending_fault() {
+    int f = g_fault.load();
+    if (f < 0) {  // first use: the environment's fault, if any
+        int env = fault_site(std::getenv("ATTT_FAULT"));
+        if (env < 0) env = FAULT_NONE;
+        g_fault.compare_exchange_strong(f, env);
+        f = g_fault.load();
+    }
+    return f;
+}
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     std::lock_guard<std::mutex> lk(g_mu);
@@ -37,6 +59,11 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }  // namespace
 
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+bool fault_take(FaultSite site) {
+    int expected = pending_fault();
+    return expected == site && g_fault.compare_exchange_strong(expected, FAULT_NONE);
+}
 
 attt_status current_device(int *dev) {
     if (cudaGetDevice(dev) != cudaSuccess) return ATTT_ERR_CUDA;
@@ -159,3 +186,11 @@ attt_status attt_device_status(attt_stream stream) {
 }
 
 }  // extern "C"
+
+extern "C" attt_status attt_fault_inject(const char *site) {
+    const int f = attt::fault_site(site);
+    if (f < 0) return ATTT_ERR_INVALID_ARG;
+    attt::pending_fault();  // the environment is read first, so this call wins
+    attt::g_fault.store(f);
+    return ATTT_OK;
+}

@@ -35,6 +35,12 @@ bool make_tmap_f32(CUtensorMap *map, const void *base, uint64_t inner, uint64_t 
 // Counts one kernel launch (attt_kernel_launches).
 void count_launch();
 
+// Host fault injection (attt_fault_inject, or the ATTT_FAULT environment
+// variable read at first use): one pending fault, taken by the first site of
+// its kind that asks.
+enum FaultSite : int { FAULT_NONE = 0, FAULT_ALLOC = 1, FAULT_TABLE_FULL = 2 };
+bool fault_take(FaultSite site);
+
 // Raises the dynamic shared memory limit of `func` once per device.
 bool set_smem_limit(const void *func, size_t bytes, int dev);
 

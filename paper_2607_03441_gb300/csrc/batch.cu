@@ -48,6 +48,7 @@ constexpr int kMaxEpisodes = 32;
 template <class T>
 bool dev_alloc(T **p, size_t count) {
     *p = nullptr;
+    if (attt::fault_take(attt::FAULT_ALLOC)) return false;  // an injected allocation failure
     return cudaMalloc(reinterpret_cast<void **>(p), (count > 0 ? count : 1) * sizeof(T)) == cudaSuccess;
 }
 

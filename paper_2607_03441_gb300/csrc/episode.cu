@@ -56,6 +56,7 @@ namespace {
 template <class T>
 bool dev_alloc(T **p, size_t count) {
     *p = nullptr;
+    if (attt::fault_take(attt::FAULT_ALLOC)) return false;  // an injected allocation failure
     return cudaMalloc(reinterpret_cast<void **>(p), (count > 0 ? count : 1) * sizeof(T)) == cudaSuccess;
 }
 

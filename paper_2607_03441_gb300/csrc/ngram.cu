@@ -281,6 +281,7 @@ attt_status attt_history_create(int n, int64_t max_tokens, attt_history **out) {
     h->len = 0;
     h->capacity = cap;
     if (cudaMalloc(&h->d_tokens, (size_t)(max_tokens > 0 ? max_tokens : 1) * sizeof(int32_t)) != cudaSuccess ||
+        attt::fault_take(attt::FAULT_ALLOC) ||  // an injected allocation failure
         cudaMalloc(&h->d_table, cap * sizeof(attt::Slot)) != cudaSuccess ||
         cudaMalloc(&h->d_status, 256) != cudaSuccess) {
         cudaFree(h->d_tokens);
@@ -345,6 +346,13 @@ attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_
     h->len = new_len;
     if (p_end < p_begin) return ATTT_OK;
     const int64_t count = p_end - p_begin + 1;
+    if (attt::fault_take(attt::FAULT_TABLE_FULL)) {
+        // an injected full table: the status word reports it as the kernel would
+        static const int code = ATTT_ERR_TABLE_FULL;
+        return cudaMemcpyAsync(h->d_status, &code, sizeof code, cudaMemcpyHostToDevice, stream) == cudaSuccess
+                   ? ATTT_OK
+                   : ATTT_ERR_CUDA;
+    }
     const int threads = 256;
     const int64_t blocks = (count + attt::kInsTile - 1) / attt::kInsTile;
     attt::history_insert_kernel<<<(unsigned)blocks, threads, 0, stream>>>(h->d_tokens, p_begin, count, h->n,

@@ -75,3 +75,13 @@ def test_missing_library_fails_loudly(tmp_path):
             attt.load_library(str(tmp_path / "nope.so"))
     finally:
         attt._lib = saved
+
+
+def test_fault_injection_switch_is_host_only():
+    """attt_fault_inject only arms a host-side fault (no device needed)."""
+    from paper_2607_03441_gb300 import attt
+    attt.attt_fault_inject("table_full")
+    attt.attt_fault_inject("alloc")
+    attt.attt_fault_inject("none")
+    with pytest.raises(attt.AtttError):
+        attt.attt_fault_inject("network")

@@ -43,3 +43,45 @@ def test_wait_runs_out_and_the_context_survives(attt):
     ref, _, _, _ = oracle.ce_loss(h, W, tgt, w)
     assert abs(loss.item() - ref) <= 1e-3 * abs(ref)
     assert attt.attt_device_status() == 0
+
+
+def test_injected_allocation_failure_cleans_up(attt):
+    ew = wk.EPISODES["tiny-episode"]
+    dense = wk.episode_dense(ew)
+    args = (bf16_dev(dense["W0"]), bf16_dev(dense["W"]), f32_dev(dense["A0"]), f32_dev(dense["B0"]))
+    kw = dict(n=ew.n, max_history=4 * ew.L, max_update=ew.L, scale=ew.scale, lr=1.0)
+    free0 = torch.cuda.mem_get_info()[0]
+    for make in (lambda: attt.History(4, 1000), lambda: attt.Episode(*args, **kw),
+                 lambda: attt.Batch(*args, episodes=3, **kw)):
+        attt.attt_fault_inject("alloc")
+        with pytest.raises(attt.AtttError) as e:
+            make()
+        assert e.value.code == attt.ATTT_ERR_CUDA
+        obj = make()                     # the fault was taken once: the next create works
+        obj.close()
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] >= free0 - (64 << 20)  # nothing of the failed creates kept
+    ep = attt.Episode(*args, **kw)       # and an update runs after it
+    ep.update(i32_dev(wk.episode_texts(ew)[0]), bf16_dev(wk.episode_x(ew, 1)))
+    assert attt.attt_device_status() == 0
+    ep.close()
+
+
+def test_injected_full_table_reaches_the_status_word(attt):
+    h = attt.History(3, 1000)
+    toks = i32_dev(np.arange(50, dtype=np.int32))
+    attt.attt_fault_inject("table_full")
+    attt.attt_history_insert(h, toks)
+    assert attt.attt_history_status(h) == attt.ATTT_ERR_TABLE_FULL
+    assert attt.attt_history_status(h) == 0          # read and cleared
+    attt.attt_history_insert(h, toks)                 # the fault was taken: counts as usual
+    q = i32_dev(np.array([[0, 1, 2], [10, 11, 12]], np.int32))
+    assert attt.attt_history_count(h, q).cpu().tolist() == [1, 1]
+    # a pending fault can be withdrawn; an unknown site is refused
+    attt.attt_fault_inject("table_full")
+    attt.attt_fault_inject("none")
+    attt.attt_history_insert(h, toks)
+    assert attt.attt_history_status(h) == 0
+    with pytest.raises(attt.AtttError):
+        attt.attt_fault_inject("disk")
+    h.close()
