@@ -60,7 +60,8 @@ typedef enum attt_status {
     ATTT_ERR_WORKSPACE = 5,    /* workspace missing or smaller than required   */
     ATTT_ERR_CUDA = 6,         /* a CUDA runtime call failed                   */
     ATTT_ERR_UNSUPPORTED = 7,  /* not a GB300-class (sm_103) device, or shape  */
-    ATTT_ERR_CAPACITY = 8      /* history would exceed its max_tokens          */
+    ATTT_ERR_CAPACITY = 8,     /* history would exceed its max_tokens          */
+    ATTT_ERR_CHECK = 9         /* a bounds check of the checked build failed   */
 } attt_status;
 
 /* Human-readable name of a status code.  Never NULL. */

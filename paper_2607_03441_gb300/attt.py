@@ -17,6 +17,8 @@ import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libattt.so")
+# ATTT_CHECKED=1 selects the checked build (device-side bounds checks)
+LIB_CHECKED_PATH = os.path.join(_HERE, "libattt_checked.so")
 
 ATTT_OK = 0
 ATTT_ERR_INVALID_ARG = 1
@@ -27,10 +29,11 @@ ATTT_ERR_WORKSPACE = 5
 ATTT_ERR_CUDA = 6
 ATTT_ERR_UNSUPPORTED = 7
 ATTT_ERR_CAPACITY = 8
+ATTT_ERR_CHECK = 9
 STATUS_NAMES = {
     0: "ATTT_OK", 1: "ATTT_ERR_INVALID_ARG", 2: "ATTT_ERR_TABLE_FULL", 3: "ATTT_ERR_TOKEN_RANGE",
     4: "ATTT_ERR_TIMEOUT", 5: "ATTT_ERR_WORKSPACE", 6: "ATTT_ERR_CUDA", 7: "ATTT_ERR_UNSUPPORTED",
-    8: "ATTT_ERR_CAPACITY",
+    8: "ATTT_ERR_CAPACITY", 9: "ATTT_ERR_CHECK",
 }
 
 _lock = threading.Lock()
@@ -67,7 +70,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     with _lock:
         if _lib is not None:
             return _lib
-        p = path or LIB_PATH
+        p = path or (LIB_CHECKED_PATH if os.environ.get("ATTT_CHECKED") == "1" else LIB_PATH)
         if not os.path.exists(p):
             raise RuntimeError(f"libattt.so not found at {p}; run paper_2607_03441_gb300.build.build()")
         lib = ctypes.CDLL(p)

@@ -157,6 +157,7 @@ const char *attt_status_string(int status) {
         case ATTT_ERR_CUDA: return "ATTT_ERR_CUDA";
         case ATTT_ERR_UNSUPPORTED: return "ATTT_ERR_UNSUPPORTED";
         case ATTT_ERR_CAPACITY: return "ATTT_ERR_CAPACITY";
+        case ATTT_ERR_CHECK: return "ATTT_ERR_CHECK";
         default: return "ATTT_ERR_UNKNOWN";
     }
 }

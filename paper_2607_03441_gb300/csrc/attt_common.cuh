@@ -35,6 +35,19 @@ __device__ __forceinline__ void record_error(int *status, int code) {
     if (status) atomicCAS(status, 0, code);
 }
 
+// The checked build (-DATTT_CHECKED=1, libattt_checked.so) tests `cond`
+// before an access that the host's validation already makes safe; a failure
+// records ATTT_ERR_CHECK in the status word and the access is skipped.  The
+// normal build compiles the test away (the guard is then always true).
+#ifndef ATTT_CHECKED
+#define ATTT_CHECKED 0
+#endif
+__device__ __forceinline__ bool check_guard(bool ok, int *status) {
+    if (!ok) record_error(status, ATTT_ERR_CHECK);
+    return ok;
+}
+#define ATTT_GUARD(cond, status) (!ATTT_CHECKED || ::attt::check_guard((cond), (status)))
+
 // Programmatic dependent launch.  griddep_wait: block until the grid launched
 // before this one in the stream has completed and its writes are visible (a
 // no-op when this grid was launched without the programmatic attribute).

@@ -65,13 +65,15 @@ __device__ __forceinline__ bool ngram_equal(const int32_t *a, const int32_t *b, 
 // count, or 0 if absent.  `hist` is the history token stream.
 __device__ __forceinline__ unsigned int table_lookup(const Slot *table, unsigned long long mask,
                                                      const int32_t *hist, const int32_t *g, int n,
-                                                     unsigned long long hsh) {
+                                                     unsigned long long hsh, int64_t hist_len, int *status) {
     const unsigned int tag = slot_tag(hsh);
     unsigned long long idx = hsh & mask;
     for (int probe = 0; probe < kMaxProbe; ++probe) {
         const Slot k = __ldcg(table + idx);
         if (k == 0ull) return 0u;
-        if ((unsigned int)(k >> 48) == tag && ngram_equal(hist + slot_pos(k), g, n)) return slot_count(k);
+        if ((unsigned int)(k >> 48) == tag && ATTT_GUARD((int64_t)slot_pos(k) + n <= hist_len, status) &&
+            ngram_equal(hist + slot_pos(k), g, n))
+            return slot_count(k);
         idx = (idx + 1) & mask;
     }
     return 0u;
@@ -81,11 +83,12 @@ __device__ __forceinline__ unsigned int table_lookup(const Slot *table, unsigned
 // hsh, starting from the result k of the optimistic claim of slot idx.
 __device__ __forceinline__ bool insert_rest(Slot *table, unsigned long long mask, const int32_t *hist,
                                             const int32_t *g, int n, unsigned long long hsh, Slot claim,
-                                            unsigned long long idx, Slot k) {
+                                            unsigned long long idx, Slot k, int64_t hist_len, int *status) {
     const unsigned int tag = slot_tag(hsh);
     for (int probe = 0; probe < kMaxProbe; ++probe) {
         if (k == 0ull) return true;  // claimed with count 1
-        if ((unsigned int)(k >> 48) == tag && ngram_equal(hist + slot_pos(k), g, n)) {
+        if ((unsigned int)(k >> 48) == tag && ATTT_GUARD((int64_t)slot_pos(k) + n <= hist_len, status) &&
+            ngram_equal(hist + slot_pos(k), g, n)) {
             atomicAdd(table + idx, 1ull);  // count lives in the low 24 bits
             return true;
         }
@@ -135,7 +138,8 @@ __device__ __forceinline__ void insert_block(const int32_t *__restrict__ hist, i
 #pragma unroll
     for (int q = 0; q < kInsPer; ++q) {
         const int li = q * blockDim.x + threadIdx.x;
-        if (i0 + li < count && !insert_rest(table, mask, hist, tok + li, n, hsh[q], claim[q], idx[q], k[q]))
+        if (i0 + li < count && !insert_rest(table, mask, hist, tok + li, n, hsh[q], claim[q], idx[q], k[q],
+                                            p_begin + count + n - 1, status))
             record_error(status, ATTT_ERR_TABLE_FULL);
     }
 }
@@ -164,13 +168,14 @@ __global__ void __launch_bounds__(256) history_insert_batch_kernel(const __grid_
 }
 
 // count(g, H) for m query n-grams stored row-major [m, n].
-__global__ void __launch_bounds__(256) history_count_kernel(const int32_t *__restrict__ hist, const Slot *table,
-                                                            unsigned long long mask, const int32_t *__restrict__ q,
-                                                            int64_t m, int n, unsigned int *out) {
+__global__ void __launch_bounds__(256) history_count_kernel(const int32_t *__restrict__ hist, int64_t hist_len,
+                                                            const Slot *table, unsigned long long mask,
+                                                            const int32_t *__restrict__ q, int64_t m, int n,
+                                                            unsigned int *out, int *status) {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= m) return;
     const int32_t *g = q + i * n;
-    out[i] = table_lookup(table, mask, hist, g, n, ngram_hash(g, n));
+    out[i] = table_lookup(table, mask, hist, g, n, ngram_hash(g, n), hist_len, status);
 }
 
 constexpr int kWTile = 256;                 // positions j per block
@@ -199,7 +204,8 @@ __device__ __forceinline__ void weights_block(const int32_t *__restrict__ x, int
     for (int i = threadIdx.x; i < nwin; i += blockDim.x) {
         const int64_t s = s_lo + i;
         unsigned int c = 0u;
-        if (s >= 0 && s + n <= L && hist_len >= n) c = table_lookup(table, mask, hist, tok + i, n, ngram_hash(tok + i, n));
+        if (s >= 0 && s + n <= L && hist_len >= n)
+            c = table_lookup(table, mask, hist, tok + i, n, ngram_hash(tok + i, n), hist_len, nullptr);
         cnt[i] = c;
     }
     __syncthreads();
@@ -407,7 +413,7 @@ attt_status attt_history_count(const attt_history *h, const int32_t *d_ngrams, i
     if (m == 0) return ATTT_OK;
     const int threads = 256;
     attt::history_count_kernel<<<(unsigned)((m + threads - 1) / threads), threads, 0, stream>>>(
-        h->d_tokens, h->d_table, h->capacity - 1, d_ngrams, m, h->n, d_counts);
+        h->d_tokens, h->len, h->d_table, h->capacity - 1, d_ngrams, m, h->n, d_counts, h->d_status);
     attt::count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }

@@ -474,9 +474,9 @@ __device__ __forceinline__ void epilogue_kl(const GemmArgs &g, int gm_base, int 
                 }
         }
     }
-    if (gm < g.M) {
-        const EpiParams &ep = g.ep;
-        const int64_t o = (int64_t)(ep.tile0 + tn) * g.M + gm, P = ep.kl_plane;
+    const EpiParams &ep = g.ep;
+    const int64_t o = (int64_t)(ep.tile0 + tn) * g.M + gm, P = ep.kl_plane;
+    if (gm < g.M && ATTT_GUARD(o < P, g.status)) {
         if (isp) {
             ep.kl_part[o] = m2;
             ep.kl_part[P + o] = sm;

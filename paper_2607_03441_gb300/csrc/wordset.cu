@@ -120,7 +120,9 @@ __device__ __forceinline__ const unsigned long long *record_word(const RepArgs &
     unsigned long long idx = h & a.cap_mask;
     for (int probe = 0; probe < kProbeLimit; ++probe) {
         const unsigned long long k0 = atomicCAS(a.keys + idx, 0ull, key);
-        if (k0 == 0ull || ((k0 >> 32) == (key >> 32) && word_equal(v, (int64_t)(k0 & 0xFFFFFFFFull) - 1, p))) {
+        if (k0 == 0ull || ((k0 >> 32) == (key >> 32) &&
+                           ATTT_GUARD((int64_t)(k0 & 0xFFFFFFFFull) - 1 < a.base + a.n, a.status) &&
+                           word_equal(v, (int64_t)(k0 & 0xFFFFFFFFull) - 1, p))) {
             unsigned long long *m = a.masks + (size_t)idx * a.W;
             *old = atomicOr(m + kw, kbit);
             return (*old & kbit) ? nullptr : m;  // else another block owns it

@@ -85,3 +85,14 @@ def test_fault_injection_switch_is_host_only():
     attt.attt_fault_inject("none")
     with pytest.raises(attt.AtttError):
         attt.attt_fault_inject("network")
+
+
+def test_checked_build_exports_the_same_calls():
+    """The checked build (-DATTT_CHECKED=1: device-side bounds checks) builds
+    and exports every declared entry point, as the normal build does."""
+    from paper_2607_03441_gb300 import build
+    path = build.build(checked=True)
+    out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (attt_\w+)", out))
+    assert not [s for s in declared_symbols() if s not in exported]
+    assert ctypes.CDLL(path).attt_status_string(9) is not None
