@@ -13,7 +13,8 @@
 //                 each row with its own episode's 1/L_e; loss_e from the rows'
 //                 NLL in a fixed order
 //     dy = bf16(dh)                            one launch
-//     dA_e, dB_e (and dx_e)                    per episode (grouped passes)
+//     dA_e, dB_e                               one grouped launch per pass (16 episodes each)
+//     dx_e                                     per episode (if asked)
 //     A, B <- A - lr dA, B - lr dB             one launch over every adapter
 //   H_e <- H_e || x_e                          one launch over every history
 // The adapters live stacked (A [E][din][r], B [E][r][d]), so the SGD step of
@@ -134,7 +135,7 @@ attt_status attt_batch_create(const attt_batch_config *cfg, const attt_bf16 *d_W
     // row count, since its vocabulary chunk depends on it), the per-episode
     // adapter calls over up to max_update rows
     size_t ws = ce_workspace_bound(rows, c.d, c.V);
-    const size_t per_ep[] = {attt_lora_workspace_bytes(c.max_update, c.din, 1, &c.d, c.r),
+    const size_t per_ep[] = {lora_grad_batch_workspace(E, rows + 8 * E, c.din, c.d, c.r),
                              attt_lora_forward_workspace_bytes(c.max_update, c.din, c.d, c.r),
                              attt_lora_input_grad_workspace_bytes(c.max_update, c.din, c.d, c.r)};
     for (size_t v : per_ep)
@@ -205,6 +206,7 @@ attt_status attt_batch_update(attt_batch *b, const int32_t *d_tokens, const attt
     attt_status st = current_device(&dev);
     if (st != ATTT_OK) return st;
     const size_t nA = (size_t)c.din * c.r, nB = (size_t)c.r * c.d;
+    const int64_t rows = (int64_t)E * c.max_update;  // the row bound the workspace was sized for
     float *losses = d_losses ? d_losses : b->loss_scratch;
 
     st = ngram_weights_batch(b->hist.data(), E, d_tokens, off, c.w_min, b->w, b->rowscale, stream);
@@ -225,15 +227,15 @@ attt_status attt_batch_update(attt_batch *b, const int32_t *d_tokens, const attt
         if (st == ATTT_OK && (cudaMemsetAsync(b->dA, 0, E * nA * sizeof(float), stream) != cudaSuccess ||
                               cudaMemsetAsync(b->dB, 0, E * nB * sizeof(float), stream) != cudaSuccess))
             st = ATTT_ERR_CUDA;
-        for (int e = 0; e < E && st == ATTT_OK; ++e) {
+        // every episode's adapter gradients: one grouped launch per pass
+        if (st == ATTT_OK)
+            st = lora_grad_batch_run(d_x, b->dy, off, E, c.din, c.d, c.r, c.scale, b->A16, b->B16, b->dA, b->dB,
+                                     rows + 8 * E, b->ws, b->ws_bytes, stream);
+        for (int e = 0; e < E && st == ATTT_OK && d_dx; ++e) {
             if (lens[e] == 0) continue;
-            const attt_bf16 *dys[1] = {b->dy + off[e] * c.d}, *As[1] = {b->A16 + e * nA}, *Bs[1] = {b->B16 + e * nB};
-            float *dAs[1] = {b->dA + e * nA}, *dBs[1] = {b->dB + e * nB};
-            st = attt_lora_grad(d_x + off[e] * c.din, lens[e], c.din, 1, dys, &c.d, As, Bs, c.r, c.scale, dAs, dBs,
-                                b->ws, b->ws_bytes, stream);
-            if (st == ATTT_OK && d_dx)
-                st = attt_lora_input_grad(dys[0], b->W0, As[0], Bs[0], lens[e], c.din, c.d, c.r, c.scale,
-                                          d_dx + ((size_t)g * R + off[e]) * c.din, b->ws, b->ws_bytes, stream);
+            st = attt_lora_input_grad(b->dy + off[e] * c.d, b->W0, b->A16 + e * nA, b->B16 + e * nB, lens[e], c.din,
+                                      c.d, c.r, c.scale, d_dx + ((size_t)g * R + off[e]) * c.din, b->ws,
+                                      b->ws_bytes, stream);
         }
         // every adapter of the batch in one step: A as [E din, r], B as [r, E d]
         if (st == ATTT_OK)

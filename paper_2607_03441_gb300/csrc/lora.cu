@@ -211,13 +211,13 @@ constexpr int kGroupMinStages = 2;
 
 // Launches every problem of `specs` in one grouped kernel; every CTA streams
 // the same number of K stages (stream-K split, tc_group.cuh).
-template <bool A_MN, bool B_MN>
+template <bool A_MN, bool B_MN, int NP = kMaxGroup>
 static attt_status launch_group(const GroupSpec *specs, int n, int BN, float *part, unsigned int *tickets, int dev,
                                 cudaStream_t stream, int *status) {
-    if (n < 1 || n > kMaxGroup || BN < 16 || BN > 256 || BN % 16 != 0) return ATTT_ERR_INVALID_ARG;
+    if (n < 1 || n > NP || BN < 16 || BN > 256 || BN % 16 != 0) return ATTT_ERR_INVALID_ARG;
     static_assert(!B_MN, "grouped B operands are K-major");
-    GroupMaps maps;
-    GroupArgs g{};
+    GroupMaps<NP> maps;
+    GroupArgs<NP> g{};
     g.nprob = n;
     g.BN = BN;
     g.part = part;
@@ -277,7 +277,7 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, float *pa
     g.total_stages = stages;
     const size_t smem =
         1024 + (size_t)g.stages * g.kbs * (kABytes + gemm_b_stage_bytes(BN)) + 8 * (2 * g.stages + 5) + 16;
-    auto kern = tc_gemm_group_kernel<A_MN, B_MN>;
+    auto kern = tc_gemm_group_kernel<A_MN, B_MN, NP>;
     if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
     // every CTA gets at least kGroupMinStages stages (at least one), so that a
     // tile is not cut into more pieces than its final sum can afford
@@ -395,6 +395,173 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
     return ATTT_OK;
 }
 
+
+// ---------------------------------------------------------------------------
+// The adapter gradients of a batch of episodes (attt_batch_update): each
+// episode has its own rows of the stacked x and dy and its own adapter, and
+// the u, v (pass 1) and dA, dB (pass 2) of up to kGroupEpisodes episodes run as
+// the problems of one grouped launch each.
+// ---------------------------------------------------------------------------
+
+struct BatchLoraLayout {
+    int rpad;
+    __nv_bfloat16 *AT, *BT;    // [E rpad, din], [E rpad, d]: episode e's rows at e rpad
+    __nv_bfloat16 *uT, *vT;    // per episode [rpad, Lp_e], laid one after another
+    int64_t tiles;
+    unsigned int *tickets;
+    float *part;
+    size_t bytes;
+};
+
+// rows_bound: an upper bound of sum_e round_up(L_e, 8) (sizes every buffer)
+static BatchLoraLayout batch_lora_layout(void *ws, int E, int64_t rows_bound, int64_t din, int64_t d, int r) {
+    BatchLoraLayout c{};
+    c.rpad = (int)round_up(r, 16);
+    const int64_t t1 = 2 * (cdiv(rows_bound, 128) + E), t2 = (int64_t)E * (cdiv(din, 128) + cdiv(d, 128));
+    c.tiles = t1 > t2 ? t1 : t2;
+    Carve cv{static_cast<char *>(ws), 0};
+    c.AT = cv.take<__nv_bfloat16>((size_t)E * c.rpad * din);
+    c.BT = cv.take<__nv_bfloat16>((size_t)E * c.rpad * d);
+    c.uT = cv.take<__nv_bfloat16>((size_t)c.rpad * rows_bound);
+    c.vT = cv.take<__nv_bfloat16>((size_t)c.rpad * rows_bound);
+    c.tickets = cv.take<unsigned int>((size_t)c.tiles);
+    c.part = cv.take<float>((size_t)(c.tiles + kGroupMaxGrid) * 128 * c.rpad);
+    c.bytes = (size_t)round_up((int64_t)cv.used, 256);
+    return c;
+}
+
+struct BatchPrepArgs {
+    const __nv_bfloat16 *A, *B;  // stacked [E][din][r], [E][r][d]
+    __nv_bfloat16 *AT, *BT;
+    int r, rpad;
+    int64_t din, d;
+    unsigned int *tickets;
+    int64_t ntickets;
+};
+
+// As lora_prep_kernel, for episode e = blockIdx.y of a batch's stacked
+// adapters: AT[e rpad + c, i] = A_e[i, c], BT[e rpad + c, o] = B_e[c, o]
+// (zero for c >= r), and the tickets zeroed (each episode row a slice).
+__global__ void __launch_bounds__(256) lora_prep_batch_kernel(BatchPrepArgs a) {
+    __shared__ __nv_bfloat16 slab[kPrepRows][64 + 2];
+    griddep_launch_dependents();
+    const int e = blockIdx.y;
+    const __nv_bfloat16 *A = a.A + (int64_t)e * a.din * a.r;
+    const __nv_bfloat16 *B = a.B + (int64_t)e * a.r * a.d;
+    __nv_bfloat16 *AT = a.AT + (int64_t)e * a.rpad * a.din;
+    __nv_bfloat16 *BT = a.BT + (int64_t)e * a.rpad * a.d;
+    const int64_t nslab = (a.din + kPrepRows - 1) / kPrepRows;
+    for (int64_t sb = blockIdx.x; sb < nslab; sb += gridDim.x) {
+        const int64_t k0 = sb * kPrepRows;
+        const int rows = (int)min((int64_t)kPrepRows, a.din - k0);
+        for (int i = threadIdx.x; i < rows * a.r; i += blockDim.x) {
+            const int kk = i / a.r, c = i - kk * a.r;
+            slab[kk][c] = A[(k0 + kk) * a.r + c];
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < a.rpad * kPrepRows; i += blockDim.x) {
+            const int c = i / kPrepRows, kk = i - c * kPrepRows;
+            if (kk < rows) AT[(int64_t)c * a.din + k0 + kk] = c < a.r ? slab[kk][c] : __float2bfloat16_rn(0.f);
+        }
+        __syncthreads();
+    }
+    const int64_t nB = (int64_t)a.rpad * a.d;
+    const int64_t ztk = (a.ntickets + gridDim.y - 1) / gridDim.y;
+    const int64_t n = nB > ztk ? nB : ztk;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        if (i < nB) {
+            const int c = (int)(i / a.d);
+            BT[i] = c < a.r ? B[i] : __float2bfloat16_rn(0.f);
+        }
+        if (i < ztk && e * ztk + i < a.ntickets) a.tickets[e * ztk + i] = 0u;
+    }
+}
+
+size_t lora_grad_batch_workspace(int E, int64_t rows_bound, int64_t din, int64_t d, int r) {
+    return batch_lora_layout(nullptr, E, rows_bound, din, d, r).bytes;
+}
+
+attt_status lora_grad_batch_run(const attt_bf16 *d_x, const attt_bf16 *d_dy, const int64_t *off, int E, int64_t din,
+                                int64_t d, int r, float scale, const attt_bf16 *d_A16, const attt_bf16 *d_B16,
+                                float *d_dA, float *d_dB, int64_t rows_bound, void *d_ws, size_t ws_bytes,
+                                cudaStream_t stream) {
+    if (E < 1 || r < 1 || r > 64 || din < 8 || d < 8 || din % 8 || d % 8) return ATTT_ERR_INVALID_ARG;
+    if (!d_ws || ws_bytes < lora_grad_batch_workspace(E, rows_bound, din, d, r)) return ATTT_ERR_WORKSPACE;
+    int dev;
+    attt_status st = current_device(&dev);
+    if (st != ATTT_OK) return st;
+    BatchLoraLayout c = batch_lora_layout(d_ws, E, rows_bound, din, d, r);
+    const int BN = c.rpad;
+    {
+        BatchPrepArgs a{};
+        a.A = reinterpret_cast<const __nv_bfloat16 *>(d_A16);
+        a.B = reinterpret_cast<const __nv_bfloat16 *>(d_B16);
+        a.AT = c.AT; a.BT = c.BT; a.r = r; a.rpad = c.rpad; a.din = din; a.d = d;
+        a.tickets = c.tickets; a.ntickets = c.tiles;
+        int64_t maxn = cdiv(din, kPrepRows) * 256;
+        if (c.rpad * d > maxn) maxn = c.rpad * d;
+        if (cdiv(c.tiles, E) > maxn) maxn = cdiv(c.tiles, E);
+        lora_prep_batch_kernel<<<dim3(grid_for(maxn, 256, dev), (unsigned)E), 256, 0, stream>>>(a);
+        count_launch();
+        if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
+    }
+    // each episode's place in uT / vT
+    int64_t toff[kGroupEpisodes] = {0};
+    for (int e0 = 0; e0 < E; e0 += kGroupEpisodes) {
+        const int e1 = e0 + kGroupEpisodes < E ? e0 + kGroupEpisodes : E;
+        int64_t acc = 0;
+        for (int e = e0; e < e1; ++e) {
+            toff[e - e0] = acc;
+            acc += (int64_t)c.rpad * round_up(off[e + 1] - off[e], 8);
+        }
+        // pass 1: u_e^T = (x_e AT_e^T)^T and v_e^T = (dy_e BT_e^T)^T, bf16
+        GroupSpec sp[kMaxGroupBatch];
+        int n = 0;
+        for (int e = e0; e < e1; ++e) {
+            const int64_t L = off[e + 1] - off[e];
+            if (L == 0) continue;
+            const int64_t Lp = round_up(L, 8);
+            GroupSpec &u = sp[n++];
+            u = GroupSpec{};
+            u.a = d_x + off[e] * din; u.a_rows_ld = din; u.a_rows = L; u.a_k = din;
+            u.b = c.AT + (int64_t)e * c.rpad * din; u.b_rows_ld = din; u.b_rows = c.rpad; u.b_k = din;
+            u.M = (int)L; u.N = c.rpad; u.K = (int)din;
+            u.out = GOUT_T16; u.out16 = c.uT + toff[e - e0]; u.ld = Lp; u.alpha = 1.0f; u.r = c.rpad; u.rpad = c.rpad;
+            GroupSpec &v = sp[n++];
+            v = GroupSpec{};
+            v.a = d_dy + off[e] * d; v.a_rows_ld = d; v.a_rows = L; v.a_k = d;
+            v.b = c.BT + (int64_t)e * c.rpad * d; v.b_rows_ld = d; v.b_rows = c.rpad; v.b_k = d;
+            v.M = (int)L; v.N = c.rpad; v.K = (int)d;
+            v.out = GOUT_T16; v.out16 = c.vT + toff[e - e0]; v.ld = Lp; v.alpha = 1.0f; v.r = c.rpad; v.rpad = c.rpad;
+        }
+        if (n == 0) continue;
+        st = launch_group<false, false, kMaxGroupBatch>(sp, n, BN, c.part, c.tickets, dev, stream, nullptr);
+        if (st != ATTT_OK) return st;
+        // pass 2: dA_e = s x_e^T v_e (x MN-major), dB_e^T = s dy_e^T u_e (dy MN-major)
+        n = 0;
+        for (int e = e0; e < e1; ++e) {
+            const int64_t L = off[e + 1] - off[e];
+            if (L == 0) continue;
+            const int64_t Lp = round_up(L, 8);
+            GroupSpec &a = sp[n++];
+            a = GroupSpec{};
+            a.a = d_x + off[e] * din; a.a_rows_ld = din; a.a_rows = din; a.a_k = L;
+            a.b = c.vT + toff[e - e0]; a.b_rows_ld = Lp; a.b_rows = c.rpad; a.b_k = L;
+            a.M = (int)din; a.N = c.rpad; a.K = (int)L;
+            a.out = GOUT_N32; a.outp[0] = d_dA + (int64_t)e * din * r; a.alpha = scale; a.r = r; a.rpad = c.rpad;
+            GroupSpec &b = sp[n++];
+            b = GroupSpec{};
+            b.a = d_dy + off[e] * d; b.a_rows_ld = d; b.a_rows = d; b.a_k = L;
+            b.b = c.uT + toff[e - e0]; b.b_rows_ld = Lp; b.b_rows = c.rpad; b.b_k = L;
+            b.M = (int)d; b.N = c.rpad; b.K = (int)L;
+            b.out = GOUT_T32; b.out32 = d_dB + (int64_t)e * r * d; b.ld = d; b.alpha = scale; b.r = r;
+            b.rpad = c.rpad;
+        }
+        st = launch_group<true, false, kMaxGroupBatch>(sp, n, BN, c.part, c.tickets, dev, stream, nullptr);
+        if (st != ATTT_OK) return st;
+    }
+    return ATTT_OK;
+}
 
 // ---------------------------------------------------------------------------
 // The adapted projection: forward and input gradient

@@ -25,7 +25,14 @@
 
 namespace attt {
 
+// Problems of one grouped launch at most.  The tensor maps and problems
+// travel in the kernel's parameters, so the capacity is a template argument:
+// kMaxGroup (u and every v of kMaxProj projections, ~3.7 KB) for one group
+// of projections, kMaxGroupBatch (the u and v, or dA and dB, of kGroupEpisodes
+// episodes of a batch, ~14 KB of the 32 KB parameter space) for a batch.
 constexpr int kMaxGroup = kMaxProj + 1;
+constexpr int kGroupEpisodes = 16;
+constexpr int kMaxGroupBatch = 2 * kGroupEpisodes;
 constexpr int kGroupMaxGrid = 256;  // CTAs of a grouped launch at most: partial slots are CTA + tile
 
 // How a problem writes its result D (fp32 accumulator, rows m < M, columns
@@ -53,11 +60,13 @@ struct GroupProblem {
     float *outp[kMaxProj];
 };
 
+template <int NP>
 struct GroupMaps {
-    CUtensorMap a[kMaxGroup];
-    CUtensorMap b[kMaxGroup];
+    CUtensorMap a[NP];
+    CUtensorMap b[NP];
 };
 
+template <int NP>
 struct GroupArgs {
     int nprob;
     int64_t total_stages;  // S; the grid G is at most S, so no CTA's range is empty
@@ -67,7 +76,7 @@ struct GroupArgs {
     int *status;
     float *part;            // partial slots of 128 x BN fp32, [BN / 4][128] float4 each; CTA + tile slots
     unsigned int *tickets;  // one arrival counter per group-wide tile, 0 between launches
-    GroupProblem prob[kMaxGroup];
+    GroupProblem prob[NP];
 };
 
 // One segment of a CTA's stage range: problem q, tile (tm, tn), K blocks
@@ -78,7 +87,8 @@ struct GroupSeg {
 };
 
 // The segment that starts at stage x of a range ending at xend; advances x.
-__device__ __forceinline__ bool group_next(const GroupArgs &g, int64_t &x, int64_t xend, GroupSeg &sg) {
+template <int NP>
+__device__ __forceinline__ bool group_next(const GroupArgs<NP> &g, int64_t &x, int64_t xend, GroupSeg &sg) {
     if (x >= xend) return false;
     int q = 0;
     while (q + 1 < g.nprob && x >= g.prob[q + 1].stage_begin) ++q;
@@ -99,7 +109,8 @@ __device__ __forceinline__ bool group_next(const GroupArgs &g, int64_t &x, int64
 }
 
 // The CTA whose range holds stage x: the largest c with floor(c S / G) <= x.
-__device__ __forceinline__ int64_t group_owner(const GroupArgs &g, int64_t x, int64_t G) {
+template <int NP>
+__device__ __forceinline__ int64_t group_owner(const GroupArgs<NP> &g, int64_t x, int64_t G) {
     return ((x + 1) * G - 1) / g.total_stages;
 }
 
@@ -152,7 +163,8 @@ __device__ __forceinline__ void group_store16(const GroupProblem &p, int m, int 
 }
 
 // Epilogue of one segment, on CTA `cta` of G (four warps, thread = row).
-__device__ __forceinline__ void group_segment_epilogue(const GroupArgs &g, const GroupSeg &sg, int64_t cta, int64_t G,
+template <int NP>
+__device__ __forceinline__ void group_segment_epilogue(const GroupArgs<NP> &g, const GroupSeg &sg, int64_t cta, int64_t G,
                                                        int row, uint32_t taddr) {
     const GroupProblem &p = g.prob[sg.q];
     const int gm = sg.tm * 128 + row;
@@ -228,9 +240,9 @@ __device__ __forceinline__ void group_segment_epilogue(const GroupArgs &g, const
     }
 }
 
-template <bool A_MN, bool B_MN>
+template <bool A_MN, bool B_MN, int NP>
 __global__ void __launch_bounds__(kGemmThreads, 1)
-    tc_gemm_group_kernel(const __grid_constant__ GroupMaps maps, const GroupArgs g) {
+    tc_gemm_group_kernel(const __grid_constant__ GroupMaps<NP> maps, const GroupArgs<NP> g) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = g.stages;
