@@ -564,7 +564,7 @@ typedef struct attt_batch_config {
     int64_t max_history; /* tokens each episode's history may hold              */
     int64_t max_update;  /* largest update text of one episode (<= max_history) */
     int64_t din, d, V;   /* adapted projection [din, d], LM head [V, d]         */
-    int r;               /* adapter rank, 1..64 (a multiple of 8 for dx)        */
+    int r;               /* adapter rank, 1..64                                 */
     float scale, lr;     /* s = alpha / r; SGD rate of Eq. 2                    */
     int grad_steps;      /* gradient steps per update (Appendix C: 2)           */
 } attt_batch_config;
@@ -594,9 +594,11 @@ ATTT_API attt_status attt_batch_reset(attt_batch *b, int e, attt_stream stream);
  * NULL) receives each episode's Eq. 10 loss per step (0 for an episode
  * without rows); d_dx (fp32 [grad_steps, sum lens, din], 16-byte aligned, or
  * NULL) the projection-input gradients.  Eq. 8/9, the dh -> dy cast, the SGD
- * step and the history append each run as one launch for the whole batch
- * and Eq. 10 as one call over every row; the adapter contractions run per
- * episode.  ATTT_ERR_CAPACITY (nothing launched) if an episode's history
+ * step and the history append each run as one launch for the whole batch,
+ * Eq. 10 as one call over every row, the projection forward and dx as one
+ * contraction each over every row, and the adapter gradients as one grouped
+ * launch per pass (16 episodes per launch).  ATTT_ERR_CAPACITY (nothing
+ * launched) if an episode's history
  * would exceed max_history.  Async on `stream`.
  */
 ATTT_API attt_status attt_batch_update(attt_batch *b, const int32_t *d_tokens, const attt_bf16 *d_x,

@@ -68,17 +68,26 @@ attt_status ce_fwd_bwd_run(const attt_bf16 *d_h, const attt_bf16 *d_W, const int
 // The largest Eq. 10 workspace over every row count up to Lmax (ce.cu).
 size_t ce_workspace_bound(int64_t Lmax, int64_t d, int64_t V);
 
-// The adapter gradients of E episodes of a batch (lora.cu): episode e owns
+// The adapted projections of E episodes of a batch (lora.cu): episode e owns
 // rows [off[e], off[e+1]) of the stacked x [*, din] and dy [*, d] (off: host
-// array) and slot e of the stacked adapters A16 [E][din][r], B16 [E][r][d] and
-// gradients dA [E][din][r], dB [E][r][d] (slots of episodes without rows are
-// left as they are).  rows_bound >= sum_e round_up(L_e, 8) sizes the
-// workspace (lora_grad_batch_workspace).
-size_t lora_grad_batch_workspace(int E, int64_t rows_bound, int64_t din, int64_t d, int r);
-attt_status lora_grad_batch_run(const attt_bf16 *d_x, const attt_bf16 *d_dy, const int64_t *off, int E, int64_t din,
-                                int64_t d, int r, float scale, const attt_bf16 *d_A16, const attt_bf16 *d_B16,
-                                float *d_dA, float *d_dB, int64_t rows_bound, void *d_ws, size_t ws_bytes,
-                                cudaStream_t stream);
+// array of E + 1) and slot e of the stacked adapters A16 [E][din][r], B16
+// [E][r][d] and gradients dA [E][din][r], dB [E][r][d] (slots of episodes
+// without rows are left as they are).  rows_bound >= sum_e round_up(L_e, 8)
+// sizes the workspace.  batch_adapter_prep (the current adapters) comes first;
+// forward (h bf16 [R, d]), grads and input_grad (dx fp32 [R, din]) then read
+// what it wrote.
+size_t batch_adapter_workspace(int E, int64_t rows_bound, int64_t din, int64_t d, int r);
+attt_status batch_adapter_prep(const attt_bf16 *d_A16, const attt_bf16 *d_B16, int E, int64_t din, int64_t d, int r,
+                               int64_t rows_bound, void *d_ws, size_t ws_bytes, cudaStream_t stream);
+attt_status batch_forward(const attt_bf16 *d_x, const int64_t *off, int E, const attt_bf16 *d_W0, int64_t din,
+                          int64_t d, int r, float scale, attt_bf16 *d_h, int64_t rows_bound, void *d_ws,
+                          size_t ws_bytes, cudaStream_t stream);
+attt_status batch_grads(const attt_bf16 *d_x, const attt_bf16 *d_dy, const int64_t *off, int E, int64_t din,
+                        int64_t d, int r, float scale, float *d_dA, float *d_dB, int64_t rows_bound, void *d_ws,
+                        size_t ws_bytes, cudaStream_t stream);
+attt_status batch_input_grad(const attt_bf16 *d_dy, const int64_t *off, int E, const attt_bf16 *d_W0, int64_t din,
+                             int64_t d, int r, float scale, float *d_dx, int64_t rows_bound, void *d_ws,
+                             size_t ws_bytes, cudaStream_t stream);
 
 // Device address of attt_lora_grad_noalloc's static status word on `dev`, or
 // nullptr if that entry point has not been set up on the device.

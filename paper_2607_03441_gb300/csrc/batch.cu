@@ -8,13 +8,14 @@
 // for an episode without an update this round):
 //   w, 1/L_e    one launch over every episode (each against its own history)
 //   grad_steps times:
-//     h_e = x_e W0 + s (x_e A_e) B_e           per episode (attt_lora_forward)
+//     h_e = x_e W0 + s (x_e A_e) B_e           one contraction over every row
+//                                              (block-diagonal adapter terms)
 //     loss_e, dh  Eq. 10 over every row in one call (the LM head is shared),
 //                 each row with its own episode's 1/L_e; loss_e from the rows'
 //                 NLL in a fixed order
 //     dy = bf16(dh)                            one launch
 //     dA_e, dB_e                               one grouped launch per pass (16 episodes each)
-//     dx_e                                     per episode (if asked)
+//     dx_e                                     one contraction over every row (if asked)
 //     A, B <- A - lr dA, B - lr dB             one launch over every adapter
 //   H_e <- H_e || x_e                          one launch over every history
 // The adapters live stacked (A [E][din][r], B [E][r][d]), so the SGD step of
@@ -37,8 +38,10 @@ struct attt_batch {
     attt_bf16 *A16, *B16;
     float *w, *rowscale, *nll, *dh, *loss_scratch;
     attt_bf16 *h, *dy;
-    void *ws;
+    void *ws;   // Eq. 10's workspace
     size_t ws_bytes;
+    void *aws;  // the adapted projections' workspace (kept across Eq. 10 within a step)
+    size_t aws_bytes;
 };
 
 namespace {
@@ -57,7 +60,7 @@ void free_all(attt_batch *b) {
     for (attt_history *h : b->hist)
         if (h) attt_history_destroy(h);
     void *bufs[] = {b->A32, b->B32, b->A0, b->B0, b->dA, b->dB, b->A16, b->B16, b->w, b->rowscale,
-                    b->nll, b->dh, b->loss_scratch, b->h, b->dy, b->ws};
+                    b->nll, b->dh, b->loss_scratch, b->h, b->dy, b->ws, b->aws};
     for (void *p : bufs) cudaFree(p);
 }
 
@@ -130,17 +133,11 @@ attt_status attt_batch_create(const attt_batch_config *cfg, const attt_bf16 *d_W
     const int E = c.episodes;
     const int64_t rows = (int64_t)E * c.max_update;
     const size_t nA = (size_t)c.din * c.r, nB = (size_t)c.r * c.d;
-    // one workspace for the calls of an update (they run in order on the
-    // stream): Eq. 10 over up to E max_update rows (its bound taken over every
-    // row count, since its vocabulary chunk depends on it), the per-episode
-    // adapter calls over up to max_update rows
-    size_t ws = ce_workspace_bound(rows, c.d, c.V);
-    const size_t per_ep[] = {lora_grad_batch_workspace(E, rows + 8 * E, c.din, c.d, c.r),
-                             attt_lora_forward_workspace_bytes(c.max_update, c.din, c.d, c.r),
-                             attt_lora_input_grad_workspace_bytes(c.max_update, c.din, c.d, c.r)};
-    for (size_t v : per_ep)
-        if (v > ws) ws = v;
-    b->ws_bytes = ws;
+    // Eq. 10 over up to E max_update rows (its bound taken over every row
+    // count, since its vocabulary chunk depends on it); the adapted
+    // projections' own workspace for up to E max_update rows
+    b->ws_bytes = ce_workspace_bound(rows, c.d, c.V);
+    b->aws_bytes = batch_adapter_workspace(E, rows + 8 * E, c.din, c.d, c.r);
     b->hist.assign(E, nullptr);
     bool ok = true;
     for (int e = 0; e < E && ok; ++e) ok = attt_history_create(c.n, c.max_history, &b->hist[e]) == ATTT_OK;
@@ -150,7 +147,8 @@ attt_status attt_batch_create(const attt_batch_config *cfg, const attt_bf16 *d_W
          dev_alloc(&b->rowscale, (size_t)rows) && dev_alloc(&b->nll, (size_t)rows) &&
          dev_alloc(&b->dh, (size_t)rows * c.d) && dev_alloc(&b->loss_scratch, (size_t)E * c.grad_steps + 1) &&
          dev_alloc(&b->h, (size_t)rows * c.d) && dev_alloc(&b->dy, (size_t)rows * c.d) &&
-         dev_alloc(reinterpret_cast<char **>(&b->ws), b->ws_bytes);
+         dev_alloc(reinterpret_cast<char **>(&b->ws), b->ws_bytes) &&
+         dev_alloc(reinterpret_cast<char **>(&b->aws), b->aws_bytes);
     if (ok)
         ok = cudaMemcpy(b->A0, d_A0, nA * sizeof(float), cudaMemcpyDeviceToDevice) == cudaSuccess &&
              cudaMemcpy(b->B0, d_B0, nB * sizeof(float), cudaMemcpyDeviceToDevice) == cudaSuccess &&
@@ -201,20 +199,19 @@ attt_status attt_batch_update(attt_batch *b, const int32_t *d_tokens, const attt
     const int64_t R = off[E];
     if (R == 0) return ATTT_OK;
     if (!d_tokens || !d_x || !aligned16(d_x) || (d_dx && !aligned16(d_dx))) return ATTT_ERR_INVALID_ARG;
-    if (d_dx && c.r % 8 != 0) return ATTT_ERR_UNSUPPORTED;
     int dev;
     attt_status st = current_device(&dev);
     if (st != ATTT_OK) return st;
     const size_t nA = (size_t)c.din * c.r, nB = (size_t)c.r * c.d;
-    const int64_t rows = (int64_t)E * c.max_update;  // the row bound the workspace was sized for
+    const int64_t rb = (int64_t)E * c.max_update + 8 * E;  // the row bound the adapter workspace was sized for
     float *losses = d_losses ? d_losses : b->loss_scratch;
 
     st = ngram_weights_batch(b->hist.data(), E, d_tokens, off, c.w_min, b->w, b->rowscale, stream);
     for (int g = 0; g < c.grad_steps && st == ATTT_OK; ++g) {
-        for (int e = 0; e < E && st == ATTT_OK; ++e)
-            if (lens[e] > 0)
-                st = attt_lora_forward(d_x + off[e] * c.din, b->W0, b->A16 + e * nA, b->B16 + e * nB, lens[e], c.din,
-                                       c.d, c.r, c.scale, b->h + off[e] * c.d, b->ws, b->ws_bytes, stream);
+        // every episode's current adapter padded and stacked, then h for every row
+        st = batch_adapter_prep(b->A16, b->B16, E, c.din, c.d, c.r, rb, b->aws, b->aws_bytes, stream);
+        if (st == ATTT_OK)
+            st = batch_forward(d_x, off, E, b->W0, c.din, c.d, c.r, c.scale, b->h, rb, b->aws, b->aws_bytes, stream);
         if (st == ATTT_OK)
             st = ce_fwd_bwd_run(b->h, b->Wlm, d_tokens, b->w, b->rowscale, R, c.d, c.V, b->loss_scratch + E * c.grad_steps,
                                 b->dh, nullptr, b->nll, b->ws, b->ws_bytes, stream);
@@ -229,14 +226,11 @@ attt_status attt_batch_update(attt_batch *b, const int32_t *d_tokens, const attt
             st = ATTT_ERR_CUDA;
         // every episode's adapter gradients: one grouped launch per pass
         if (st == ATTT_OK)
-            st = lora_grad_batch_run(d_x, b->dy, off, E, c.din, c.d, c.r, c.scale, b->A16, b->B16, b->dA, b->dB,
-                                     rows + 8 * E, b->ws, b->ws_bytes, stream);
-        for (int e = 0; e < E && st == ATTT_OK && d_dx; ++e) {
-            if (lens[e] == 0) continue;
-            st = attt_lora_input_grad(b->dy + off[e] * c.d, b->W0, b->A16 + e * nA, b->B16 + e * nB, lens[e], c.din,
-                                      c.d, c.r, c.scale, d_dx + ((size_t)g * R + off[e]) * c.din, b->ws,
-                                      b->ws_bytes, stream);
-        }
+            st = batch_grads(d_x, b->dy, off, E, c.din, c.d, c.r, c.scale, b->dA, b->dB, rb, b->aws, b->aws_bytes,
+                             stream);
+        if (st == ATTT_OK && d_dx)
+            st = batch_input_grad(b->dy, off, E, b->W0, c.din, c.d, c.r, c.scale, d_dx + (size_t)g * R * c.din, rb,
+                                  b->aws, b->aws_bytes, stream);
         // every adapter of the batch in one step: A as [E din, r], B as [r, E d]
         if (st == ATTT_OK)
             st = attt_lora_step(b->A32, b->B32, b->dA, b->dB, (int64_t)E * c.din, (int64_t)E * c.d, c.r, c.lr, b->A16,

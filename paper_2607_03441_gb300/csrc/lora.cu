@@ -397,19 +397,36 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
 
 
 // ---------------------------------------------------------------------------
-// The adapter gradients of a batch of episodes (attt_batch_update): each
-// episode has its own rows of the stacked x and dy and its own adapter, and
-// the u, v (pass 1) and dA, dB (pass 2) of up to kGroupEpisodes episodes run as
-// the problems of one grouped launch each.
+// The adapted projections of a batch of episodes (attt_batch_update): each
+// episode has its own rows of the stacked x and dy and its own adapter.
+//   prep      every episode's A^T and B padded to rpad rows (stacked by
+//             episode), and A concatenated along the rank, [din, E rpad];
+//   forward   h = [x | S] [W0 ; B_all] over every row in one contraction, S
+//             block-diagonal: row j of episode e holds s (x_j A_e) in columns
+//             [e rpad, (e + 1) rpad) and zeros elsewhere (a grouped pass with one
+//             problem per episode writes the blocks);
+//   grads     u, v (pass 1) and dA, dB (pass 2) of up to kGroupEpisodes
+//             episodes as the problems of one grouped launch each;
+//   dx        [dy | S'] [W0^T ; A_cat^T] in one contraction, S' block-diagonal
+//             with s (dy_j B_e^T).
+// Every episode's rpad values fall in one 16-deep MMA step of the adapter
+// part of K and the other episodes' blocks add exact zeros, so each row's h
+// and dx are those of the episode's own call.
 // ---------------------------------------------------------------------------
+
+// Split slots of the dx contraction's tail split (as for the CE's dh).
+constexpr int kDxSplitRegions = 160;
 
 struct BatchLoraLayout {
     int rpad;
-    __nv_bfloat16 *AT, *BT;    // [E rpad, din], [E rpad, d]: episode e's rows at e rpad
-    __nv_bfloat16 *uT, *vT;    // per episode [rpad, Lp_e], laid one after another
+    int64_t Ncat;                   // E rpad
+    __nv_bfloat16 *AT, *BT;         // [E rpad, din], [E rpad, d]: episode e's rows at e rpad
+    __nv_bfloat16 *ACAT;            // [din, E rpad]
+    __nv_bfloat16 *uT, *vT;         // per episode [rpad, Lp_e], laid one after another
+    __nv_bfloat16 *S;               // [rows_bound, E rpad] block-diagonal s u or s v
     int64_t tiles;
-    unsigned int *tickets;
-    float *part;
+    unsigned int *tickets;          // [tiles + kDxSplitRegions]
+    float *part, *split_ws;
     size_t bytes;
 };
 
@@ -417,30 +434,34 @@ struct BatchLoraLayout {
 static BatchLoraLayout batch_lora_layout(void *ws, int E, int64_t rows_bound, int64_t din, int64_t d, int r) {
     BatchLoraLayout c{};
     c.rpad = (int)round_up(r, 16);
+    c.Ncat = (int64_t)E * c.rpad;
     const int64_t t1 = 2 * (cdiv(rows_bound, 128) + E), t2 = (int64_t)E * (cdiv(din, 128) + cdiv(d, 128));
     c.tiles = t1 > t2 ? t1 : t2;
     Carve cv{static_cast<char *>(ws), 0};
-    c.AT = cv.take<__nv_bfloat16>((size_t)E * c.rpad * din);
-    c.BT = cv.take<__nv_bfloat16>((size_t)E * c.rpad * d);
+    c.AT = cv.take<__nv_bfloat16>((size_t)c.Ncat * din);
+    c.BT = cv.take<__nv_bfloat16>((size_t)c.Ncat * d);
+    c.ACAT = cv.take<__nv_bfloat16>((size_t)din * c.Ncat);
     c.uT = cv.take<__nv_bfloat16>((size_t)c.rpad * rows_bound);
     c.vT = cv.take<__nv_bfloat16>((size_t)c.rpad * rows_bound);
-    c.tickets = cv.take<unsigned int>((size_t)c.tiles);
+    c.S = cv.take<__nv_bfloat16>((size_t)rows_bound * c.Ncat);
+    c.tickets = cv.take<unsigned int>((size_t)(c.tiles + kDxSplitRegions));
     c.part = cv.take<float>((size_t)(c.tiles + kGroupMaxGrid) * 128 * c.rpad);
+    c.split_ws = cv.take<float>((size_t)kDxSplitRegions * 128 * 256);
     c.bytes = (size_t)round_up((int64_t)cv.used, 256);
     return c;
 }
 
 struct BatchPrepArgs {
     const __nv_bfloat16 *A, *B;  // stacked [E][din][r], [E][r][d]
-    __nv_bfloat16 *AT, *BT;
+    __nv_bfloat16 *AT, *BT, *ACAT;
     int r, rpad;
-    int64_t din, d;
+    int64_t din, d, Ncat;
     unsigned int *tickets;
     int64_t ntickets;
 };
 
-// As lora_prep_kernel, for episode e = blockIdx.y of a batch's stacked
-// adapters: AT[e rpad + c, i] = A_e[i, c], BT[e rpad + c, o] = B_e[c, o]
+// For episode e = blockIdx.y of a batch's stacked adapters: AT[e rpad + c, i]
+// = A_e[i, c], ACAT[i, e rpad + c] = A_e[i, c], BT[e rpad + c, o] = B_e[c, o]
 // (zero for c >= r), and the tickets zeroed (each episode row a slice).
 __global__ void __launch_bounds__(256) lora_prep_batch_kernel(BatchPrepArgs a) {
     __shared__ __nv_bfloat16 slab[kPrepRows][64 + 2];
@@ -463,6 +484,10 @@ __global__ void __launch_bounds__(256) lora_prep_batch_kernel(BatchPrepArgs a) {
             const int c = i / kPrepRows, kk = i - c * kPrepRows;
             if (kk < rows) AT[(int64_t)c * a.din + k0 + kk] = c < a.r ? slab[kk][c] : __float2bfloat16_rn(0.f);
         }
+        for (int i = threadIdx.x; i < rows * a.rpad; i += blockDim.x) {
+            const int kk = i / a.rpad, c = i - kk * a.rpad;
+            a.ACAT[(k0 + kk) * a.Ncat + (int64_t)e * a.rpad + c] = c < a.r ? slab[kk][c] : __float2bfloat16_rn(0.f);
+        }
         __syncthreads();
     }
     const int64_t nB = (int64_t)a.rpad * a.d;
@@ -477,35 +502,106 @@ __global__ void __launch_bounds__(256) lora_prep_batch_kernel(BatchPrepArgs a) {
     }
 }
 
-size_t lora_grad_batch_workspace(int E, int64_t rows_bound, int64_t din, int64_t d, int r) {
+size_t batch_adapter_workspace(int E, int64_t rows_bound, int64_t din, int64_t d, int r) {
     return batch_lora_layout(nullptr, E, rows_bound, din, d, r).bytes;
 }
 
-attt_status lora_grad_batch_run(const attt_bf16 *d_x, const attt_bf16 *d_dy, const int64_t *off, int E, int64_t din,
-                                int64_t d, int r, float scale, const attt_bf16 *d_A16, const attt_bf16 *d_B16,
-                                float *d_dA, float *d_dB, int64_t rows_bound, void *d_ws, size_t ws_bytes,
-                                cudaStream_t stream) {
+static attt_status batch_check(int E, int64_t din, int64_t d, int r, int64_t rows_bound, size_t ws_bytes,
+                               const void *ws) {
     if (E < 1 || r < 1 || r > 64 || din < 8 || d < 8 || din % 8 || d % 8) return ATTT_ERR_INVALID_ARG;
-    if (!d_ws || ws_bytes < lora_grad_batch_workspace(E, rows_bound, din, d, r)) return ATTT_ERR_WORKSPACE;
+    if (!ws || !aligned256(ws) || ws_bytes < batch_adapter_workspace(E, rows_bound, din, d, r))
+        return ATTT_ERR_WORKSPACE;
+    return ATTT_OK;
+}
+
+attt_status batch_adapter_prep(const attt_bf16 *d_A16, const attt_bf16 *d_B16, int E, int64_t din, int64_t d, int r,
+                               int64_t rows_bound, void *d_ws, size_t ws_bytes, cudaStream_t stream) {
+    attt_status st = batch_check(E, din, d, r, rows_bound, ws_bytes, d_ws);
+    if (st != ATTT_OK) return st;
     int dev;
-    attt_status st = current_device(&dev);
+    st = current_device(&dev);
+    if (st != ATTT_OK) return st;
+    BatchLoraLayout c = batch_lora_layout(d_ws, E, rows_bound, din, d, r);
+    BatchPrepArgs a{};
+    a.A = reinterpret_cast<const __nv_bfloat16 *>(d_A16);
+    a.B = reinterpret_cast<const __nv_bfloat16 *>(d_B16);
+    a.AT = c.AT; a.BT = c.BT; a.ACAT = c.ACAT; a.r = r; a.rpad = c.rpad; a.din = din; a.d = d; a.Ncat = c.Ncat;
+    a.tickets = c.tickets; a.ntickets = c.tiles + kDxSplitRegions;
+    int64_t maxn = cdiv(din, kPrepRows) * 256;
+    if (c.rpad * d > maxn) maxn = c.rpad * d;
+    if (cdiv(a.ntickets, E) > maxn) maxn = cdiv(a.ntickets, E);
+    lora_prep_batch_kernel<<<dim3(grid_for(maxn, 256, dev), (unsigned)E), 256, 0, stream>>>(a);
+    count_launch();
+    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+}
+
+// S = block-diagonal alpha (rows_e M_e) for M_e = AT_e (mats = c.AT, K = din,
+// src = x) or BT_e (mats = c.BT, K = d, src = dy): zeroed, then one grouped
+// launch per kGroupEpisodes episodes writes the diagonal blocks.
+static attt_status batch_blockdiag(const BatchLoraLayout &c, const attt_bf16 *src, int64_t K,
+                                   const __nv_bfloat16 *mats, const int64_t *off, int E, float alpha, int dev,
+                                   cudaStream_t stream) {
+    if (cudaMemsetAsync(c.S, 0, (size_t)off[E] * c.Ncat * sizeof(__nv_bfloat16), stream) != cudaSuccess)
+        return ATTT_ERR_CUDA;
+    for (int e0 = 0; e0 < E; e0 += kMaxGroupBatch) {
+        const int e1 = e0 + kMaxGroupBatch < E ? e0 + kMaxGroupBatch : E;
+        GroupSpec sp[kMaxGroupBatch];
+        int n = 0;
+        for (int e = e0; e < e1; ++e) {
+            const int64_t L = off[e + 1] - off[e];
+            if (L == 0) continue;
+            GroupSpec &u = sp[n++];
+            u = GroupSpec{};
+            u.a = src + off[e] * K; u.a_rows_ld = K; u.a_rows = L; u.a_k = K;
+            u.b = mats + (int64_t)e * c.rpad * K; u.b_rows_ld = K; u.b_rows = c.rpad; u.b_k = K;
+            u.M = (int)L; u.N = c.rpad; u.K = (int)K;
+            u.out = GOUT_N16; u.out16 = c.S + off[e] * c.Ncat + (int64_t)e * c.rpad; u.ld = c.Ncat;
+            u.alpha = alpha; u.r = c.rpad; u.rpad = c.rpad;
+        }
+        if (n == 0) continue;
+        attt_status st = launch_group<false, false, kMaxGroupBatch>(sp, n, c.rpad, c.part, c.tickets, dev, stream,
+                                                                    nullptr);
+        if (st != ATTT_OK) return st;
+    }
+    return ATTT_OK;
+}
+
+attt_status batch_forward(const attt_bf16 *d_x, const int64_t *off, int E, const attt_bf16 *d_W0, int64_t din,
+                          int64_t d, int r, float scale, attt_bf16 *d_h, int64_t rows_bound, void *d_ws,
+                          size_t ws_bytes, cudaStream_t stream) {
+    attt_status st = batch_check(E, din, d, r, rows_bound, ws_bytes, d_ws);
+    if (st != ATTT_OK) return st;
+    const int64_t R = off[E];
+    if (R == 0) return ATTT_OK;
+    int dev;
+    st = current_device(&dev);
+    if (st != ATTT_OK) return st;
+    BatchLoraLayout c = batch_lora_layout(d_ws, E, rows_bound, din, d, r);
+    st = batch_blockdiag(c, d_x, din, c.AT, off, E, scale, dev, stream);
+    if (st != ATTT_OK) return st;
+    // h = [x | S] [W0 ; BT]: W0 [din, d] and the padded B rows [E rpad, d] read MN-major
+    GemmProblem p{};
+    p.a = d_x; p.a_rows_ld = din; p.a_rows = R; p.a_k = din;
+    p.b = d_W0; p.b_rows_ld = d; p.b_rows = d; p.b_k = din;
+    p.a2 = c.S; p.a2_rows_ld = c.Ncat; p.a2_rows = R; p.a2_k = c.Ncat;
+    p.b2 = c.BT; p.b2_rows_ld = d; p.b2_rows = d; p.b2_k = c.Ncat;
+    p.M = (int)R; p.N = (int)d; p.K = (int)din; p.K2 = (int)c.Ncat; p.BN = 256; p.pair = R > 128;
+    p.pdl = true;
+    EpiParams ep{};
+    ep.out16 = reinterpret_cast<__nv_bfloat16 *>(d_h); ep.out_ld = d; ep.alpha = 1.0f;
+    return launch_gemm<EPI_BF16, false, true>(p, ep, dev, stream);
+}
+
+attt_status batch_grads(const attt_bf16 *d_x, const attt_bf16 *d_dy, const int64_t *off, int E, int64_t din,
+                        int64_t d, int r, float scale, float *d_dA, float *d_dB, int64_t rows_bound, void *d_ws,
+                        size_t ws_bytes, cudaStream_t stream) {
+    attt_status st = batch_check(E, din, d, r, rows_bound, ws_bytes, d_ws);
+    if (st != ATTT_OK) return st;
+    int dev;
+    st = current_device(&dev);
     if (st != ATTT_OK) return st;
     BatchLoraLayout c = batch_lora_layout(d_ws, E, rows_bound, din, d, r);
     const int BN = c.rpad;
-    {
-        BatchPrepArgs a{};
-        a.A = reinterpret_cast<const __nv_bfloat16 *>(d_A16);
-        a.B = reinterpret_cast<const __nv_bfloat16 *>(d_B16);
-        a.AT = c.AT; a.BT = c.BT; a.r = r; a.rpad = c.rpad; a.din = din; a.d = d;
-        a.tickets = c.tickets; a.ntickets = c.tiles;
-        int64_t maxn = cdiv(din, kPrepRows) * 256;
-        if (c.rpad * d > maxn) maxn = c.rpad * d;
-        if (cdiv(c.tiles, E) > maxn) maxn = cdiv(c.tiles, E);
-        lora_prep_batch_kernel<<<dim3(grid_for(maxn, 256, dev), (unsigned)E), 256, 0, stream>>>(a);
-        count_launch();
-        if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
-    }
-    // each episode's place in uT / vT
     int64_t toff[kGroupEpisodes] = {0};
     for (int e0 = 0; e0 < E; e0 += kGroupEpisodes) {
         const int e1 = e0 + kGroupEpisodes < E ? e0 + kGroupEpisodes : E;
@@ -563,12 +659,37 @@ attt_status lora_grad_batch_run(const attt_bf16 *d_x, const attt_bf16 *d_dy, con
     return ATTT_OK;
 }
 
+attt_status batch_input_grad(const attt_bf16 *d_dy, const int64_t *off, int E, const attt_bf16 *d_W0, int64_t din,
+                             int64_t d, int r, float scale, float *d_dx, int64_t rows_bound, void *d_ws,
+                             size_t ws_bytes, cudaStream_t stream) {
+    attt_status st = batch_check(E, din, d, r, rows_bound, ws_bytes, d_ws);
+    if (st != ATTT_OK) return st;
+    const int64_t R = off[E];
+    if (R == 0) return ATTT_OK;
+    int dev;
+    st = current_device(&dev);
+    if (st != ATTT_OK) return st;
+    BatchLoraLayout c = batch_lora_layout(d_ws, E, rows_bound, din, d, r);
+    st = batch_blockdiag(c, d_dy, d, c.BT, off, E, scale, dev, stream);
+    if (st != ATTT_OK) return st;
+    // dx = [dy | S'] [W0^T ; A_cat^T]: W0 [din, d] and A_cat [din, E rpad] read K-major
+    GemmProblem p{};
+    p.a = d_dy; p.a_rows_ld = d; p.a_rows = R; p.a_k = d;
+    p.b = d_W0; p.b_rows_ld = d; p.b_rows = din; p.b_k = d;
+    p.a2 = c.S; p.a2_rows_ld = c.Ncat; p.a2_rows = R; p.a2_k = c.Ncat;
+    p.b2 = c.ACAT; p.b2_rows_ld = c.Ncat; p.b2_rows = din; p.b2_k = c.Ncat;
+    p.M = (int)R; p.N = (int)din; p.K = (int)d; p.K2 = (int)c.Ncat; p.BN = 256; p.pair = R > 128;
+    p.pdl = true;
+    p.split_ws = c.split_ws; p.split_tick = c.tickets + c.tiles; p.split_regions = kDxSplitRegions;
+    EpiParams ep{};
+    ep.out = d_dx; ep.out_ld = din; ep.accumulate = 0; ep.alpha = 1.0f;
+    return launch_gemm<EPI_F32_ACC, false, false>(p, ep, dev, stream);
+}
+
 // ---------------------------------------------------------------------------
 // The adapted projection: forward and input gradient
 // ---------------------------------------------------------------------------
 
-// Split slots of the dx contraction's tail split (as for the CE's dh).
-constexpr int kDxSplitRegions = 160;
 
 struct ProjLayout {
     int rpad;
