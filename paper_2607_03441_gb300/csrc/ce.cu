@@ -31,6 +31,8 @@ constexpr int kChunkRows = 32;
 // fp32 partials of 128 x kCeBN (128 KB each) for the tail split of the dh
 // contraction: enough for every CTA of a 160-SM part to hold one piece.
 constexpr int kCeSplitRegions = 160;
+// Bound of the chunk's bf16 block E [L, Vc] in bytes.
+constexpr int64_t kCeEBytes = 1024ll << 20;
 
 struct CeLayout {
     int64_t nvt, Vc, nblk;
@@ -46,11 +48,11 @@ struct CeLayout {
 };
 
 // Upper bound of the vocab chunk: the chunk's bf16 block E (L x Vc) is kept
-// near 256 MB, so the workspace stays bounded whatever V is.  Each chunk costs
+// near kCeEBytes (1 GB), so the workspace stays bounded whatever V is.  Each chunk costs
 // about 20 us of launch, ramp and tail on top of its FLOPs, and E is streamed
 // once from L2 or HBM either way, so wider chunks are faster up to this bound.
 static int64_t ce_chunk_max(int64_t L, int64_t V) {
-    int64_t vc = (256ll << 20) / (2 * L);
+    int64_t vc = kCeEBytes / (2 * L);
     vc = (vc / kCeBN) * kCeBN;
     if (vc < 4096) vc = 4096;
     if (vc > kCeMaxTiles * kCeBN) vc = kCeMaxTiles * kCeBN;
@@ -336,12 +338,12 @@ namespace attt {
 // The largest attt_ce_workspace_bytes(L, d, V) over 1 <= L <= Lmax.  The
 // workspace grows with L while the vocabulary chunk Vc stays the same, and Vc
 // (a multiple of kCeBN, clamped to [4096, kCeMaxTiles kCeBN] and to V) only
-// changes where 256 MB / (2 L) crosses a multiple of kCeBN, so the maximum is
+// changes where kCeEBytes / (2 L) crosses a multiple of kCeBN, so the maximum is
 // at Lmax or at the last L of one of those ranges.
 size_t ce_workspace_bound(int64_t Lmax, int64_t d, int64_t V) {
     if (Lmax < 1) return 0;
     size_t best = attt_ce_workspace_bytes(Lmax, d, V);
-    const int64_t budget = (256ll << 20) / 2;
+    const int64_t budget = kCeEBytes / 2;
     for (int64_t vc = kCeBN; vc <= kCeMaxTiles * kCeBN; vc += kCeBN) {
         const int64_t L = budget / vc;  // the last L whose unclamped chunk is at least vc
         for (int64_t c = L - 1; c <= L + 1; ++c)
