@@ -170,3 +170,33 @@ def test_7b_shapes_batch_equals_episodes(attt):
         ep.close()
     assert attt.attt_device_status() == 0
     b.close()
+
+
+def test_batch_of_twenty_episodes(attt):
+    """20 episodes: the adapter gradients run as two grouped launches per pass
+    (16 episodes each at most); every episode against the oracle."""
+    E = 20
+    base, eps, dense = _episodes(E if E <= 6 else 6)
+    # 20 episodes from 6 generated ones, with their lengths cut apart
+    eps = [dict(eps[e % 6], cut=min(eps[e % 6]["texts"][0].size, base.L - 9 * e)) for e in range(E)]
+    b = _batch(attt, base, [{"H": ep["H"]} for ep in eps], dense, E)
+    lens = [ep["cut"] for ep in eps]
+    toks = np.concatenate([ep["texts"][0][:n] for ep, n in zip(eps, lens)])
+    xs = np.concatenate([ep["xs"][0][:n] for ep, n in zip(eps, lens)])
+    losses = torch.empty(E, base.grad_steps, dtype=torch.float32, device=DEV)
+    R = int(sum(lens))
+    dx = torch.empty(base.grad_steps, R, base.din, dtype=torch.float32, device=DEV)
+    b.update(i32_dev(toks), bf16_dev(xs), lens, losses=losses, dx=dx)
+    off = np.concatenate([[0], np.cumsum(lens)])
+    for e in (0, 7, 15, 16, 19):     # both launches of each pass, and their edges
+        ep = eps[e]
+        ref = oracle.episode_update(ep["H"], ep["texts"][0][:lens[e]], ep["xs"][0][:lens[e]], dense["W0"],
+                                    dense["W"], dense["A0"], dense["B0"], n=base.n, w_min=base.w_min,
+                                    scale=base.scale, lr=LR, grad_steps=base.grad_steps)
+        np.testing.assert_allclose(losses[e].cpu().numpy(), ref["losses"], rtol=1e-3)
+        A, B = (t.cpu().numpy() for t in b.read_adapter(e))
+        assert rel_l2(A - dense["A0"], ref["A32"] - dense["A0"]) < 2e-2, e
+        assert rel_l2(B - dense["B0"], ref["B32"] - dense["B0"]) < 2e-2, e
+        assert rel_l2(dx[1, off[e]:off[e + 1]].cpu().numpy(), ref["dx"][1]) < 2e-2, e
+    assert attt.attt_device_status() == 0
+    b.close()
