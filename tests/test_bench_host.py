@@ -1,0 +1,43 @@
+"""Host-side logic of bench.py (no GPU): the clock summary, the agent-step
+split of an update, the algorithmic work of each row, the replica
+throughput."""
+import bench
+from paper_2607_03441_gb300 import workloads as wk
+
+
+def test_clock_summary():
+    lines = ["0, 2070, 2070, 900.1, 0x0, Not Active, Not Active, Not Active, Not Active\n",
+             "0, 1500, 2070, 1400.0, 0x4, Not Active, Not Active, Not Active, Active\n",
+             "0, 1800, 2070, 1300.0, 0x0, Not Active, Not Active, Not Active, Not Active\n",
+             "garbage\n"]
+    out = bench.ClockSampler.summarize(lines)
+    assert out == {"sm_mhz": 1800.0, "sm_max_mhz": 2070.0, "samples": 3, "reasons": ["sw_power_cap"]}
+    assert bench.ClockSampler.summarize([]) is None
+
+
+def test_agent_cuts_split_an_update_evenly():
+    for L, K in ((2048, 5), (256, 3), (7, 5), (5, 5)):
+        cuts = bench._agent_cuts(L, K)
+        assert len(cuts) == K + 1 and cuts[0] == 0 and cuts[-1] == L
+        steps = [b - a for a, b in zip(cuts, cuts[1:])]
+        assert min(steps) >= 0 and max(steps) - min(steps) <= 1
+
+
+def test_work_accounting():
+    wl = wk.WORKLOADS["7b"]
+    work = bench.row_work(wl)
+    assert work["weighted_ce_fwd_bwd"] == ("tensor", 4.0 * 2048 * 152064 * 3584, "FLOP")
+    # LoRA bytes: x once, every dy once, adapters in and gradients out
+    x = 2 * 2048 * 3584
+    dys = 2 * 2048 * (3584 + 512)
+    ad = 6 * 3584 * 16 * 2 + 6 * 16 * (3584 + 512)
+    assert work["lora_grad"] == ("hbm", x + dys + ad, "B")
+    ew = wk.EPISODES["7b-episode"]
+    L, V, d = ew.L, ew.V, ew.d
+    per_step = 4.0 * L * V * d + 2 * (2.0 * L * d * d + 2.0 * L * 16 * 2 * d) + 4.0 * L * 16 * 2 * d
+    assert bench.episode_flops(ew) == 2 * per_step
+
+
+def test_replica_throughput():
+    # 4 replicas, 10 steps of 2,048 tokens in 50 ms: 1.6384 M tokens/s
+    assert abs(bench.replica_throughput(2048, 10, 4, 50.0) - 1638400.0) < 1e-6
