@@ -22,7 +22,7 @@ def lib_path():
     return build.build()
 
 
-def test_header_declares_north_star_calls():
+def test_header_declares_the_update_calls():
     names = declared_symbols()
     for must in ("attt_history_insert", "attt_ngram_weights", "attt_weighted_ce_fwd_bwd", "attt_lora_grad",
                  "attt_lora_step"):
