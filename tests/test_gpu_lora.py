@@ -54,6 +54,12 @@ def test_shapes(attt, L, din, douts, r):
     _check_group(attt, *_inputs(L + din, L, din, douts, r))
 
 
+def test_largest_group(attt):
+    """Eight projections on one x (the largest group), ragged douts."""
+    douts = [64, 72, 128, 200, 8, 136, 256, 24]
+    _check_group(attt, *_inputs(99, 330, 136, douts, 12))
+
+
 def test_zero_B_and_zero_x(attt):
     x, dys, As, Bs = _inputs(7, 200, 128, [96], 8)
     gA, gB = _group(attt, x, dys, As, [np.zeros_like(Bs[0])], 2.0)

@@ -167,3 +167,28 @@ def test_invalid_args(attt):
     with pytest.raises(AtttError):
         attt.attt_ngram_weights(h, i32_dev(np.zeros(4, np.int32)), 0.0)
     h.close()
+
+
+def test_extreme_ids_and_every_n(attt):
+    """Any int32 token value (the sign bit set, 0, INT32_MAX) and n from 1 up
+    to the largest, 16: five symbols with copied spans, so that long n-grams
+    repeat; weights bit-exact and table counts equal to brute force."""
+    rng = wk.rng_for(11, "extreme")
+    i32 = np.iinfo(np.int32)
+    alphabet = np.array([i32.min, -1, 0, 1, i32.max], np.int32)
+    H0 = alphabet[rng.integers(0, 5, 3000)]
+    H = wk.copy_spans(rng, H0, H0[:800], 0.5)
+    x = wk.copy_spans(rng, alphabet[rng.integers(0, 5, 600)], H, 0.6)
+    for n in (1, 2, 3, 8, 15, 16):
+        ref = oracle.ngram_weights(H, x, n)
+        if n >= 8:
+            assert (ref < 1.0).any()  # some n-grams of x do repeat from H
+        _assert_bit_exact(_weights(attt, H, x, n), ref)
+    n = 16
+    h = attt.attt_history_create(n, len(H))
+    attt.attt_history_insert(h, i32_dev(H))
+    q = np.stack([H[p:p + n] for p in range(0, len(H) - n, 37)] + [x[p:p + n] for p in range(0, 580, 29)])
+    got = attt.attt_history_count(h, i32_dev(q)).cpu().numpy()
+    np.testing.assert_array_equal(got, [oracle.count_naive(H, g) for g in q])
+    assert attt.attt_history_status(h) == 0
+    h.close()
