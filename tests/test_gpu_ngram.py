@@ -192,3 +192,34 @@ def test_extreme_ids_and_every_n(attt):
     np.testing.assert_array_equal(got, [oracle.count_naive(H, g) for g in q])
     assert attt.attt_history_status(h) == 0
     h.close()
+
+
+@pytest.mark.slow
+def test_history_at_maximum_length(attt):
+    """A history filled to its limit, 2^24 - 2 tokens (the 24-bit position and
+    count fields at their largest), inserted in three chunks: weights
+    bit-exact, counts exact (an n-gram whose only occurrence ends the history
+    included), and one token more is refused."""
+    from paper_2607_03441_gb300.attt import AtttError
+    MAXH = (1 << 24) - 2
+    n = 4
+    rng = wk.rng_for(12, "maxhist")
+    H = wk.zipf_ids(rng, MAXH, 128256)
+    tail = np.arange(40, dtype=np.int32) + 200000  # ids that occur nowhere else
+    H[-40:] = tail
+    x = wk.copy_spans(rng, wk.zipf_ids(rng, 1024, 128256), H[-2_000_000:], 0.4)
+    x[500:540] = tail
+    h = attt.attt_history_create(n, MAXH)
+    for a, b in ((0, 5_000_001), (5_000_001, MAXH - 20), (MAXH - 20, MAXH)):
+        attt.attt_history_insert(h, i32_dev(H[a:b]))
+    assert attt.attt_history_length(h) == MAXH
+    with pytest.raises(AtttError):
+        attt.attt_history_insert(h, i32_dev(H[:1]))
+    w = attt.attt_ngram_weights(h, i32_dev(x), 0.05).cpu().numpy()
+    _assert_bit_exact(w, oracle.ngram_weights(H, x, n))
+    assert np.all(w[500:540] == np.float32(0.5))
+    q = np.stack([H[p:p + n] for p in (0, 1, 12345, MAXH // 2, MAXH - 41, MAXH - n)] + [tail[:n], tail[-n:]])
+    got = attt.attt_history_count(h, i32_dev(q)).cpu().numpy()
+    np.testing.assert_array_equal(got, [oracle.count_naive(H, g) for g in q])
+    assert got[-1] == 1 and attt.attt_history_status(h) == 0
+    h.close()
