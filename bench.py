@@ -120,10 +120,11 @@ class Update:
     it.  Projections that share an input x (q/k/v; gate/up) form one group
     and one attt_lora_grad call."""
 
-    def __init__(self, wl, dev, max_steps):
+    def __init__(self, wl, dev, max_steps, grad_steps=1):
         import torch
         from paper_2607_03441_gb300 import attt
         self.attt = attt
+        self.grad_steps = grad_steps
         self.torch = torch
         self.wl = wl
         self.dev = dev
@@ -171,35 +172,38 @@ class Update:
     ROWS = ("ngram_weights", "weighted_ce_fwd_bwd", "lora_grad", "lora_step", "history_insert")
 
     def step(self, events=None, part="all"):
-        """One update.  `events` (optional) maps each row name to a pair of
-        CUDA events recorded around that row's calls on the current stream."""
+        """One update: the weights, `grad_steps` rounds of Eq. 10, the LoRA
+        gradients and the SGD step, then the history insert.  `events`
+        (optional) maps each row name to a pair of CUDA events recorded around
+        that row's calls (the first round's) on the current stream."""
         a = self.attt
 
-        def mark(name, k):
-            if events is not None:
+        def mark(name, k, g=0):
+            if events is not None and g == 0:
                 events[name][k].record()
 
         if part in ("all", "ngram"):
             mark("ngram_weights", 0)
             a.attt_ngram_weights(self.hist, self.x, self.wl.w_min, out=self.w)
             mark("ngram_weights", 1)
-        if part in ("all", "ce"):
-            mark("weighted_ce_fwd_bwd", 0)
-            a.attt_weighted_ce_fwd_bwd(self.h, self.W, self.x, self.w, loss=self.loss, dh=self.dh,
-                                       workspace=self.ws_ce)
-            mark("weighted_ce_fwd_bwd", 1)
-        if part in ("all", "lora"):
-            mark("lora_grad", 0)
-            for gname, idx in self.groups.items():
-                a.attt_lora_grad(self.xin[gname], [self.dy[i] for i in idx], [self.A16[i] for i in idx],
-                                 [self.B16[i] for i in idx], self.wl.scale, dAs=[self.dA[i] for i in idx],
-                                 dBs=[self.dB[i] for i in idx], workspace=self.ws_lora)
-            mark("lora_grad", 1)
-            mark("lora_step", 0)
-            for i in range(len(self.projs)):
-                a.attt_lora_step(self.A32[i], self.B32[i], self.dA[i], self.dB[i], wk.LORA_LR, self.A16[i],
-                                 self.B16[i])
-            mark("lora_step", 1)
+        for g in range(self.grad_steps):
+            if part in ("all", "ce"):
+                mark("weighted_ce_fwd_bwd", 0, g)
+                a.attt_weighted_ce_fwd_bwd(self.h, self.W, self.x, self.w, loss=self.loss, dh=self.dh,
+                                           workspace=self.ws_ce)
+                mark("weighted_ce_fwd_bwd", 1, g)
+            if part in ("all", "lora"):
+                mark("lora_grad", 0, g)
+                for gname, idx in self.groups.items():
+                    a.attt_lora_grad(self.xin[gname], [self.dy[i] for i in idx], [self.A16[i] for i in idx],
+                                     [self.B16[i] for i in idx], self.wl.scale, dAs=[self.dA[i] for i in idx],
+                                     dBs=[self.dB[i] for i in idx], workspace=self.ws_lora)
+                mark("lora_grad", 1, g)
+                mark("lora_step", 0, g)
+                for i in range(len(self.projs)):
+                    a.attt_lora_step(self.A32[i], self.B32[i], self.dA[i], self.dB[i], wk.LORA_LR, self.A16[i],
+                                     self.B16[i])
+                mark("lora_step", 1, g)
         if part in ("all", "ngram"):
             mark("history_insert", 0)
             a.attt_history_insert(self.hist, self.x)
@@ -303,21 +307,22 @@ class OracleSample:
         self.x = wk.update_tokens(wl, self.H) if x is None else x
         self.dense = wk.dense_inputs(wl) if dense is None else dense
 
-    def run(self, rows: int):
+    def run(self, rows: int, grad_steps: int = 1):
         o, wl, dense = self.oracle, self.wl, self.dense
         sel = np.sort(wk.rng_for(wl.seed, "cpu_sample").choice(wl.L, rows, replace=False)).astype(np.int64)
         t0 = time.perf_counter()
         w = o.ngram_weights(self.H, self.x, wl.n, wl.w_min)
-        o.ce_rows(dense["h"], dense["W"], self.x, w, sel)
-        for p in wl.projs:
-            dA, dB = o.lora_grad(dense[f"x/{p.name}"][sel], dense[f"dy/{p.name}"][sel], dense[f"A/{p.name}"],
-                                 dense[f"B/{p.name}"], wl.scale)
-            o.sgd_step(wk.bf16_to_f32(dense[f"A/{p.name}"]), dA.astype(np.float32), wk.LORA_LR)
-            o.sgd_step(wk.bf16_to_f32(dense[f"B/{p.name}"]), dB.astype(np.float32), wk.LORA_LR)
+        for _ in range(grad_steps):
+            o.ce_rows(dense["h"], dense["W"], self.x, w, sel)
+            for p in wl.projs:
+                dA, dB = o.lora_grad(dense[f"x/{p.name}"][sel], dense[f"dy/{p.name}"][sel], dense[f"A/{p.name}"],
+                                     dense[f"B/{p.name}"], wl.scale)
+                o.sgd_step(wk.bf16_to_f32(dense[f"A/{p.name}"]), dA.astype(np.float32), wk.LORA_LR)
+                o.sgd_step(wk.bf16_to_f32(dense[f"B/{p.name}"]), dB.astype(np.float32), wk.LORA_LR)
         dt = time.perf_counter() - t0
         desc = (f"{rows} of {wl.L} update tokens of the {wl.name} workload per sample: full Eq. 8/9 weights, "
                 f"Eq. 10 lse+dh for {rows} rows over all {wl.V} vocab entries, LoRA grads and SGD for those "
-                f"rows; fp64 C oracle with OpenMP")
+                f"rows" + (f", {grad_steps} times" if grad_steps > 1 else "") + "; fp64 C oracle with OpenMP")
         return dt, {"value": round(rows / dt, 3), "unit": UNIT, "cores": o.num_threads(), "kind": "oracle",
                     "sample": desc + f", {dt:.1f} s"}
 
@@ -361,7 +366,7 @@ def run_gpu(args):
     wl = wk.WORKLOADS[args.workload]
     peaks = _peaks()
     max_steps = 2 * (args.warmup + args.steps) + 4
-    u = Update(wl, dev, max_steps)
+    u = Update(wl, dev, max_steps, args.grad_steps)
     torch.cuda.synchronize()
 
     part = args.part
@@ -485,7 +490,7 @@ def run_gpu(args):
         traffic = _stored_traffic(wl)
         cpu = None
         if ws == 1 and args.cpu_rows > 0:
-            _, cpu = OracleSample(wl, dense=u.dense, x=u.x_host, H=u.H0).run(args.cpu_rows)
+            _, cpu = OracleSample(wl, dense=u.dense, x=u.x_host, H=u.H0).run(args.cpu_rows, args.grad_steps)
         out = {
             "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(t_ms / args.steps, 4), "higher_is_better": True,
@@ -493,7 +498,10 @@ def run_gpu(args):
             "config": {"workload": (f"{wl.name}: one aTTT update, L={wl.L} tokens, V={wl.V}, d={wl.d}, n={wl.n}, "
                                     f"history {len(u.H0)} tokens at the start (+L per step), LoRA r={wl.r} on " +
                                     ", ".join(f"{p.name} {p.din}x{p.dout}" for p in wl.projs) +
-                                    ", one SGD step"),
+                                    (", one SGD step" if args.grad_steps == 1 else
+                                     f", {args.grad_steps} SGD steps (weights and insert once; Eq. 10, LoRA "
+                                     f"grads and SGD per step)")),
+                       "grad_steps": args.grad_steps,
                        "global_batch": wl.L * ws, "seq_len": wl.L, "parallelism": f"replicas{ws}",
                        "l2": f"inputs larger than L2 (LM head {2 * wl.V * wl.d / 1e9:.2f} GB streamed every step)"},
             "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
@@ -972,14 +980,15 @@ def run_reference(args):
     t = 0.0
     last = None
     for _ in range(args.steps):
-        dt, last = sample.run(args.ref_rows)
+        dt, last = sample.run(args.ref_rows, args.grad_steps)
         t += dt
     value = args.ref_rows * args.steps / t
     return {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * t / args.steps, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": f"{wl.name} (oracle sample of {args.ref_rows} update tokens per step)",
-                       "global_batch": wl.L, "seq_len": wl.L, "parallelism": "host cores"},
+                       "global_batch": wl.L, "seq_len": wl.L, "parallelism": "host cores",
+                       "grad_steps": args.grad_steps},
             "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": last["cores"], "kind": "oracle",
                              "sample": last["sample"]},
             "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -999,6 +1008,9 @@ def main():
     ap.add_argument("--part", default="all", choices=["all", "ce", "lora", "ngram"],
                     help="time one stage alone (profiling aid); 'all' is the benchmark")
     ap.add_argument("--cpu-rows", type=int, default=64, help="rows of the oracle CPU-baseline sample (0: skip)")
+    ap.add_argument("--grad-steps", type=int, default=1, choices=range(1, 9), metavar="G",
+                    help="gradient steps per update of the single-update workloads (the paper takes 2: "
+                         "weights and insert once, Eq. 10, LoRA grads and SGD per step)")
     ap.add_argument("--ref-rows", type=int, default=4, help="rows per step of the reference arm")
     args = ap.parse_args()
     if args.warmup < 3:

@@ -41,3 +41,34 @@ def test_work_accounting():
 def test_replica_throughput():
     # 4 replicas, 10 steps of 2,048 tokens in 50 ms: 1.6384 M tokens/s
     assert abs(bench.replica_throughput(2048, 10, 4, 50.0) - 1638400.0) < 1e-6
+
+
+class _Recorder:
+    """Stands in for the binding: records the order of the calls."""
+
+    def __init__(self):
+        self.calls = []
+
+    def __getattr__(self, name):
+        def call(*args, **kwargs):
+            self.calls.append(name)
+        return call
+
+
+def test_update_step_order_with_gradient_steps():
+    """Algorithm 1 per update: the weights once, then per gradient step
+    Eq. 10, the LoRA gradients of every group and the SGD step of every
+    projection, then the history insert once."""
+    wl = wk.WORKLOADS["7b"]
+    for G in (1, 2):
+        u = object.__new__(bench.Update)
+        u.attt, u.wl, u.grad_steps = _Recorder(), wl, G
+        u.hist = u.x = u.w = u.h = u.W = u.loss = u.dh = u.ws_ce = u.ws_lora = None
+        u.projs = list(wl.projs)
+        u.groups = {"attn": list(range(len(u.projs)))}
+        u.xin = {"attn": None}
+        u.dy = u.A16 = u.B16 = u.A32 = u.B32 = u.dA = u.dB = [None] * len(u.projs)
+        u.step()
+        P = len(u.projs)
+        round_ = ["attt_weighted_ce_fwd_bwd", "attt_lora_grad"] + ["attt_lora_step"] * P
+        assert u.attt.calls == ["attt_ngram_weights"] + round_ * G + ["attt_history_insert"]
