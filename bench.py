@@ -1007,7 +1007,7 @@ def main():
                          "'*-episode' runs chained updates through attt_episode_*")
     ap.add_argument("--part", default="all", choices=["all", "ce", "lora", "ngram"],
                     help="time one stage alone (profiling aid); 'all' is the benchmark")
-    ap.add_argument("--cpu-rows", type=int, default=64, help="rows of the oracle CPU-baseline sample (0: skip)")
+    ap.add_argument("--cpu-rows", type=int, default=256, help="rows of the oracle CPU-baseline sample (0: skip)")
     ap.add_argument("--grad-steps", type=int, default=1, choices=range(1, 9), metavar="G",
                     help="gradient steps per update of the single-update workloads (the paper takes 2: "
                          "weights and insert once, Eq. 10, LoRA grads and SGD per step)")
