@@ -1,7 +1,7 @@
 """Plain CPU oracle for the aTTT update step -- TEST INFRASTRUCTURE ONLY.
 
-Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
-``bench.py`` may import this package.  The CUDA library never imports, links
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg and
+reference arm (``--impl reference``) of ``bench.py`` may import this package.  The CUDA library never imports, links
 or calls it, and it shares no code with that library.
 
 The arithmetic lives in ``attt_oracle.c`` (fp64 sums over the bf16 inputs,

@@ -2,8 +2,8 @@
  * attt_oracle.c -- plain, slow CPU oracle for the aTTT update step.
  *
  * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may call, link or
- * load this file; only the tests, the smoke check and the CPU baseline leg of
- * the benchmark do.  It shares no code, header, table or helper with the CUDA
+ * load this file; only the tests, the smoke check and the CPU baseline leg and
+ * reference arm of the benchmark do.  It shares no code, header, table or helper with the CUDA
  * library under paper_2607_03441_gb300/csrc.
  *
  * What it computes (aTTT, "Agentic Test-Time Training", Sec. 3.3):
