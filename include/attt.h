@@ -203,6 +203,14 @@ ATTT_API attt_status attt_ngram_weights(const attt_history *h, const int32_t *d_
 ATTT_API size_t attt_ce_workspace_bytes(int64_t L, int64_t d, int64_t V);
 
 /*
+ * The largest attt_ce_workspace_bytes(L, d, V) over 1 <= L <= Lmax: one
+ * workspace that serves every update length up to Lmax (the size is not
+ * monotone in L, because the vocabulary chunk depends on L).  0 if Lmax < 1.
+ * Host-only.
+ */
+ATTT_API size_t attt_ce_workspace_max_bytes(int64_t Lmax, int64_t d, int64_t V);
+
+/*
  * With h = d_h (bf16 [L, d], row j is the state that predicts target x_j),
  * W = d_W (bf16 [V, d], the frozen LM head), z_j = h_j W^T:
  *   lse_j  = log sum_v exp(z_jv)

@@ -93,6 +93,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
             "attt_history_count": (i32, [P, P, i64, P, P]),
             "attt_ngram_weights": (i32, [P, P, i64, f32, P, P]),
             "attt_ce_workspace_bytes": (sz, [i64, i64, i64]),
+            "attt_ce_workspace_max_bytes": (sz, [i64, i64, i64]),
             "attt_weighted_ce_fwd_bwd": (i32, [P, P, P, P, i64, i64, i64, P, P, P, P, sz, P]),
             "attt_lora_workspace_bytes": (sz, [i64, i64, i32, P, i32]),
             "attt_lora_grad": (i32, [P, i64, i64, i32, P, P, P, P, i32, f32, P, P, P, sz, P]),
@@ -321,6 +322,11 @@ def attt_ngram_weights(h: History, tokens: torch.Tensor, w_min: float = 0.05,
 
 def attt_ce_workspace_bytes(L: int, d: int, V: int) -> int:
     return int(load_library().attt_ce_workspace_bytes(int(L), int(d), int(V)))
+
+
+def attt_ce_workspace_max_bytes(Lmax: int, d: int, V: int) -> int:
+    """One workspace for every update length 1..Lmax (host-only)."""
+    return int(load_library().attt_ce_workspace_max_bytes(int(Lmax), int(d), int(V)))
 
 
 def attt_weighted_ce_fwd_bwd(h: torch.Tensor, W: torch.Tensor, tgt: torch.Tensor, w: torch.Tensor,

@@ -359,6 +359,11 @@ size_t ce_workspace_bound(int64_t Lmax, int64_t d, int64_t V) {
 
 extern "C" {
 
+size_t attt_ce_workspace_max_bytes(int64_t Lmax, int64_t d, int64_t V) {
+    if (Lmax < 1 || V <= 0 || d <= 0) return 0;
+    return attt::ce_workspace_bound(Lmax, d, V);
+}
+
 attt_status attt_weighted_ce_fwd_bwd(const attt_bf16 *d_h, const attt_bf16 *d_W, const int32_t *d_tgt,
                                      const float *d_w, int64_t L, int64_t d, int64_t V, float *d_loss,
                                      float *d_dh, float *d_lse, void *d_ws, size_t ws_bytes, attt_stream stream) {

@@ -96,3 +96,16 @@ def test_checked_build_exports_the_same_calls():
     exported = set(re.findall(r"\bT (attt_\w+)", out))
     assert not [s for s in declared_symbols() if s not in exported]
     assert ctypes.CDLL(path).attt_status_string(9) is not None
+
+
+def test_ce_workspace_max_is_the_maximum_over_lengths(lib_path):
+    """attt_ce_workspace_max_bytes(Lmax) equals the largest
+    attt_ce_workspace_bytes(L) over every L <= Lmax (host-only; the size is
+    not monotone in L because the vocabulary chunk depends on L)."""
+    from paper_2607_03441_gb300 import attt
+    lib = attt.load_library()
+    assert attt.attt_ce_workspace_max_bytes(0, 512, 8192) == 0
+    for Lmax, d, V in ((256, 512, 8192), (2048, 3584, 152064), (4096, 4096, 128256), (9000, 5120, 152064),
+                       (40000, 3584, 152064), (3000, 64, 300), (5000, 128, 100000)):
+        exhaustive = max(lib.attt_ce_workspace_bytes(L, d, V) for L in range(1, Lmax + 1))
+        assert attt.attt_ce_workspace_max_bytes(Lmax, d, V) == exhaustive, (Lmax, d, V)
