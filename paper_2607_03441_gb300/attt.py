@@ -169,6 +169,18 @@ def _bf16(t: torch.Tensor) -> int:
     return _ptr(t)
 
 
+def _expect(t: Optional[torch.Tensor], shape, dtype, name: str) -> None:
+    """Raises ValueError unless t (when given) has this shape and dtype: the
+    C ABI takes sizes on trust, so a smaller tensor would be read or written
+    past its end."""
+    if t is None:
+        return
+    if tuple(t.shape) != tuple(int(x) for x in shape):
+        raise ValueError(f"{name}: expected shape {tuple(shape)}, got {tuple(t.shape)}")
+    if t.dtype != dtype:
+        raise ValueError(f"{name}: expected {dtype}, got {t.dtype}")
+
+
 # --------------------------------------------------------------------------
 # status
 # --------------------------------------------------------------------------
@@ -337,6 +349,13 @@ def attt_weighted_ce_fwd_bwd(h: torch.Tensor, W: torch.Tensor, tgt: torch.Tensor
     L, d = h.shape
     V = W.shape[0]
     dev = h.device
+    _expect(W, (V, d), torch.bfloat16, "W")
+    _expect(tgt, (L,), torch.int32, "tgt")
+    _expect(w, (L,), torch.float32, "w")
+    _expect(dh, (L, d), torch.float32, "dh")
+    _expect(lse, (L,), torch.float32, "lse")
+    if loss is not None and (loss.numel() < 1 or loss.dtype != torch.float32):
+        raise ValueError("loss: expected a float32 tensor of at least one element")
     if loss is None:
         loss = torch.empty(1, dtype=torch.float32, device=dev)
     if dh is None:
@@ -370,6 +389,14 @@ def attt_lora_grad(x: torch.Tensor, dys: Sequence[torch.Tensor], As: Sequence[to
     r = As[0].shape[1]
     douts = [int(t.shape[1]) for t in dys]
     dev = x.device
+    if not (len(As) == len(Bs) == k) or (dAs is not None and len(dAs) != k) or (dBs is not None and len(dBs) != k):
+        raise ValueError("dys, As, Bs (and dAs, dBs) must have one entry per projection")
+    for p in range(k):
+        _expect(dys[p], (L, douts[p]), torch.bfloat16, f"dys[{p}]")
+        _expect(As[p], (din, r), torch.bfloat16, f"As[{p}]")
+        _expect(Bs[p], (r, douts[p]), torch.bfloat16, f"Bs[{p}]")
+        _expect(dAs[p] if dAs is not None else None, (din, r), torch.float32, f"dAs[{p}]")
+        _expect(dBs[p] if dBs is not None else None, (r, douts[p]), torch.float32, f"dBs[{p}]")
     if dAs is None:
         dAs = [torch.empty(din, r, dtype=torch.float32, device=dev) for _ in range(k)]
     if dBs is None:
@@ -411,6 +438,12 @@ def attt_lora_step(A32: torch.Tensor, B32: torch.Tensor, dA: torch.Tensor, dB: t
     """In-place SGD step on the fp32 masters and bf16 refresh (Eq. 2)."""
     din, r = A32.shape
     dout = B32.shape[1]
+    _expect(A32, (din, r), torch.float32, "A32")
+    _expect(B32, (r, dout), torch.float32, "B32")
+    _expect(dA, (din, r), torch.float32, "dA")
+    _expect(dB, (r, dout), torch.float32, "dB")
+    _expect(A16, (din, r), torch.bfloat16, "A16")
+    _expect(B16, (r, dout), torch.bfloat16, "B16")
     _check(load_library().attt_lora_step(
         _ptr(A32), _ptr(B32), _ptr(dA), _ptr(dB), din, dout, r, float(lr),
         _bf16(A16) if A16 is not None else None, _bf16(B16) if B16 is not None else None, _stream(stream)),
@@ -436,6 +469,10 @@ def attt_lora_forward(x: torch.Tensor, W0: torch.Tensor, A: torch.Tensor, B: tor
     L, din = x.shape
     dout = W0.shape[1]
     r = A.shape[1]
+    _expect(W0, (din, dout), torch.bfloat16, "W0")
+    _expect(A, (din, r), torch.bfloat16, "A")
+    _expect(B, (r, dout), torch.bfloat16, "B")
+    _expect(h, (L, dout), torch.bfloat16, "h")
     if h is None:
         h = torch.empty(L, dout, dtype=torch.bfloat16, device=x.device)
     if workspace is None:
@@ -454,6 +491,10 @@ def attt_lora_input_grad(dy: torch.Tensor, W0: torch.Tensor, A: torch.Tensor, B:
     L, dout = dy.shape
     din = W0.shape[0]
     r = A.shape[1]
+    _expect(W0, (din, dout), torch.bfloat16, "W0")
+    _expect(A, (din, r), torch.bfloat16, "A")
+    _expect(B, (r, dout), torch.bfloat16, "B")
+    _expect(dx, (L, din), torch.float32, "dx")
     if dx is None:
         dx = torch.empty(L, din, dtype=torch.float32, device=dy.device)
     if workspace is None:
@@ -471,6 +512,8 @@ def attt_cast_bf16(src: torch.Tensor, dst: Optional[torch.Tensor] = None, stream
         raise ValueError(f"expected float32, got {src.dtype}")
     if dst is None:
         dst = torch.empty(src.shape, dtype=torch.bfloat16, device=src.device)
+    if dst.numel() != src.numel():
+        raise ValueError(f"dst: expected {src.numel()} elements, got {dst.numel()}")
     _check(load_library().attt_cast_bf16(_ptr(src), _bf16(dst), src.numel(), _stream(stream)), "attt_cast_bf16")
     return dst
 

@@ -109,3 +109,37 @@ def test_ce_workspace_max_is_the_maximum_over_lengths(lib_path):
                        (40000, 3584, 152064), (3000, 64, 300), (5000, 128, 100000)):
         exhaustive = max(lib.attt_ce_workspace_bytes(L, d, V) for L in range(1, Lmax + 1))
         assert attt.attt_ce_workspace_max_bytes(Lmax, d, V) == exhaustive, (Lmax, d, V)
+
+
+def test_binding_rejects_mismatched_shapes():
+    """The C ABI takes sizes on trust, so the binding checks every tensor's
+    shape and dtype against the sizes it passes (host-only: the checks run
+    before any pointer is taken)."""
+    import torch
+    from paper_2607_03441_gb300 import attt
+    bf, f32 = torch.bfloat16, torch.float32
+    x = torch.zeros(8, 16, dtype=bf)
+    with pytest.raises(ValueError, match="dys"):
+        attt.attt_lora_grad(x, [torch.zeros(7, 32, dtype=bf)], [torch.zeros(16, 4, dtype=bf)],
+                            [torch.zeros(4, 32, dtype=bf)], 2.0)
+    with pytest.raises(ValueError, match="Bs"):
+        attt.attt_lora_grad(x, [torch.zeros(8, 32, dtype=bf)], [torch.zeros(16, 4, dtype=bf)],
+                            [torch.zeros(4, 24, dtype=bf)], 2.0)
+    with pytest.raises(ValueError, match="one entry per projection"):
+        attt.attt_lora_grad(x, [torch.zeros(8, 32, dtype=bf)] * 2, [torch.zeros(16, 4, dtype=bf)],
+                            [torch.zeros(4, 32, dtype=bf)], 2.0)
+    with pytest.raises(ValueError, match="tgt"):
+        attt.attt_weighted_ce_fwd_bwd(x, torch.zeros(10, 16, dtype=bf), torch.zeros(7, dtype=torch.int32),
+                                      torch.zeros(8, dtype=f32))
+    with pytest.raises(ValueError, match="W"):
+        attt.attt_weighted_ce_fwd_bwd(x, torch.zeros(10, 12, dtype=bf), torch.zeros(8, dtype=torch.int32),
+                                      torch.zeros(8, dtype=f32))
+    with pytest.raises(ValueError, match="dB"):
+        attt.attt_lora_step(torch.zeros(16, 4), torch.zeros(4, 32), torch.zeros(16, 4), torch.zeros(4, 31), 1e-3)
+    with pytest.raises(ValueError, match="B"):
+        attt.attt_lora_forward(x, torch.zeros(16, 32, dtype=bf), torch.zeros(16, 4, dtype=bf),
+                               torch.zeros(4, 33, dtype=bf), 2.0)
+    with pytest.raises(ValueError, match="dx"):
+        attt.attt_lora_input_grad(torch.zeros(8, 32, dtype=bf), torch.zeros(16, 32, dtype=bf),
+                                  torch.zeros(16, 4, dtype=bf), torch.zeros(4, 32, dtype=bf), 2.0,
+                                  dx=torch.zeros(8, 15))
