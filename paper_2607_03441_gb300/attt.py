@@ -308,6 +308,7 @@ def attt_history_count(h: History, ngrams: torch.Tensor, out: Optional[torch.Ten
     if ngrams.dtype != torch.int32 or ngrams.dim() != 2 or ngrams.shape[1] != h.n:
         raise ValueError("ngrams must be int32 [m, n]")
     m = ngrams.shape[0]
+    _expect(out, (m,), torch.int32, "out")
     if out is None:
         out = torch.empty(m, dtype=torch.int32, device=ngrams.device)
     _check(load_library().attt_history_count(h.handle, _ptr(ngrams), m, _ptr(out), _stream(stream)),
@@ -321,6 +322,7 @@ def attt_ngram_weights(h: History, tokens: torch.Tensor, w_min: float = 0.05,
     if tokens.dtype != torch.int32:
         raise ValueError("tokens must be int32")
     L = tokens.numel()
+    _expect(out, (L,), torch.float32, "out")
     if out is None:
         out = torch.empty(L, dtype=torch.float32, device=tokens.device)
     _check(load_library().attt_ngram_weights(h.handle, _ptr(tokens), L, float(w_min), _ptr(out), _stream(stream)),
@@ -665,6 +667,8 @@ def attt_kl_drift(hp: torch.Tensor, hq: torch.Tensor, W: torch.Tensor, kl: Optio
     V = W.shape[0]
     if tuple(hq.shape) != (L, d) or W.shape[1] != d:
         raise ValueError("shape mismatch")
+    _expect(kl, (L,), torch.float32, "kl")
+    _expect(kl_mean, (1,), torch.float32, "kl_mean")
     dev = hp.device
     if kl is None:
         kl = torch.empty(L, dtype=torch.float32, device=dev)
@@ -732,6 +736,8 @@ def attt_repetition(s: WordSets, text: torch.Tensor, tau: float = 0.5, out: Opti
     returns (out, keep) with out = float32 [2] (rho, nu) and keep = int32 [1]."""
     if text.dtype != torch.uint8:
         raise ValueError("text must be uint8 bytes")
+    _expect(out, (2,), torch.float32, "out")
+    _expect(keep, (1,), torch.int32, "keep")
     dev = text.device
     if out is None:
         out = torch.empty(2, dtype=torch.float32, device=dev)
