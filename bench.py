@@ -683,25 +683,45 @@ def run_episode(args):
         raise RuntimeError("device status error in the timed region")
 
     # end to end: each update's text and projection inputs copied from pinned
-    # host memory every step (on the same stream, before its agent steps), the
-    # losses read back every step
+    # host memory every step, the losses read back every step.  The copies run
+    # on a copy stream into two device buffer sets: step i computes on set
+    # i % 2 while the inputs of step i + 1 land in the other (the copy of step
+    # i + 1 waits until step i - 1, the set's last user, is done; step i waits
+    # for its own copy).  Every copy is inside the timed region.
     tok_h = [torch.from_numpy(t).pin_memory() for t in texts]
     xs_h = [torch.from_numpy(x.view(np.int16)).pin_memory() for x in xs_host]
-    tok_d = torch.empty(ew.L, dtype=torch.int32, device=dev)
-    x_d = torch.empty(ew.L, ew.din, dtype=torch.int16, device=dev)
+    tok_d = [torch.empty(ew.L, dtype=torch.int32, device=dev) for _ in range(2)]
+    x_d = [torch.empty(ew.L, ew.din, dtype=torch.int16, device=dev) for _ in range(2)]
     loss_host = torch.empty(ew.grad_steps, dtype=torch.float32).pin_memory()
-    h2d = tok_d.numel() * 4 + x_d.numel() * 2
+    h2d = tok_d[0].numel() * 4 + x_d[0].numel() * 2
     d2h = loss_host.numel() * 4
+    cs = torch.cuda.Stream(device=dev)
+    main = torch.cuda.current_stream()
+    ready = [torch.cuda.Event() for _ in range(args.steps)]
+    done = [torch.cuda.Event() for _ in range(args.steps)]
+
+    def upload(i):
+        k = i % ew.updates  # the update step i runs (state["k"] starts at 0)
+        with torch.cuda.stream(cs):
+            if i >= 2:
+                cs.wait_event(done[i - 2])
+            tok_d[i % 2].copy_(tok_h[k], non_blocking=True)
+            x_d[i % 2].copy_(xs_h[k], non_blocking=True)
+            ready[i].record(cs)
+
     state["k"] = 0
     barrier()
     torch.cuda.synchronize()
     f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     f0.record()
-    for _ in range(args.steps):
-        k = state["k"]
-        tok_d.copy_(tok_h[k], non_blocking=True)
-        x_d.copy_(xs_h[k], non_blocking=True)
-        step(tok_d, x_d.view(torch.bfloat16))
+    cs.wait_event(f0)
+    upload(0)
+    for i in range(args.steps):
+        if i + 1 < args.steps:
+            upload(i + 1)
+        main.wait_event(ready[i])
+        step(tok_d[i % 2], x_d[i % 2].view(torch.bfloat16))
+        done[i].record(main)
         loss_host.copy_(losses, non_blocking=True)
     f1.record()
     torch.cuda.synchronize()
@@ -734,7 +754,7 @@ def run_episode(args):
         ach = flops / (t_ms / args.steps * 1e-3) / 1e12
         cpu = None
         if ws == 1 and args.cpu_rows > 0:
-            cpu = _episode_oracle_sample(ew, texts, dense, xs_host, min(args.cpu_rows, 16))[1]
+            cpu = _episode_oracle_sample(ew, texts, dense, xs_host, min(args.cpu_rows, 128))[1]
         out = {
             "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(t_ms / args.steps, 4), "higher_is_better": True,
