@@ -1,13 +1,16 @@
 #!/usr/bin/env python3
 """aTTT update-step benchmark: update tokens/sec on GB300.
 
-One step = one aTTT update (Algorithm 1) of the 7B-class workload:
-  Eq. 8/9 weights of the 2,048-token update against the n = 4 history
-  (65,536 prior tokens at start), Eq. 10 weighted CE forward + backward
-  through the frozen 152,064 x 3,584 bf16 LM head, LoRA rank-16 gradients of
-  the q (3584x3584) and v (3584x512) projections, the SGD step on both
-  adapters, and the history insert of the update.
+One step = one aTTT update (Algorithm 1) of the 32B-class workload, the
+largest configuration that one GPU holds:
+  Eq. 8/9 weights of the 8,192-token update against the n = 4 history
+  (262,144 prior tokens at start), Eq. 10 weighted CE forward + backward
+  through the frozen 152,064 x 5,120 bf16 LM head, LoRA rank-64 gradients of
+  the q, k, v (one shared input) and o projections, the SGD step on every
+  adapter, and the history insert of the update.
 The whole step runs in libattt's CUDA kernels, called through the C ABI.
+The same run adds, under "extra", the paper's two gradient steps per update
+on that workload and the 7B-class single update.
 
 Contract: `python bench.py --gpus N --steps K --warmup W` prints one JSON line.
 N > 1 runs N independent replicas (one per GPU, no data-path collective;
@@ -38,7 +41,7 @@ from paper_2607_03441_gb300 import workloads as wk  # noqa: E402
 
 METRIC = "aTTT update tokens/sec on 1 GB300 and % of roofline (tensor peak / HBM)"
 UNIT = "update tokens/s"
-WORKLOAD = "7b"
+WORKLOAD = "32b"
 
 
 def _peaks():
@@ -236,21 +239,79 @@ def row_work(wl):
     }
 
 
-def row_report(wl, events, peaks):
+def peak_kind(region_ms, clk):
+    """Which measured bf16 peak a contraction timed in this region is held
+    to: the burst figure (cuBLAS timed alone at full clock) when the timed
+    region is shorter than a second and its median SM clock stayed within 3%
+    of the maximum; the sustained figure (a seconds-long loop at the power
+    cap) otherwise.  Without a clock record the region's length decides."""
+    short = region_ms < 1000.0
+    if clk is None:
+        return "burst" if short else "sustained"
+    at_max = clk["sm_mhz"] >= 0.97 * clk["sm_max_mhz"]
+    return "burst" if (short and at_max) else "sustained"
+
+
+def _bf16_peak(peaks, kind):
+    return peaks["bf16"] if kind == "burst" else peaks["bf16_sustained"]
+
+
+def row_report(wl, events, peaks, kind="sustained"):
     out = {}
     work = row_work(wl)
     for name, evs in events.items():
         ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
-        kind, amount, _ = work[name]
-        if kind == "tensor":
+        amount_kind, amount, _ = work[name]
+        if amount_kind == "tensor":
             ach = amount / (ms * 1e-3) / 1e12
             out[name] = {"ms": round(ms, 4), "bound": "tensor", "achieved_tflops": round(ach, 1),
-                         "frac": round(ach / peaks["bf16_sustained"], 4), "flop": amount}
+                         "frac": round(ach / _bf16_peak(peaks, kind), 4), "peak_kind": kind,
+                         "frac_of_burst": round(ach / peaks["bf16"], 4),
+                         "frac_of_sustained": round(ach / peaks["bf16_sustained"], 4), "flop": amount}
         else:
             ach = amount / (ms * 1e-3) / 1e9
             out[name] = {"ms": round(ms, 4), "bound": "hbm", "achieved_gbs": round(ach, 1),
                          "frac": round(ach / peaks["hbm_gbs"], 4), "bytes": int(amount)}
     return out
+
+
+def _tensor_roofline(achieved, peaks, kind, kernel):
+    peak = _bf16_peak(peaks, kind)
+    return {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
+            "frac": round(achieved / peak, 4), "traffic": None, "kernel": kernel,
+            "peak_kind": f"bf16 {kind}, {peaks['src']}", "frac_of_burst": round(achieved / peaks["bf16"], 4),
+            "frac_of_sustained": round(achieved / peaks["bf16_sustained"], 4)}
+
+
+def path_work(wl, grad_steps):
+    """Algorithmic FLOPs and bytes of one whole update: the weights and the
+    insert once, and per gradient step Eq. 10 (4 L V d; W, h, dh once), the
+    LoRA gradients (4 L r (din + dout) per projection; each distinct x and
+    each dy once, the adapters) and the SGD step."""
+    work = row_work(wl)
+    L, V, d = wl.L, wl.V, wl.d
+    lora_flops = sum(4.0 * L * wl.r * (p.din + p.dout) for p in wl.projs)
+    flops = grad_steps * (work["weighted_ce_fwd_bwd"][1] + lora_flops)
+    ce_bytes = 2.0 * V * d + 2.0 * L * d + 4.0 * L * d + 8.0 * L
+    nbytes = (work["ngram_weights"][1] + work["history_insert"][1]
+              + grad_steps * (ce_bytes + work["lora_grad"][1] + work["lora_step"][1]))
+    return flops, nbytes
+
+
+def path_roofline(wl, grad_steps, ms_per_step, peaks, kind):
+    """The whole update against the slower of its FLOPs at the bf16 tensor
+    peak and its bytes at the HBM bandwidth (the path roofline)."""
+    flops, nbytes = path_work(wl, grad_steps)
+    t_tensor = flops / (_bf16_peak(peaks, kind) * 1e12)
+    t_hbm = nbytes / (peaks["hbm_gbs"] * 1e9)
+    t_roof = max(t_tensor, t_hbm)
+    t = ms_per_step * 1e-3
+    return {"bound": "tensor" if t_tensor >= t_hbm else "hbm", "flop": flops, "bytes": nbytes,
+            "roofline_ms": round(t_roof * 1e3, 4), "ms_per_step": round(ms_per_step, 4),
+            "frac": round(t_roof / t, 4), "peak_kind": kind,
+            "frac_of_burst": round(max(flops / (peaks["bf16"] * 1e12), t_hbm) / t, 4),
+            "frac_of_sustained": round(max(flops / (peaks["bf16_sustained"] * 1e12), t_hbm) / t, 4),
+            "achieved_tflops": round(flops / t / 1e12, 1)}
 
 
 # The sources the Eq. 10 call is built from (its kernels, the contraction
@@ -284,14 +345,17 @@ def _stored_traffic(wl):
     return rec.get("traffic_bytes_per_call")
 
 
-def _ce_roofline(wl, t_ce_ms, peaks, traffic):
+def _ce_roofline(wl, t_ce_ms, peaks, traffic, kind):
     flops = 4.0 * wl.L * wl.V * wl.d
     achieved = flops / (t_ce_ms * 1e-3) / 1e12
-    peak = peaks["bf16_sustained"]
+    peak = _bf16_peak(peaks, kind)
     return {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
             "frac": round(achieved / peak, 4), "traffic": traffic,
             "kernel": "attt_weighted_ce_fwd_bwd (Eq. 10 fwd+bwd; 4*L*V*d algorithmic FLOPs per call)",
-            "peak_kind": f"bf16 sustained, {peaks['src']}"}
+            "peak_kind": f"bf16 {kind}, {peaks['src']}",
+            "peak_burst": peaks["bf16"], "frac_of_burst": round(achieved / peaks["bf16"], 4),
+            "peak_sustained": peaks["bf16_sustained"],
+            "frac_of_sustained": round(achieved / peaks["bf16_sustained"], 4)}
 
 
 class OracleSample:
@@ -350,44 +414,16 @@ def _dist():
     return ws, rank, local
 
 
-def run_gpu(args):
+def _measure_update(wl, dev, steps, warmup, grad_steps, pg, local, e2e=True):
+    """Times `steps` updates of workload `wl` (after `warmup` untimed ones) on
+    the device, then (if `e2e`) the same number again with every step's inputs
+    copied from pinned host memory and the loss read back.  Returns the
+    timings and the per-row CUDA-event report inputs."""
     import torch
     from paper_2607_03441_gb300 import attt
-    from paper_2607_03441_gb300 import build
-    ws, rank, local = _dist()
-    build.build()
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    pg = None
-    if ws > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=dev)
-        pg = dist
-    wl = wk.WORKLOADS[args.workload]
-    peaks = _peaks()
-    max_steps = 2 * (args.warmup + args.steps) + 4
-    u = Update(wl, dev, max_steps, args.grad_steps)
+    u = Update(wl, dev, 2 * (warmup + steps) + 4, grad_steps)
     torch.cuda.synchronize()
-
-    part = args.part
-    if part != "all":
-        # one stage alone, for profiling: a single timed loop, no e2e, no baseline
-        u.w.fill_(1.0)
-        for _ in range(args.warmup):
-            u.step(part=part)
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        for _ in range(args.steps):
-            u.step(part=part)
-        e1.record()
-        torch.cuda.synchronize()
-        status = attt.attt_device_status()
-        u.hist.close()
-        return {"part": part, "workload": wl.name, "steps": args.steps,
-                "ms_per_step": round(e0.elapsed_time(e1) / args.steps, 4), "device_status": status}
-
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         u.step()
     torch.cuda.synchronize()
     if attt.attt_device_status() != 0 or attt.attt_history_status(u.hist) != 0:
@@ -399,7 +435,7 @@ def run_gpu(args):
 
     # ---------------- device-timed region ----------------
     events = {name: [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                     for _ in range(args.steps)] for name in Update.ROWS}
+                     for _ in range(steps)] for name in Update.ROWS}
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
     clocks.start()
@@ -407,7 +443,7 @@ def run_gpu(args):
     torch.cuda.synchronize()
     n0 = attt.attt_kernel_launches()
     e0.record()
-    for i in range(args.steps):
+    for i in range(steps):
         u.step({k: v[i] for k, v in events.items()})
     e1.record()
     torch.cuda.synchronize()
@@ -415,10 +451,11 @@ def run_gpu(args):
     barrier()
     clk = clocks.stop()
     t_ms = e0.elapsed_time(e1)
-    rows = row_report(wl, events, peaks)
-    t_ce = rows["weighted_ce_fwd_bwd"]["ms"]
     if attt.attt_device_status() != 0 or attt.attt_history_status(u.hist) != 0:
         raise RuntimeError("device status error in the timed region")
+    res = {"u": u, "t_ms": t_ms, "events": events, "clk": clk, "launches": int(n1 - n0)}
+    if not e2e:
+        return res
 
     # ---------------- end to end through host buffers ----------------
     # Every step's inputs (tokens, h, each distinct x, each dy) are copied from
@@ -450,8 +487,8 @@ def run_gpu(args):
     d2h = loss_host.numel() * loss_host.element_size()
     cs = torch.cuda.Stream(device=dev)
     main = torch.cuda.current_stream()
-    ready = [torch.cuda.Event() for _ in range(args.steps)]
-    done = [torch.cuda.Event() for _ in range(args.steps)]
+    ready = [torch.cuda.Event() for _ in range(steps)]
+    done = [torch.cuda.Event() for _ in range(steps)]
 
     def upload(i):
         with torch.cuda.stream(cs):
@@ -467,8 +504,8 @@ def run_gpu(args):
     f0.record()
     cs.wait_event(f0)
     upload(0)
-    for i in range(args.steps):
-        if i + 1 < args.steps:
+    for i in range(steps):
+        if i + 1 < steps:
             upload(i + 1)
         main.wait_event(ready[i])
         use_set(sets[i % 2])
@@ -478,45 +515,131 @@ def run_gpu(args):
     f1.record()
     torch.cuda.synchronize()
     barrier()
-    t_e2e = f0.elapsed_time(f1)
+    res.update({"t_e2e": f0.elapsed_time(f1), "h2d": h2d, "d2h": d2h})
+    return res
 
+
+def _workload_desc(wl, hist_tokens, grad_steps):
+    return (f"{wl.name}: one aTTT update, L={wl.L} tokens, V={wl.V}, d={wl.d}, n={wl.n}, history {hist_tokens} "
+            f"tokens at the start (+L per step), LoRA r={wl.r} on " +
+            ", ".join(f"{p.name} {p.din}x{p.dout}" for p in wl.projs) +
+            (", one SGD step" if grad_steps == 1 else
+             f", {grad_steps} SGD steps (weights and insert once; Eq. 10, LoRA grads and SGD per step)") +
+            "; every step re-inserts the same update tokens, so from the second step on the Eq. 8/9 weights see a "
+            "fully repeated text")
+
+
+def run_gpu(args):
+    import torch
+    from paper_2607_03441_gb300 import attt  # noqa: F401  (fails loudly without the CUDA library)
+    from paper_2607_03441_gb300 import build
+    ws, rank, local = _dist()
+    build.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+    wl = wk.WORKLOADS[args.workload]
+    peaks = _peaks()
+
+    if args.part != "all":
+        # one stage alone, for profiling: a single timed loop, no e2e, no baseline
+        u = Update(wl, dev, 2 * (args.warmup + args.steps) + 4, args.grad_steps)
+        u.w.fill_(1.0)
+        for _ in range(args.warmup):
+            u.step(part=args.part)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(args.steps):
+            u.step(part=args.part)
+        e1.record()
+        torch.cuda.synchronize()
+        status = attt.attt_device_status()
+        u.hist.close()
+        return {"part": args.part, "workload": wl.name, "steps": args.steps,
+                "ms_per_step": round(e0.elapsed_time(e1) / args.steps, 4), "device_status": status}
+
+    m = _measure_update(wl, dev, args.steps, args.warmup, args.grad_steps, pg, local, e2e=True)
+    u = m["u"]
+    t_ms, t_e2e = m["t_ms"], m["t_e2e"]
     if pg is not None:
         t_ms, t_e2e = max_over_ranks([t_ms, t_e2e], pg, dev)
-
+    kind = peak_kind(t_ms, m["clk"])
+    rows = row_report(wl, m["events"], peaks, kind)
+    t_ce = rows["weighted_ce_fwd_bwd"]["ms"]
     value = replica_throughput(wl.L, args.steps, ws, t_ms)
     e2e_value = replica_throughput(wl.L, args.steps, ws, t_e2e)
+    hist0 = len(u.H0)
+    x_host, dense, H0 = u.x_host, u.dense, u.H0
+    u.hist.close()
+    del u, m["u"]
+    torch.cuda.empty_cache()
+
+    # Extra lines of the same run (one GPU only): the paper's two gradient
+    # steps per update on this workload, and the 7B-class single update.
+    extras = {}
+    if ws == 1 and args.extras:
+        gs2 = 2 if args.grad_steps == 1 else 1
+        steps2 = max(10, args.steps // 5)
+        e = _measure_update(wl, dev, steps2, args.warmup, gs2, None, local, e2e=False)
+        k2 = peak_kind(e["t_ms"], e["clk"])
+        r2 = row_report(wl, e["events"], peaks, k2)
+        extras[f"grad_steps_{gs2}"] = {
+            "workload": _workload_desc(wl, hist0, gs2), "value": round(replica_throughput(wl.L, steps2, 1, e["t_ms"]), 1),
+            "unit": UNIT, "steps": steps2, "ms_per_step": round(e["t_ms"] / steps2, 4),
+            "path_roofline": path_roofline(wl, gs2, e["t_ms"] / steps2, peaks, k2),
+            "roofline": _ce_roofline(wl, r2["weighted_ce_fwd_bwd"]["ms"], peaks, None, k2),
+            "clocks": e["clk"], "gpu_launches": e["launches"]}
+        e["u"].hist.close()
+        del e
+        torch.cuda.empty_cache()
+        if wl.name != "7b":
+            w7 = wk.WORKLOADS["7b"]
+            e = _measure_update(w7, dev, args.steps, args.warmup, 1, None, local, e2e=False)
+            k7 = peak_kind(e["t_ms"], e["clk"])
+            r7 = row_report(w7, e["events"], peaks, k7)
+            extras["7b"] = {
+                "workload": _workload_desc(w7, len(e["u"].H0), 1),
+                "value": round(replica_throughput(w7.L, args.steps, 1, e["t_ms"]), 1), "unit": UNIT,
+                "steps": args.steps, "ms_per_step": round(e["t_ms"] / args.steps, 4),
+                "path_roofline": path_roofline(w7, 1, e["t_ms"] / args.steps, peaks, k7),
+                "roofline": _ce_roofline(w7, r7["weighted_ce_fwd_bwd"]["ms"], peaks, _stored_traffic(w7), k7),
+                "rows": r7, "clocks": e["clk"], "gpu_launches": e["launches"]}
+            e["u"].hist.close()
+            del e
+            torch.cuda.empty_cache()
+
     out = None
     if rank == 0:
-        traffic = _stored_traffic(wl)
         cpu = None
         if ws == 1 and args.cpu_rows > 0:
-            _, cpu = OracleSample(wl, dense=u.dense, x=u.x_host, H=u.H0).run(args.cpu_rows, args.grad_steps)
+            _, cpu = OracleSample(wl, dense=dense, x=x_host, H=H0).run(args.cpu_rows, args.grad_steps)
         out = {
             "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(t_ms / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": (f"{wl.name}: one aTTT update, L={wl.L} tokens, V={wl.V}, d={wl.d}, n={wl.n}, "
-                                    f"history {len(u.H0)} tokens at the start (+L per step), LoRA r={wl.r} on " +
-                                    ", ".join(f"{p.name} {p.din}x{p.dout}" for p in wl.projs) +
-                                    (", one SGD step" if args.grad_steps == 1 else
-                                     f", {args.grad_steps} SGD steps (weights and insert once; Eq. 10, LoRA "
-                                     f"grads and SGD per step)")),
+            "config": {"workload": _workload_desc(wl, hist0, args.grad_steps),
                        "grad_steps": args.grad_steps,
                        "global_batch": wl.L * ws, "seq_len": wl.L, "parallelism": f"replicas{ws}",
                        "l2": f"inputs larger than L2 (LM head {2 * wl.V * wl.d / 1e9:.2f} GB streamed every step)"},
-            "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h},
-            "gpu_launches": int(n1 - n0),
-            "roofline": _ce_roofline(wl, t_ce, peaks, traffic),
+            "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": m["h2d"],
+                    "d2h_bytes_per_step": m["d2h"]},
+            "gpu_launches": m["launches"],
+            "roofline": _ce_roofline(wl, t_ce, peaks, _stored_traffic(wl), kind),
+            "path_roofline": path_roofline(wl, args.grad_steps, t_ms / args.steps, peaks, kind),
             "ce_ms_per_call": round(t_ce, 4),
             "rows": rows,
-            "clocks": clk,
+            "clocks": m["clk"],
             "cpu_baseline": cpu,
+            "extra": extras,
         }
     if pg is not None:
         pg.barrier()
         pg.destroy_process_group()
-    u.hist.close()
     return out
 
 
@@ -768,15 +891,14 @@ def run_episode(args):
             "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "gpu_launches": int(n1 - n0),
-            "roofline": {"bound": "tensor", "achieved": round(ach, 1), "peak": peaks["bf16_sustained"],
-                         "unit": "TFLOP/s", "frac": round(ach / peaks["bf16_sustained"], 4), "traffic": None,
-                         "kernel": "whole update (two Eq. 10 calls, projection forward and dx, adapter grads)",
-                         "peak_kind": f"bf16 sustained, {peaks['src']}"},
+            "roofline": _tensor_roofline(ach, peaks, peak_kind(t_ms, clk),
+                                         "whole update (two Eq. 10 calls, projection forward and dx, adapter grads)"),
             "clocks": clk,
             "cpu_baseline": cpu,
             "kl_drift": {"ms": round(t_kl, 4), "kl_mean": round(kl_mean.item(), 6),
                          "achieved_tflops": round(kl_flops / (t_kl * 1e-3) / 1e12, 1),
-                         "frac": round(kl_flops / (t_kl * 1e-3) / 1e12 / peaks["bf16_sustained"], 4),
+                         "frac": round(kl_flops / (t_kl * 1e-3) / 1e12 / _bf16_peak(peaks, peak_kind(t_kl, clk)), 4),
+                         "peak_kind": peak_kind(t_kl, clk),
                          "work": "attt_episode_drift: adapted and base projection forward, then the KL through "
                                  "the LM head (4 L V d + 4 L din d FLOPs)"},
         }
@@ -890,10 +1012,9 @@ def run_batch(args):
                       "global_batch": R, "seq_len": ew.L, "parallelism": "replicas1",
                       "l2": "inputs larger than L2 (LM head streamed by every Eq. 10 chunk)"},
            "gpu_launches": int(n1 - n0),
-           "roofline": {"bound": "tensor", "achieved": round(ach, 1), "peak": peaks["bf16_sustained"],
-                        "unit": "TFLOP/s", "frac": round(ach / peaks["bf16_sustained"], 4), "traffic": None,
-                        "kernel": "whole batched update (Eq. 10 over all rows twice, projection forward and dx, "
-                                  "adapter grads)", "peak_kind": f"bf16 sustained, {peaks['src']}"},
+           "roofline": _tensor_roofline(ach, peaks, peak_kind(t_ms, clk),
+                                        "whole batched update (Eq. 10 over all rows twice, projection forward and "
+                                        "dx, adapter grads)"),
            "clocks": clk}
     b.close()
     return out
@@ -1032,6 +1153,8 @@ def main():
                     help="gradient steps per update of the single-update workloads (the paper takes 2: "
                          "weights and insert once, Eq. 10, LoRA grads and SGD per step)")
     ap.add_argument("--ref-rows", type=int, default=4, help="rows per step of the reference arm")
+    ap.add_argument("--no-extras", dest="extras", action="store_false",
+                    help="skip the extra lines (the other gradient-step count and the 7B-class update)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

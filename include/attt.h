@@ -282,7 +282,10 @@ ATTT_API attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din
  *
  * The first call on a device (with that device current) looks up the static
  * array's device address and caches it; make that first call before any
- * stream capture begins.  Every call shares the one array per device and the
+ * stream capture begins.  The cached address belongs to the device's current
+ * context: after cudaDeviceReset() the array is re-created, possibly at
+ * another address, so calling this entry point after a device reset is not
+ * supported.  Every call shares the one array per device and the
  * array keeps the last call's contents (the call clears what must start at
  * zero itself), so calls that overlap on the GPU -- on two streams, or from
  * two host threads -- race and must be serialised by the caller.  A timed-out

@@ -342,11 +342,6 @@ void oracle_lora_input_grad(const uint16_t *dy, const uint16_t *W0, const uint16
     }
 }
 
-/* ------------------------------------------------------------------------ */
-/* Eq. 2 / Algorithm 1: the SGD step on the fp32 adapter masters            */
-/* ------------------------------------------------------------------------ */
-
-/* p <- p - lr * g, in fp32, multiply then subtract (no fused multiply-add). */
 /*
  * Adapter drift (Sec. 4, Fig. 6): per row j, the KL divergence of the
  * adapted model's next-token distribution p_j = softmax(h_p[j] W^T) from the
@@ -401,6 +396,11 @@ void oracle_kl_rows(const uint16_t *hp, const uint16_t *hq, const uint16_t *W, i
     }
 }
 
+/* ------------------------------------------------------------------------ */
+/* Eq. 2 / Algorithm 1: the SGD step on the fp32 adapter masters            */
+/* ------------------------------------------------------------------------ */
+
+/* p <- p - lr * g, in fp32, multiply then subtract (no fused multiply-add). */
 void oracle_sgd_step(float *p, const float *g, int64_t n, float lr)
 {
     for (int64_t i = 0; i < n; ++i) {

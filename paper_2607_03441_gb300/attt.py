@@ -381,24 +381,45 @@ def attt_lora_workspace_bytes(L: int, din: int, douts: Sequence[int], r: int) ->
     return int(load_library().attt_lora_workspace_bytes(int(L), int(din), len(douts), arr, int(r)))
 
 
-def attt_lora_grad(x: torch.Tensor, dys: Sequence[torch.Tensor], As: Sequence[torch.Tensor],
-                   Bs: Sequence[torch.Tensor], scale: float, dAs: Optional[Sequence[torch.Tensor]] = None,
-                   dBs: Optional[Sequence[torch.Tensor]] = None, workspace: Optional[torch.Tensor] = None,
-                   stream=None):
-    """Adapter gradients for projections sharing the input x.  Returns (dAs, dBs)."""
+def _lora_check(x: torch.Tensor, dys, As, Bs, dAs, dBs):
+    """Shapes of one attt_lora_grad group: (L, din, r, douts).  Raises
+    ValueError before any launch unless every list has one entry per
+    projection and every tensor has its shape and dtype (the C ABI takes the
+    sizes on trust, so a smaller or wider-typed tensor would be read or written
+    past its end)."""
+    if x.dim() != 2:
+        raise ValueError(f"x: expected a 2-D [L, din] tensor, got shape {tuple(x.shape)}")
     L, din = x.shape
     k = len(dys)
-    r = As[0].shape[1]
-    douts = [int(t.shape[1]) for t in dys]
-    dev = x.device
+    if k < 1:
+        raise ValueError("at least one projection (dys) is required")
     if not (len(As) == len(Bs) == k) or (dAs is not None and len(dAs) != k) or (dBs is not None and len(dBs) != k):
         raise ValueError("dys, As, Bs (and dAs, dBs) must have one entry per projection")
+    _expect(x, (L, din), torch.bfloat16, "x")
+    if As[0].dim() != 2:
+        raise ValueError(f"As[0]: expected a 2-D [din, r] tensor, got shape {tuple(As[0].shape)}")
+    r = int(As[0].shape[1])
+    douts = []
     for p in range(k):
+        if dys[p].dim() != 2:
+            raise ValueError(f"dys[{p}]: expected a 2-D [L, dout] tensor, got shape {tuple(dys[p].shape)}")
+        douts.append(int(dys[p].shape[1]))
         _expect(dys[p], (L, douts[p]), torch.bfloat16, f"dys[{p}]")
         _expect(As[p], (din, r), torch.bfloat16, f"As[{p}]")
         _expect(Bs[p], (r, douts[p]), torch.bfloat16, f"Bs[{p}]")
         _expect(dAs[p] if dAs is not None else None, (din, r), torch.float32, f"dAs[{p}]")
         _expect(dBs[p] if dBs is not None else None, (r, douts[p]), torch.float32, f"dBs[{p}]")
+    return int(L), int(din), r, douts
+
+
+def attt_lora_grad(x: torch.Tensor, dys: Sequence[torch.Tensor], As: Sequence[torch.Tensor],
+                   Bs: Sequence[torch.Tensor], scale: float, dAs: Optional[Sequence[torch.Tensor]] = None,
+                   dBs: Optional[Sequence[torch.Tensor]] = None, workspace: Optional[torch.Tensor] = None,
+                   stream=None):
+    """Adapter gradients for projections sharing the input x.  Returns (dAs, dBs)."""
+    L, din, r, douts = _lora_check(x, dys, As, Bs, dAs, dBs)
+    k = len(dys)
+    dev = x.device
     if dAs is None:
         dAs = [torch.empty(din, r, dtype=torch.float32, device=dev) for _ in range(k)]
     if dBs is None:
@@ -422,13 +443,15 @@ def attt_lora_grad_noalloc(x: torch.Tensor, dys: Sequence[torch.Tensor], As: Seq
                            dBs: Sequence[torch.Tensor], stream=None):
     """attt_lora_grad without a workspace: the library uses its own static
     16 MiB device scratch and allocates nothing.  The caller passes the output
-    tensors.  Returns (dAs, dBs)."""
-    L, din = x.shape
+    tensors, which are checked like every other argument before the call.
+    Returns (dAs, dBs)."""
+    if dAs is None or dBs is None:
+        raise ValueError("attt_lora_grad_noalloc: the caller passes the output tensors dAs and dBs")
+    L, din, r, douts = _lora_check(x, dys, As, Bs, dAs, dBs)
     k = len(dys)
-    r = As[0].shape[1]
     P = ctypes.c_void_p
     arr = lambda ts, f: (P * k)(*[f(t) for t in ts])  # noqa: E731
-    douts_arr = (ctypes.c_int64 * k)(*[int(t.shape[1]) for t in dys])
+    douts_arr = (ctypes.c_int64 * k)(*douts)
     _check(load_library().attt_lora_grad_noalloc(
         _bf16(x), L, din, k, arr(dys, _bf16), douts_arr, arr(As, _bf16), arr(Bs, _bf16), int(r), float(scale),
         arr(dAs, _ptr), arr(dBs, _ptr), _stream(stream)), "attt_lora_grad_noalloc")

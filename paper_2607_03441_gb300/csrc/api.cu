@@ -171,17 +171,17 @@ attt_status attt_device_status(attt_stream stream) {
     attt_status st = attt::current_device(&dev);
     if (st != ATTT_OK) return st;
     if (cudaStreamSynchronize(stream) != cudaSuccess) return ATTT_ERR_CUDA;
-    int *w = attt::device_status_word(dev);
-    if (!w) return ATTT_ERR_CUDA;
+    // Both words are read and every one that holds an error is cleared, so a
+    // single call drains them; the library-wide word's error is reported first.
+    int *words[2] = {attt::device_status_word(dev), attt::noalloc_status_word(dev)};
+    if (!words[0]) return ATTT_ERR_CUDA;
     int v = 0;
-    if (cudaMemcpy(&v, w, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return ATTT_ERR_CUDA;
-    if (v != 0 && cudaMemset(w, 0, sizeof v) != cudaSuccess) return ATTT_ERR_CUDA;
-    if (v == 0) {
-        int *nw = attt::noalloc_status_word(dev);  // attt_lora_grad_noalloc's own word
-        if (nw) {
-            if (cudaMemcpy(&v, nw, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return ATTT_ERR_CUDA;
-            if (v != 0 && cudaMemset(nw, 0, sizeof v) != cudaSuccess) return ATTT_ERR_CUDA;
-        }
+    for (int *w : words) {
+        if (!w) continue;  // attt_lora_grad_noalloc has not been set up on this device
+        int x = 0;
+        if (cudaMemcpy(&x, w, sizeof x, cudaMemcpyDeviceToHost) != cudaSuccess) return ATTT_ERR_CUDA;
+        if (x != 0 && cudaMemset(w, 0, sizeof x) != cudaSuccess) return ATTT_ERR_CUDA;
+        if (v == 0) v = x;
     }
     return (attt_status)v;
 }

@@ -15,7 +15,10 @@
 // array's device address with cudaGetSymbolAddress (in host code the array's
 // name is only a host-side stand-in, never a device address) and caches it.
 // The same is done for a static status word that records a timed-out device
-// wait of this entry point's kernels; attt_device_status() reports it.
+// wait of this entry point's kernels; attt_device_status() reports it.  The
+// cached addresses hold for the life of the device's context: a call after
+// cudaDeviceReset() (which re-creates the module's static arrays) is not
+// supported.
 #include <mutex>
 
 #include "attt_host.h"

@@ -143,3 +143,45 @@ def test_binding_rejects_mismatched_shapes():
         attt.attt_lora_input_grad(torch.zeros(8, 32, dtype=bf), torch.zeros(16, 32, dtype=bf),
                                   torch.zeros(16, 4, dtype=bf), torch.zeros(4, 32, dtype=bf), 2.0,
                                   dx=torch.zeros(8, 15))
+
+
+def test_noalloc_scratch_size_matches_the_header():
+    """The binding's size constant is the header's ATTT_LORA_NOALLOC_SCRATCH_BYTES."""
+    from paper_2607_03441_gb300 import attt
+    m = re.search(r"#define\s+ATTT_LORA_NOALLOC_SCRATCH_BYTES\s+\(\(size_t\)(\d+)\s*<<\s*(\d+)\)", open(HEADER).read())
+    assert m, "ATTT_LORA_NOALLOC_SCRATCH_BYTES not found in include/attt.h"
+    assert int(m.group(1)) << int(m.group(2)) == attt.LORA_NOALLOC_SCRATCH_BYTES
+    src = open(os.path.join(ROOT, "paper_2607_03441_gb300", "csrc", "lora_noalloc.cu")).read()
+    assert re.search(r"static __device__ __align__\(256\) unsigned char g_scratch\[kScratchBytes\]", src)
+    assert "kScratchBytes = ATTT_LORA_NOALLOC_SCRATCH_BYTES" in src
+
+
+@pytest.mark.parametrize("entry", ["attt_lora_grad", "attt_lora_grad_noalloc"])
+def test_lora_entry_points_check_arguments_before_any_call(entry):
+    """A wrong dtype, shape or list length raises ValueError on the host,
+    before a pointer reaches the C ABI (CPU tensors: nothing could launch)."""
+    import torch
+    from paper_2607_03441_gb300 import attt
+    L, din, douts, r = 32, 16, [24, 8], 4
+    bf = torch.bfloat16
+
+    def args(**over):
+        a = dict(x=torch.zeros(L, din, dtype=bf), dys=[torch.zeros(L, d, dtype=bf) for d in douts],
+                 As=[torch.zeros(din, r, dtype=bf) for _ in douts], Bs=[torch.zeros(r, d, dtype=bf) for d in douts],
+                 dAs=[torch.zeros(din, r) for _ in douts], dBs=[torch.zeros(r, d) for d in douts])
+        a.update(over)
+        return a
+
+    bad = {
+        "dys[1]": args(dys=[torch.zeros(L, 24, dtype=bf), torch.zeros(L, 8)]),             # fp32 dy
+        "As[0]": args(As=[torch.zeros(din + 1, r, dtype=bf), torch.zeros(din, r, dtype=bf)]),
+        "Bs[1]": args(Bs=[torch.zeros(r, 24, dtype=bf), torch.zeros(r, 16, dtype=bf)]),    # narrower than dout
+        "dAs[0]": args(dAs=[torch.zeros(din, r, dtype=bf), torch.zeros(din, r)]),           # bf16 gradient
+        "dBs[1]": args(dBs=[torch.zeros(r, 24), torch.zeros(r, 4)]),                       # smaller than r x dout
+        "x": args(x=torch.zeros(L, din)),                                                    # fp32 x
+        "one entry per projection": args(Bs=[torch.zeros(r, 24, dtype=bf)]),
+    }
+    fn = getattr(attt, entry)
+    for name, a in bad.items():
+        with pytest.raises(ValueError, match=re.escape(name)):
+            fn(a["x"], a["dys"], a["As"], a["Bs"], 2.0, a["dAs"], a["dBs"])

@@ -72,3 +72,41 @@ def test_update_step_order_with_gradient_steps():
         P = len(u.projs)
         round_ = ["attt_weighted_ce_fwd_bwd", "attt_lora_grad"] + ["attt_lora_step"] * P
         assert u.attt.calls == ["attt_ngram_weights"] + round_ * G + ["attt_history_insert"]
+
+
+def test_peak_kind_follows_region_length_and_clock():
+    """A short region at full clock is held to the burst peak; a long one, or
+    one whose median clock fell below the maximum (power cap), to the
+    sustained peak."""
+    full = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "samples": 5, "reasons": []}
+    capped = {"sm_mhz": 1440.0, "sm_max_mhz": 2070.0, "samples": 5, "reasons": ["sw_power_cap"]}
+    assert bench.peak_kind(53.0, full) == "burst"
+    assert bench.peak_kind(53.0, capped) == "sustained"
+    assert bench.peak_kind(1700.0, full) == "sustained"
+    assert bench.peak_kind(200.0, None) == "burst"
+    assert bench.peak_kind(2000.0, None) == "sustained"
+
+
+def test_ce_roofline_frac_follows_from_the_record():
+    """frac = 4 L V d / ce_ms / the named peak, with both peaks' fractions."""
+    wl = wk.WORKLOADS["32b"]
+    peaks = {"hbm_gbs": 6780.0, "bf16": 1908.6, "bf16_sustained": 1705.1, "src": "measured"}
+    for kind, peak in (("burst", 1908.6), ("sustained", 1705.1)):
+        r = bench._ce_roofline(wl, 15.0, peaks, None, kind)
+        ach = 4.0 * wl.L * wl.V * wl.d / 15e-3 / 1e12
+        assert abs(r["frac"] - ach / peak) < 1e-4 and r["peak"] == peak
+        assert abs(r["frac_of_burst"] - ach / 1908.6) < 1e-4
+        assert abs(r["frac_of_sustained"] - ach / 1705.1) < 1e-4
+
+
+def test_path_roofline_is_the_slower_bound_of_the_whole_update():
+    wl = wk.WORKLOADS["32b"]
+    peaks = {"hbm_gbs": 6780.0, "bf16": 1908.6, "bf16_sustained": 1705.1, "src": "measured"}
+    flops, nbytes = bench.path_work(wl, 1)
+    ce = 4.0 * wl.L * wl.V * wl.d
+    lora = sum(4.0 * wl.L * wl.r * (p.din + p.dout) for p in wl.projs)
+    assert flops == ce + lora
+    assert bench.path_work(wl, 2)[0] == 2 * flops
+    r = bench.path_roofline(wl, 1, 20.0, peaks, "sustained")
+    t_roof = max(flops / 1705.1e12, nbytes / 6780e9)
+    assert r["bound"] == "tensor" and abs(r["frac"] - t_roof / 20e-3) < 1e-4
