@@ -84,12 +84,10 @@ ATTT_API uint64_t attt_kernel_launches(void);
 ATTT_API attt_status attt_device_status(attt_stream stream);
 
 /*
- * Failure-detection self-test: launches one kernel with the two kinds of
- * device-side wait the library uses -- on an mbarrier that nothing completes,
- * and on a global counter that no CTA raises (as between the passes of
- * attt_lora_grad) -- side by side.  Both run out after the library's
- * wall-clock limit of 2 s and return; only then does the kernel record
- * ATTT_ERR_TIMEOUT in the device status word (attt_device_status), and the
+ * Failure-detection self-test: launches one kernel whose only wait (on an
+ * mbarrier that nothing completes) runs out after the library's wall-clock
+ * limit of 2 s, as any device-side wait of the library would, so the device
+ * status word then reads ATTT_ERR_TIMEOUT (attt_device_status) and the
  * context stays usable.  No fault, trap or hang.  Async on `stream`.
  */
 ATTT_API attt_status attt_selftest_wait_timeout(attt_stream stream);
@@ -251,13 +249,8 @@ ATTT_API size_t attt_lora_workspace_bytes(int64_t L, int64_t din, int nproj, con
  *   d_dB[p] = scale * u_p^T dy_p                              (fp32 [r, dout[p]])
  *   d_dA[p] = scale * x^T v_p                                 (fp32 [din, r])
  * u and v are rounded to bf16 before the second contraction; products are
- * bf16, accumulation fp32.  Every sum is taken in a fixed order (the rows in
- * chunks of the call's plan, then the chunks in order), so repeated calls
- * give the same bits.  Two launches: a prep kernel, then one persistent
- * kernel whose CTAs take work items in order from a counter and wait (bounded,
- * ATTT_ERR_TIMEOUT in the device status word) only for items taken earlier.
- * The arrays d_dy, dout, d_A, d_B, d_dA, d_dB are HOST arrays of nproj
- * entries holding device pointers / sizes.
+ * bf16, accumulation fp32.  The arrays d_dy, dout, d_A, d_B, d_dA, d_dB are
+ * HOST arrays of nproj entries holding device pointers / sizes.
  * Requirements: 1 <= nproj <= 8, 1 <= r <= 64, L >= 1, din and every dout
  * >= 8 and multiples of 8, all tensor pointers 16-byte aligned, d_ws at least
  * attt_lora_workspace_bytes(...) bytes and 256-byte aligned.

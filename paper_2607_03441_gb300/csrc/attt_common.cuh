@@ -148,44 +148,6 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
 }
 
 // ---------------------------------------------------------------------------
-// Counters in global memory shared by the CTAs of one grid
-// ---------------------------------------------------------------------------
-
-__device__ __forceinline__ unsigned int ld_acquire_gpu(const unsigned int *p) {
-    unsigned int v;
-    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-
-__device__ __forceinline__ void st_release_gpu(unsigned int *p, unsigned int v) {
-    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
-}
-
-// Orders this thread's generic-proxy global accesses with its later
-// async-proxy (TMA) accesses of global memory (both sides of a hand-off of
-// data that one CTA writes with ordinary stores and another reads by TMA).
-__device__ __forceinline__ void fence_proxy_async_global() {
-    asm volatile("fence.proxy.async.global;" ::: "memory");
-}
-
-// Waits until *ctr >= target (acquire loads at GPU scope).  Returns false if
-// the CTA's abort flag is raised or the wall-clock limit passes first.
-__device__ __forceinline__ bool wait_counter_geq(const unsigned int *ctr, unsigned int target,
-                                                 volatile int *abort_flag) {
-    if (ld_acquire_gpu(ctr) >= target) return true;
-    const unsigned long long t0 = global_ns();
-    uint32_t spins = 0;
-    while (true) {
-        __nanosleep(64);
-        if (ld_acquire_gpu(ctr) >= target) return true;
-        if ((++spins & 15u) == 0u) {
-            if (*abort_flag) return false;
-            if (global_ns() - t0 > kWaitLimitNs) return false;
-        }
-    }
-}
-
-// ---------------------------------------------------------------------------
 // TMA (tensor memory accelerator) tiled loads
 // ---------------------------------------------------------------------------
 

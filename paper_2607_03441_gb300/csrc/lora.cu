@@ -8,10 +8,12 @@
 //   dA  = s x^T [v_0 | v_1 | ...]    one contraction for all p (x read once)
 //   dB_p^T = s dy_p^T u_p            (dout on the 128-row side)
 // Every contraction puts the long dimension (L, din or dout) on the 128-row
-// MMA side and the rank on N, so the tensor core streams x and dy at HBM
-// rate.  Two launches per call: prep (adapters to K-major, counters zeroed)
-// and one persistent launch of both passes over row chunks that stay in L2
-// between the passes (lora_fused.cuh).
+// MMA side and the rank on N, so the tensor core streams x and dy once per
+// pass at HBM rate.  Reductions over L (or din/dout) are split across CTAs
+// (stream-K, tc_group.cuh) and summed in a fixed order by the piece that
+// finishes each tile last; u and v go to bf16 in between.  Three launches per
+// call: prep (adapters to K-major), pass 1 (u and every v_p, grouped), pass 2
+// (dA and every dB_p, grouped).
 //
 // The adapted projection itself (for a chained update, where the projection
 // feeds the LM head): the forward h = x W0 + s (x A) B and the input gradient
@@ -21,118 +23,44 @@
 #include <cmath>
 
 #include "gemm_launch.cuh"
-#include "lora_fused.cuh"
 #include "tc_group.cuh"
 
 namespace attt {
 
-// Rows of x and dy per chunk of the fused launch: two chunks (the one pass 2
-// reads back and the one pass 1 streams) stay in the 126 MB L2 together.
-constexpr int64_t kFusedChunkBytes = 24ll << 20;
-// Work-item size: about six items per SM over both passes (152 SMs; a plan
-// constant, so the workspace size does not depend on the device), each
-// streaming between 64 KB and 256 KB of x or dy.
-constexpr int64_t kFusedPlanSms = 152;
-constexpr int64_t kFusedItemsPerSm = 6;
-constexpr int64_t kFusedItemMin = 64ll << 10, kFusedItemMax = 256ll << 10;
-
-// The plan of one attt_lora_grad call: the fused launch's sizes (FusedArgs
-// without its pointers) and the workspace layout.
-struct LoraPlan {
-    FusedArgs a;
-    __nv_bfloat16 *AT;             // [Nu, din]
-    __nv_bfloat16 *BT[kMaxProj];   // [rpad, dout_p]
-    unsigned int *counters;        // head, p1done [C], tickets [C * t1_full], flags [n2]
-    int64_t ncounters;
-    int64_t total_items;
+struct LoraLayout {
+    int rpad, Nu, BN;
+    int64_t Lp;
+    __nv_bfloat16 *AT;            // [Nu, din]
+    __nv_bfloat16 *BT[kMaxProj];  // [rpad, dout_p]
+    __nv_bfloat16 *uT16, *vT16;   // [Nu, Lp] each, contiguous
+    int64_t tiles;                // group-wide tiles of the larger pass
+    unsigned int *tickets;        // [tiles] arrival counters (both passes)
+    float *part;                  // [tiles + kGroupMaxGrid] partial slots of 128 x BN fp32
     size_t bytes;
 };
 
-static LoraPlan lora_plan(void *ws, int64_t L, int64_t din, int nproj, const int64_t *dout, int r) {
-    LoraPlan pl{};
-    FusedArgs &a = pl.a;
-    a.P = nproj;
-    a.r = r;
-    a.rpad = (int)round_up(r, 16);
-    a.Nu = nproj * a.rpad;
-    a.BNu = a.Nu <= 256 ? a.Nu : 256;
-    a.tn_u = (int)cdiv(a.Nu, a.BNu);
-    a.L = (int)L;
-    a.Lp = (int)round_up(L, 8);
-    a.din = (int)din;
-    int64_t row_bytes = 2 * din;
+static LoraLayout lora_layout(void *ws, int64_t L, int64_t din, int nproj, const int64_t *dout, int r) {
+    LoraLayout c{};
+    c.rpad = (int)round_up(r, 16);
+    c.Nu = nproj * c.rpad;
+    c.BN = c.Nu <= 256 ? c.Nu : 256;
+    c.Lp = round_up(L, 8);
+    // pass 1: u (L x Nu) and each v_p (L x rpad); pass 2: dA (din x Nu) and each dB_p (dout_p x rpad)
+    int64_t t1 = cdiv(L, 128) * cdiv(c.Nu, c.BN), t2 = cdiv(din, 128) * cdiv(c.Nu, c.BN);
     for (int p = 0; p < nproj; ++p) {
-        a.dout[p] = (int)dout[p];
-        row_bytes += 2 * dout[p];
+        t1 += cdiv(L, 128) * cdiv(c.rpad, c.BN);
+        t2 += cdiv(dout[p], 128) * cdiv(c.rpad, c.BN);
     }
-    // chunk rows: the L2 bound, and the item bound (a pass-2 item streams 128
-    // columns of x or dy over the chunk's rows, 256 bytes per row)
-    int64_t item = 2 * L * row_bytes / (kFusedPlanSms * kFusedItemsPerSm);
-    item = item < kFusedItemMin ? kFusedItemMin : (item > kFusedItemMax ? kFusedItemMax : item);
-    int64_t lc = kFusedChunkBytes / row_bytes;
-    if (lc > item / 256) lc = item / 256;
-    lc = lc / 128 * 128;
-    if (lc < 128) lc = 128;
-    const int64_t C = cdiv(L, lc);
-    const int64_t Lc = round_up(cdiv(L, C), 128);
-    a.Lc = (int)Lc;
-    a.C = (int)cdiv(L, Lc);
-    a.mt_full = (int)(Lc / 128);
-    a.mt_last = (int)cdiv(L - (int64_t)(a.C - 1) * Lc, 128);
-    a.kpiece = (int)(Lc / 64 > 4 ? Lc / 64 : 4);
-    a.kb_u = (int)cdiv(din, 64);
-    a.np_u = (int)cdiv(a.kb_u, a.kpiece);
-    a.tm_dA = (int)cdiv(din, 128);
-    int64_t n1_per_mt = (int64_t)a.tn_u * a.np_u;
-    int64_t n2 = (int64_t)a.tn_u * a.tm_dA;
-    for (int p = 0; p < nproj; ++p) {
-        a.kb_v[p] = (int)cdiv(dout[p], 64);
-        a.np_v[p] = (int)cdiv(a.kb_v[p], a.kpiece);
-        a.tm_dB[p] = (int)cdiv(dout[p], 128);
-        a.t2_dB[p] = (int)n2;
-        n1_per_mt += a.np_v[p];
-        n2 += a.tm_dB[p];
-    }
-    const int64_t n1_full = n1_per_mt * a.mt_full, n1_last = n1_per_mt * a.mt_last;
-    pl.total_items = a.C == 1 ? n1_last + n2 : (int64_t)(a.C - 1) * n1_full + n1_last + (int64_t)a.C * n2;
-    a.n1_full = (int)n1_full;
-    a.n1_last = (int)n1_last;
-    a.n2 = (int)n2;
-    a.t1_full = (a.tn_u + nproj) * a.mt_full;
-    a.total_items = (int)(pl.total_items < (1ll << 30) ? pl.total_items : 0);
-    // pass-1 partial slots of one chunk (only tiles cut into pieces), pass-2 running sums
-    int64_t sl = 0;
-    a.slot_u = sl;
-    if (a.np_u > 1) sl += (int64_t)a.tn_u * a.mt_full * a.np_u * 128 * a.BNu;
-    for (int p = 0; p < nproj; ++p) {
-        a.slot_v[p] = sl;
-        if (a.np_v[p] > 1) sl += (int64_t)a.mt_full * a.np_v[p] * 128 * a.rpad;
-    }
-    a.slot_chunk = sl;
-    int64_t ac = 0;
-    if (a.C > 1) {
-        a.acc_dA = ac;
-        ac += (int64_t)a.tn_u * a.tm_dA * 128 * a.BNu;
-        for (int p = 0; p < nproj; ++p) {
-            a.acc_dB[p] = ac;
-            ac += (int64_t)a.tm_dB[p] * 128 * a.rpad;
-        }
-    }
-    pl.ncounters = 1 + a.C + (int64_t)a.C * a.t1_full + n2;
+    c.tiles = t1 > t2 ? t1 : t2;
     Carve cv{static_cast<char *>(ws), 0};
-    pl.AT = cv.take<__nv_bfloat16>((size_t)a.Nu * din);
-    for (int p = 0; p < nproj; ++p) pl.BT[p] = cv.take<__nv_bfloat16>((size_t)a.rpad * dout[p]);
-    a.uT = cv.take<__nv_bfloat16>((size_t)a.Nu * a.Lp);
-    a.vT = cv.take<__nv_bfloat16>((size_t)a.Nu * a.Lp);
-    pl.counters = cv.take<unsigned int>((size_t)pl.ncounters);
-    a.slots = cv.take<float>((size_t)(a.C * sl));
-    a.acc = cv.take<float>((size_t)ac);
-    a.head = pl.counters;
-    a.p1done = pl.counters + 1;
-    a.tickets = a.p1done + a.C;
-    a.flags = a.tickets + (int64_t)a.C * a.t1_full;
-    pl.bytes = (size_t)round_up((int64_t)cv.used, 256);
-    return pl;
+    c.AT = cv.take<__nv_bfloat16>((size_t)(c.Nu * din));
+    for (int p = 0; p < nproj; ++p) c.BT[p] = cv.take<__nv_bfloat16>((size_t)(c.rpad * dout[p]));
+    c.uT16 = cv.take<__nv_bfloat16>((size_t)(2 * c.Nu * c.Lp));
+    c.vT16 = c.uT16 + (size_t)c.Nu * c.Lp;
+    c.tickets = cv.take<unsigned int>((size_t)c.tiles);
+    c.part = cv.take<float>((size_t)(c.tiles + kGroupMaxGrid) * 128 * c.BN);
+    c.bytes = (size_t)round_up((int64_t)cv.used, 256);
+    return c;
 }
 
 struct PrepArgs {
@@ -393,22 +321,22 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
     attt_status st = current_device(&dev);
     if (st != ATTT_OK) return st;
 
-    LoraPlan pl = lora_plan(d_ws, L, din, nproj, dout, r);
-    if (pl.a.total_items <= 0) return ATTT_ERR_UNSUPPORTED;
+    LoraLayout c = lora_layout(d_ws, L, din, nproj, dout, r);
+    const int BN = c.BN;
 
-    // prep: adapters to K-major (rank padded with zeros), counters zeroed
+    // prep: adapters to K-major (rank padded with zeros), accumulators zeroed
     {
         PrepArgs a{};
         int64_t maxn = cdiv(din, kPrepRows) * 256;  // the transpose slabs (one block each)
         for (int p = 0; p < nproj; ++p) {
             a.A[p] = reinterpret_cast<const __nv_bfloat16 *>(d_A[p]);
             a.B[p] = reinterpret_cast<const __nv_bfloat16 *>(d_B[p]);
-            a.BT[p] = pl.BT[p];
+            a.BT[p] = c.BT[p];
             a.dout[p] = dout[p];
-            if (pl.a.rpad * dout[p] > maxn) maxn = pl.a.rpad * dout[p];
+            if (c.rpad * dout[p] > maxn) maxn = c.rpad * dout[p];
         }
-        a.nproj = nproj; a.r = r; a.rpad = pl.a.rpad; a.din = din; a.AT = pl.AT;
-        a.tickets = pl.counters; a.ntickets = pl.ncounters;
+        a.nproj = nproj; a.r = r; a.rpad = c.rpad; a.din = din; a.AT = c.AT;
+        a.tickets = c.tickets; a.ntickets = c.tiles;
         if (a.ntickets / nproj > maxn) maxn = a.ntickets / nproj + 1;
         dim3 grid(grid_for(maxn, 256, dev), nproj);
         lora_prep_kernel<<<grid, 256, 0, stream>>>(a);
@@ -416,52 +344,55 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
         if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
     }
 
-    // both passes in one persistent launch (lora_fused.cuh)
-    FusedArgs g = pl.a;
-    FusedMaps maps;
-    const int BNu = g.BNu, rpad = g.rpad;
-    bool ok = make_tmap_bf16(&maps.x_k, d_x, (uint64_t)din, (uint64_t)L, (uint64_t)din * 2, 64, 128) &&
-              make_tmap_bf16(&maps.x_mn, d_x, (uint64_t)din, (uint64_t)L, (uint64_t)din * 2, 64, 64) &&
-              make_tmap_bf16(&maps.at, pl.AT, (uint64_t)din, (uint64_t)g.Nu, (uint64_t)din * 2, 64, (uint32_t)BNu) &&
-              make_tmap_bf16(&maps.ut, g.uT, (uint64_t)L, (uint64_t)g.Nu, (uint64_t)g.Lp * 2, 64, (uint32_t)rpad) &&
-              make_tmap_bf16(&maps.vt, g.vT, (uint64_t)L, (uint64_t)g.Nu, (uint64_t)g.Lp * 2, 64, (uint32_t)BNu);
-    for (int p = 0; ok && p < nproj; ++p) {
-        ok = make_tmap_bf16(&maps.dy_k[p], d_dy[p], (uint64_t)dout[p], (uint64_t)L, (uint64_t)dout[p] * 2, 64, 128) &&
-             make_tmap_bf16(&maps.dy_mn[p], d_dy[p], (uint64_t)dout[p], (uint64_t)L, (uint64_t)dout[p] * 2, 64, 64) &&
-             make_tmap_bf16(&maps.bt[p], pl.BT[p], (uint64_t)dout[p], (uint64_t)rpad, (uint64_t)dout[p] * 2, 64,
-                            (uint32_t)rpad);
+    // pass 1: u^T = (x AT^T)^T and v_p^T = (dy_p BT_p^T)^T, fp32 sums then bf16
+    {
+        GroupSpec sp[kMaxGroup];
+        int n = 0;
+        GroupSpec &u = sp[n++];
+        u = GroupSpec{};
+        u.a = d_x; u.a_rows_ld = din; u.a_rows = L; u.a_k = din;
+        u.b = c.AT; u.b_rows_ld = din; u.b_rows = c.Nu; u.b_k = din;
+        u.M = (int)L; u.N = c.Nu; u.K = (int)din;
+        u.out = GOUT_T16; u.out16 = c.uT16; u.ld = c.Lp; u.alpha = 1.0f; u.r = c.rpad; u.rpad = c.rpad;
+        for (int q = 0; q < nproj; ++q) {
+            GroupSpec &v = sp[n++];
+            v = GroupSpec{};
+            v.a = d_dy[q]; v.a_rows_ld = dout[q]; v.a_rows = L; v.a_k = dout[q];
+            v.b = c.BT[q]; v.b_rows_ld = dout[q]; v.b_rows = c.rpad; v.b_k = dout[q];
+            v.M = (int)L; v.N = c.rpad; v.K = (int)dout[q];
+            v.out = GOUT_T16; v.out16 = c.vT16 + (size_t)q * c.rpad * c.Lp; v.ld = c.Lp; v.alpha = 1.0f;
+            v.r = c.rpad; v.rpad = c.rpad;
+        }
+        st = launch_group<false, false>(sp, n, BN, c.part, c.tickets, dev, stream, status);
+        if (st != ATTT_OK) return st;
     }
-    if (!ok) return ATTT_ERR_INVALID_ARG;
-    g.scale = scale;
-    for (int p = 0; p < nproj; ++p) {
-        g.dA[p] = d_dA[p];
-        g.dB[p] = d_dB[p];
+
+    // pass 2: dA_p = s x^T v_p (all p at once, x MN-major) and
+    //         dB_p^T = s dy_p^T u_p (dy MN-major), stored transposed into dB_p
+    {
+        GroupSpec sp[kMaxGroup];
+        int n = 0;
+        GroupSpec &a = sp[n++];
+        a = GroupSpec{};
+        a.a = d_x; a.a_rows_ld = din; a.a_rows = din; a.a_k = L;
+        a.b = c.vT16; a.b_rows_ld = c.Lp; a.b_rows = c.Nu; a.b_k = L;  // padding columns read as zeros
+        a.M = (int)din; a.N = c.Nu; a.K = (int)L;
+        a.out = GOUT_N32;
+        for (int q = 0; q < nproj; ++q) a.outp[q] = d_dA[q];
+        a.alpha = scale; a.r = r; a.rpad = c.rpad;
+        for (int q = 0; q < nproj; ++q) {
+            GroupSpec &b = sp[n++];
+            b = GroupSpec{};
+            b.a = d_dy[q]; b.a_rows_ld = dout[q]; b.a_rows = dout[q]; b.a_k = L;
+            b.b = c.uT16; b.b_rows_ld = c.Lp; b.b_rows = c.Nu; b.b_k = L;
+            b.b_n_off = q * c.rpad;
+            b.M = (int)dout[q]; b.N = c.rpad; b.K = (int)L;
+            b.out = GOUT_T32; b.out32 = d_dB[q]; b.ld = dout[q]; b.alpha = scale; b.r = r; b.rpad = c.rpad;
+        }
+        st = launch_group<true, false>(sp, n, BN, c.part, c.tickets, dev, stream, status);
+        if (st != ATTT_OK) return st;
     }
-    g.status = status ? status : device_status_word(dev);
-    g.b_stage_bytes = gemm_b_stage_bytes(BNu);
-    g.acc_cols = gemm_tmem_cols(BNu) / 2;
-    const size_t fixed = 1024 + 8 * (5 + 2 * kFusedRing) + 16 + 16;
-    const size_t per_stage = kABytes + g.b_stage_bytes;
-    int st_n = 8;
-    while (st_n > 2 && fixed + st_n * (per_stage + 16) > kMaxSmem) --st_n;
-    g.stages = st_n;
-    const size_t smem = fixed + (size_t)st_n * (per_stage + 16);
-    if (!set_smem_limit(reinterpret_cast<const void *>(lora_fused_kernel), smem, dev)) return ATTT_ERR_CUDA;
-    const int sms = num_sms(dev);
-    const int grid = pl.total_items < sms ? (int)pl.total_items : sms;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)grid);
-    cfg.blockDim = dim3(kGemmThreads);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    if (cudaLaunchKernelEx(&cfg, lora_fused_kernel, maps, g) != cudaSuccess) return ATTT_ERR_CUDA;
-    count_launch();
-    return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
+    return ATTT_OK;
 }
 
 
@@ -910,9 +841,7 @@ attt_status attt_lora_input_grad(const attt_bf16 *d_dy, const attt_bf16 *d_W0, c
 
 size_t attt_lora_workspace_bytes(int64_t L, int64_t din, int nproj, const int64_t *dout, int r) {
     if (L < 1 || din < 1 || nproj < 1 || nproj > attt::kMaxProj || !dout || r < 1 || r > 64) return 0;
-    for (int p = 0; p < nproj; ++p)
-        if (dout[p] < 1) return 0;
-    return attt::lora_plan(nullptr, L, din, nproj, dout, r).bytes;
+    return attt::lora_layout(nullptr, L, din, nproj, dout, r).bytes;
 }
 
 attt_status attt_lora_grad(const attt_bf16 *d_x, int64_t L, int64_t din, int nproj, const attt_bf16 *const *d_dy,

@@ -128,12 +128,12 @@ def test_sgd_step_bit_exact(attt):
 
 
 def test_launch_counter_counts_every_kernel(attt):
-    """Two projections: prep and one persistent launch of both passes = 2
-    kernels; the SGD step is one more."""
+    """Two projections: prep, pass 1 (u and both v, grouped), pass 2 (dA and
+    both dB, grouped) = 3 kernels; the SGD step is one more."""
     x, dys, As, Bs = _inputs(9, 200, 128, [64, 128], 8)
     n0 = attt.attt_kernel_launches()
     _group(attt, x, dys, As, Bs, 2.0)
-    assert attt.attt_kernel_launches() - n0 == 2
+    assert attt.attt_kernel_launches() - n0 == 3
     A32 = f32_dev(np.zeros((128, 8), np.float32))
     B32 = f32_dev(np.zeros((8, 64), np.float32))
     n1 = attt.attt_kernel_launches()
@@ -142,14 +142,14 @@ def test_launch_counter_counts_every_kernel(attt):
 
 
 @pytest.mark.parametrize("L,din,douts,r", [
-    (2000, 3584, [3584, 512], 16),                               # 8 row chunks, the last one ragged
+    (2000, 3584, [3584, 512], 16),                               # ragged last row tile, tiles split over CTAs
     (1500, 256, [64, 72, 128, 200, 8, 136, 256, 24], 40),        # 8 x 48 = 384 rank columns: two N tiles
-    (777, 1032, [520, 1032], 64),                                # ragged din / dout tiles, pieces of K
+    (777, 1032, [520, 1032], 64),                                # ragged din / dout tiles
 ])
-def test_chunked_shapes_and_repeatability(attt, L, din, douts, r):
-    """Shapes whose plan cuts the rows into several chunks (a pass-2 sum
-    folded in chunk order), splits K into pieces, or tiles the rank columns
-    of u and dA twice; two calls give the same bits."""
+def test_ragged_shapes_and_repeatability(attt, L, din, douts, r):
+    """Ragged row, din and dout tiles, a group whose rank columns take two N
+    tiles of u and dA, and the stream-K split of long tiles; two calls give
+    the same bits."""
     host = _inputs(L + r, L, din, douts, r)
     gA, gB = _check_group(attt, *host)
     hA, hB = _group(attt, *host, 2.0)
