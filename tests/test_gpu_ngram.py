@@ -194,6 +194,47 @@ def test_extreme_ids_and_every_n(attt):
     h.close()
 
 
+def _count_check(attt, h, H, n, rng, picks=300, absent=100, vocab=60):
+    q = np.concatenate([np.stack([H[p:p + n] for p in rng.integers(0, len(H) - n + 1, picks)]),
+                        rng.integers(0, vocab, (absent, n)).astype(np.int32)])
+    got = attt.attt_history_count(h, i32_dev(q)).cpu().numpy()
+    np.testing.assert_array_equal(got, [oracle.count_naive(H, g) for g in q])
+
+
+def test_large_append_between_small_ones_heavy_repeats(attt):
+    """A 180,000-token append between small appends, into one table, over a
+    50-symbol vocabulary (most n-grams repeat, so most inserts compare tokens
+    and add to a count): weights bit-exact, counts exact."""
+    rng = wk.rng_for(13, "bulk")
+    n = 3
+    H = wk.zipf_ids(rng, 200_000, 50)
+    h = attt.attt_history_create(n, len(H))
+    for a, b in ((0, 5000), (5000, 185_000), (185_000, len(H))):
+        attt.attt_history_insert(h, i32_dev(H[a:b]))
+    x = wk.copy_spans(rng, wk.zipf_ids(rng, 3000, 50), H, 0.5)
+    w = attt.attt_ngram_weights(h, i32_dev(x), 0.05).cpu().numpy()
+    _assert_bit_exact(w, oracle.ngram_weights(H, x, n))
+    _count_check(attt, h, H, n, rng, vocab=50)
+    assert attt.attt_history_status(h) == 0
+    h.close()
+
+
+def test_append_of_two_and_a_half_million_tokens(attt):
+    """One append of 2.5 M Zipf tokens over 128,256 ids (a 16 M-slot table):
+    weights bit-exact on an update of copied spans, counts exact."""
+    rng = wk.rng_for(14, "bulk_rounds")
+    n = 4
+    H = wk.zipf_ids(rng, 2_500_000, 128256)
+    h = attt.attt_history_create(n, len(H))
+    attt.attt_history_insert(h, i32_dev(H))
+    x = wk.copy_spans(rng, wk.zipf_ids(rng, 4096, 128256), H, 0.5)
+    w = attt.attt_ngram_weights(h, i32_dev(x), 0.05).cpu().numpy()
+    _assert_bit_exact(w, oracle.ngram_weights(H, x, n))
+    _count_check(attt, h, H, n, rng, vocab=128256)
+    assert attt.attt_history_status(h) == 0
+    h.close()
+
+
 @pytest.mark.slow
 def test_history_at_maximum_length(attt):
     """A history filled to its limit, 2^24 - 2 tokens (the 24-bit position and
