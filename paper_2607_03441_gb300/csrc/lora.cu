@@ -78,38 +78,44 @@ struct PrepArgs {
 // AT[p*rpad + c, i] = A_p[i, c] (zero for c >= r); BT_p[c, o] = B_p[c, o]
 // (zero rows for c >= r); and the tile tickets set to zero, block row p of
 // the grid doing projection p's share.  The transpose goes through shared
-// memory in slabs of 64 rows of A_p (read row-contiguous, written as 128-byte
-// runs of AT).
+// memory in slabs of 64 rows of A_p: a slab is contiguous in A_p and is read
+// as 16-byte vectors, and each thread writes 8 consecutive elements of a row
+// of AT as one 16-byte vector (din, dout and every tensor pointer are
+// multiples of 8 elements / 16 bytes, and a slab starts at a multiple of 64
+// rows).  BT is copied 16 bytes at a time.
 constexpr int kPrepRows = 64;
 
 __global__ void __launch_bounds__(256) lora_prep_kernel(PrepArgs a) {
-    __shared__ __nv_bfloat16 slab[kPrepRows][64 + 2];  // [row of A_p][column c], r <= 64
+    __shared__ __align__(16) __nv_bfloat16 slab[kPrepRows * 64];  // [row of A_p][column c], r <= 64
     griddep_launch_dependents();  // pass 1 may launch; it waits for this grid before reading AT, BT
     const int p = blockIdx.y;
     const int64_t nslab = (a.din + kPrepRows - 1) / kPrepRows;
     for (int64_t sb = blockIdx.x; sb < nslab; sb += gridDim.x) {
         const int64_t k0 = sb * kPrepRows;
-        const int rows = (int)min((int64_t)kPrepRows, a.din - k0);
-        for (int e = threadIdx.x; e < rows * a.r; e += blockDim.x) {
-            const int kk = e / a.r, c = e - kk * a.r;
-            slab[kk][c] = a.A[p][(k0 + kk) * a.r + c];
-        }
+        const int rows = (int)min((int64_t)kPrepRows, a.din - k0);  // a multiple of 8
+        const uint4 *src = reinterpret_cast<const uint4 *>(a.A[p] + k0 * a.r);
+        uint4 *dst = reinterpret_cast<uint4 *>(slab);
+        for (int e = threadIdx.x; e < rows * a.r / 8; e += blockDim.x) dst[e] = src[e];  // slab[kk * r + c]
         __syncthreads();
-        for (int e = threadIdx.x; e < a.rpad * kPrepRows; e += blockDim.x) {
-            const int c = e / kPrepRows, kk = e - c * kPrepRows;
-            if (kk < rows)
-                a.AT[((int64_t)p * a.rpad + c) * a.din + k0 + kk] = c < a.r ? slab[kk][c] : __float2bfloat16_rn(0.f);
+        const int runs = rows / 8;  // 8-row runs per column of AT
+        for (int e = threadIdx.x; e < a.rpad * runs; e += blockDim.x) {
+            const int c = e / runs, kk0 = (e - c * runs) * 8;
+            __align__(16) __nv_bfloat16 v[8];
+#pragma unroll
+            for (int t = 0; t < 8; ++t) v[t] = c < a.r ? slab[(kk0 + t) * a.r + c] : __float2bfloat16_rn(0.f);
+            *reinterpret_cast<uint4 *>(a.AT + ((int64_t)p * a.rpad + c) * a.din + k0 + kk0) =
+                *reinterpret_cast<const uint4 *>(v);
         }
         __syncthreads();
     }
-    const int64_t nB = (int64_t)a.rpad * a.dout[p];
+    const int64_t nB8 = (int64_t)a.rpad * a.dout[p] / 8;  // 16-byte vectors of BT_p
+    const int64_t rB8 = (int64_t)a.r * a.dout[p] / 8;     // of them copied from B_p (rows c < r)
     const int64_t ztk = (a.ntickets + a.nproj - 1) / a.nproj;  // this row's slice of the tickets
-    const int64_t n = nB > ztk ? nB : ztk;
+    const int64_t n = nB8 > ztk ? nB8 : ztk;
+    const uint4 *b_src = reinterpret_cast<const uint4 *>(a.B[p]);
+    uint4 *b_dst = reinterpret_cast<uint4 *>(a.BT[p]);
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-        if (i < nB) {
-            const int c = (int)(i / a.dout[p]);
-            a.BT[p][i] = c < a.r ? a.B[p][i] : __float2bfloat16_rn(0.f);
-        }
+        if (i < nB8) b_dst[i] = i < rB8 ? b_src[i] : make_uint4(0u, 0u, 0u, 0u);
         if (i < ztk && p * ztk + i < a.ntickets) a.tickets[p * ztk + i] = 0u;
     }
 }
@@ -313,7 +319,7 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
     for (int p = 0; p < nproj; ++p) {
         if (!d_dy[p] || !d_A[p] || !d_B[p] || !d_dA[p] || !d_dB[p]) return ATTT_ERR_INVALID_ARG;
         if (dout[p] < 8 || dout[p] % 8 != 0 || dout[p] > (1ll << 30)) return ATTT_ERR_INVALID_ARG;
-        if (!aligned16(d_dy[p])) return ATTT_ERR_INVALID_ARG;
+        if (!aligned16(d_dy[p]) || !aligned16(d_A[p]) || !aligned16(d_B[p])) return ATTT_ERR_INVALID_ARG;
     }
     if (!d_ws || !aligned256(d_ws) || ws_bytes < attt_lora_workspace_bytes(L, din, nproj, dout, r))
         return ATTT_ERR_WORKSPACE;
@@ -333,7 +339,7 @@ attt_status lora_grad_run(const attt_bf16 *d_x, int64_t L, int64_t din, int npro
             a.B[p] = reinterpret_cast<const __nv_bfloat16 *>(d_B[p]);
             a.BT[p] = c.BT[p];
             a.dout[p] = dout[p];
-            if (c.rpad * dout[p] > maxn) maxn = c.rpad * dout[p];
+            if (c.rpad * dout[p] / 8 > maxn) maxn = c.rpad * dout[p] / 8;
         }
         a.nproj = nproj; a.r = r; a.rpad = c.rpad; a.din = din; a.AT = c.AT;
         a.tickets = c.tickets; a.ntickets = c.tiles;
@@ -764,7 +770,7 @@ attt_status attt_lora_forward(const attt_bf16 *d_x, const attt_bf16 *d_W0, const
         a.nproj = 1; a.r = r; a.rpad = c.rpad; a.din = din; a.AT = c.AT;
         a.tickets = c.tickets; a.ntickets = c.tiles;
         int64_t maxn = cdiv(din, kPrepRows) * 256;
-        if (c.rpad * dout > maxn) maxn = c.rpad * dout;
+        if (c.rpad * dout / 8 > maxn) maxn = c.rpad * dout / 8;
         lora_prep_kernel<<<dim3(grid_for(maxn, 256, dev), 1), 256, 0, stream>>>(a);
         count_launch();
         if (cudaGetLastError() != cudaSuccess) return ATTT_ERR_CUDA;
