@@ -68,6 +68,20 @@ def test_ragged_shapes(attt, L, V, d):
     _full_check(attt, h, W, tgt, w)
 
 
+def test_every_row_at_a_multi_tile_size(attt):
+    """L 2,048, d 3,584 (the 7B-class rows and hidden size), V 4,000: eight
+    256-row pair tiles of the logits contraction and 112 tiles of the dh
+    contraction on 76 CTA pairs (a partial last wave, so the tail split);
+    the loss, every row's lse and all of dh against the oracle."""
+    L, V, d = 2048, 4000, 3584
+    h = wk.normal_bf16(21, "h", (L, d), 1.0)
+    W = wk.normal_bf16(21, "W", (V, d), 0.02)
+    rng = wk.rng_for(21, "t")
+    tgt = rng.integers(0, V, L).astype(np.int32)
+    w = rng.choice(np.array([1.0, 0.5, 0.25, 0.05], np.float32), L).astype(np.float32)
+    _full_check(attt, h, W, tgt, w)
+
+
 def test_zero_weights_and_unit_weights(attt):
     L, V, d = 200, 700, 96
     h = wk.normal_bf16(3, "h", (L, d), 1.0)
