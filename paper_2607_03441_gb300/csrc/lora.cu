@@ -294,7 +294,7 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, float *pa
     // a programmatic dependent of the previous kernel of the call (prep, or pass 1)
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid);
-    cfg.blockDim = dim3(kGemmThreads);
+    cfg.blockDim = dim3(kGroupThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];

@@ -648,10 +648,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (!ok) {
                 *abort_flag = 1;
                 record_error(g.status, ATTT_ERR_TIMEOUT);
-                // Let every load already issued land before the CTA retires.
+                // Let every load already issued land before the CTA retires (a wait
+                // of its own, bounded, that the raised abort flag does not cut short).
+                volatile int no_abort = 0;
                 for (int s = 0; s < S; ++s)
                     if (issued_mask & (1u << s))
-                        (void)mbar_wait(full0 + 8 * s, (issued_parity >> s) & 1u, abort_flag);
+                        (void)mbar_wait(full0 + 8 * s, (issued_parity >> s) & 1u, &no_abort);
             }
         }
     } else if (warp == 1) {
@@ -836,6 +838,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (!g.operands_ready) griddep_wait();
             int stage = 0;
             uint32_t phase = 0;
+            uint32_t issued_mask = 0, issued_parity = 0;  // leader: stages whose bytes it expects
             bool ok = true;
             for (int w = cid; w < nwork && ok; w += ncl) {
                 const Work wi = work_item(g, w, tiles_m2);
@@ -844,7 +847,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const int brow0 = wi.tn * g.BN + BNh * (int)rank;
                 for (int kb = wi.kb0; kb < wi.kb1; ++kb) {
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
-                    if (leader) mbar_arrive_expect_tx(full0 + 8 * stage, 2u * (a_bytes + b_bytes));
+                    if (leader) {
+                        mbar_arrive_expect_tx(full0 + 8 * stage, 2u * (a_bytes + b_bytes));
+                        issued_mask |= 1u << stage;
+                        issued_parity = (issued_parity & ~(1u << stage)) | (phase << stage);
+                    }
                     const uint32_t fb = lead_full0 + 8 * stage;
                     const uint32_t a_dst = smem_u32(sA + (size_t)stage * a_bytes);
                     const uint32_t b_dst = smem_u32(sB + (size_t)stage * b_bytes);
@@ -876,6 +883,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (!ok) {
                 *abort_flag = 1;
                 record_error(g.status, ATTT_ERR_TIMEOUT);
+                // The pair's loads of every stage the leader expects land on its barrier:
+                // wait (bounded, a flag of its own) for them before the pair retires.
+                volatile int no_abort = 0;
+                for (int s = 0; s < S; ++s)
+                    if (issued_mask & (1u << s))
+                        (void)mbar_wait(full0 + 8 * s, (issued_parity >> s) & 1u, &no_abort);
             }
         }
     } else if (warp == 1) {

@@ -5,9 +5,9 @@
 // rank on N); launched one by one, each pays a launch, a ramp and a tail
 // that cost more than streaming its operands.  Grouping runs every
 // contraction of a pass in one launch.  The pipeline is the single-CTA one
-// of tc_gemm.cuh (TMA producer warp, MMA warp, four epilogue warps, two TMEM
-// accumulators); only the work decode, the per-problem tensor maps and the
-// epilogue differ.  All problems of a group share BN and the operand majors.
+// of tc_gemm.cuh (MMA warp, four epilogue warps, two TMEM accumulators) with
+// two TMA producer warps instead of one; the work decode, the per-problem
+// tensor maps and the epilogue differ.  All problems of a group share BN and the operand majors.
 //
 // Work is split stream-K style: the K stages of every tile of every problem
 // are laid end to end (problem by problem, tile by tile), and CTA c takes the
@@ -240,8 +240,14 @@ __device__ __forceinline__ void group_segment_epilogue(const GroupArgs<NP> &g, c
     }
 }
 
+// Warps 0 and 6 both feed the ring, taking alternate stages: one thread keeps
+// about one stage of TMA loads in flight at a time (measured on GB300), so two
+// producers double what a CTA streams.  Warp 1 issues the MMAs, warps 2-5 run
+// the epilogue.
+constexpr int kGroupThreads = 224;
+
 template <bool A_MN, bool B_MN, int NP>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+__global__ void __launch_bounds__(kGroupThreads, 1)
     tc_gemm_group_kernel(const __grid_constant__ GroupMaps<NP> maps, const GroupArgs<NP> g) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -292,9 +298,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int64_t x0 = (int64_t)blockIdx.x * g.total_stages / G;
     const int64_t x1 = ((int64_t)blockIdx.x + 1) * g.total_stages / G;
 
-    if (warp == 0) {
+    if (warp == 0 || warp == 6) {
         if (lane == 0) {
             griddep_wait();  // the B operands (adapters, u, v) come from the previous grid
+            const uint32_t pid = warp == 0 ? 0u : 1u;  // this producer's stages: pos % 2 == pid
+            uint32_t pos = 0;
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_parity = 0;
@@ -306,6 +314,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const CUtensorMap *tb = &maps.b[sg.q];
                 const int tm = sg.tm, tn = sg.tn;
                 for (int kb = sg.kb0; kb < sg.kb1; kb += KBS) {
+                    if (((pos++) & 1u) != pid) {  // the other producer's stage
+                        if (++stage == S) { stage = 0; phase ^= 1u; }
+                        continue;
+                    }
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
                     const uint32_t fb = full0 + 8 * stage;
                     mbar_arrive_expect_tx(fb, kABytesS + b_bytes);  // blocks past K arrive as zeros
@@ -334,9 +346,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (!ok) {
                 *abort_flag = 1;
                 record_error(g.status, ATTT_ERR_TIMEOUT);
+                // the loads already issued still land in shared memory: wait (bounded)
+                // for them with a flag of its own, which the raised abort flag does not cut short
+                volatile int no_abort = 0;
                 for (int s = 0; s < S; ++s)
                     if (issued_mask & (1u << s))
-                        (void)mbar_wait(full0 + 8 * s, (issued_parity >> s) & 1u, abort_flag);
+                        (void)mbar_wait(full0 + 8 * s, (issued_parity >> s) & 1u, &no_abort);
             }
         }
     } else if (warp == 1) {
@@ -382,7 +397,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             volatile int no_abort = 0;
             if (!mbar_wait(drain0, 0u, &no_abort)) record_error(g.status, ATTT_ERR_TIMEOUT);
         }
-    } else {
+    } else if (warp >= 2 && warp <= 5) {
         griddep_wait();  // tickets, slots and outputs follow the previous grid
         const int qw = warp & 3;
         const int row = qw * 32 + lane;
