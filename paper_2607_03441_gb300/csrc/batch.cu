@@ -42,6 +42,10 @@ struct attt_batch {
     size_t ws_bytes;
     void *aws;  // the adapted projections' workspace (kept across Eq. 10 within a step)
     size_t aws_bytes;
+    // the histories' append of an update runs on this stream beside the update's
+    // contractions; the update's own stream waits for it before the call returns
+    cudaStream_t side;
+    cudaEvent_t ev_weights, ev_append;
 };
 
 namespace {
@@ -62,6 +66,9 @@ void free_all(attt_batch *b) {
     void *bufs[] = {b->A32, b->B32, b->A0, b->B0, b->dA, b->dB, b->A16, b->B16, b->w, b->rowscale,
                     b->nll, b->dh, b->loss_scratch, b->h, b->dy, b->ws, b->aws};
     for (void *p : bufs) cudaFree(p);
+    if (b->ev_weights) cudaEventDestroy(b->ev_weights);
+    if (b->ev_append) cudaEventDestroy(b->ev_append);
+    if (b->side) cudaStreamDestroy(b->side);
 }
 
 bool config_ok(const attt_batch_config *c) {
@@ -149,6 +156,9 @@ attt_status attt_batch_create(const attt_batch_config *cfg, const attt_bf16 *d_W
          dev_alloc(&b->h, (size_t)rows * c.d) && dev_alloc(&b->dy, (size_t)rows * c.d) &&
          dev_alloc(reinterpret_cast<char **>(&b->ws), b->ws_bytes) &&
          dev_alloc(reinterpret_cast<char **>(&b->aws), b->aws_bytes);
+    ok = ok && cudaStreamCreateWithFlags(&b->side, cudaStreamNonBlocking) == cudaSuccess &&
+         cudaEventCreateWithFlags(&b->ev_weights, cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&b->ev_append, cudaEventDisableTiming) == cudaSuccess;
     if (ok)
         ok = cudaMemcpy(b->A0, d_A0, nA * sizeof(float), cudaMemcpyDeviceToDevice) == cudaSuccess &&
              cudaMemcpy(b->B0, d_B0, nB * sizeof(float), cudaMemcpyDeviceToDevice) == cudaSuccess &&
@@ -207,6 +217,15 @@ attt_status attt_batch_update(attt_batch *b, const int32_t *d_tokens, const attt
     float *losses = d_losses ? d_losses : b->loss_scratch;
 
     st = ngram_weights_batch(b->hist.data(), E, d_tokens, off, c.w_min, b->w, b->rowscale, stream);
+    // nothing below reads the tables, so the histories' append (last in
+    // Algorithm 1) runs on the side stream beside the update's contractions
+    if (st == ATTT_OK) {
+        if (cudaEventRecord(b->ev_weights, stream) != cudaSuccess ||
+            cudaStreamWaitEvent(b->side, b->ev_weights, 0) != cudaSuccess)
+            st = ATTT_ERR_CUDA;
+        if (st == ATTT_OK) st = history_insert_batch(b->hist.data(), E, d_tokens, off, b->side);
+        if (cudaEventRecord(b->ev_append, b->side) != cudaSuccess && st == ATTT_OK) st = ATTT_ERR_CUDA;
+    }
     for (int g = 0; g < c.grad_steps && st == ATTT_OK; ++g) {
         // every episode's current adapter padded and stacked, then h for every row
         st = batch_adapter_prep(b->A16, b->B16, E, c.din, c.d, c.r, rb, b->aws, b->aws_bytes, stream);
@@ -236,7 +255,8 @@ attt_status attt_batch_update(attt_batch *b, const int32_t *d_tokens, const attt
             st = attt_lora_step(b->A32, b->B32, b->dA, b->dB, (int64_t)E * c.din, (int64_t)E * c.d, c.r, c.lr, b->A16,
                                 b->B16, stream);
     }
-    if (st == ATTT_OK) st = history_insert_batch(b->hist.data(), E, d_tokens, off, stream);
+    // the update's stream waits for the append (a no-op before the first one)
+    if (cudaStreamWaitEvent(stream, b->ev_append, 0) != cudaSuccess && st == ATTT_OK) st = ATTT_ERR_CUDA;
     return st;
 }
 

@@ -48,6 +48,11 @@ struct attt_episode {
     int pend_steps;
     void *ws;
     size_t ws_bytes;
+    // Algorithm 1's history append of an update runs on this stream, beside
+    // the update's contractions (it only needs the weights to have read the
+    // table); the update's own stream waits for it before the call returns.
+    cudaStream_t side;
+    cudaEvent_t ev_weights, ev_append;
 };
 
 namespace {
@@ -65,6 +70,19 @@ void free_all(attt_episode *e) {
     void *bufs[] = {e->A32, e->B32, e->A0, e->B0, e->dA, e->dB, e->mA, e->vA, e->mB, e->vB, e->A16, e->B16, e->w,
                     e->dh,  e->losses, e->h, e->dy, e->h_base, e->pend_tok, e->pend_x, e->ws};
     for (void *b : bufs) cudaFree(b);
+    if (e->ev_weights) cudaEventDestroy(e->ev_weights);
+    if (e->ev_append) cudaEventDestroy(e->ev_append);
+    if (e->side) cudaStreamDestroy(e->side);
+}
+
+// H <- H || x on the side stream once the update's weights (enqueued on
+// `stream`) have read the table; ev_append marks its end.
+attt_status append_beside(attt_episode *e, const int32_t *d_tokens, int64_t L, cudaStream_t stream) {
+    if (cudaEventRecord(e->ev_weights, stream) != cudaSuccess ||
+        cudaStreamWaitEvent(e->side, e->ev_weights, 0) != cudaSuccess)
+        return ATTT_ERR_CUDA;
+    const attt_status st = attt_history_insert(e->hist, d_tokens, L, e->side);
+    return cudaEventRecord(e->ev_append, e->side) == cudaSuccess ? st : ATTT_ERR_CUDA;
 }
 
 bool config_ok(const attt_episode_config *c) {
@@ -143,6 +161,9 @@ attt_status attt_episode_create(const attt_episode_config *cfg, const attt_bf16 
          dev_alloc(reinterpret_cast<char **>(&e->ws), e->ws_bytes);
     if (ok && c.optimizer == 1)
         ok = dev_alloc(&e->mA, nA) && dev_alloc(&e->vA, nA) && dev_alloc(&e->mB, nB) && dev_alloc(&e->vB, nB);
+    ok = ok && cudaStreamCreateWithFlags(&e->side, cudaStreamNonBlocking) == cudaSuccess &&
+         cudaEventCreateWithFlags(&e->ev_weights, cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&e->ev_append, cudaEventDisableTiming) == cudaSuccess;
     if (ok) {
         // The initial adapter is copied once; later resets restore it.
         ok = cudaMemcpy(e->A0, d_A0, nA * sizeof(float), cudaMemcpyDeviceToDevice) == cudaSuccess &&
@@ -189,6 +210,9 @@ attt_status attt_episode_update(attt_episode *e, const int32_t *d_tokens, const 
     float *losses = d_losses ? d_losses : e->losses;
 
     attt_status st = attt_ngram_weights(e->hist, d_tokens, L, c.w_min, e->w, stream);
+    // nothing below reads the table, so the append (last in Algorithm 1) runs
+    // beside the update's contractions
+    if (st == ATTT_OK) st = append_beside(e, d_tokens, L, stream);
     for (int g = 0; g < c.grad_steps && st == ATTT_OK; ++g) {
         st = attt_lora_forward(d_x, e->W0, e->A16, e->B16, L, c.din, c.d, c.r, c.scale, e->h, e->ws, e->ws_bytes,
                                stream);
@@ -216,7 +240,8 @@ attt_status attt_episode_update(attt_episode *e, const int32_t *d_tokens, const 
             }
         }
     }
-    if (st == ATTT_OK) st = attt_history_insert(e->hist, d_tokens, L, stream);
+    // the update's stream waits for the append (a no-op before the first one)
+    if (cudaStreamWaitEvent(stream, e->ev_append, 0) != cudaSuccess && st == ATTT_OK) st = ATTT_ERR_CUDA;
     return st;
 }
 
