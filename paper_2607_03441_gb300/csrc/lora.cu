@@ -214,6 +214,13 @@ struct GroupSpec {
 };
 
 constexpr int kGroupMinStages = 2;
+// Ring stages a grouped launch's shared-memory ring keeps when it can (the
+// stage shape: the most K blocks per stage that leaves this many).  Measured
+// on GB300 with two producer warps: five stages of one K block against two of
+// two took the 32B q/k/v group from 158 to 140 us and the o group from 118
+// to 104 us; rings of three or four stages were as fast at 32B and slower for
+// the long episode's q/k/v group.
+constexpr int kGroupMinRing = 5;
 
 // Launches every problem of `specs` in one grouped kernel; every CTA streams
 // the same number of K stages (stream-K split, tc_group.cuh).
@@ -233,11 +240,13 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, float *pa
     // row per block), as long as at least two stages fit in shared memory.
     g.kbs = 1;
     g.stages = 0;
+    // the most K blocks per stage that leaves at least kGroupMinRing stages
+    // (the two producers each keep a few stages in flight), else one block
     for (int kbs = 4; kbs >= 1 && g.stages == 0; kbs /= 2) {
         const size_t per_stage = (size_t)kbs * (kABytes + gemm_b_stage_bytes(BN));
         int st = 8;
         while (st >= 2 && 1024 + st * per_stage + 8 * (2 * st + 5) + 16 > kMaxSmem) --st;
-        if (st >= 2) { g.kbs = kbs; g.stages = st; }
+        if (st >= kGroupMinRing || (kbs == 1 && st >= 2)) { g.kbs = kbs; g.stages = st; }
     }
     if (g.stages == 0) return ATTT_ERR_UNSUPPORTED;
     g.tmem_cols = gemm_tmem_cols(BN);
