@@ -245,7 +245,7 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, float *pa
     for (int kbs = 4; kbs >= 1 && g.stages == 0; kbs /= 2) {
         const size_t per_stage = (size_t)kbs * (kABytes + gemm_b_stage_bytes(BN));
         int st = 8;
-        while (st >= 2 && 1024 + st * per_stage + 8 * (2 * st + 5) + 16 > kMaxSmem) --st;
+        while (st >= 2 && 1024 + st * per_stage + kGroupTBytes + 8 * (2 * st + 5) + 16 > kMaxSmem) --st;
         if (st >= kGroupMinRing || (kbs == 1 && st >= 2)) { g.kbs = kbs; g.stages = st; }
     }
     if (g.stages == 0) return ATTT_ERR_UNSUPPORTED;
@@ -291,7 +291,7 @@ static attt_status launch_group(const GroupSpec *specs, int n, int BN, float *pa
     }
     g.total_stages = stages;
     const size_t smem =
-        1024 + (size_t)g.stages * g.kbs * (kABytes + gemm_b_stage_bytes(BN)) + 8 * (2 * g.stages + 5) + 16;
+        1024 + (size_t)g.stages * g.kbs * (kABytes + gemm_b_stage_bytes(BN)) + kGroupTBytes + 8 * (2 * g.stages + 5) + 16;
     auto kern = tc_gemm_group_kernel<A_MN, B_MN, NP>;
     if (!set_smem_limit(reinterpret_cast<const void *>(kern), smem, dev)) return ATTT_ERR_CUDA;
     // every CTA gets at least kGroupMinStages stages (at least one), so that a

@@ -162,10 +162,49 @@ __device__ __forceinline__ void group_store16(const GroupProblem &p, int m, int 
     }
 }
 
+// Shared memory of the GOUT_T16 stores: two buffers of 16 columns x 128 rows
+// of bf16.
+constexpr uint32_t kGroupTBytes = 2 * 16 * 128 * 2;
+
+// GOUT_T16 columns [col0, col0 + 16) of the tile's 128 rows (m0 + row), all
+// four epilogue warps together: each thread puts its row's 16 values into a
+// 16 x 128 buffer, then 16 rows of out16 go out as 16-byte vectors of 8
+// consecutive m (out16 rows are ld elements long, ld a multiple of 8; rows m
+// past M but below ld hold the accumulator's zero rows and are never read).
+// Two buffers alternate, so one barrier per call orders the writes of a
+// buffer after the reads of its previous use.
+__device__ __forceinline__ void group_store_t16(const GroupProblem &p, int m0, int row, int col0, int n_end,
+                                                const float (&v)[16], uint32_t sbase, uint32_t &chunk) {
+    const uint32_t buf = sbase + (chunk & 1u) * (kGroupTBytes / 2);
+    ++chunk;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const __nv_bfloat16 b = __float2bfloat16_rn(p.alpha * v[i]);
+        asm volatile("st.shared.b16 [%0], %1;" ::"r"(buf + (uint32_t)(i * 128 + row) * 2u),
+                     "h"(*reinterpret_cast<const unsigned short *>(&b))
+                     : "memory");
+    }
+    named_barrier_sync(1, 128);
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const int idx = row + 128 * k;  // 16 rows of out16 x 16 vectors of 8 m
+        const int i = idx >> 4, j = idx & 15;
+        const int col = col0 + i, m = m0 + j * 8;
+        if (col < n_end && m < p.ld) {
+            uint4 val;
+            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(val.x), "=r"(val.y), "=r"(val.z), "=r"(val.w)
+                         : "r"(buf + (uint32_t)(i * 256 + j * 16)));
+            *reinterpret_cast<uint4 *>(p.out16 + (int64_t)col * p.ld + m) = val;
+        }
+    }
+}
+
 // Epilogue of one segment, on CTA `cta` of G (four warps, thread = row).
+// sT / tchunk: the GOUT_T16 buffers (group_store_t16).
 template <int NP>
 __device__ __forceinline__ void group_segment_epilogue(const GroupArgs<NP> &g, const GroupSeg &sg, int64_t cta, int64_t G,
-                                                       int row, uint32_t taddr) {
+                                                       int row, uint32_t taddr, uint32_t sT, uint32_t &tchunk) {
     const GroupProblem &p = g.prob[sg.q];
     const int gm = sg.tm * 128 + row;
     const bool rv = gm < p.M;
@@ -177,7 +216,8 @@ __device__ __forceinline__ void group_segment_epilogue(const GroupArgs<NP> &g, c
             if (n_base + c >= n_end) break;
             float v[16];
             tmem_ld_x16(taddr + (uint32_t)c, v);
-            if (rv) group_store16(p, gm, n_base + c, n_end, v);
+            if (p.out == GOUT_T16) group_store_t16(p, sg.tm * 128, row, n_base + c, n_end, v, sT, tchunk);
+            else if (rv) group_store16(p, gm, n_base + c, n_end, v);
         }
         return;
     }
@@ -236,7 +276,8 @@ __device__ __forceinline__ void group_segment_epilogue(const GroupArgs<NP> &g, c
                 }
             }
         }
-        if (rv) group_store16(p, gm, n_base + c, n_end, s);
+        if (p.out == GOUT_T16) group_store_t16(p, sg.tm * 128, row, n_base + c, n_end, s, sT, tchunk);
+        else if (rv) group_store16(p, gm, n_base + c, n_end, s);
     }
 }
 
@@ -258,7 +299,8 @@ __global__ void __launch_bounds__(kGroupThreads, 1)
     const uint32_t b_bytes = b1 * KBS;
     uint8_t *sA = smem;
     uint8_t *sB = smem + (size_t)S * kABytesS;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + (size_t)S * b_bytes);
+    uint8_t *sT = sB + (size_t)S * b_bytes;  // the GOUT_T16 store buffers
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sT + kGroupTBytes);
     const uint32_t full0 = smem_u32(bars);
     const uint32_t empty0 = smem_u32(bars + S);
     const uint32_t tfull0 = smem_u32(bars + 2 * S);
@@ -402,6 +444,7 @@ __global__ void __launch_bounds__(kGroupThreads, 1)
         const int qw = warp & 3;
         const int row = qw * 32 + lane;
         int it = 0;
+        uint32_t tchunk = 0;
         GroupSeg sg;
         for (int64_t x = x0; group_next(g, x, x1, sg); ++it) {
             const int acc = it & 1;
@@ -416,7 +459,7 @@ __global__ void __launch_bounds__(kGroupThreads, 1)
             (void)mbar_try_wait(tfull0 + 8 * acc, par);
             tc_fence_after();
             const uint32_t taddr = tmem_base + ((uint32_t)(qw * 32) << 16) + (uint32_t)(acc * g.BN);
-            group_segment_epilogue(g, sg, (int64_t)blockIdx.x, G, row, taddr);
+            group_segment_epilogue(g, sg, (int64_t)blockIdx.x, G, row, taddr, smem_u32(sT), tchunk);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
