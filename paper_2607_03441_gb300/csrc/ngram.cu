@@ -79,16 +79,35 @@ __device__ __forceinline__ unsigned int table_lookup(const Slot *table, unsigned
     return 0u;
 }
 
+// The history stream during an insert: positions below old_len from the
+// stream itself, the appended tokens from the caller's buffer (src; null when
+// they are already in the stream), which the insert kernel copies into the
+// stream as it goes, so nothing of that launch reads them there.
+struct HistTokens {
+    const int32_t *hist;
+    const int32_t *src;
+    int64_t old_len;
+    __device__ __forceinline__ int32_t at(int64_t pos) const {
+        return (src && pos >= old_len) ? __ldg(src + (pos - old_len)) : hist[pos];
+    }
+};
+
+__device__ __forceinline__ bool ngram_equal_at(const HistTokens &ht, int64_t pos, const int32_t *g, int n) {
+    for (int i = 0; i < n; ++i)
+        if (ht.at(pos + i) != g[i]) return false;
+    return true;
+}
+
 // Inserts one occurrence (at history position p) of the n-gram g with hash
 // hsh, starting from the result k of the optimistic claim of slot idx.
-__device__ __forceinline__ bool insert_rest(Slot *table, unsigned long long mask, const int32_t *hist,
+__device__ __forceinline__ bool insert_rest(Slot *table, unsigned long long mask, const HistTokens &ht,
                                             const int32_t *g, int n, unsigned long long hsh, Slot claim,
                                             unsigned long long idx, Slot k, int64_t hist_len, int *status) {
     const unsigned int tag = slot_tag(hsh);
     for (int probe = 0; probe < kMaxProbe; ++probe) {
         if (k == 0ull) return true;  // claimed with count 1
         if ((unsigned int)(k >> 48) == tag && ATTT_GUARD((int64_t)slot_pos(k) + n <= hist_len, status) &&
-            ngram_equal(hist + slot_pos(k), g, n)) {
+            ngram_equal_at(ht, slot_pos(k), g, n)) {
             atomicAdd(table + idx, 1ull);  // count lives in the low 24 bits
             return true;
         }
@@ -114,13 +133,13 @@ constexpr int kInsTile = 256 * kInsPer;
 
 // One block of history_insert_kernel's work: new n-gram starts
 // p = p_begin + blk * kInsTile + threadIdx.x, p - p_begin < count.
-__device__ __forceinline__ void insert_block(const int32_t *__restrict__ hist, int64_t p_begin, int64_t count, int n,
+__device__ __forceinline__ void insert_block(const HistTokens &ht, int64_t p_begin, int64_t count, int n,
                                              Slot *table, unsigned long long mask, int *status, int64_t blk) {
     __shared__ int32_t tok[kInsTile + kMaxN];
     const int64_t i0 = blk * kInsTile;
     const int64_t rem = count - i0;
     const int nt = (int)(rem < kInsTile ? rem : kInsTile) + n - 1;  // tokens of this block's n-grams
-    for (int t = threadIdx.x; t < nt; t += blockDim.x) tok[t] = hist[p_begin + i0 + t];
+    for (int t = threadIdx.x; t < nt; t += blockDim.x) tok[t] = ht.at(p_begin + i0 + t);
     __syncthreads();
     unsigned long long hsh[kInsPer], idx[kInsPer];
     Slot claim[kInsPer], k[kInsPer];
@@ -138,16 +157,26 @@ __device__ __forceinline__ void insert_block(const int32_t *__restrict__ hist, i
 #pragma unroll
     for (int q = 0; q < kInsPer; ++q) {
         const int li = q * blockDim.x + threadIdx.x;
-        if (i0 + li < count && !insert_rest(table, mask, hist, tok + li, n, hsh[q], claim[q], idx[q], k[q],
+        if (i0 + li < count && !insert_rest(table, mask, ht, tok + li, n, hsh[q], claim[q], idx[q], k[q],
                                             p_begin + count + n - 1, status))
             record_error(status, ATTT_ERR_TABLE_FULL);
     }
 }
 
-__global__ void __launch_bounds__(256) history_insert_kernel(const int32_t *__restrict__ hist, int64_t p_begin,
+// src (may be null): the appended tokens, new_len - old_len of them, not yet
+// in the stream; the launch copies them to hist[old_len, new_len) besides
+// inserting (one D2D copy fewer per append).
+__global__ void __launch_bounds__(256) history_insert_kernel(int32_t *hist, const int32_t *__restrict__ src,
+                                                             int64_t old_len, int64_t new_len, int64_t p_begin,
                                                              int64_t count, int n, Slot *table,
                                                              unsigned long long mask, int *status) {
-    insert_block(hist, p_begin, count, n, table, mask, status, blockIdx.x);
+    if (src) {
+        const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+        for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < new_len - old_len; j += stride)
+            hist[old_len + j] = __ldg(src + j);
+    }
+    const HistTokens ht{hist, src, src ? old_len : INT64_MAX};
+    insert_block(ht, p_begin, count, n, table, mask, status, blockIdx.x);
 }
 
 // The histories of a batch of episodes (one per blockIdx.y).
@@ -164,7 +193,8 @@ struct InsertBatch {
 __global__ void __launch_bounds__(256) history_insert_batch_kernel(const __grid_constant__ InsertBatch b) {
     const int e = blockIdx.y;
     if ((int64_t)blockIdx.x * kInsTile >= b.count[e]) return;
-    insert_block(b.hist[e], b.p_begin[e], b.count[e], b.n, b.table[e], b.mask[e], b.status[e], blockIdx.x);
+    const HistTokens ht{b.hist[e], nullptr, INT64_MAX};
+    insert_block(ht, b.p_begin[e], b.count[e], b.n, b.table[e], b.mask[e], b.status[e], blockIdx.x);
 }
 
 // count(g, H) for m query n-grams stored row-major [m, n].
@@ -340,9 +370,7 @@ attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_
     if (!h || len < 0 || (len > 0 && !d_tokens)) return ATTT_ERR_INVALID_ARG;
     if (len == 0) return ATTT_OK;
     if (h->len + len > h->max_tokens) return ATTT_ERR_CAPACITY;
-    if (cudaMemcpyAsync(h->d_tokens + h->len, d_tokens, (size_t)len * sizeof(int32_t), cudaMemcpyDeviceToDevice,
-                        stream) != cudaSuccess)
-        return ATTT_ERR_CUDA;
+    const int64_t old_len = h->len;
     const int64_t new_len = h->len + len;
     // New n-grams: every start p whose last token p+n-1 is new, i.e.
     // p in [max(0, old_len - n + 1), new_len - n].
@@ -350,19 +378,27 @@ attt_status attt_history_insert(attt_history *h, const int32_t *d_tokens, int64_
     if (p_begin < 0) p_begin = 0;
     const int64_t p_end = new_len - h->n;  // inclusive
     h->len = new_len;
-    if (p_end < p_begin) return ATTT_OK;
+    if (p_end < p_begin)  // no new n-gram: the tokens only
+        return cudaMemcpyAsync(h->d_tokens + old_len, d_tokens, (size_t)len * sizeof(int32_t),
+                               cudaMemcpyDeviceToDevice, stream) == cudaSuccess
+                   ? ATTT_OK
+                   : ATTT_ERR_CUDA;
     const int64_t count = p_end - p_begin + 1;
     if (attt::fault_take(attt::FAULT_TABLE_FULL)) {
         // an injected full table: the status word reports it as the kernel would
+        // (the tokens are still appended)
         static const int code = ATTT_ERR_TABLE_FULL;
-        return cudaMemcpyAsync(h->d_status, &code, sizeof code, cudaMemcpyHostToDevice, stream) == cudaSuccess
+        return cudaMemcpyAsync(h->d_tokens + old_len, d_tokens, (size_t)len * sizeof(int32_t),
+                               cudaMemcpyDeviceToDevice, stream) == cudaSuccess &&
+                       cudaMemcpyAsync(h->d_status, &code, sizeof code, cudaMemcpyHostToDevice, stream) == cudaSuccess
                    ? ATTT_OK
                    : ATTT_ERR_CUDA;
     }
     const int threads = 256;
     const int64_t blocks = (count + attt::kInsTile - 1) / attt::kInsTile;
-    attt::history_insert_kernel<<<(unsigned)blocks, threads, 0, stream>>>(h->d_tokens, p_begin, count, h->n,
-                                                                          h->d_table, h->capacity - 1, h->d_status);
+    attt::history_insert_kernel<<<(unsigned)blocks, threads, 0, stream>>>(h->d_tokens, d_tokens, old_len, new_len,
+                                                                          p_begin, count, h->n, h->d_table,
+                                                                          h->capacity - 1, h->d_status);
     attt::count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
@@ -392,7 +428,7 @@ attt_status attt_history_restore(attt_history *h, const int32_t *host_tokens, in
     const int64_t count = len - h->n + 1;
     if (count <= 0) return ATTT_OK;
     attt::history_insert_kernel<<<(unsigned)((count + attt::kInsTile - 1) / attt::kInsTile), 256, 0, stream>>>(
-        h->d_tokens, 0, count, h->n, h->d_table, h->capacity - 1, h->d_status);
+        h->d_tokens, nullptr, len, len, 0, count, h->n, h->d_table, h->capacity - 1, h->d_status);
     attt::count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
 }
