@@ -176,7 +176,7 @@ attt_status launch_gemm(const GemmProblem &p, const EpiParams &ep, int dev, cuda
     const size_t smem = gemm_smem_bytes(bn_cta, g.stages, g.e_stage_bytes);
     const int ntiles = g.whole_tiles + (tiles - g.whole_tiles) * g.tail_s;  // work items
     cudaLaunchConfig_t cfg = {};
-    cfg.blockDim = dim3(kGemmThreads);
+    cfg.blockDim = dim3(p.pair ? kGemmPairThreads : kGemmThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[2];

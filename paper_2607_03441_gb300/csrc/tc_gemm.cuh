@@ -90,6 +90,9 @@ struct GemmArgs {
 
 constexpr uint32_t kABytes = 128 * 64 * 2;  // one A stage: 128 rows x 64 bf16
 constexpr int kGemmThreads = 192;
+// The pair kernel runs a second TMA producer warp (warp 6): the two take
+// alternate stages (one issuing thread keeps about one stage in flight).
+constexpr int kGemmPairThreads = 224;
 
 __host__ __device__ inline uint32_t gemm_b_stage_bytes(int BN) { return (uint32_t)BN * 128u; }
 
@@ -767,7 +770,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 // ---------------------------------------------------------------------------
 
 template <int EPI, bool A_MN, bool B_MN>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+__global__ void __launch_bounds__(kGemmPairThreads, 1)
     tc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmA2,
                    const __grid_constant__ CUtensorMap tmB2, const GemmArgs g) {
@@ -832,10 +835,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t lead_full0 = mapa_shared(full0, 0);
     const uint32_t lead_tempty0 = mapa_shared(tempty0, 0);
 
-    if (warp == 0) {
+    if (warp == 0 || warp == 6) {
         if (lane == 0) {
-            // ---------------- TMA producer (both CTAs) ----------------
+            // ---------------- TMA producers (both CTAs; warp 0 even, warp 6 odd stages) ----------------
             if (!g.operands_ready) griddep_wait();
+            const uint32_t pid = warp == 0 ? 0u : 1u;  // this producer's stages: pos % 2 == pid
+            uint32_t pos = 0;
             int stage = 0;
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_parity = 0;  // leader: stages whose bytes it expects
@@ -846,6 +851,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const int arow0 = EPI == EPI_KL ? wi.tm * 128 + 64 * (int)rank : wi.tm * 256 + 128 * (int)rank;
                 const int brow0 = wi.tn * g.BN + BNh * (int)rank;
                 for (int kb = wi.kb0; kb < wi.kb1; ++kb) {
+                    if (((pos++) & 1u) != pid) {
+                        if (++stage == S) { stage = 0; phase ^= 1u; }
+                        continue;
+                    }
                     if (!mbar_wait(empty0 + 8 * stage, phase ^ 1u, abort_flag)) { ok = false; break; }
                     if (leader) {
                         mbar_arrive_expect_tx(full0 + 8 * stage, 2u * (a_bytes + b_bytes));
@@ -933,7 +942,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             volatile int no_abort = 0;
             if (!mbar_wait(drain0, 0u, &no_abort)) record_error(g.status, ATTT_ERR_TIMEOUT);
         }
-    } else {
+    } else if (warp >= 2 && warp <= 5) {
         // ---------------- epilogue (warps 2..5, both CTAs) ----------------
         griddep_wait();  // what the epilogue reads or overwrites may come from the previous grid
         const int q = warp & 3;
