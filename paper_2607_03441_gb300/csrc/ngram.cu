@@ -14,10 +14,14 @@
 //     24 bits).  Equality is decided by comparing the n tokens in the
 //     device-resident history stream (exact, any vocabulary, any n up to 16)
 //     after a tag match;
+//   * lookups are warp-cooperative: eight lanes load eight consecutive
+//     slots of an n-gram's probe run at once and ballots find the empty
+//     slots and the tag matches, which the group then checks token by token
+//     together (one round trip to the table, one per candidate);
 //   * the weights kernel stages the update's tokens for a block in shared
-//     memory with coalesced loads, probes once per n-gram, takes the window
-//     max of the counts from shared memory and applies Eq. 9 with an IEEE
-//     round-to-nearest division (bit-exact with the definition).
+//     memory with coalesced loads, looks up each window once, takes the
+//     window max of the counts from shared memory and applies Eq. 9 with an
+//     IEEE round-to-nearest division (bit-exact with the definition).
 #include <cuda_runtime.h>
 
 #include <new>
@@ -55,28 +59,69 @@ __device__ __forceinline__ unsigned long long ngram_hash(const int32_t *t, int n
     return mix64(h);
 }
 
-__device__ __forceinline__ bool ngram_equal(const int32_t *a, const int32_t *b, int n) {
-    for (int i = 0; i < n; ++i)
-        if (a[i] != b[i]) return false;
-    return true;
-}
+// Lookups are warp-cooperative: a group of kProbeLanes lanes takes one
+// n-gram and loads kProbeLanes consecutive slots of its probe sequence at
+// once (one 64-byte window, at most three 32-byte sectors), and ballots give
+// the group the empty slots and the tag matches.  The candidates are the
+// tag matches before the first empty slot (linear probing places an n-gram
+// before any slot that was empty when it was inserted); each is checked by
+// the group together, lane j comparing tokens j and j + 8, and one more
+// ballot.  A lookup thus costs one round trip to the table and one to the
+// history per candidate, however long the probe run.
+constexpr int kProbeLanes = 8;
 
-// Finds the slot of n-gram `g` (n tokens, anywhere in memory) and returns its
-// count, or 0 if absent.  `hist` is the history token stream.
-__device__ __forceinline__ unsigned int table_lookup(const Slot *table, unsigned long long mask,
+// Count of the n-gram g (n tokens in shared or global memory) with hash hsh,
+// for the group of kProbeLanes lanes that holds it; lanes of groups with
+// active == false take part in the ballots only.  Every lane of the warp
+// calls it (the ballots are over the full warp); the result is returned to
+// every lane of the group.
+__device__ __forceinline__ unsigned int group_lookup(const Slot *table, unsigned long long mask,
                                                      const int32_t *hist, const int32_t *g, int n,
-                                                     unsigned long long hsh, int64_t hist_len, int *status) {
+                                                     unsigned long long hsh, int64_t hist_len, bool active,
+                                                     int *status) {
+    const int lane = threadIdx.x & 31;
+    const int j = lane & (kProbeLanes - 1);
+    const int gsh = lane & ~(kProbeLanes - 1);  // first lane of the group, and its ballot shift
     const unsigned int tag = slot_tag(hsh);
-    unsigned long long idx = hsh & mask;
-    for (int probe = 0; probe < kMaxProbe; ++probe) {
-        const Slot k = __ldcg(table + idx);
-        if (k == 0ull) return 0u;
-        if ((unsigned int)(k >> 48) == tag && ATTT_GUARD((int64_t)slot_pos(k) + n <= hist_len, status) &&
-            ngram_equal(hist + slot_pos(k), g, n))
-            return slot_count(k);
-        idx = (idx + 1) & mask;
+    unsigned long long base = hsh & mask;
+    unsigned int result = 0u;
+    // the n-gram's tokens this lane compares: j and j + 8 (n <= 16)
+    const int32_t g0 = (active && j < n) ? g[j] : 0;
+    const int32_t g1 = (active && j + kProbeLanes < n) ? g[j + kProbeLanes] : 0;
+    for (int round = 0; round < kMaxProbe / kProbeLanes; ++round) {
+        if (!__any_sync(0xffffffffu, active)) break;
+        const Slot k = active ? __ldcg(table + ((base + j) & mask)) : 0ull;
+        const unsigned int empty = (__ballot_sync(0xffffffffu, active && k == 0ull) >> gsh) & 0xFFu;
+        const unsigned int hit =
+            (__ballot_sync(0xffffffffu, active && k != 0ull && (unsigned int)(k >> 48) == tag) >> gsh) & 0xFFu;
+        const int stop = empty ? __ffs(empty) - 1 : kProbeLanes;
+        unsigned int cand = hit & ((1u << stop) - 1u);
+        bool found = false;
+        // the candidates in probe order, one group-wide token compare each
+        for (;;) {
+            const bool have = cand != 0u;
+            if (!__any_sync(0xffffffffu, have)) break;
+            const int src = gsh + (have ? __ffs(cand) - 1 : 0);
+            const Slot kc = __shfl_sync(0xffffffffu, k, src);
+            const int64_t pos = (int64_t)slot_pos(kc);
+            bool ok = have && ATTT_GUARD(pos + n <= hist_len, status);
+            if (ok && j < n) ok = __ldcg(hist + pos + j) == g0;
+            if (ok && j + kProbeLanes < n) ok = __ldcg(hist + pos + j + kProbeLanes) == g1;
+            const unsigned int bad = (__ballot_sync(0xffffffffu, have && !ok) >> gsh) & 0xFFu;
+            if (have && bad == 0u) {
+                result = slot_count(kc);
+                found = true;
+                cand = 0u;
+            } else if (have) {
+                cand &= cand - 1u;
+            }
+        }
+        if (active) {
+            if (found || empty) active = false;
+            else base += kProbeLanes;
+        }
     }
-    return 0u;
+    return result;
 }
 
 // The history stream during an insert: positions below old_len from the
@@ -197,47 +242,51 @@ __global__ void __launch_bounds__(256) history_insert_batch_kernel(const __grid_
     insert_block(ht, b.p_begin[e], b.count[e], b.n, b.table[e], b.mask[e], b.status[e], blockIdx.x);
 }
 
-// count(g, H) for m query n-grams stored row-major [m, n].
+// count(g, H) for m query n-grams stored row-major [m, n], one probe group
+// per query.
 __global__ void __launch_bounds__(256) history_count_kernel(const int32_t *__restrict__ hist, int64_t hist_len,
                                                             const Slot *table, unsigned long long mask,
                                                             const int32_t *__restrict__ q, int64_t m, int n,
                                                             unsigned int *out, int *status) {
-    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= m) return;
-    const int32_t *g = q + i * n;
-    out[i] = table_lookup(table, mask, hist, g, n, ngram_hash(g, n), hist_len, status);
+    const int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / kProbeLanes;
+    const bool active = i < m;
+    const int32_t *g = q + (active ? i : 0) * n;
+    const unsigned int c = group_lookup(table, mask, hist, g, n, active ? ngram_hash(g, n) : 0ull, hist_len,
+                                        active, status);
+    if (active && (threadIdx.x & (kProbeLanes - 1)) == 0) out[i] = c;
 }
 
-constexpr int kWTile = 256;                 // positions j per block
-constexpr int kWThreads = kWTile + kMaxN;  // one thread per candidate window (at most kWTile + n - 1)
+constexpr int kWTile = 48;                              // positions j per block
+constexpr int kWWin = kWTile + kMaxN;                       // candidate windows (at most kWTile + n - 1)
+constexpr int kWThreads = kProbeLanes * kWWin;              // one probe group per window
 
 // Eq. 8 then Eq. 9 for positions [j0, j0 + kWTile) of the update.  Each
-// window has its own thread, so a block's critical path is one lookup.
+// window has its own probe group, so a block's critical path is one
+// cooperative lookup; the window max and Eq. 9 take one thread per position.
 // rowscale (may be null) receives `scale` at every position written.
 __device__ __forceinline__ void weights_block(const int32_t *__restrict__ x, int64_t L, int n,
                                               const int32_t *__restrict__ hist, int64_t hist_len, const Slot *table,
                                               unsigned long long mask, float w_min, float *__restrict__ w,
                                               float *__restrict__ rowscale, float scale, int64_t j0) {
     __shared__ int32_t tok[kWTile + 2 * kMaxN];
-    __shared__ unsigned int cnt[kWTile + kMaxN];
+    __shared__ unsigned int cnt[kWWin];
     // Window starts s that cover some j in the tile: s in [j0-n+1, j0+kWTile-1]
     // clipped to [0, L-n].  Tokens needed: x[s0 .. s1+n-1].
     const int64_t s_lo = j0 - (n - 1);
-    const int64_t nwin = kWTile + n - 1;  // candidate windows, indexed by s - s_lo
+    const int nwin = kWTile + n - 1;  // candidate windows, indexed by s - s_lo
     // stage tokens x[s_lo .. s_lo + nwin + n - 2] (coalesced)
-    const int ntok = (int)(nwin + n - 1);
+    const int ntok = nwin + n - 1;
     for (int i = threadIdx.x; i < ntok; i += blockDim.x) {
         const int64_t pos = s_lo + i;
         tok[i] = (pos >= 0 && pos < L) ? __ldg(x + pos) : 0;
     }
     __syncthreads();
-    for (int i = threadIdx.x; i < nwin; i += blockDim.x) {
-        const int64_t s = s_lo + i;
-        unsigned int c = 0u;
-        if (s >= 0 && s + n <= L && hist_len >= n)
-            c = table_lookup(table, mask, hist, tok + i, n, ngram_hash(tok + i, n), hist_len, nullptr);
-        cnt[i] = c;
-    }
+    const int i = threadIdx.x / kProbeLanes;  // this lane's window
+    const int64_t s = s_lo + i;
+    const bool valid = i < nwin && s >= 0 && s + n <= L && hist_len >= n;
+    const unsigned long long hsh = valid ? ngram_hash(tok + i, n) : 0ull;
+    const unsigned int c = group_lookup(table, mask, hist, tok + (valid ? i : 0), n, hsh, hist_len, valid, nullptr);
+    if ((threadIdx.x & (kProbeLanes - 1)) == 0 && i < nwin) cnt[i] = c;
     __syncthreads();
     const int64_t j = j0 + threadIdx.x;
     if (threadIdx.x >= kWTile || j >= L) return;
@@ -448,7 +497,8 @@ attt_status attt_history_count(const attt_history *h, const int32_t *d_ngrams, i
     if (!h || m < 0 || (m > 0 && (!d_ngrams || !d_counts))) return ATTT_ERR_INVALID_ARG;
     if (m == 0) return ATTT_OK;
     const int threads = 256;
-    attt::history_count_kernel<<<(unsigned)((m + threads - 1) / threads), threads, 0, stream>>>(
+    const int64_t per_block = threads / attt::kProbeLanes;
+    attt::history_count_kernel<<<(unsigned)((m + per_block - 1) / per_block), threads, 0, stream>>>(
         h->d_tokens, h->len, h->d_table, h->capacity - 1, d_ngrams, m, h->n, d_counts, h->d_status);
     attt::count_launch();
     return cudaGetLastError() == cudaSuccess ? ATTT_OK : ATTT_ERR_CUDA;
