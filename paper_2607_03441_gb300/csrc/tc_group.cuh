@@ -242,43 +242,42 @@ __device__ __forceinline__ void group_segment_epilogue(const GroupArgs<NP> &g, c
         __threadfence();
     }
     if (!named_barrier_or(1, 128, last)) return;
-    // The last piece sums the tile 64 columns at a time: each other piece's 64
-    // columns are 16 float4 loads in flight together (one round trip per piece
-    // and 64 columns instead of per 16), added in CTA order.
-    for (int c = 0; c < g.BN; c += 64) {
+    for (int c = 0; c < g.BN; c += 16) {
         if (n_base + c >= n_end) break;
-        const int nq = min(4, (n_end - n_base - c + 15) / 16);  // 16-column chunks of this batch
-        float s[64];
-        for (int64_t j = c0; j <= c1; ++j) {
-            float f[64];
-            if (j == cta) {
+        float own[16];
+        tmem_ld_x16(taddr + (uint32_t)c, own);
+        float s[16];
+        // pieces in CTA order, four partials loaded together (their loads in
+        // flight at once), summed in order after they land
+        for (int64_t j0 = c0; j0 <= c1; j0 += 4) {
+            float4 f[4][4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    if (i < nq) tmem_ld_x16(taddr + (uint32_t)(c + 16 * i), *reinterpret_cast<float(*)[16]>(f + 16 * i));
-            } else {
-                const float4 *src = reinterpret_cast<const float4 *>(g.part + (size_t)(j + gtile) * slot) + row;
+            for (int b = 0; b < 4; ++b) {
+                const int64_t j = j0 + b;
+                if (j <= c1 && j != cta) {
+                    const float4 *src = reinterpret_cast<const float4 *>(g.part + (size_t)(j + gtile) * slot) + row;
 #pragma unroll
-                for (int i = 0; i < 16; ++i)
-                    if (i < 4 * nq) {
-                        const float4 x = __ldcg(src + (size_t)(c / 4 + i) * 128);
-                        f[4 * i] = x.x; f[4 * i + 1] = x.y; f[4 * i + 2] = x.z; f[4 * i + 3] = x.w;
+                    for (int q = 0; q < 4; ++q) f[b][q] = __ldcg(src + (size_t)(c / 4 + q) * 128);
+                }
+            }
+#pragma unroll
+            for (int b = 0; b < 4; ++b) {
+                const int64_t j = j0 + b;
+                if (j > c1) break;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 x = (j == cta) ? make_float4(own[4 * q], own[4 * q + 1], own[4 * q + 2], own[4 * q + 3])
+                                                : f[b][q];
+                    if (j == c0) {
+                        s[4 * q] = x.x; s[4 * q + 1] = x.y; s[4 * q + 2] = x.z; s[4 * q + 3] = x.w;
+                    } else {
+                        s[4 * q] += x.x; s[4 * q + 1] += x.y; s[4 * q + 2] += x.z; s[4 * q + 3] += x.w;
                     }
-            }
-            if (j == c0) {
-#pragma unroll
-                for (int i = 0; i < 64; ++i) s[i] = f[i];
-            } else {
-#pragma unroll
-                for (int i = 0; i < 64; ++i) s[i] += f[i];
+                }
             }
         }
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            if (i >= nq) break;
-            const float(&v)[16] = *reinterpret_cast<const float(*)[16]>(s + 16 * i);
-            if (p.out == GOUT_T16) group_store_t16(p, sg.tm * 128, row, n_base + c + 16 * i, n_end, v, sT, tchunk);
-            else if (rv) group_store16(p, gm, n_base + c + 16 * i, n_end, v);
-        }
+        if (p.out == GOUT_T16) group_store_t16(p, sg.tm * 128, row, n_base + c, n_end, s, sT, tchunk);
+        else if (rv) group_store16(p, gm, n_base + c, n_end, s);
     }
 }
 
