@@ -121,21 +121,37 @@ __global__ void __launch_bounds__(256) lora_prep_kernel(PrepArgs a) {
 }
 
 // SGD: p <- p - lr * g (product then difference, both rounded), bf16 refresh.
-__global__ void lora_step_kernel(float *A32, const float *dA, __nv_bfloat16 *A16, int64_t nA, float *B32,
-                                 const float *dB, __nv_bfloat16 *B16, int64_t nB, float lr) {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nA + nB;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        if (i < nA) {
-            const float v = __fsub_rn(A32[i], __fmul_rn(lr, dA[i]));
-            A32[i] = v;
-            if (A16) A16[i] = __float2bfloat16_rn(v);
-        } else {
-            const int64_t k = i - nA;
-            const float v = __fsub_rn(B32[k], __fmul_rn(lr, dB[k]));
-            B32[k] = v;
-            if (B16) B16[k] = __float2bfloat16_rn(v);
+// One tensor (n elements): four elements per thread step (16-byte loads of p
+// and g, a 16-byte store of p, an 8-byte store of the bf16 copy) when every
+// pointer allows it, else one.
+__device__ __forceinline__ void sgd_range(float *p32, const float *g, __nv_bfloat16 *p16, int64_t n, float lr,
+                                          int64_t t0, int64_t stride) {
+    const bool vec = ((reinterpret_cast<uintptr_t>(p32) | reinterpret_cast<uintptr_t>(g)) & 15) == 0 &&
+                     (reinterpret_cast<uintptr_t>(p16) & 7) == 0;
+    const int64_t n4 = vec ? n / 4 : 0;
+    for (int64_t i = t0; i < n4; i += stride) {
+        const float4 p = reinterpret_cast<const float4 *>(p32)[i];
+        const float4 d = reinterpret_cast<const float4 *>(g)[i];
+        const float4 v = make_float4(__fsub_rn(p.x, __fmul_rn(lr, d.x)), __fsub_rn(p.y, __fmul_rn(lr, d.y)),
+                                     __fsub_rn(p.z, __fmul_rn(lr, d.z)), __fsub_rn(p.w, __fmul_rn(lr, d.w)));
+        reinterpret_cast<float4 *>(p32)[i] = v;
+        if (p16) {
+            __nv_bfloat162 o[2] = {__floats2bfloat162_rn(v.x, v.y), __floats2bfloat162_rn(v.z, v.w)};
+            reinterpret_cast<uint2 *>(p16)[i] = *reinterpret_cast<uint2 *>(o);
         }
     }
+    for (int64_t i = 4 * n4 + t0; i < n; i += stride) {
+        const float v = __fsub_rn(p32[i], __fmul_rn(lr, g[i]));
+        p32[i] = v;
+        if (p16) p16[i] = __float2bfloat16_rn(v);
+    }
+}
+
+__global__ void lora_step_kernel(float *A32, const float *dA, __nv_bfloat16 *A16, int64_t nA, float *B32,
+                                 const float *dB, __nv_bfloat16 *B16, int64_t nB, float lr) {
+    const int64_t t0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x, stride = (int64_t)gridDim.x * blockDim.x;
+    sgd_range(A32, dA, A16, nA, lr, t0, stride);
+    sgd_range(B32, dB, B16, nB, lr, t0, stride);
 }
 
 // AdamW (decoupled weight decay) on the fp32 masters of A and B, with the
@@ -877,7 +893,7 @@ attt_status attt_lora_step(float *d_A32, float *d_B32, const float *d_dA, const 
     attt_status st = current_device(&dev);
     if (st != ATTT_OK) return st;
     const int64_t nA = din * r, nB = (int64_t)r * dout;
-    lora_step_kernel<<<grid_for(nA + nB, 256, dev), 256, 0, stream>>>(
+    lora_step_kernel<<<grid_for((nA + nB) / 4 + 1, 256, dev), 256, 0, stream>>>(
         d_A32, d_dA, reinterpret_cast<__nv_bfloat16 *>(d_A16), nA, d_B32, d_dB,
         reinterpret_cast<__nv_bfloat16 *>(d_B16), nB, lr);
     count_launch();

@@ -108,17 +108,32 @@ def test_workload(attt, name):
                      [dense[f"B/{p.name}"] for p in projs], wl.scale)
 
 
-def test_sgd_step_bit_exact(attt):
-    din, dout, r = 384, 200, 16
-    rng = np.random.default_rng(0)
+def _offset_view(arr, dtype, off):
+    """A contiguous device copy of arr that starts `off` elements into its
+    allocation (off = 1 leaves it without 16-byte alignment)."""
+    n = int(np.prod(arr.shape))
+    buf = torch.empty(n + off, dtype=dtype, device=DEV)
+    v = buf[off:].view(*arr.shape)
+    if arr.dtype != np.float32 or dtype != torch.float32:
+        return v
+    v.copy_(torch.from_numpy(arr))
+    return v
+
+
+@pytest.mark.parametrize("din,dout,r,off", [(384, 200, 16, 0), (37, 19, 3, 1), (130, 66, 5, 1), (64, 64, 4, 2)])
+def test_sgd_step_bit_exact(attt, din, dout, r, off):
+    """Both the four-wide path (aligned, sizes a multiple of four) and the
+    one-wide path (offset buffers, ragged sizes) against the oracle."""
+    rng = np.random.default_rng(din + dout + r + off)
     A = rng.standard_normal((din, r)).astype(np.float32) * 0.02
     B = rng.standard_normal((r, dout)).astype(np.float32) * 0.01
     dA = rng.standard_normal((din, r)).astype(np.float32)
     dB = rng.standard_normal((r, dout)).astype(np.float32)
-    A32, B32 = f32_dev(A), f32_dev(B)
-    A16 = torch.empty(din, r, dtype=torch.bfloat16, device=DEV)
-    B16 = torch.empty(r, dout, dtype=torch.bfloat16, device=DEV)
-    attt.attt_lora_step(A32, B32, f32_dev(dA), f32_dev(dB), 5e-4, A16, B16)
+    A32, B32 = _offset_view(A, torch.float32, off), _offset_view(B, torch.float32, off)
+    A16 = _offset_view(A, torch.bfloat16, off)
+    B16 = _offset_view(B, torch.bfloat16, off)
+    attt.attt_lora_step(A32, B32, _offset_view(dA, torch.float32, off), _offset_view(dB, torch.float32, off), 5e-4,
+                        A16, B16)
     pA, bA = oracle.sgd_step(A, dA, 5e-4)
     pB, bB = oracle.sgd_step(B, dB, 5e-4)
     np.testing.assert_array_equal(A32.cpu().numpy(), pA)
