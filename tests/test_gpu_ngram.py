@@ -116,9 +116,9 @@ def test_edge_cases(attt):
     rng = wk.rng_for(3, "edge")
     H = wk.zipf_ids(rng, 3000, 16)
     # L < n, L == n, L == 1, L == 0, and ragged tile tails
-    for L in (0, 1, 2, 3, 4, 5, 255, 256, 257, 511, 513):
+    for L in (0, 1, 2, 3, 4, 5, 47, 48, 49, 95, 96, 97, 255, 256, 257, 511, 513):
         x = wk.zipf_ids(rng, L, 16)
-        for n in (1, 4):
+        for n in (1, 4, 16):
             if L == 0:
                 h = attt.attt_history_create(n, len(H))
                 attt.attt_history_insert(h, i32_dev(H))
@@ -264,3 +264,58 @@ def test_history_at_maximum_length(attt):
     np.testing.assert_array_equal(got, [oracle.count_naive(H, g) for g in q])
     assert got[-1] == 1 and attt.attt_history_status(h) == 0
     h.close()
+
+
+_M64 = (1 << 64) - 1
+
+
+def _table_home(tokens, mask):
+    """Home slot of an n-gram in the device table: the table's 64-bit hash
+    (an odd multiply per token, then a finalizer) masked to the capacity.
+    White-box: used only to build inputs with long probe runs."""
+    h = (0x9e3779b97f4a7c15 * (len(tokens) + 1)) & _M64
+    for t in tokens:
+        h = ((h ^ (int(t) & 0xFFFFFFFF)) * 0xbf58476d1ce4e5b9) & _M64
+    for mul in (0xff51afd7ed558ccd, 0xc4ceb9fe1a85ec53):
+        h ^= h >> 33
+        h = (h * mul) & _M64
+    h ^= h >> 33
+    return h & mask
+
+
+@pytest.mark.parametrize("n", [1, 2])
+def test_long_probe_runs(attt, n):
+    """N-grams whose home slots crowd into a few slots of a 1,024-slot table
+    form one probe run of ~40 slots, so inserts probe past their home and a
+    lookup (present or absent) reads several eight-slot windows.  Weights and
+    counts against the oracle."""
+    mask = 1023  # the table of a history of <= 256 tokens
+    rng = np.random.default_rng(40 + n)
+    crowd = []
+    while len(crowd) < 60:
+        g = rng.integers(0, 1 << 20, n).astype(np.int32)
+        if 500 <= _table_home(g, mask) < 504:
+            crowd.append(g)
+    present, absent = crowd[:40], crowd[40:]
+    H = np.concatenate(present).astype(np.int32)  # every window of H starting at a multiple of n is crowded
+    # the run: linear probing of H's n-grams, in order, from their home slots
+    used = set()
+    for p in range(len(H) - n + 1):
+        s = _table_home(H[p:p + n], mask)
+        while s in used:
+            s = (s + 1) & mask
+        used.add(s)
+    run = 0
+    while (500 + run) & mask in used:
+        run += 1
+    assert run > 3 * 8, run
+    x = np.concatenate(present[::3] + absent + present[1::5]).astype(np.int32)
+    w = _weights(attt, H, x, n, max_tokens=len(H))
+    _assert_bit_exact(w, oracle.ngram_weights(H, x, n))
+    h = attt.attt_history_create(n, len(H))
+    attt.attt_history_insert(h, i32_dev(H))
+    q = np.stack(crowd).astype(np.int32)
+    got = attt.attt_history_count(h, i32_dev(q)).cpu().numpy()
+    assert attt.attt_history_status(h) == 0
+    h.close()
+    np.testing.assert_array_equal(got, [oracle.count_naive(H, g) for g in q])
