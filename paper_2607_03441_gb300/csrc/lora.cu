@@ -232,10 +232,9 @@ struct GroupSpec {
 constexpr int kGroupMinStages = 2;
 // Ring stages a grouped launch's shared-memory ring keeps when it can (the
 // stage shape: the most K blocks per stage that leaves this many).  Measured
-// on GB300 with two producer warps: five stages of one K block against two of
-// two took the 32B q/k/v group from 158 to 140 us and the o group from 118
-// to 104 us; rings of three or four stages were as fast at 32B and slower for
-// the long episode's q/k/v group.
+// on GB300 (A/B in one process, the order of the two builds alternating):
+// five stages of one K block against two of two took the 32B-class q/k/v
+// group from 145.5 to 131.7 us and the o group from 121.5 to 106.6 us.
 constexpr int kGroupMinRing = 5;
 
 // Launches every problem of `specs` in one grouped kernel; every CTA streams

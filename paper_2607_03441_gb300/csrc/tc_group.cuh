@@ -282,9 +282,10 @@ __device__ __forceinline__ void group_segment_epilogue(const GroupArgs<NP> &g, c
 }
 
 // Warps 0 and 6 both feed the ring, taking alternate stages: one thread keeps
-// about one stage of TMA loads in flight at a time (measured on GB300), so two
-// producers double what a CTA streams.  Warp 1 issues the MMAs, warps 2-5 run
-// the epilogue.
+// about one stage of TMA loads in flight at a time (measured on GB300 for a CTA
+// streaming alone), so two producers double what a lone CTA streams; with every
+// SM streaming, the grid's read rate is HBM's either way.  Warp 1 issues the
+// MMAs, warps 2-5 run the epilogue.
 constexpr int kGroupThreads = 224;
 
 template <bool A_MN, bool B_MN, int NP>
