@@ -167,10 +167,14 @@ class Update:
         self.loss = torch.empty(1, dtype=torch.float32, device=dev)
         self.dh = torch.empty(L, d, dtype=torch.float32, device=dev)
         self.ws_ce = torch.empty(attt.attt_ce_workspace_bytes(L, d, V), dtype=torch.uint8, device=dev)
-        ws = max(attt.attt_lora_workspace_bytes(L, self.projs[idx[0]].din, [self.projs[i].dout for i in idx], r)
-                 for idx in self.groups.values())
-        self.ws_lora = torch.empty(ws, dtype=torch.uint8, device=dev)  # groups run one after another
+        # The groups' gradients are independent (own x, dy, adapters and outputs): the first group runs
+        # on the update's stream and every other one on a side stream of its own, each with its own
+        # workspace, so one group's ramp and tail overlap another's streaming.
+        self.ws_lora = {gname: torch.empty(attt.attt_lora_workspace_bytes(
+            L, self.projs[idx[0]].din, [self.projs[i].dout for i in idx], r), dtype=torch.uint8, device=dev)
+            for gname, idx in self.groups.items()}
         self.stream = torch.cuda.current_stream()
+        self.side = [torch.cuda.Stream(device=dev) for _ in list(self.groups)[1:]]
 
     ROWS = ("ngram_weights", "weighted_ce_fwd_bwd", "lora_grad", "lora_step", "history_insert")
 
@@ -197,10 +201,25 @@ class Update:
                 mark("weighted_ce_fwd_bwd", 1, g)
             if part in ("all", "lora"):
                 mark("lora_grad", 0, g)
-                for gname, idx in self.groups.items():
+                names = list(self.groups)
+                main = self.torch.cuda.current_stream() if len(names) > 1 else None
+                if main is not None:
+                    fork = self.torch.cuda.Event()
+                    fork.record(main)
+                for k, gname in enumerate(names):
+                    idx = self.groups[gname]
+                    kw = {}
+                    if k > 0:  # a side stream of its own, after everything before the fork
+                        self.side[k - 1].wait_event(fork)
+                        kw["stream"] = self.side[k - 1]
                     a.attt_lora_grad(self.xin[gname], [self.dy[i] for i in idx], [self.A16[i] for i in idx],
                                      [self.B16[i] for i in idx], self.wl.scale, dAs=[self.dA[i] for i in idx],
-                                     dBs=[self.dB[i] for i in idx], workspace=self.ws_lora)
+                                     dBs=[self.dB[i] for i in idx], workspace=self.ws_lora[gname], **kw)
+                if main is not None:
+                    for st in self.side:
+                        join = self.torch.cuda.Event()
+                        join.record(st)
+                        main.wait_event(join)
                 mark("lora_grad", 1, g)
                 mark("lora_step", 0, g)
                 for i in range(len(self.projs)):

@@ -63,7 +63,8 @@ def test_update_step_order_with_gradient_steps():
     for G in (1, 2):
         u = object.__new__(bench.Update)
         u.attt, u.wl, u.grad_steps = _Recorder(), wl, G
-        u.hist = u.x = u.w = u.h = u.W = u.loss = u.dh = u.ws_ce = u.ws_lora = None
+        u.hist = u.x = u.w = u.h = u.W = u.loss = u.dh = u.ws_ce = None
+        u.ws_lora = {"attn": None}
         u.projs = list(wl.projs)
         u.groups = {"attn": list(range(len(u.projs)))}
         u.xin = {"attn": None}
