@@ -111,3 +111,79 @@ def test_path_roofline_is_the_slower_bound_of_the_whole_update():
     r = bench.path_roofline(wl, 1, 20.0, peaks, "sustained")
     t_roof = max(flops / 1705.1e12, nbytes / 6780e9)
     assert r["bound"] == "tensor" and abs(r["frac"] - t_roof / 20e-3) < 1e-4
+
+
+class _FakeCuda:
+    """Stands in for torch.cuda's streams and events: records, on one shared
+    log, which stream each event is recorded on and what each stream waits
+    for."""
+
+    def __init__(self):
+        self.log = []
+        outer = self
+
+        class Stream:
+            def __init__(self, name):
+                self.name = name
+
+            def wait_event(self, ev):
+                outer.log.append(("wait", self.name, ev.name))
+
+        class Event:
+            n = 0
+
+            def __init__(self, *a, **k):
+                Event.n += 1
+                self.name = f"ev{Event.n}"
+
+            def record(self, stream=None):
+                outer.log.append(("record", stream.name if stream else "main", self.name))
+
+        self.Stream, self.Event = Stream, Event
+        self.main = Stream("main")
+
+    def current_stream(self):
+        return self.main
+
+
+class _StreamRecorder(_Recorder):
+    """Records each call's name and the stream it was given."""
+
+    def __getattr__(self, name):
+        def call(*args, **kwargs):
+            st = kwargs.get("stream")
+            self.calls.append((name, st.name if st is not None else "main"))
+        return call
+
+
+def test_update_runs_independent_lora_groups_on_their_own_streams():
+    """Two projection groups: the first group's gradients on the update's
+    stream, the second on a side stream that waits for an event recorded on
+    the update's stream before the first call (after Eq. 10) and is joined
+    before the SGD steps."""
+    import types
+    wl = wk.WORKLOADS["32b"]
+    fake = _FakeCuda()
+    u = object.__new__(bench.Update)
+    u.attt, u.wl, u.grad_steps = _StreamRecorder(), wl, 1
+    u.torch = types.SimpleNamespace(cuda=fake)
+    u.hist = u.x = u.w = u.h = u.W = u.loss = u.dh = u.ws_ce = None
+    u.projs = list(wl.projs)
+    u.groups = {}
+    for i, p in enumerate(u.projs):
+        u.groups.setdefault(p.x_group, []).append(i)
+    assert len(u.groups) == 2
+    u.ws_lora = {g: None for g in u.groups}
+    u.xin = {g: None for g in u.groups}
+    u.dy = u.A16 = u.B16 = u.A32 = u.B32 = u.dA = u.dB = [None] * len(u.projs)
+    u.side = [fake.Stream("side0")]
+    u.step()
+    names = [c[0] for c in u.attt.calls]
+    P = len(u.projs)
+    assert names == (["attt_ngram_weights", "attt_weighted_ce_fwd_bwd", "attt_lora_grad", "attt_lora_grad"]
+                     + ["attt_lora_step"] * P + ["attt_history_insert"])
+    lora = [c for c in u.attt.calls if c[0] == "attt_lora_grad"]
+    assert lora == [("attt_lora_grad", "main"), ("attt_lora_grad", "side0")]
+    (_, s0, fork), (_, s1, waited), (_, s2, join), (_, s3, joined) = fake.log
+    assert (s0, s1, s2, s3) == ("main", "side0", "side0", "main")
+    assert waited == fork and joined == join
