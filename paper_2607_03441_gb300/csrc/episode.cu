@@ -19,6 +19,9 @@
 // owns its device buffers (allocated once at create) and one workspace that
 // the calls share, since they run one after another on the caller's stream
 // and the first kernel of each call waits for the previous call to finish.
+// Two calls run beside that chain on streams of their own, ordered by events:
+// the history append (after the weights) and dx (after dy is written; joined
+// before the SGD step), the latter with a workspace of its own.
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -53,6 +56,13 @@ struct attt_episode {
     // table); the update's own stream waits for it before the call returns.
     cudaStream_t side;
     cudaEvent_t ev_weights, ev_append;
+    // dx of a gradient step runs on its own stream with its own workspace,
+    // beside the adapter gradients: both read dy and the adapter, neither
+    // writes what the other reads, and the step waits for both.
+    cudaStream_t side_dx;
+    cudaEvent_t ev_dy, ev_dx;
+    void *ws_dx;
+    size_t ws_dx_bytes;
 };
 
 namespace {
@@ -68,11 +78,14 @@ bool dev_alloc(T **p, size_t count) {
 void free_all(attt_episode *e) {
     if (e->hist) attt_history_destroy(e->hist);
     void *bufs[] = {e->A32, e->B32, e->A0, e->B0, e->dA, e->dB, e->mA, e->vA, e->mB, e->vB, e->A16, e->B16, e->w,
-                    e->dh,  e->losses, e->h, e->dy, e->h_base, e->pend_tok, e->pend_x, e->ws};
+                    e->dh,  e->losses, e->h, e->dy, e->h_base, e->pend_tok, e->pend_x, e->ws, e->ws_dx};
     for (void *b : bufs) cudaFree(b);
     if (e->ev_weights) cudaEventDestroy(e->ev_weights);
     if (e->ev_append) cudaEventDestroy(e->ev_append);
     if (e->side) cudaStreamDestroy(e->side);
+    if (e->ev_dy) cudaEventDestroy(e->ev_dy);
+    if (e->ev_dx) cudaEventDestroy(e->ev_dx);
+    if (e->side_dx) cudaStreamDestroy(e->side_dx);
 }
 
 // H <- H || x on the side stream once the update's weights (enqueued on
@@ -105,7 +118,6 @@ size_t workspace_bound(const attt_episode_config &c) {
     const int64_t L = c.max_update;
     upd(attt_lora_workspace_bytes(L, c.din, 1, &c.d, c.r));
     upd(attt_lora_forward_workspace_bytes(L, c.din, c.d, c.r));
-    upd(attt_lora_input_grad_workspace_bytes(L, c.din, c.d, c.r));
     upd(attt_kl_workspace_bytes(L, c.d, c.V));  // grows with L
     return ws;
 }
@@ -159,11 +171,16 @@ attt_status attt_episode_create(const attt_episode_config *cfg, const attt_bf16 
          dev_alloc(&e->pend_tok, (size_t)c.max_update) &&
          dev_alloc(&e->pend_x, (size_t)c.max_update * c.din) &&
          dev_alloc(reinterpret_cast<char **>(&e->ws), e->ws_bytes);
+    e->ws_dx_bytes = attt_lora_input_grad_workspace_bytes(c.max_update, c.din, c.d, c.r);
+    ok = ok && dev_alloc(reinterpret_cast<char **>(&e->ws_dx), e->ws_dx_bytes);
     if (ok && c.optimizer == 1)
         ok = dev_alloc(&e->mA, nA) && dev_alloc(&e->vA, nA) && dev_alloc(&e->mB, nB) && dev_alloc(&e->vB, nB);
     ok = ok && cudaStreamCreateWithFlags(&e->side, cudaStreamNonBlocking) == cudaSuccess &&
          cudaEventCreateWithFlags(&e->ev_weights, cudaEventDisableTiming) == cudaSuccess &&
-         cudaEventCreateWithFlags(&e->ev_append, cudaEventDisableTiming) == cudaSuccess;
+         cudaEventCreateWithFlags(&e->ev_append, cudaEventDisableTiming) == cudaSuccess &&
+         cudaStreamCreateWithFlags(&e->side_dx, cudaStreamNonBlocking) == cudaSuccess &&
+         cudaEventCreateWithFlags(&e->ev_dy, cudaEventDisableTiming) == cudaSuccess &&
+         cudaEventCreateWithFlags(&e->ev_dx, cudaEventDisableTiming) == cudaSuccess;
     if (ok) {
         // The initial adapter is copied once; later resets restore it.
         ok = cudaMemcpy(e->A0, d_A0, nA * sizeof(float), cudaMemcpyDeviceToDevice) == cudaSuccess &&
@@ -220,15 +237,28 @@ attt_status attt_episode_update(attt_episode *e, const int32_t *d_tokens, const 
             st = attt_weighted_ce_fwd_bwd(e->h, e->Wlm, d_tokens, e->w, L, c.d, c.V, losses + g, e->dh, nullptr,
                                           e->ws, e->ws_bytes, stream);
         if (st == ATTT_OK) st = attt_cast_bf16(e->dh, e->dy, L * c.d, stream);
+        // dx on its own stream once dy is written, beside the adapter gradients
+        bool dx_beside = false;
+        if (st == ATTT_OK && d_dx) {
+            if (cudaEventRecord(e->ev_dy, stream) != cudaSuccess ||
+                cudaStreamWaitEvent(e->side_dx, e->ev_dy, 0) != cudaSuccess) {
+                st = ATTT_ERR_CUDA;
+            } else {
+                st = attt_lora_input_grad(e->dy, e->W0, e->A16, e->B16, L, c.din, c.d, c.r, c.scale,
+                                          d_dx + (size_t)g * L * c.din, e->ws_dx, e->ws_dx_bytes, e->side_dx);
+                dx_beside = true;
+                if (cudaEventRecord(e->ev_dx, e->side_dx) != cudaSuccess && st == ATTT_OK) st = ATTT_ERR_CUDA;
+            }
+        }
         if (st == ATTT_OK) {
             const attt_bf16 *dys[1] = {e->dy}, *As[1] = {e->A16}, *Bs[1] = {e->B16};
             float *dAs[1] = {e->dA}, *dBs[1] = {e->dB};
             st = attt_lora_grad(d_x, L, c.din, 1, dys, &c.d, As, Bs, c.r, c.scale, dAs, dBs, e->ws, e->ws_bytes,
                                 stream);
         }
-        if (st == ATTT_OK && d_dx)
-            st = attt_lora_input_grad(e->dy, e->W0, e->A16, e->B16, L, c.din, c.d, c.r, c.scale,
-                                      d_dx + (size_t)g * L * c.din, e->ws, e->ws_bytes, stream);
+        // the step changes the adapter that dx reads: it waits for dx
+        if (dx_beside && cudaStreamWaitEvent(stream, e->ev_dx, 0) != cudaSuccess && st == ATTT_OK)
+            st = ATTT_ERR_CUDA;
         if (st == ATTT_OK) {
             if (c.optimizer == 0) {
                 st = attt_lora_step(e->A32, e->B32, e->dA, e->dB, c.din, c.d, c.r, c.lr, e->A16, e->B16, stream);
