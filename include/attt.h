@@ -31,6 +31,11 @@
  *   - No call aborts, traps or throws.  Every device-side wait is bounded;
  *     a wait that runs out sets ATTT_ERR_TIMEOUT and the kernel returns.
  *   - Inputs must not alias outputs unless a call says so.
+ *   - Calls may run concurrently on different streams when they share no
+ *     written buffer: each its own outputs and workspace, and no history or
+ *     episode object used by two of them at once (attt_lora_grad_noalloc's
+ *     static scratch is one per device: its calls are serialised by the
+ *     caller).  Kernel errors of either land in the same status word.
  */
 #ifndef ATTT_H
 #define ATTT_H
